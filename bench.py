@@ -1,0 +1,431 @@
+#!/usr/bin/env python
+"""Benchmark of the Chameleon format-adaptive quantized linear path on GB300.
+
+Workload: the SDXL-UNet attention/FFN projections at batch 2 with classifier-free guidance, W8A8
+(q/k/v/out 8192x640x640 x4, 2048x1280x1280 x4, GEGLU-in 2048x1280->10240, FF-out 2048x5120->1280),
+seeded synthetic activations over the 10 timestep buckets.  One step is one pass of the whole hot
+path: per-channel weight-format selection and pack of all 10 layers, then for every bucket and
+layer the activation quantizer in the format the (layer, bucket) LUT picks and the tcgen05 GEMM.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on a bounded sample of the
+same workload instead.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")   # the oracle's timed leg runs on one core
+os.environ.setdefault("OMP_NUM_THREADS", "1")
+
+import numpy as np  # noqa: E402
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "mixed-format linear TFLOP/s & % tensor peak; act-quant HBM GB/s"
+WORKLOAD = "SDXL-UNet attention/FFN projections, W8A8, batch 2 (CFG), 10 timestep buckets"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_BYTES = 126 * 2 ** 20
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of the dominant kernel from an ncu
+# capture (None until a capture of the current kernel exists)
+GEMM_TRAFFIC_PER_LAUNCH = None
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return PEAKS_FALLBACK, "fallback"
+
+
+# ------------------------------------------------------------------ clocks during the timed region
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+        return False
+
+    def summary(self):
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ workload
+def layer_flops(M, K, N):
+    return 2.0 * M * K * N
+
+
+def host_inputs(WL):
+    """Weights, biases and the activations of every (layer, bucket), generated once on the host."""
+    layers = WL.SDXL_PROJ_LAYERS
+    Wn, bn, Xn = [], [], []
+    for li in range(len(layers)):
+        w, b = WL.sdxl_layer_weights(li)
+        Wn.append(w)
+        bn.append(b)
+        Xn.append([WL.sdxl_layer_activation(li, bk) for bk in range(10)])
+    return Wn, bn, Xn
+
+
+def build_inputs(torch, host, device):
+    Wn, bn, Xn = host
+    W = [torch.from_numpy(w).to(device) for w in Wn]
+    bias = [torch.from_numpy(b).to(device) for b in bn]
+    X = [[torch.from_numpy(x).to(device) for x in xs] for xs in Xn]
+    return W, bias, X
+
+
+def calibrate_lut(torch, cl, X, device):
+    """Alg. 1 on the synthetic activations: power sums on the GPU, kappa, SNR at the bucket
+    midpoint (scaled-linear schedule), Route -> F[l, b]."""
+    snr = cl.snr(cl.SCHEDULE_SCALED_LINEAR, 1000)
+    lut = np.zeros((len(X), 10), dtype=np.int64)
+    kappa = np.zeros((len(X), 10))
+    for li, xs in enumerate(X):
+        for bk, x in enumerate(xs):
+            sums = cl.act_moments(x).cpu().numpy()
+            kappa[li, bk] = cl.kurtosis(sums[:5])
+            lut[li, bk] = cl.route(kappa[li, bk], snr[bk * 100 + 50], False)
+    return lut, kappa
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        print(json.dumps(reference_arm(args, world)), flush=True)
+        return 0
+
+    import torch
+    import torch.distributed as dist
+    import paper_2609_33496_gb300 as P
+    from paper_2609_33496_gb300 import build as B
+    from paper_2609_33496_gb300 import workloads as WL
+
+    B.build()
+    cl = P.chameleon
+    cl.lib()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=device)
+
+    layers = WL.SDXL_PROJ_LAYERS
+    host = host_inputs(WL)
+    W, bias, X = build_inputs(torch, host, device)
+    lut, kappa = calibrate_lut(torch, cl, X, device)
+    st = torch.zeros(1, dtype=torch.int32, device=device)
+    stream = torch.cuda.current_stream()
+
+    # buffers reused every step
+    Y = [torch.empty((M, N), dtype=torch.float32, device=device) for (_, M, K, N) in layers]
+    ws = [torch.empty(max(cl.linear_workspace_size(M, cl.pack_plan(N, K, np.zeros(N, np.uint8)), f)
+                          for f in range(6)), dtype=torch.uint8, device=device) for (_, M, K, N) in layers]
+
+    def select_pack():
+        descs, blobs = [], []
+        fmts = [cl.select_weight_formats(W[li], cl.PALETTE_W8)[0] for li in range(len(layers))]
+        fmts_host = [f.cpu().numpy() for f in fmts]           # the plan needs the counts on the host
+        for li, (_, M, K, N) in enumerate(layers):
+            d = cl.pack_plan(N, K, fmts_host[li])
+            blob, _ = cl.pack_weights(W[li], fmts[li], d, dev_status=st)
+            descs.append(d)
+            blobs.append(blob)
+        return descs, blobs, fmts_host
+
+    flops_step = 10 * sum(layer_flops(M, K, N) for (_, M, K, N) in layers)
+    quant_bytes_step = 0.0
+    gemm_bytes_step = 0.0
+
+    def run_step(descs, blobs, ev):
+        for bk in range(10):
+            for li, (_, M, K, N) in enumerate(layers):
+                f = int(lut[li, bk])
+                if ev is not None:
+                    ev.append(("q", li, bk, torch.cuda.Event(enable_timing=True)))
+                    ev[-1][3].record(stream)
+                cl.linear_prepare(X[li][bk], f, ws[li], st)
+                if ev is not None:
+                    ev.append(("g", li, bk, torch.cuda.Event(enable_timing=True)))
+                    ev[-1][3].record(stream)
+                cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
+        if ev is not None:
+            ev.append(("end", -1, -1, torch.cuda.Event(enable_timing=True)))
+            ev[-1][3].record(stream)
+
+    # warm-up
+    for _ in range(args.warmup):
+        descs, blobs, fmts_host = select_pack()
+        run_step(descs, blobs, None)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0, "device status %d" % int(st.item())
+
+    # kernel launches per step: select 1 + pack 3 per layer; per linear 2 (per-tensor) or 1 (MX)
+    # quantizer kernels + 1 GEMM
+    launches = 4 * len(layers) + sum(
+        (2 if lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(10))
+    for li, (_, M, K, N) in enumerate(layers):
+        for bk in range(10):
+            mx = lut[li, bk] >= 3
+            quant_bytes_step += M * K * 2 + M * K * 2 + (M * K / 32 if mx else 0)
+            gemm_bytes_step += M * K * 1 + N * K * 1 + N * (4 + 1) + 4 * N + M * N * 4
+    # ---------------------------------------------------------------- timed region (device)
+    all_ev = []
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for _ in range(args.steps):
+            descs, blobs, fmts_host = select_pack()
+            ev = []
+            run_step(descs, blobs, ev)
+            all_ev.append(ev)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([elapsed_ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(tt.item())
+    assert int(st.item()) == 0, "device status %d" % int(st.item())
+
+    # per-kernel durations from the events
+    gemm_ms, quant_ms, gemm_launch_ms = 0.0, 0.0, []
+    for ev in all_ev:
+        for i in range(len(ev) - 1):
+            kind, li, bk, e = ev[i]
+            d = e.elapsed_time(ev[i + 1][3])
+            if kind == "g":
+                gemm_ms += d
+                gemm_launch_ms.append(d)
+            elif kind == "q":
+                quant_ms += d
+    K_ = args.steps
+    value = world * flops_step * K_ / (elapsed_ms * 1e-3) / 1e12
+    pk, pk_kind = peaks()
+    peak_tensor = pk.get("bf16_tflops_sustained", pk.get("bf16_tflops"))
+    gemm_tflops = flops_step * K_ / (gemm_ms * 1e-3) / 1e12
+    quant_gbs = quant_bytes_step * K_ / (quant_ms * 1e-3) / 1e9
+    # roofline time of every GEMM launch: max(flops / tensor peak, algorithmic bytes / HBM peak)
+    t_roof = 0.0
+    for li, (_, M, K, N) in enumerate(layers):
+        b = M * K + N * K + 5 * N + 4 * N + 4 * M * N
+        t_roof += 10 * max(layer_flops(M, K, N) / (peak_tensor * 1e12), b / (pk["hbm_gbs"] * 1e9))
+    clocks = clk.summary()
+
+    result = {
+        "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
+        "warmup": args.warmup, "ms_per_step": round(elapsed_ms / K_, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "layers": len(layers), "buckets": 10, "global_batch": 2 * world,
+                   "tokens": [M for (_, M, _, _) in layers], "weight_palette": "W8 {INT8-sym, INT8-asym, MXINT8}",
+                   "activation_formats_used": sorted(set(int(v) for v in lut.ravel())),
+                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant + GEMM",
+                   "l2": "inputs larger than L2 (%.0f MB of activations per step)" %
+                         (sum(x.numel() * 2 for xs in X for x in xs) / 1e6),
+                   "parallelism": "replicas" if world > 1 else "single-gpu"},
+        "roofline": {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak_tensor,
+                     "unit": "TFLOP/s", "frac": round(gemm_tflops / peak_tensor, 4),
+                     "traffic": GEMM_TRAFFIC_PER_LAUNCH,
+                     "kernel": "k_gemm_ts_f16 (tcgen05 kind::f16, weights decoded into TMEM)",
+                     "peak_source": "%s bf16_tflops_sustained (fp16 MMA rate = bf16 rate)" % pk_kind,
+                     "roofline_time_frac": round(t_roof * K_ / (gemm_ms * 1e-3), 4),
+                     "gemm_ms_per_step": round(gemm_ms / K_, 4),
+                     "gemm_launch_ms_mean": round(statistics.mean(gemm_launch_ms), 5)},
+        "act_quant": {"achieved_gbs": round(quant_gbs, 1), "peak_gbs": pk["hbm_gbs"],
+                      "frac": round(quant_gbs / pk["hbm_gbs"], 4), "ms_per_step": round(quant_ms / K_, 4),
+                      "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"},
+        "gpu_launches": launches * K_,
+        "clocks": clocks,
+    }
+    if not args.no_e2e:
+        del X
+        result["e2e"] = e2e_leg(args, torch, cl, host, layers, lut, device, stream, world, flops_step)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline()
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def e2e_leg(args, torch, cl, host, layers, lut, device, stream, world, flops_step):
+    """Same step through the public calls with HOST buffers: the weights and every activation are
+    copied host->device from pinned memory and every output device->host inside the timed
+    region."""
+    import torch.distributed as dist
+    Wn, bn, Xn = host
+    Wh = [torch.from_numpy(w).pin_memory() for w in Wn]
+    bh = [torch.from_numpy(b).pin_memory() for b in bn]
+    Xh = [[torch.from_numpy(x).pin_memory() for x in xs] for xs in Xn]
+    Yh = [torch.empty((M, N), dtype=torch.float32).pin_memory() for (_, M, K, N) in layers]
+    Wd = [w.to(device) for w in Wh]
+    bd = [b.to(device) for b in bh]
+    Xd = [torch.empty_like(Xh[li][0], device=device) for li in range(len(layers))]
+    Yd = [torch.empty((M, N), dtype=torch.float32, device=device) for (_, M, K, N) in layers]
+    st = torch.zeros(1, dtype=torch.int32, device=device)
+    ws = [torch.empty(max(cl.linear_workspace_size(M, cl.pack_plan(N, K, np.zeros(N, np.uint8)), f)
+                          for f in range(6)), dtype=torch.uint8, device=device) for (_, M, K, N) in layers]
+    h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + sum(x.numel() * 2 for xs in Xh for x in xs)
+    d2h = 10 * sum(M * N * 4 for (_, M, K, N) in layers)
+
+    def step():
+        fmts, descs, blobs = [], [], []
+        for li in range(len(layers)):
+            Wd[li].copy_(Wh[li], non_blocking=True)
+            bd[li].copy_(bh[li], non_blocking=True)
+            fmts.append(cl.select_weight_formats(Wd[li], cl.PALETTE_W8)[0])
+        for li, (_, M, K, N) in enumerate(layers):
+            d = cl.pack_plan(N, K, fmts[li].cpu().numpy())
+            descs.append(d)
+            blobs.append(cl.pack_weights(Wd[li], fmts[li], d, dev_status=st)[0])
+        for bk in range(10):
+            for li in range(len(layers)):
+                Xd[li].copy_(Xh[li][bk], non_blocking=True)
+                cl.linear(Xd[li], descs[li], blobs[li], int(lut[li, bk]), bias=bd[li], Y=Yd[li], ws=ws[li],
+                          dev_status=st)
+                Yh[li].copy_(Yd[li], non_blocking=True)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        step()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    assert int(st.item()) == 0
+    return {"value": round(world * flops_step * args.steps / (ms * 1e-3) / 1e12, 3), "unit": "TFLOP/s",
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "ms_per_step": round(ms / args.steps, 3)}
+
+
+# ------------------------------------------------------------------ the oracle as CPU baseline
+def oracle_sample(layers_idx=(4,), buckets=(0, 9)):
+    """The oracle on a bounded sample of the workload: for each (layer, bucket) of the sample,
+    per-channel selection over the W8 palette, the activation quantizer in the format the route
+    picks, and the fp64 GEMM over all rows.  Returns (flops, seconds, description)."""
+    from oracle import formats as F
+    from oracle import gemm as G
+    from oracle import schedule as S
+    from oracle import select as SEL
+    from paper_2609_33496_gb300 import workloads as WL
+    snr = S.snr(S.betas_scaled_linear())
+    flops, t = 0.0, 0.0
+    for li in layers_idx:
+        name, M, K, N = WL.SDXL_PROJ_LAYERS[li]
+        W, bias = WL.sdxl_layer_weights(li)
+        for bk in buckets:
+            X = WL.sdxl_layer_activation(li, bk)
+            t0 = time.perf_counter()
+            fmt, _, _ = SEL.select_formats(W, 0x007)
+            f = S.route(S.kurtosis(X), snr[int(S.bucket_midpoint(bk))])
+            G.linear_reference(X, f, W, fmt, bias)
+            t += time.perf_counter() - t0
+            flops += layer_flops(M, K, N)
+    desc = "oracle select(W8)+act-quant+fp64 GEMM of layer(s) %s at buckets %s" % (
+        [WL.SDXL_PROJ_LAYERS[i][0] for i in layers_idx], list(buckets))
+    return flops, t, desc
+
+
+def cpu_baseline():
+    flops, t, desc = oracle_sample()
+    return {"value": round(flops / t / 1e12, 6), "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+            "sample": desc, "seconds": round(t, 2)}
+
+
+def reference_arm(args, world):
+    for _ in range(args.warmup):
+        oracle_sample(buckets=(9,))
+    flops, t = 0.0, 0.0
+    desc = ""
+    for _ in range(args.steps):
+        f, s, desc = oracle_sample(buckets=(9,))
+        flops += f
+        t += s
+    value = flops / t / 1e12
+    return {"metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(1e3 * t / args.steps, 2), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": WORKLOAD, "sample": desc},
+            "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,215 @@
+/*
+ * chameleon.h -- C ABI of the Chameleon format-adaptive quantized linear layer on GB300 (sm_103a).
+ *
+ * Method: arXiv 2609.33496 ("Chameleon: Dynamic Format Adapter for Efficient Diffusion").
+ * Activations are quantized per tensor in the format a per-(layer, timestep-bucket) table picks
+ * (Sec. 3.2-3.3, Alg. 2/3); every weight output channel carries its own format, chosen offline by
+ * reconstruction error (Sec. 3.4); the layer multiplies the two on tcgen05 tensor cores.
+ *
+ * Conventions (all entry points):
+ *   - every call returns a cham_status; CHAM_OK is 0.  chameleon_last_error_detail() gives a
+ *     one-line message for the last failure on the calling host thread.
+ *   - pointers marked (device) are CUDA device pointers owned by the caller; (host) are host
+ *     pointers.  The library never allocates device memory: size queries come first and the caller
+ *     passes buffers of at least the returned size.
+ *   - calls are asynchronous on `stream` (a cudaStream_t passed as void*; NULL = legacy stream) and
+ *     never synchronise, except where a host value is computed.  Errors detected by the kernels
+ *     (non-finite input, a wait that timed out, an MX weight outside fp16) are written to the
+ *     caller's device status word `dev_status` (int32, device): the kernels only ever store a
+ *     non-zero cham_status there; the caller zeroes it and reads it after synchronising.
+ *   - X is fp16, M x K, row-major (K contiguous); W is fp16, N x K (nn.Linear layout); Y is fp32
+ *     M x N row-major; bias is fp32 [N].  Row pitches are exactly K (resp. N) elements.
+ *   - all device pointers must be 16-byte aligned; K must be a multiple of 32.
+ */
+#ifndef CHAMELEON_H
+#define CHAMELEON_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int cham_status;
+#define CHAM_OK 0
+#define CHAM_ERR_INVALID_ARG 1  /* bad size, pointer, alignment or format code (host check) */
+#define CHAM_ERR_UNSUPPORTED 2  /* a valid request this build does not handle */
+#define CHAM_ERR_WORKSPACE 3    /* a buffer is smaller than its size query returned */
+#define CHAM_ERR_NONFINITE 4    /* device: the activation tensor holds Inf or NaN */
+#define CHAM_ERR_TIMEOUT 5      /* device: a bounded wait inside a kernel gave up */
+#define CHAM_ERR_CUDA 6         /* a CUDA runtime/driver call failed */
+#define CHAM_ERR_RANGE 7        /* device: an MX weight block does not decode exactly in fp16 */
+
+/* Activation formats: the runtime LUT codes 0..4 of Sec. 3.2 (F_a), plus 5 = fp16 operands for the
+ * weight-only few-step fork of Sec. 3.5. */
+#define CHAM_A_INT8_ASYM 0
+#define CHAM_A_E4M3 1
+#define CHAM_A_E5M2 2
+#define CHAM_A_MXFP8 3
+#define CHAM_A_MXINT8 4
+#define CHAM_A_FP16 5
+
+/* Weight formats (Sec. 3.2: F_w^(8) and F_w^(4), in palette order = tie-break order). */
+#define CHAM_W_INT8_SYM 0
+#define CHAM_W_INT8_ASYM 1
+#define CHAM_W_MXINT8 2
+#define CHAM_W_INT4_SYM 3
+#define CHAM_W_INT4_ASYM 4
+#define CHAM_W_NF4 5
+#define CHAM_W_E2M1 6
+#define CHAM_W_MXINT4 7
+#define CHAM_W_MXFP4 8
+#define CHAM_W_NFORMATS 9
+#define CHAM_PALETTE_W8 0x007u   /* INT8-sym, INT8-asym, MXINT8 */
+#define CHAM_PALETTE_W4 0x1F8u   /* INT4-sym, INT4-asym, NF4, E2M1, MXINT4, MXFP4 */
+
+/* Noise schedules for chameleon_snr (App. A.1, A.11): scaled-linear (SDXL, beta 0.00085 -> 0.012)
+ * and linear (PixArt-alpha, beta 1e-4 -> 0.02). */
+#define CHAM_SCHEDULE_SCALED_LINEAR 0
+#define CHAM_SCHEDULE_LINEAR 1
+
+const char* chameleon_status_string(cham_status s);
+const char* chameleon_last_error_detail(void);
+int chameleon_version(void);
+
+/* ------------------------------------------------------------------ host helpers (a1, L2) */
+
+/* Bucket of timestep t: b = min(floor(t / (T/B)), B-1) (Alg. 2 and Alg. 3).  Returns -1 when
+ * T <= 0, B <= 0 or t < 0. */
+int chameleon_bucket(int t, int T, int B);
+
+/* SNR(t) = abar_t / (1 - abar_t), abar_t = prod_{s<=t} (1 - beta_s), t = 0..T-1 (Sec. 2.1,
+ * Eq. snr).  snr_out (host) receives T doubles. */
+cham_status chameleon_snr(int schedule, int T, double* snr_out);
+
+/* Kurtosis kappa = m4 / m2^2 from the power sums {n, S1, S2, S3, S4} (App. A.2 Eq. kurt, Alg. 1);
+ * 0 when the variance is 0. */
+double chameleon_kurtosis(const double sums[5]);
+
+/* Routing rule of Sec. 3.3 at SNR(t_b): shortcut -> MXFP8; kappa > 5 or snr < 0.2 -> E5M2;
+ * kappa <= 3 and snr > 2 -> INT8-asym; else E4M3.  Returns an activation format code. */
+int chameleon_route(double kappa, double snr_b, int is_shortcut);
+
+/* ------------------------------------------------------------------ calibration statistics */
+
+/* Power sums of one activation tensor, the accumulator of Alg. 1 (Sec. 3.5):
+ * out (device, 7 doubles) = {n, sum x, sum x^2, sum x^3, sum x^4, min, max}, ADDED to what `out`
+ * holds for n and the sums, min/max merged (so calls accumulate across steps like Alg. 1; zero
+ * the first five and set min = +inf, max = -inf before the first call).  X fp16 (device), count
+ * elements.  ws (device) >= chameleon_act_moments_workspace_size bytes. */
+cham_status chameleon_act_moments_workspace_size(int64_t count, size_t* ws_bytes);
+cham_status chameleon_act_moments(const void* X, int64_t count, double* out, void* ws,
+                                  size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------ a2-a4: activation quantizer */
+
+/* Quantized-activation buffer layout (qact, device), for fmt in 0..4:
+ *   [0, M*K)                codes, uint8 row-major: INT8-asym q; E4M3 / E5M2 / MXFP8 bit pattern;
+ *                           MXINT8 two's-complement int8
+ *   [P, P+16), P = round_up(M*K, 256): cham_qparams {float s; int32 z; float inv; int32 fmt}
+ *                           (per-tensor formats; MX formats store s = 1, z = 0, inv = 1)
+ *   [P+256, P+256+M*K/32)   E8M0 block exponents, uint8 M x (K/32) row-major (MX formats only)
+ * Dequantized value: INT8-asym (q - z) * s; E4M3/E5M2 value(code) * s; MXFP8 value(code) * 2^(e-127);
+ * MXINT8 code * 2^-6 * 2^(e-127)  (App. A.7 ScaleZP, App. A.11; readings R1-R8 in the design doc). */
+typedef struct {
+  float s;
+  int32_t z;
+  float inv;
+  int32_t fmt;
+} cham_qparams;
+
+cham_status chameleon_act_quant_size(int M, int K, int fmt, size_t* qact_bytes, size_t* ws_bytes);
+
+/* Quantize X (device, fp16 M x K) in activation format fmt with its own dynamic range (Alg. 3:
+ * lo, hi = min x, max x; ScaleZP; fq_f).  Writes qact (device, qact_bytes); ws (device) is
+ * scratch of ws_bytes.  Non-finite input sets *dev_status = CHAM_ERR_NONFINITE (codes then
+ * unspecified). */
+cham_status chameleon_act_quant(const void* X, int M, int K, int fmt, void* qact, size_t qact_bytes,
+                                void* ws, size_t ws_bytes, int* dev_status, void* stream);
+
+/* ------------------------------------------------------------------ a5: weight-format selection */
+
+/* Per output channel c of W (device, fp16 N x K): SSE_f(c) = sum_k (w - DQ_f(Q_f(w)))^2 for every
+ * format f in palette_mask (bits = weight format codes; all members of one bit width), and
+ * fmt_out[c] (device, uint8 [N]) = argmin, first in palette order on ties (Sec. 3.4, Eq.
+ * weight-argmax: the SQNR argmax is the SSE argmin).  sse_out (device, double N x 9, row c holds
+ * the 9 format slots, +inf for non-members) may be NULL. */
+cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_t palette_mask,
+                                            uint8_t* fmt_out, double* sse_out, void* stream);
+
+/* ------------------------------------------------------------------ a6: weight pack */
+
+/* Packed-weight descriptor.  Channels are permuted (Sec. 5: "same-format sub-GEMMs after a
+ * channel permutation") into two MMA classes, each padded to 128-channel tiles:
+ *   class 0 = 4-bit formats with an 8-bit tensor-core path (INT4-sym, INT4-asym, E2M1, MXINT4,
+ *             MXFP4), class 1 = the rest (NF4, INT8-sym, INT8-asym, MXINT8);
+ * inside a class by format in that order, then by original channel index.  Offsets are from the
+ * blob base, 256-byte aligned.  Blob regions:
+ *   [0, 256)       a copy of this descriptor
+ *   codes          per tile t (128 packed channels) and K-chunk c (64 elements): 128 * CB bytes,
+ *                  CB = 64 (8-bit) or 32 (4-bit) bytes per channel, stored as CB/16 slabs of
+ *                  128 x 16 bytes: slab j holds bytes [16j, 16j+16) of every channel's CB bytes.
+ *                  8-bit: byte i = element i of the chunk (int8 two's complement for INT8-sym and
+ *                  MXINT8, uint8 q for INT8-asym).  4-bit: each 32-bit word holds 8 elements
+ *                  e0..e7, nibble j (bits 4j..4j+3) = e_{2j} for j < 4 and e_{2(j-4)+1} for j >= 4;
+ *                  INT4-sym/MXINT4 two's complement, INT4-asym q, NF4 level index, E2M1/MXFP4
+ *                  bit pattern.  Elements k >= K are code 0.
+ *   scale          float [Np]: per-channel scale s (1 for MX and padding)
+ *   zero           uint8 [Np]: zero point z (asym formats, else 0)
+ *   e8m0           uint8 [tiles][Kp/64][128][2]: the two E8M0 exponents of each channel's chunk
+ *                  (MX formats; 127 otherwise)
+ *   fmt            uint8 [Np]: format of each packed channel, 255 for padding
+ *   perm           int32 [Np]: original channel of each packed channel, -1 for padding
+ * with Np = 128 * (n_tiles[0] + n_tiles[1]) and Kp = K rounded up to 64. */
+typedef struct {
+  uint32_t magic;    /* 0x574D4843 ("CHMW") */
+  uint32_t version;  /* 1 */
+  int32_t N, K, Kp, bits;
+  int32_t n_class[2];
+  int32_t n_tiles[2];
+  int32_t n_fmt[CHAM_W_NFORMATS];
+  int32_t reserved0;
+  uint64_t off_codes, off_scale, off_zero, off_e8m0, off_fmt, off_perm, bytes;
+  uint8_t reserved[120];      /* pads the descriptor to 256 bytes */
+} cham_wpack_desc;
+
+/* Fill *desc for N x K weights whose selected formats are fmt_host (host, uint8 [N], all of one
+ * bit width).  desc->bytes is the blob size. */
+cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* desc);
+
+/* Encode W (device, fp16 N x K) with each channel in fmt_dev[c] (device copy of the formats the
+ * plan was made from) into blob (device, >= desc->bytes).  An MX channel whose dequantized values
+ * are not all exact fp16 values sets *dev_status = CHAM_ERR_RANGE. */
+cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const cham_wpack_desc* desc,
+                                   void* blob, size_t blob_bytes, int* dev_status, void* stream);
+
+/* ------------------------------------------------------------------ a7/a8: quantized linear */
+
+cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* desc, int act_fmt,
+                                            size_t* ws_bytes);
+
+/* Y = DQ(Q_act_fmt(X)) . DQ(W)^T + bias: X (device, fp16 M x desc->K) is quantized in act_fmt
+ * (= F[layer, bucket] resolved on the host, Alg. 2/3) with its own range, multiplied on tcgen05
+ * tensor cores with the packed weights (device blob made from *desc, host), fp32 accumulation;
+ * Y (device, fp32 M x desc->N) in original channel order.  bias (device, fp32 [N]) may be NULL.
+ * act_fmt = CHAM_A_FP16 multiplies X itself (weight-only fork).  ws (device) >= the size query. */
+cham_status chameleon_linear(const void* X, int M, const cham_wpack_desc* desc, const void* blob,
+                             int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
+                             int* dev_status, void* stream);
+
+/* The two halves of chameleon_linear, for callers that schedule or time them separately.
+ * chameleon_linear_prepare quantizes X (device, fp16 M x K) in act_fmt into ws (the GEMM operand:
+ * the exact fp16 value of every code, R13, plus the per-tensor scale; nothing for CHAM_A_FP16).
+ * chameleon_linear_gemm multiplies that operand (or X itself for CHAM_A_FP16; X may be NULL
+ * otherwise) with the packed weights.  Same arguments, workspace and errors as chameleon_linear. */
+cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, void* ws, size_t ws_bytes,
+                                     int* dev_status, void* stream);
+cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* desc, const void* blob,
+                                  int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
+                                  int* dev_status, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CHAMELEON_H */

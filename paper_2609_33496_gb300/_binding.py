@@ -1,0 +1,259 @@
+"""ctypes binding of libchameleon (include/chameleon.h): argument marshalling only.
+
+Every step of the quantized linear runs in the library's CUDA kernels; this module only turns torch
+tensors into pointers, allocates the buffers the size queries ask for (through torch) and raises
+when a call fails.  There is no fallback: without the built library every call raises.
+"""
+import ctypes
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libchameleon.so")
+
+# status codes
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_WORKSPACE, ERR_NONFINITE, ERR_TIMEOUT, ERR_CUDA, ERR_RANGE = range(8)
+# activation formats (Sec. 3.2 codes) and the fp16 operand of the weight-only fork
+A_INT8_ASYM, A_E4M3, A_E5M2, A_MXFP8, A_MXINT8, A_FP16 = range(6)
+# weight formats in palette order
+(W_INT8_SYM, W_INT8_ASYM, W_MXINT8, W_INT4_SYM, W_INT4_ASYM, W_NF4, W_E2M1, W_MXINT4,
+ W_MXFP4) = range(9)
+PALETTE_W8 = 0x007
+PALETTE_W4 = 0x1F8
+SCHEDULE_SCALED_LINEAR, SCHEDULE_LINEAR = 0, 1
+
+EXPORTS = [
+    "chameleon_status_string", "chameleon_last_error_detail", "chameleon_version",
+    "chameleon_bucket", "chameleon_snr", "chameleon_kurtosis", "chameleon_route",
+    "chameleon_act_moments_workspace_size", "chameleon_act_moments",
+    "chameleon_act_quant_size", "chameleon_act_quant",
+    "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_weights",
+    "chameleon_linear_workspace_size", "chameleon_linear", "chameleon_linear_prepare",
+    "chameleon_linear_gemm",
+]
+
+
+class WPackDesc(ctypes.Structure):
+    """cham_wpack_desc (256 bytes)."""
+    _fields_ = [("magic", ctypes.c_uint32), ("version", ctypes.c_uint32),
+                ("N", ctypes.c_int32), ("K", ctypes.c_int32), ("Kp", ctypes.c_int32),
+                ("bits", ctypes.c_int32), ("n_class", ctypes.c_int32 * 2),
+                ("n_tiles", ctypes.c_int32 * 2), ("n_fmt", ctypes.c_int32 * 9),
+                ("reserved0", ctypes.c_int32),
+                ("off_codes", ctypes.c_uint64), ("off_scale", ctypes.c_uint64),
+                ("off_zero", ctypes.c_uint64), ("off_e8m0", ctypes.c_uint64),
+                ("off_fmt", ctypes.c_uint64), ("off_perm", ctypes.c_uint64),
+                ("bytes", ctypes.c_uint64), ("reserved", ctypes.c_uint8 * 120)]
+
+
+assert ctypes.sizeof(WPackDesc) == 256
+
+_lib = None
+
+
+class ChameleonError(RuntimeError):
+    def __init__(self, status, detail):
+        super().__init__("chameleon status %d (%s): %s" % (status, STATUS_NAMES.get(status, "?"), detail))
+        self.status = status
+
+
+STATUS_NAMES = {OK: "ok", ERR_INVALID_ARG: "invalid argument", ERR_UNSUPPORTED: "unsupported",
+                ERR_WORKSPACE: "workspace too small", ERR_NONFINITE: "non-finite activation",
+                ERR_TIMEOUT: "device wait timed out", ERR_CUDA: "CUDA error",
+                ERR_RANGE: "MX weight outside fp16"}
+
+
+def lib():
+    """The loaded library (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError("libchameleon.so is not built: run `python -m paper_2609_33496_gb300.build` "
+                           "(there is no fallback path)")
+    L = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64, u32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_uint32, ctypes.c_size_t
+    psz = ctypes.POINTER(ctypes.c_size_t)
+    pdesc = ctypes.POINTER(WPackDesc)
+    sig = {
+        "chameleon_status_string": (ctypes.c_char_p, [i32]),
+        "chameleon_last_error_detail": (ctypes.c_char_p, []),
+        "chameleon_version": (i32, []),
+        "chameleon_bucket": (i32, [i32, i32, i32]),
+        "chameleon_snr": (i32, [i32, i32, ctypes.POINTER(ctypes.c_double)]),
+        "chameleon_kurtosis": (ctypes.c_double, [ctypes.POINTER(ctypes.c_double)]),
+        "chameleon_route": (i32, [ctypes.c_double, ctypes.c_double, i32]),
+        "chameleon_act_moments_workspace_size": (i32, [i64, psz]),
+        "chameleon_act_moments": (i32, [vp, i64, vp, vp, sz, vp]),
+        "chameleon_act_quant_size": (i32, [i32, i32, i32, psz, psz]),
+        "chameleon_act_quant": (i32, [vp, i32, i32, i32, vp, sz, vp, sz, vp, vp]),
+        "chameleon_select_weight_formats": (i32, [vp, i32, i32, u32, vp, vp, vp]),
+        "chameleon_pack_plan": (i32, [i32, i32, vp, pdesc]),
+        "chameleon_pack_weights": (i32, [vp, vp, pdesc, vp, sz, vp, vp]),
+        "chameleon_linear_workspace_size": (i32, [i32, pdesc, i32, psz]),
+        "chameleon_linear": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
+        "chameleon_linear_prepare": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
+        "chameleon_linear_gemm": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = L
+    return L
+
+
+def check(status):
+    if status != OK:
+        raise ChameleonError(status, lib().chameleon_last_error_detail().decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _bytes(n, device):
+    import torch
+    return torch.empty(max(int(n), 16), dtype=torch.uint8, device=device)
+
+
+# ------------------------------------------------------------------ host helpers
+def bucket(t, T=1000, B=10):
+    return lib().chameleon_bucket(int(t), int(T), int(B))
+
+
+def snr(schedule=SCHEDULE_SCALED_LINEAR, T=1000):
+    out = np.zeros(T, dtype=np.float64)
+    check(lib().chameleon_snr(schedule, T, out.ctypes.data_as(ctypes.POINTER(ctypes.c_double))))
+    return out
+
+
+def kurtosis(sums):
+    arr = (ctypes.c_double * 5)(*[float(s) for s in sums[:5]])
+    return lib().chameleon_kurtosis(arr)
+
+
+def route(kappa, snr_b, is_shortcut=False):
+    return lib().chameleon_route(float(kappa), float(snr_b), int(bool(is_shortcut)))
+
+
+# ------------------------------------------------------------------ calibration sums
+def act_moments(X, out=None, stream=None):
+    """Alg. 1 accumulator {n, S1..S4, min, max} of the fp16 tensor X, added into `out` (a
+    7-element float64 CUDA tensor; a fresh one when None)."""
+    import torch
+    if out is None:
+        out = torch.tensor([0, 0, 0, 0, 0, float("inf"), float("-inf")], dtype=torch.float64, device=X.device)
+    n = X.numel()
+    ws_b = ctypes.c_size_t()
+    check(lib().chameleon_act_moments_workspace_size(n, ctypes.byref(ws_b)))
+    ws = _bytes(ws_b.value, X.device)
+    check(lib().chameleon_act_moments(_ptr(X), n, _ptr(out), _ptr(ws), ws_b.value, _stream(stream)))
+    return out
+
+
+# ------------------------------------------------------------------ a2-a4
+def act_quant_size(M, K, fmt):
+    q, w = ctypes.c_size_t(), ctypes.c_size_t()
+    check(lib().chameleon_act_quant_size(M, K, fmt, ctypes.byref(q), ctypes.byref(w)))
+    return q.value, w.value
+
+
+def act_quant(X, fmt, dev_status=None, stream=None):
+    """Quantize fp16 X (M x K, CUDA) in activation format fmt.  Returns the raw qact byte buffer
+    (layout of include/chameleon.h) and the device status word."""
+    import torch
+    M, K = X.shape
+    qb, wb = act_quant_size(M, K, fmt)
+    qact = _bytes(qb, X.device)
+    ws = _bytes(wb, X.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
+    check(lib().chameleon_act_quant(_ptr(X), M, K, fmt, _ptr(qact), qb, _ptr(ws), wb, _ptr(dev_status),
+                                    _stream(stream)))
+    return qact, dev_status
+
+
+def split_qact(qact, M, K):
+    """Views of a qact buffer: codes (M x K uint8), params (s, z, inv, fmt), e8m0 (M x K/32)."""
+    import torch
+    n = M * K
+    P = (n + 255) // 256 * 256
+    codes = qact[:n].view(M, K)
+    pbytes = qact[P:P + 16].cpu().numpy().tobytes()
+    s, inv = np.frombuffer(pbytes[0:4], np.float32)[0], np.frombuffer(pbytes[8:12], np.float32)[0]
+    z, fmt = int(np.frombuffer(pbytes[4:8], np.int32)[0]), int(np.frombuffer(pbytes[12:16], np.int32)[0])
+    e8 = qact[P + 256:P + 256 + n // 32].view(M, K // 32)
+    return codes, {"s": s, "z": z, "inv": inv, "fmt": fmt}, e8
+
+
+# ------------------------------------------------------------------ a5
+def select_weight_formats(W, palette_mask, want_sse=False, stream=None):
+    import torch
+    N, K = W.shape
+    fmt = torch.empty(N, dtype=torch.uint8, device=W.device)
+    sse = torch.empty((N, 9), dtype=torch.float64, device=W.device) if want_sse else None
+    check(lib().chameleon_select_weight_formats(_ptr(W), N, K, palette_mask, _ptr(fmt), _ptr(sse),
+                                                _stream(stream)))
+    return fmt, sse
+
+
+# ------------------------------------------------------------------ a6
+def pack_plan(N, K, fmt_host):
+    f = np.ascontiguousarray(np.asarray(fmt_host, dtype=np.uint8))
+    d = WPackDesc()
+    check(lib().chameleon_pack_plan(N, K, f.ctypes.data_as(ctypes.c_void_p), ctypes.byref(d)))
+    return d
+
+
+def pack_weights(W, fmt_dev, desc, dev_status=None, stream=None):
+    import torch
+    blob = _bytes(desc.bytes, W.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=W.device)
+    check(lib().chameleon_pack_weights(_ptr(W), _ptr(fmt_dev), ctypes.byref(desc), _ptr(blob), desc.bytes,
+                                       _ptr(dev_status), _stream(stream)))
+    return blob, dev_status
+
+
+# ------------------------------------------------------------------ a7/a8
+def linear_workspace_size(M, desc, act_fmt):
+    w = ctypes.c_size_t()
+    check(lib().chameleon_linear_workspace_size(M, ctypes.byref(desc), act_fmt, ctypes.byref(w)))
+    return w.value
+
+
+def linear(X, desc, blob, act_fmt, bias=None, Y=None, ws=None, dev_status=None, stream=None):
+    """Y = DQ(Q_act_fmt(X)) DQ(W)^T + bias on the GPU.  Buffers may be passed in for reuse."""
+    import torch
+    M = X.shape[0]
+    need = linear_workspace_size(M, desc, act_fmt)
+    if ws is None or ws.numel() < need:
+        ws = _bytes(need, X.device)
+    if Y is None:
+        Y = torch.empty((M, desc.N), dtype=torch.float32, device=X.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
+    check(lib().chameleon_linear(_ptr(X), M, ctypes.byref(desc), _ptr(blob), act_fmt, _ptr(bias), _ptr(Y),
+                                 _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))
+    return Y, dev_status
+
+
+def linear_prepare(X, act_fmt, ws, dev_status, stream=None):
+    """First half of linear: quantize X into the workspace operand."""
+    M, K = X.shape
+    check(lib().chameleon_linear_prepare(_ptr(X), M, K, act_fmt, _ptr(ws), ws.numel(), _ptr(dev_status),
+                                         _stream(stream)))
+
+
+def linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream=None):
+    """Second half of linear: the tcgen05 GEMM on the prepared operand."""
+    check(lib().chameleon_linear_gemm(_ptr(X), X.shape[0], ctypes.byref(desc), _ptr(blob), act_fmt, _ptr(bias),
+                                      _ptr(Y), _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))

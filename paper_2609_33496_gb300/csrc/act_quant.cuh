@@ -1,0 +1,44 @@
+// act_quant.cuh -- declarations shared by the activation-quantizer kernels and the host API.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace cham {
+
+struct RangePartial {  // one CTA's min / max / non-finite flag of an activation tensor
+  float lo, hi;
+  int nonfinite, pad;
+};
+
+struct TensorParams {  // ScaleZP result of a per-tensor format
+  float s, inv;
+  int z;
+};
+
+struct MomentPartial {  // one CTA's power sums (Alg. 1 accumulator)
+  double s[4];
+  float lo, hi;
+};
+
+struct ActQuantArgs {
+  const uint4* X;          // fp16 tensor, 8 elements per vector
+  int64_t nvec;            // M*K/8
+  RangePartial* parts;     // per-tensor formats: nparts partials (scratch)
+  int nparts;
+  uint2* codes;            // 8 code bytes per vector, or null
+  uint4* deq;              // 8 exact fp16 operand values per vector, or null
+  uint8_t* e8m0;           // MX formats: one byte per 4 vectors, or null
+  cham_qparams* params;    // per-tensor parameters, or null
+  float* scale_out;        // the per-tensor scale s as a bare float (GEMM epilogue), or null
+  int* dev_status;
+  int num_sms;
+};
+
+int range_grid(int64_t nvec, int num_sms);
+void launch_act_quant(int fmt, const ActQuantArgs& a, bool codes, bool deq, cudaStream_t st);
+void launch_act_moments(const uint4* X, int64_t nvec, int64_t count, MomentPartial* parts, int nparts,
+                        double* out, cudaStream_t st);
+
+}  // namespace cham

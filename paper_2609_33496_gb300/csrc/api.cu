@@ -1,0 +1,547 @@
+// api.cu -- the extern "C" entry points of libchameleon (include/chameleon.h).
+//
+// Host side only: argument validation, size queries, buffer carving, tensor-map encoding and
+// kernel launches.  Nothing here allocates device memory or synchronises the device.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "act_quant.cuh"
+#include "gemm.cuh"
+#include "weights.cuh"
+
+static_assert(sizeof(cham_wpack_desc) == 256, "descriptor is 256 bytes");
+static_assert(sizeof(cham_qparams) == 16, "qparams is 16 bytes");
+
+namespace {
+
+thread_local char g_detail[512] = "";
+
+cham_status fail(cham_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_detail, sizeof(g_detail), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+cham_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(CHAM_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int num_sms_current() {
+  static int cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cache[dev] == 0) {
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    cache[dev] = n > 0 ? n : 148;
+  }
+  return cache[dev];
+}
+
+// ---------------------------------------------------------------- NF4 levels (library's own)
+// Quantile construction of NormalFloat-4 (QLoRA, cited in App. A.11): positive levels are the
+// normal quantiles at 9 evenly spaced probabilities from delta to 1/2 (the last, 0, dropped),
+// negative levels the negated quantiles at 8 probabilities from delta to 1/2 (zero dropped), plus
+// one zero, all divided by the largest; delta = mean of 1 - 1/30 and 1 - 1/32.  The inverse
+// normal CDF is solved here by bisection on Phi(x) = erfc(-x / sqrt 2) / 2; the levels are then
+// rounded to fp16 (reading R9).
+double phi_inv(double p) {
+  double lo = -12.0, hi = 12.0;
+  for (int i = 0; i < 200; ++i) {
+    const double mid = 0.5 * (lo + hi);
+    if (0.5 * std::erfc(-mid / std::sqrt(2.0)) < p) lo = mid;
+    else hi = mid;
+  }
+  return 0.5 * (lo + hi);
+}
+
+uint16_t double_to_half_rne(double v) {  // finite |v| <= 65504, normal or zero range suffices here
+  if (v == 0.0) return std::signbit(v) ? 0x8000u : 0u;
+  const uint16_t sign = v < 0 ? 0x8000u : 0u;
+  double a = std::fabs(v);
+  int e;
+  std::frexp(a, &e);
+  e -= 1;                       // a in [2^e, 2^(e+1))
+  if (e < -14) e = -14;         // subnormal binade
+  const double quantum = std::ldexp(1.0, e - 10);
+  double m = std::nearbyint(a / quantum);  // default rounding mode: nearest, ties to even
+  if (m >= 2048.0) {           // rounded up into the next binade
+    m /= 2.0;
+    e += 1;
+  }
+  if (m < 1024.0) return static_cast<uint16_t>(sign | static_cast<uint16_t>(m));  // subnormal
+  return static_cast<uint16_t>(sign | ((e + 15) << 10) | (static_cast<int>(m) - 1024));
+}
+
+double half_bits_to_double(uint16_t h) {
+  const int e = (h >> 10) & 31, m = h & 1023;
+  const double v = e == 0 ? std::ldexp(m, -24) : std::ldexp(1024 + m, e - 25);
+  return (h & 0x8000u) ? -v : v;
+}
+
+const cham::NF4Table& nf4_table() {
+  static cham::NF4Table t;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    const double delta = 0.5 * ((1.0 - 1.0 / 30.0) + (1.0 - 1.0 / 32.0));
+    double v[16];
+    int n = 0;
+    for (int i = 0; i < 7; ++i) v[n++] = -phi_inv(delta + i * (0.5 - delta) / 7.0);
+    v[n++] = 0.0;
+    for (int i = 7; i >= 0; --i) v[n++] = phi_inv(delta + i * (0.5 - delta) / 8.0);
+    const double vmax = phi_inv(delta);
+    for (int i = 0; i < 16; ++i) t.level[i] = double_to_half_rne(v[i] / vmax);
+    for (int i = 0; i < 15; ++i)
+      t.mid[i] = static_cast<float>(0.5 * (half_bits_to_double(t.level[i]) + half_bits_to_double(t.level[i + 1])));
+  });
+  return t;
+}
+
+// ---------------------------------------------------------------- tensor map (TMA descriptor)
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// Row-major fp16 matrix rows x cols, box = 64 columns (128 bytes) x box_rows, 128-byte swizzle.
+cham_status make_act_map(CUtensorMap* map, const void* base, int rows, int cols, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return fail(CHAM_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(CHAM_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return CHAM_OK;
+}
+
+// ---------------------------------------------------------------- activation quantizer carving
+struct ActLayout {
+  size_t codes, params, e8m0, total;
+};
+ActLayout act_layout(int M, int K) {
+  ActLayout L;
+  const size_t n = static_cast<size_t>(M) * K;
+  L.codes = 0;
+  L.params = round_up(n, 256);
+  L.e8m0 = L.params + 256;
+  L.total = L.e8m0 + round_up(n / 32, 256);
+  return L;
+}
+
+size_t range_ws_bytes(int64_t nvec) {
+  return round_up(static_cast<size_t>(cham::range_grid(nvec, num_sms_current())) * sizeof(cham::RangePartial), 256);
+}
+
+cham_status check_act_args(const void* X, int M, int K, int fmt, bool allow_fp16) {
+  if (M <= 0 || K <= 0) return fail(CHAM_ERR_INVALID_ARG, "M=%d K=%d must be positive", M, K);
+  if (K % 32 != 0) return fail(CHAM_ERR_INVALID_ARG, "K=%d must be a multiple of 32", K);
+  if (fmt < 0 || fmt > (allow_fp16 ? CHAM_A_FP16 : CHAM_A_MXINT8))
+    return fail(CHAM_ERR_INVALID_ARG, "activation format %d is not valid here", fmt);
+  if (X == nullptr || !aligned16(X)) return fail(CHAM_ERR_INVALID_ARG, "X must be a 16-byte aligned device pointer");
+  return CHAM_OK;
+}
+
+// Per-format packing order inside each MMA class (R15).
+const int kClassOrder[2][5] = {{CHAM_W_INT4_SYM, CHAM_W_INT4_ASYM, CHAM_W_E2M1, CHAM_W_MXINT4, CHAM_W_MXFP4},
+                               {CHAM_W_NF4, CHAM_W_INT8_SYM, CHAM_W_INT8_ASYM, CHAM_W_MXINT8, -1}};
+
+cham_status check_desc(const cham_wpack_desc* d) {
+  if (d == nullptr) return fail(CHAM_ERR_INVALID_ARG, "descriptor is NULL");
+  if (d->magic != 0x574D4843u || d->version != 1) return fail(CHAM_ERR_INVALID_ARG, "not a packed-weight descriptor");
+  if (d->N <= 0 || d->K <= 0 || d->K % 32 != 0 || (d->bits != 4 && d->bits != 8))
+    return fail(CHAM_ERR_INVALID_ARG, "descriptor sizes are invalid");
+  return CHAM_OK;
+}
+
+
+// Byte offsets inside the linear workspace.
+struct LinearWs {
+  size_t scale, parts, operand;
+};
+LinearWs linear_ws(int M, int K) {
+  const int64_t nvec = static_cast<int64_t>(M) * K / 8;
+  return LinearWs{0, 256, 256 + range_ws_bytes(nvec)};
+}
+
+cham_status check_linear_common(int M, int K, int act_fmt, void* ws, size_t ws_bytes, size_t need) {
+  if (M <= 0 || K <= 0 || K % 32 != 0) return fail(CHAM_ERR_INVALID_ARG, "M=%d K=%d", M, K);
+  if (act_fmt < 0 || act_fmt > CHAM_A_FP16) return fail(CHAM_ERR_INVALID_ARG, "activation format %d", act_fmt);
+  if (ws == nullptr || !aligned16(ws)) return fail(CHAM_ERR_INVALID_ARG, "ws must be a 16-byte aligned pointer");
+  if (ws_bytes < need) return fail(CHAM_ERR_WORKSPACE, "workspace %zu < %zu bytes", ws_bytes, need);
+  return CHAM_OK;
+}
+
+size_t linear_ws_need(int M, int K, int act_fmt) {
+  if (act_fmt == CHAM_A_FP16) return 256;
+  return linear_ws(M, K).operand + round_up(static_cast<size_t>(M) * K * 2, 256);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* chameleon_status_string(cham_status s) {
+  switch (s) {
+    case CHAM_OK: return "ok";
+    case CHAM_ERR_INVALID_ARG: return "invalid argument";
+    case CHAM_ERR_UNSUPPORTED: return "unsupported";
+    case CHAM_ERR_WORKSPACE: return "workspace too small";
+    case CHAM_ERR_NONFINITE: return "non-finite activation";
+    case CHAM_ERR_TIMEOUT: return "device wait timed out";
+    case CHAM_ERR_CUDA: return "CUDA error";
+    case CHAM_ERR_RANGE: return "MX weight outside fp16";
+    default: return "unknown status";
+  }
+}
+
+const char* chameleon_last_error_detail(void) { return g_detail; }
+
+int chameleon_version(void) { return 1; }
+
+// ---------------------------------------------------------------- a1 and the LUT builder
+int chameleon_bucket(int t, int T, int B) {
+  if (T <= 0 || B <= 0 || t < 0) return -1;
+  // floor(t / (T/B)) computed exactly in integers: floor(t * B / T)
+  const long b = static_cast<long>(t) * B / T;
+  return static_cast<int>(b < B - 1 ? b : B - 1);
+}
+
+cham_status chameleon_snr(int schedule, int T, double* snr_out) {
+  if (T < 2 || snr_out == nullptr) return fail(CHAM_ERR_INVALID_ARG, "T must be >= 2 and snr_out non-NULL");
+  if (schedule != CHAM_SCHEDULE_SCALED_LINEAR && schedule != CHAM_SCHEDULE_LINEAR)
+    return fail(CHAM_ERR_INVALID_ARG, "unknown schedule %d", schedule);
+  double abar = 1.0;
+  for (int t = 0; t < T; ++t) {
+    double beta;
+    if (schedule == CHAM_SCHEDULE_SCALED_LINEAR) {
+      const double a = std::sqrt(0.00085), b = std::sqrt(0.012);
+      const double r = a + (b - a) * t / (T - 1);
+      beta = r * r;
+    } else {
+      beta = 1e-4 + (0.02 - 1e-4) * t / (T - 1);
+    }
+    abar *= 1.0 - beta;
+    snr_out[t] = abar / (1.0 - abar);
+  }
+  return CHAM_OK;
+}
+
+double chameleon_kurtosis(const double sums[5]) {
+  const double n = sums[0];
+  if (!(n > 0)) return 0.0;
+  const double mu = sums[1] / n;
+  const double m2 = sums[2] / n - mu * mu;
+  const double m4 = sums[4] / n - 4.0 * mu * sums[3] / n + 6.0 * mu * mu * sums[2] / n - 3.0 * mu * mu * mu * mu;
+  if (!(m2 > 0)) return 0.0;
+  return m4 / (m2 * m2);
+}
+
+int chameleon_route(double kappa, double snr_b, int is_shortcut) {
+  if (is_shortcut) return CHAM_A_MXFP8;
+  if (kappa > 5.0 || snr_b < 0.2) return CHAM_A_E5M2;
+  if (kappa <= 3.0 && snr_b > 2.0) return CHAM_A_INT8_ASYM;
+  return CHAM_A_E4M3;
+}
+
+// ---------------------------------------------------------------- calibration power sums
+cham_status chameleon_act_moments_workspace_size(int64_t count, size_t* ws_bytes) {
+  if (count <= 0 || count % 8 != 0 || ws_bytes == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "count must be a positive multiple of 8");
+  *ws_bytes = round_up(static_cast<size_t>(cham::range_grid(count / 8, num_sms_current())) * sizeof(cham::MomentPartial),
+                       256);
+  return CHAM_OK;
+}
+
+cham_status chameleon_act_moments(const void* X, int64_t count, double* out, void* ws, size_t ws_bytes,
+                                  void* stream) {
+  size_t need = 0;
+  cham_status s = chameleon_act_moments_workspace_size(count, &need);
+  if (s != CHAM_OK) return s;
+  if (X == nullptr || out == nullptr || ws == nullptr || !aligned16(X) || !aligned16(ws))
+    return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
+  if (ws_bytes < need) return fail(CHAM_ERR_WORKSPACE, "workspace %zu < %zu", ws_bytes, need);
+  const int64_t nvec = count / 8;
+  const int nparts = cham::range_grid(nvec, num_sms_current());
+  cham::launch_act_moments(static_cast<const uint4*>(X), nvec, count, static_cast<cham::MomentPartial*>(ws), nparts,
+                           out, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "act_moments launch");
+}
+
+// ---------------------------------------------------------------- a2-a4
+cham_status chameleon_act_quant_size(int M, int K, int fmt, size_t* qact_bytes, size_t* ws_bytes) {
+  if (M <= 0 || K <= 0 || K % 32 != 0 || fmt < 0 || fmt > CHAM_A_MXINT8)
+    return fail(CHAM_ERR_INVALID_ARG, "M=%d K=%d fmt=%d", M, K, fmt);
+  const ActLayout L = act_layout(M, K);
+  if (qact_bytes) *qact_bytes = L.total;
+  if (ws_bytes) *ws_bytes = fmt <= CHAM_A_E5M2 ? range_ws_bytes(static_cast<int64_t>(M) * K / 8) : 0;
+  return CHAM_OK;
+}
+
+cham_status chameleon_act_quant(const void* X, int M, int K, int fmt, void* qact, size_t qact_bytes, void* ws,
+                                size_t ws_bytes, int* dev_status, void* stream) {
+  cham_status s = check_act_args(X, M, K, fmt, false);
+  if (s != CHAM_OK) return s;
+  size_t need_q = 0, need_ws = 0;
+  chameleon_act_quant_size(M, K, fmt, &need_q, &need_ws);
+  if (qact == nullptr || !aligned16(qact)) return fail(CHAM_ERR_INVALID_ARG, "qact must be 16-byte aligned");
+  if (qact_bytes < need_q) return fail(CHAM_ERR_WORKSPACE, "qact %zu < %zu bytes", qact_bytes, need_q);
+  if (need_ws > 0 && (ws == nullptr || !aligned16(ws))) return fail(CHAM_ERR_INVALID_ARG, "ws must be 16-byte aligned");
+  if (ws_bytes < need_ws) return fail(CHAM_ERR_WORKSPACE, "ws %zu < %zu bytes", ws_bytes, need_ws);
+  const ActLayout L = act_layout(M, K);
+  uint8_t* q = static_cast<uint8_t*>(qact);
+  cham::ActQuantArgs a{};
+  a.X = static_cast<const uint4*>(X);
+  a.nvec = static_cast<int64_t>(M) * K / 8;
+  a.num_sms = num_sms_current();
+  a.parts = static_cast<cham::RangePartial*>(ws);
+  a.nparts = cham::range_grid(a.nvec, a.num_sms);
+  a.codes = reinterpret_cast<uint2*>(q + L.codes);
+  a.deq = nullptr;
+  a.e8m0 = fmt >= CHAM_A_MXFP8 ? q + L.e8m0 : nullptr;
+  a.params = reinterpret_cast<cham_qparams*>(q + L.params);
+  a.scale_out = nullptr;
+  a.dev_status = dev_status;
+  cham::launch_act_quant(fmt, a, true, false, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "act_quant launch");
+}
+
+// ---------------------------------------------------------------- a5
+cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_t palette_mask, uint8_t* fmt_out,
+                                            double* sse_out, void* stream) {
+  if (N <= 0 || K <= 0 || K % 32 != 0) return fail(CHAM_ERR_INVALID_ARG, "N=%d K=%d (K must be a multiple of 32)", N, K);
+  if (palette_mask == 0 || (palette_mask & ~0x1FFu) != 0) return fail(CHAM_ERR_INVALID_ARG, "palette mask 0x%x", palette_mask);
+  if ((palette_mask & CHAM_PALETTE_W8) && (palette_mask & CHAM_PALETTE_W4))
+    return fail(CHAM_ERR_INVALID_ARG, "palette mixes 8-bit and 4-bit formats");
+  if (W == nullptr || !aligned16(W) || fmt_out == nullptr) return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
+  cham::launch_select(static_cast<const __half*>(W), N, K, palette_mask, fmt_out, sse_out, nf4_table(),
+                      static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "select launch");
+}
+
+// ---------------------------------------------------------------- a6
+cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* d) {
+  if (N <= 0 || K <= 0 || K % 32 != 0 || fmt_host == nullptr || d == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "N=%d K=%d (K must be a multiple of 32)", N, K);
+  std::memset(d, 0, sizeof(*d));
+  int bits = 0;
+  for (int c = 0; c < N; ++c) {
+    const int f = fmt_host[c];
+    if (f >= CHAM_W_NFORMATS) return fail(CHAM_ERR_INVALID_ARG, "channel %d has format %d", c, f);
+    const int b = cham::wbits(f);
+    if (bits != 0 && b != bits) return fail(CHAM_ERR_INVALID_ARG, "formats of mixed bit width");
+    bits = b;
+    d->n_fmt[f] += 1;
+  }
+  d->magic = 0x574D4843u;
+  d->version = 1;
+  d->N = N;
+  d->K = K;
+  d->Kp = static_cast<int>(round_up(K, 64));
+  d->bits = bits;
+  for (int cls = 0; cls < 2; ++cls) {
+    for (int j = 0; j < 5; ++j)
+      if (kClassOrder[cls][j] >= 0) d->n_class[cls] += d->n_fmt[kClassOrder[cls][j]];
+    d->n_tiles[cls] = (d->n_class[cls] + 127) / 128;
+  }
+  const size_t tiles = static_cast<size_t>(d->n_tiles[0] + d->n_tiles[1]);
+  const size_t np = tiles * 128, chunks = d->Kp / 64;
+  size_t off = 256;
+  d->off_codes = off;
+  off = round_up(off + tiles * chunks * 128 * (bits == 8 ? 64 : 32), 256);
+  d->off_scale = off;
+  off = round_up(off + np * 4, 256);
+  d->off_zero = off;
+  off = round_up(off + np, 256);
+  d->off_e8m0 = off;
+  off = round_up(off + tiles * chunks * 128 * 2, 256);
+  d->off_fmt = off;
+  off = round_up(off + np, 256);
+  d->off_perm = off;
+  off = round_up(off + np * 4, 256);
+  d->bytes = off;
+  return CHAM_OK;
+}
+
+}  // extern "C"
+
+namespace cham {
+__global__ void k_write_desc(cham_wpack_desc d, cham_wpack_desc* out) {
+  const uint32_t* src = reinterpret_cast<const uint32_t*>(&d);
+  uint32_t* dst = reinterpret_cast<uint32_t*>(out);
+  for (int i = threadIdx.x; i < 64; i += blockDim.x) dst[i] = src[i];
+}
+}  // namespace cham
+
+extern "C" {
+
+cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const cham_wpack_desc* d, void* blob,
+                                   size_t blob_bytes, int* dev_status, void* stream) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  if (W == nullptr || fmt_dev == nullptr || blob == nullptr || !aligned16(W) || !aligned16(blob))
+    return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
+  if (blob_bytes < d->bytes) return fail(CHAM_ERR_WORKSPACE, "blob %zu < %llu bytes", blob_bytes,
+                                          static_cast<unsigned long long>(d->bytes));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* b = static_cast<uint8_t*>(blob);
+  cham::PackArgs a{};
+  a.W = static_cast<const __half*>(W);
+  a.fmt_dev = fmt_dev;
+  a.N = d->N;
+  a.K = d->K;
+  a.Kp = d->Kp;
+  a.bits = d->bits;
+  a.n_chunks = d->Kp / 64;
+  a.n_packed = 128 * (d->n_tiles[0] + d->n_tiles[1]);
+  for (int cls = 0, base = 0; cls < 2; ++cls) {
+    int slot = base;
+    for (int j = 0; j < 5; ++j) {
+      const int f = kClassOrder[cls][j];
+      if (f < 0) continue;
+      a.base[f] = slot;
+      a.count[f] = d->n_fmt[f];
+      slot += d->n_fmt[f];
+    }
+    base += 128 * d->n_tiles[cls];
+  }
+  a.codes = b + d->off_codes;
+  a.scale = reinterpret_cast<float*>(b + d->off_scale);
+  a.zero = b + d->off_zero;
+  a.e8m0 = b + d->off_e8m0;
+  a.fmtp = b + d->off_fmt;
+  a.perm = reinterpret_cast<int32_t*>(b + d->off_perm);
+  a.dev_status = dev_status;
+  cham::k_write_desc<<<1, 64, 0, st>>>(*d, reinterpret_cast<cham_wpack_desc*>(b));
+  cham::launch_pack(a, nf4_table(), st);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "pack launch");
+}
+
+// ---------------------------------------------------------------- a7/a8
+// Workspace: [0, 256) the per-tensor scale s_a; [256, 256 + R) range partials; then the M x K
+// fp16 activation operand (exact values of the codes, R13).
+cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* d, int act_fmt, size_t* ws_bytes) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  if (M <= 0 || act_fmt < 0 || act_fmt > CHAM_A_FP16 || ws_bytes == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "M=%d act_fmt=%d", M, act_fmt);
+  *ws_bytes = linear_ws_need(M, d->K, act_fmt);
+  return CHAM_OK;
+}
+
+}  // extern "C"
+
+
+extern "C" {
+
+cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, void* ws, size_t ws_bytes,
+                                     int* dev_status, void* stream) {
+  cham_status s = check_act_args(X, M, K, act_fmt, true);
+  if (s != CHAM_OK) return s;
+  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
+  if (s != CHAM_OK) return s;
+  if (act_fmt == CHAM_A_FP16) return CHAM_OK;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  const LinearWs L = linear_ws(M, K);
+  cham::ActQuantArgs a{};
+  a.X = static_cast<const uint4*>(X);
+  a.nvec = static_cast<int64_t>(M) * K / 8;
+  a.num_sms = num_sms_current();
+  a.parts = reinterpret_cast<cham::RangePartial*>(w + L.parts);
+  a.nparts = cham::range_grid(a.nvec, a.num_sms);
+  a.codes = nullptr;
+  a.deq = reinterpret_cast<uint4*>(w + L.operand);
+  a.e8m0 = nullptr;
+  a.params = nullptr;
+  a.scale_out = act_fmt <= CHAM_A_E5M2 ? reinterpret_cast<float*>(w + L.scale) : nullptr;
+  a.dev_status = dev_status;
+  cham::launch_act_quant(act_fmt, a, false, true, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "linear_prepare launch");
+}
+
+cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d, const void* blob, int act_fmt,
+                                  const float* bias, float* Y, void* ws, size_t ws_bytes, int* dev_status,
+                                  void* stream) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  const int K = d->K;
+  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
+  if (s != CHAM_OK) return s;
+  if (act_fmt == CHAM_A_FP16 && (X == nullptr || !aligned16(X)))
+    return fail(CHAM_ERR_INVALID_ARG, "X must be a 16-byte aligned device pointer");
+  if (blob == nullptr || Y == nullptr || !aligned16(blob) || !aligned16(Y) || (bias != nullptr && !aligned16(bias)))
+    return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  const LinearWs L = linear_ws(M, K);
+  const void* operand = act_fmt == CHAM_A_FP16 ? X : static_cast<const void*>(w + L.operand);
+  const float* act_scale = act_fmt <= CHAM_A_E5M2 ? reinterpret_cast<const float*>(w + L.scale) : nullptr;
+  const uint8_t* b = static_cast<const uint8_t*>(blob);
+  cham::GemmArgs g{};
+  g.codes = b + d->off_codes;
+  g.wscale = reinterpret_cast<const float*>(b + d->off_scale);
+  g.wzero = b + d->off_zero;
+  g.we8m0 = b + d->off_e8m0;
+  g.wfmt = b + d->off_fmt;
+  g.perm = reinterpret_cast<const int32_t*>(b + d->off_perm);
+  g.bias = bias;
+  g.act_scale = act_scale;
+  g.Y = Y;
+  g.M = M;
+  g.N = d->N;
+  g.n_chunks = d->Kp / 64;
+  g.bits = d->bits;
+  g.dev_status = dev_status;
+  const cham::NF4Table& nf4 = nf4_table();
+  for (int i = 0; i < 16; ++i) g.nf4_level[i] = nf4.level[i];
+  const int num_sms = num_sms_current();
+  const int tiles = d->n_tiles[0] + d->n_tiles[1];
+  const int bn = cham::gemm_pick_bn(M, tiles, num_sms);
+  CUtensorMap map;
+  s = make_act_map(&map, operand, M, K, bn);
+  if (s != CHAM_OK) return s;
+  g.tile0 = 0;
+  const cudaError_t e = cham::launch_gemm_f16(map, g, tiles, bn, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "gemm launch");
+}
+
+cham_status chameleon_linear(const void* X, int M, const cham_wpack_desc* d, const void* blob, int act_fmt,
+                             const float* bias, float* Y, void* ws, size_t ws_bytes, int* dev_status, void* stream) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  s = chameleon_linear_prepare(X, M, d->K, act_fmt, ws, ws_bytes, dev_status, stream);
+  if (s != CHAM_OK) return s;
+  return chameleon_linear_gemm(X, M, d, blob, act_fmt, bias, Y, ws, ws_bytes, dev_status, stream);
+}
+
+}  // extern "C"

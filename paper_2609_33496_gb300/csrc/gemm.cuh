@@ -1,0 +1,31 @@
+// gemm.cuh -- mixed-format quantized linear on tcgen05 (steps a7, a8): declarations.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "weights.cuh"
+
+namespace cham {
+
+struct GemmArgs {
+  const uint8_t* codes;      // blob code region (tiled, include/chameleon.h)
+  const float* wscale;       // [Np] per packed channel
+  const uint8_t* wzero;      // [Np]
+  const uint8_t* we8m0;      // [tiles][chunks][128][2]
+  const uint8_t* wfmt;       // [Np]
+  const int32_t* perm;       // [Np]
+  const float* bias;         // [N] in original order, or null
+  const float* act_scale;    // device scalar s_a (per-tensor activation formats), or null for 1
+  float* Y;                  // [M][N] fp32
+  int M, N, n_chunks;        // n_chunks = Kp / 64
+  int tile0;                 // first 128-channel tile of this launch
+  int bits;                  // 4 or 8
+  int* dev_status;
+  uint16_t nf4_level[16];    // NF4 levels as fp16 bit patterns
+};
+
+// Token-tile (MMA N) sizes the kernel is instantiated for.
+int gemm_pick_bn(int M, int n_tiles, int num_sms);
+cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int n_tiles, int bn, cudaStream_t st);
+
+}  // namespace cham

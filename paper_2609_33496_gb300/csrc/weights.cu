@@ -1,0 +1,307 @@
+// weights.cu -- weight-format selection (step a5) and weight pack (step a6).
+//
+// Selection (Sec. 3.4, Eq. weight-argmax): every output channel is round-tripped through every
+// palette format; the squared reconstruction error SSE_f(c) is accumulated in fp64 from
+// per-element errors that are exact up to one fp32 rounding; the smallest error wins, the
+// earlier palette member on ties (strict '<').  One CTA per channel: the row (at most 10 KB for
+// K = 5120) stays in L1 across the format passes.
+//
+// Pack: channels are permuted into format-homogeneous runs (Sec. 5: "same-format sub-GEMMs after
+// a channel permutation"), grouped by MMA class and padded to 128-channel tiles, and encoded in
+// the tiled layout the GEMM's decode warps read with coalesced 16-byte loads (include/chameleon.h).
+#include "weights.cuh"
+
+namespace cham {
+
+constexpr int kWThreads = 128;
+
+// Block-wide reductions for 128 threads.
+template <typename T, typename Op>
+CHAM_DEV T block_reduce(T v, Op op, T* sh) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = op(v, __shfl_xor_sync(0xffffffffu, v, o));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) sh[warp] = v;
+  __syncthreads();
+  T r = sh[0];
+#pragma unroll
+  for (int k = 1; k < kWThreads / 32; ++k) r = op(r, sh[k]);
+  return r;
+}
+
+struct FMin {
+  CHAM_DEV float operator()(float a, float b) const { return fminf(a, b); }
+};
+struct FMax {
+  CHAM_DEV float operator()(float a, float b) const { return fmaxf(a, b); }
+};
+struct DAdd {
+  CHAM_DEV double operator()(double a, double b) const { return a + b; }
+};
+
+// Eight consecutive elements of a row as fp32.
+CHAM_DEV void load8(const __half* row, int v, float (&x)[8]) {
+  const uint4 u = __ldg(reinterpret_cast<const uint4*>(row) + v);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 f = __half22float2(u32_as_h2(w[j]));
+    x[2 * j] = f.x;
+    x[2 * j + 1] = f.y;
+  }
+}
+
+// Channel statistics (amax, lo, hi) of one row, reduced over the CTA.
+CHAM_DEV ChanStats row_stats(const __half* row, int nvec, float* shf) {
+  float amax = 0.f, lo = INFINITY, hi = -INFINITY;
+  for (int v = threadIdx.x; v < nvec; v += kWThreads) {
+    float x[8];
+    load8(row, v, x);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      amax = fmaxf(amax, fabsf(x[i]));
+      lo = fminf(lo, x[i]);
+      hi = fmaxf(hi, x[i]);
+    }
+  }
+  ChanStats s;
+  s.amax = block_reduce(amax, FMax(), shf);
+  s.lo = block_reduce(lo, FMin(), shf);
+  s.hi = block_reduce(hi, FMax(), shf);
+  return s;
+}
+
+// ------------------------------------------------------------------ a5: selection
+__global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict__ W, int K, uint32_t mask,
+                                                       uint8_t* __restrict__ fmt_out, double* __restrict__ sse_out,
+                                                       NF4Table nf4) {
+  __shared__ float shf[kWThreads / 32];
+  __shared__ double shd[kWThreads / 32];
+  __shared__ double sse[CHAM_W_NFORMATS];
+  const int c = blockIdx.x;
+  const __half* row = W + static_cast<size_t>(c) * K;
+  const int nvec = K / 8;
+  const ChanStats st = row_stats(row, nvec, shf);
+  const int iters = (nvec + kWThreads - 1) / kWThreads;  // same trip count in every lane (shuffles)
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
+    if (!((mask >> f) & 1u)) continue;
+    double acc = 0.0;
+    if (w_is_mx(f)) {
+      for (int it = 0; it < iters; ++it) {
+        const int v = it * kWThreads + threadIdx.x;
+        float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        if (v < nvec) load8(row, v, x);
+        float a = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a = fmaxf(a, fabsf(x[i]));
+        a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, 1));  // 4 lanes = one 32-element block
+        a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, 2));
+        const int X = mx_exponent(f, a);
+        if (v < nvec) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            float dq;
+            encode_mx(f, x[i], X, &dq);
+            const double e = static_cast<double>(__fsub_rn(x[i], dq));
+            acc = fma(e, e, acc);
+          }
+        }
+      }
+    } else {
+      const ChanScale cs = chan_scale(f, st);
+      for (int v = threadIdx.x; v < nvec; v += kWThreads) {
+        float x[8];
+        load8(row, v, x);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float err;
+          encode_chan(f, x[i], cs, nf4, &err);
+          const double e = static_cast<double>(err);
+          acc = fma(e, e, acc);
+        }
+      }
+    }
+    const double tot = block_reduce(acc, DAdd(), shd);
+    if (threadIdx.x == 0) sse[f] = tot;
+  }
+  if (threadIdx.x == 0) {
+    int best = -1;
+    double best_e = 0.0;
+    for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
+      const bool member = (mask >> f) & 1u;
+      if (member && (best < 0 || sse[f] < best_e)) {
+        best = f;
+        best_e = sse[f];
+      }
+      if (sse_out != nullptr) sse_out[static_cast<size_t>(c) * CHAM_W_NFORMATS + f] = member ? sse[f] : INFINITY;
+    }
+    fmt_out[c] = static_cast<uint8_t>(best);
+  }
+}
+
+void launch_select(const __half* W, int N, int K, uint32_t mask, uint8_t* fmt_out, double* sse_out,
+                   const NF4Table& nf4, cudaStream_t st) {
+  k_w_select<<<N, kWThreads, 0, st>>>(W, K, mask, fmt_out, sse_out, nf4);
+}
+
+// ------------------------------------------------------------------ a6: slot assignment
+// Packed slot of every channel: base[f] + (number of earlier channels with the same format).
+// One CTA walks the channels in chunks of 1024 with per-format warp ballots.
+__global__ void __launch_bounds__(1024) k_w_slots(PackArgs a) {
+  __shared__ int warp_cnt[32][CHAM_W_NFORMATS];
+  __shared__ int running[CHAM_W_NFORMATS];
+  for (int p = threadIdx.x; p < a.n_packed; p += blockDim.x) {
+    a.perm[p] = -1;
+    a.fmtp[p] = 0xFF;
+  }
+  if (threadIdx.x < CHAM_W_NFORMATS) running[threadIdx.x] = 0;
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int c0 = 0; c0 < a.N; c0 += blockDim.x) {
+    const int c = c0 + threadIdx.x;
+    const int f = c < a.N ? a.fmt_dev[c] : -1;
+    int my_rank_in_warp = 0;
+#pragma unroll
+    for (int g = 0; g < CHAM_W_NFORMATS; ++g) {
+      const uint32_t m = __ballot_sync(0xffffffffu, f == g);
+      if (f == g) my_rank_in_warp = __popc(m & ((1u << lane) - 1u));
+      if (lane == 0) warp_cnt[warp][g] = __popc(m);
+    }
+    __syncthreads();
+    if (c < a.N) {
+      if (f < 0 || f >= CHAM_W_NFORMATS) {
+        set_status(a.dev_status, CHAM_ERR_INVALID_ARG);
+      } else {
+        int rank = running[f] + my_rank_in_warp;
+        for (int w = 0; w < warp; ++w) rank += warp_cnt[w][f];
+        if (rank < a.count[f]) {  // device formats must match the host plan
+          const int slot = a.base[f] + rank;
+          a.perm[slot] = c;
+          a.fmtp[slot] = static_cast<uint8_t>(f);
+        } else {
+          set_status(a.dev_status, CHAM_ERR_INVALID_ARG);
+        }
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x < CHAM_W_NFORMATS) {
+      int t = 0;
+      for (int w = 0; w < 32; ++w) t += warp_cnt[w][threadIdx.x];
+      running[threadIdx.x] += t;
+    }
+    __syncthreads();
+  }
+}
+
+// ------------------------------------------------------------------ a6: encode one packed slot
+// Byte offset of the 8 codes of elements [k0, k0+8) of packed slot p in the tiled code layout.
+CHAM_DEV size_t code_offset(int p, int k0, int n_chunks, int bits) {
+  const int tile = p >> 7, r = p & 127;
+  const int chunk = k0 >> 6, kk = k0 & 63;
+  const size_t chunk_base = (static_cast<size_t>(tile) * n_chunks + chunk) * (bits == 8 ? 8192u : 4096u);
+  if (bits == 8) return chunk_base + static_cast<size_t>(kk >> 4) * 2048 + r * 16 + (kk & 15);
+  return chunk_base + static_cast<size_t>(kk >> 5) * 2048 + r * 16 + ((kk & 31) >> 3) * 4;
+}
+
+__global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) {
+  __shared__ float shf[kWThreads / 32];
+  const int p = blockIdx.x;
+  const int c = a.perm[p];
+  const int nvec_p = a.Kp / 8;
+  const int tile = p >> 7, r = p & 127;
+  if (c < 0) {  // padding slot: zero codes, unit scale
+    for (int v = threadIdx.x; v < nvec_p; v += kWThreads) {
+      const size_t off = code_offset(p, v * 8, a.n_chunks, a.bits);
+      if (a.bits == 8) *reinterpret_cast<uint2*>(a.codes + off) = make_uint2(0, 0);
+      else *reinterpret_cast<uint32_t*>(a.codes + off) = 0u;
+    }
+    for (int ch = threadIdx.x; ch < a.n_chunks; ch += kWThreads) {
+      const size_t e = ((static_cast<size_t>(tile) * a.n_chunks + ch) * 128 + r) * 2;
+      a.e8m0[e] = 127;
+      a.e8m0[e + 1] = 127;
+    }
+    if (threadIdx.x == 0) {
+      a.scale[p] = 1.f;
+      a.zero[p] = 0;
+    }
+    return;
+  }
+  const int f = a.fmtp[p];
+  const __half* row = a.W + static_cast<size_t>(c) * a.K;
+  const int nvec = a.K / 8;
+  const ChanStats st = row_stats(row, nvec, shf);
+  const ChanScale cs = chan_scale(f, st);
+  const bool mx = w_is_mx(f);
+  const int iters = (nvec_p + kWThreads - 1) / kWThreads;
+  bool range_ok = true;
+  for (int it = 0; it < iters; ++it) {
+    const int v = it * kWThreads + threadIdx.x;
+    float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    if (v < nvec) load8(row, v, x);
+    int code[8];
+    int X = 0;
+    if (mx) {
+      float am = 0.f;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
+      am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 1));
+      am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 2));
+      X = mx_exponent(f, am);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        float dq;
+        code[i] = encode_mx(f, x[i], X, &dq);
+        // the GEMM's fp16 operand must equal DQ exactly (R13)
+        range_ok &= (__half2float(__float2half_rn(dq)) == dq);
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        float err;
+        code[i] = encode_chan(f, x[i], cs, nf4, &err);
+      }
+    }
+    if (v >= nvec_p) continue;
+    if (v >= nvec) {  // K padding up to a multiple of 64: code 0
+#pragma unroll
+      for (int i = 0; i < 8; ++i) code[i] = 0;
+    }
+    const size_t off = code_offset(p, v * 8, a.n_chunks, a.bits);
+    if (a.bits == 8) {
+      uint32_t lo = 0, hi = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        lo |= (static_cast<uint32_t>(code[i]) & 0xFFu) << (8 * i);
+        hi |= (static_cast<uint32_t>(code[4 + i]) & 0xFFu) << (8 * i);
+      }
+      *reinterpret_cast<uint2*>(a.codes + off) = make_uint2(lo, hi);
+    } else {
+      // nibble j (j < 4) = element 2j, nibble 4 + j = element 2j + 1
+      uint32_t w = 0;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        w |= (static_cast<uint32_t>(code[2 * j]) & 0xFu) << (4 * j);
+        w |= (static_cast<uint32_t>(code[2 * j + 1]) & 0xFu) << (4 * (j + 4));
+      }
+      *reinterpret_cast<uint32_t*>(a.codes + off) = w;
+    }
+    if ((threadIdx.x & 3) == 0) {  // one E8M0 byte per 32-element block
+      const int k0 = v * 8;
+      const size_t e = ((static_cast<size_t>(tile) * a.n_chunks + (k0 >> 6)) * 128 + r) * 2 + ((k0 & 63) >> 5);
+      a.e8m0[e] = mx ? static_cast<uint8_t>(X + 127) : 127;
+    }
+  }
+  if (mx && !range_ok) set_status(a.dev_status, CHAM_ERR_RANGE);
+  if (threadIdx.x == 0) {
+    a.scale[p] = mx ? 1.f : cs.s;
+    a.zero[p] = static_cast<uint8_t>(cs.z);
+  }
+}
+
+void launch_pack(const PackArgs& a, const NF4Table& nf4, cudaStream_t st) {
+  k_w_slots<<<1, 1024, 0, st>>>(a);
+  k_w_pack<<<a.n_packed, kWThreads, 0, st>>>(a, nf4);
+}
+
+}  // namespace cham

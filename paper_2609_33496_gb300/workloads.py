@@ -1,0 +1,92 @@
+"""Seeded synthetic inputs shaped like the paper's workloads (stand-ins for SDXL / PixArt-alpha
+activations and weights; no checkpoint or dataset is used).  Holds no arithmetic of the method:
+only value distributions, shapes and seeds.  Shared by the tests, the benchmark and the oracle's
+callers.
+
+Seeds: 20260000 + 1000 * config + index.  Values are drawn in float64 and rounded to fp16.
+"""
+import numpy as np
+
+SEED_BASE = 20260000
+
+# SDXL-UNet attention / FFN projections at batch 2 with classifier-free guidance:
+# (name, M tokens, K in-features, N out-features)
+SDXL_PROJ_LAYERS = (
+    [("down1.attn.%s" % n, 8192, 640, 640) for n in ("q", "k", "v", "out")]
+    + [("down2.attn.%s" % n, 2048, 1280, 1280) for n in ("q", "k", "v", "out")]
+    + [("down2.ff.geglu_in", 2048, 1280, 10240), ("down2.ff.out", 2048, 5120, 1280)]
+)
+
+# Student-t degrees of freedom of the activations per timestep bucket b = 0..9 (None = Gaussian):
+# near-Gaussian at high SNR (b = 0), heavy-tailed at low SNR (b = 9), App. A.3 phases.
+NU_SCHEDULE = (None, 30, 20, 12, 9, 7, 6, 5, 4, 3)
+
+
+def rng(config, index=0):
+    return np.random.default_rng(SEED_BASE + 1000 * config + index)
+
+
+def to_fp16(x):
+    return np.asarray(x, dtype=np.float64).astype(np.float16)
+
+
+def student_t(g, nu, shape):
+    return g.standard_normal(shape) if nu is None else g.standard_t(nu, shape)
+
+
+def single_layer(seed_index=0, M=256, K=320, N=320, n_outliers=4, outlier_gain=20.0):
+    """Single linear layer: X = 0.5 * StudentT(3), W ~ N(0, 0.02^2) with `n_outliers` output
+    channels scaled by `outlier_gain`, bias ~ N(0, 0.02^2)."""
+    g = rng(1, seed_index)
+    X = to_fp16(0.5 * g.standard_t(3, (M, K)))
+    W = g.normal(0.0, 0.02, (N, K))
+    if n_outliers:
+        rows = g.choice(N, n_outliers, replace=False)
+        W[rows] *= outlier_gain
+    bias = g.normal(0.0, 0.02, N).astype(np.float32)
+    return X, to_fp16(W), bias
+
+
+def channel_jitter(g, K, sigma=0.1):
+    """Per-input-channel scale c_k = exp(sigma * N(0, 1))."""
+    return np.exp(sigma * g.standard_normal(K))
+
+
+def sdxl_layer_weights(layer_index):
+    name, M, K, N = SDXL_PROJ_LAYERS[layer_index]
+    g = rng(2, layer_index)
+    W = to_fp16(g.normal(0.0, 0.02, (N, K)))
+    bias = g.normal(0.0, 0.02, N).astype(np.float32)
+    return W, bias
+
+
+def sdxl_layer_activation(layer_index, bucket, rows=None):
+    """Activation of projection layer `layer_index` at timestep bucket `bucket`:
+    StudentT(nu_b) * c_k with a per-layer channel jitter c_k.  `rows` limits M (smaller tests)."""
+    name, M, K, N = SDXL_PROJ_LAYERS[layer_index]
+    if rows is not None:
+        M = rows
+    c = channel_jitter(rng(2, 100 + layer_index), K)
+    g = rng(2, 200 + 10 * layer_index + bucket)
+    return to_fp16(student_t(g, NU_SCHEDULE[bucket], (M, K)) * c[None, :])
+
+
+def weight_mix(g, N, K, scale=0.02):
+    """Weights with per-channel distribution diversity (round-robin Gaussian, Laplace, uniform,
+    Student-t nu=4, sparse outliers) so that a format argmin yields a mix."""
+    W = np.empty((N, K))
+    for n in range(N):
+        kind = n % 5
+        if kind == 0:
+            W[n] = g.normal(0, scale, K)
+        elif kind == 1:
+            W[n] = g.laplace(0, scale / np.sqrt(2), K)
+        elif kind == 2:
+            W[n] = g.uniform(-scale * np.sqrt(3), scale * np.sqrt(3), K)
+        elif kind == 3:
+            W[n] = g.standard_t(4, K) * scale / np.sqrt(2)
+        else:
+            W[n] = g.normal(0, scale, K)
+            idx = g.choice(K, max(1, K // 64), replace=False)
+            W[n, idx] *= 12.0
+    return to_fp16(W)

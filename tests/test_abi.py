@@ -1,0 +1,89 @@
+"""The C-ABI library builds, loads and exports every entry point include/chameleon.h declares; its
+host-only helpers (no GPU needed) agree with the oracle.  No kernel is launched here."""
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+from oracle import schedule as S
+from oracle import formats as F
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "chameleon.h")
+
+
+@pytest.fixture(scope="module")
+def cl():
+    from paper_2609_33496_gb300 import build
+    build.build()
+    import paper_2609_33496_gb300 as P
+    P.chameleon.lib()
+    return P.chameleon
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(chameleon_\w+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(cl):
+    names = declared_symbols()
+    assert len(names) >= 16
+    L = ctypes.CDLL(cl.LIB_PATH)
+    for n in names:
+        assert hasattr(L, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", cl.LIB_PATH], capture_output=True, text=True).stdout
+    exported = set(re.findall(r"\b(chameleon_\w+)\b", out))
+    assert set(names) == exported
+    assert set(cl.EXPORTS) == set(names)
+
+
+def test_bucket_matches_alg2(cl):
+    for t in [0, 1, 99, 100, 101, 549, 550, 999, 1000, 1500]:
+        assert cl.bucket(t) == S.bucket(t)
+    assert cl.bucket(-1) == -1 and cl.bucket(5, 0, 10) == -1
+
+
+@pytest.mark.parametrize("sched,betas", [(0, S.betas_scaled_linear()), (1, S.betas_linear())])
+def test_snr_matches_oracle(cl, sched, betas):
+    np.testing.assert_allclose(cl.snr(sched), S.snr(betas), rtol=1e-10)
+
+
+def test_route_and_kurtosis_match_oracle(cl):
+    rng = np.random.default_rng(7)
+    for kappa in [1.0, 3.0, 3.0000001, 4.0, 5.0, 5.0000001, 9.0]:
+        for snr_b in [0.1, 0.2, 0.2000001, 1.0, 2.0, 2.0000001, 50.0]:
+            for sc in (False, True):
+                assert cl.route(kappa, snr_b, sc) == S.route(kappa, snr_b, sc)
+    for x in [rng.standard_normal(1000), 3 + rng.laplace(size=999), np.ones(5)]:
+        ps = S.power_sums(x)
+        sums = [ps["n"], ps["s1"], ps["s2"], ps["s3"], ps["s4"]]
+        assert cl.kurtosis(sums) == pytest.approx(S.kurtosis_from_sums(*sums), rel=1e-12, abs=1e-15)
+
+
+def test_pack_plan_layout(cl):
+    fmt = np.array([F.W_NF4] * 50 + [F.W_INT4_SYM] * 130 + [F.W_MXFP4] * 3 + [F.W_E2M1] * 7, np.uint8)
+    d = cl.pack_plan(len(fmt), 320, fmt)
+    assert (d.N, d.K, d.Kp, d.bits) == (190, 320, 320, 4)
+    assert list(d.n_class) == [140, 50] and list(d.n_tiles) == [2, 1]
+    offs = [d.off_codes, d.off_scale, d.off_zero, d.off_e8m0, d.off_fmt, d.off_perm, d.bytes]
+    assert all(o % 256 == 0 for o in offs) and offs == sorted(offs)
+    assert d.off_scale - d.off_codes >= 3 * 5 * 128 * 32
+
+
+def test_host_validation_errors(cl):
+    with pytest.raises(cl.ChameleonError) as e:
+        cl.pack_plan(4, 320, np.array([0, 0, 3, 3], np.uint8))     # mixed bit widths
+    assert e.value.status == cl.ERR_INVALID_ARG
+    with pytest.raises(cl.ChameleonError):
+        cl.pack_plan(2, 100, np.array([0, 0], np.uint8))           # K not a multiple of 32
+    with pytest.raises(cl.ChameleonError):
+        cl.act_quant_size(16, 48, 1)
+    with pytest.raises(cl.ChameleonError):
+        cl.act_quant_size(16, 64, 7)
+    q, w = cl.act_quant_size(256, 320, 3)
+    assert q >= 256 * 320 + 256 + 256 * 10 and w == 0

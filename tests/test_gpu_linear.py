@@ -1,0 +1,104 @@
+"""GPU quantized linear (a7, a8) against the fp64 oracle on the same dequantized operands:
+|Y - Y_ref| <= 2^-10 * sum_k |a_k w_k| per element."""
+import numpy as np
+import pytest
+
+from oracle import formats as F
+from oracle import gemm as G
+from oracle import select as SEL
+from paper_2609_33496_gb300 import workloads as WL
+from gpu_common import lib_module, cuda, host, assert_within_bound
+
+pytestmark = pytest.mark.gpu
+ACT = [F.A_INT8_ASYM, F.A_E4M3, F.A_E5M2, F.A_MXFP8, F.A_MXINT8]
+
+
+@pytest.fixture(scope="module")
+def cl():
+    return lib_module()
+
+
+def gpu_linear(cl, X, W, fmt, act_fmt, bias):
+    import torch
+    d = cl.pack_plan(W.shape[0], W.shape[1], fmt)
+    blob, st = cl.pack_weights(cuda(W), cuda(fmt), d)
+    Y, st2 = cl.linear(cuda(X), d, blob, act_fmt, bias=None if bias is None else cuda(bias))
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0 and int(st2.item()) == 0
+    return host(Y)
+
+
+def check(cl, X, W, fmt, act_fmt, bias, what):
+    Y = gpu_linear(cl, X, W, fmt, act_fmt, bias)
+    Y_ref, bound, _, _ = G.linear_reference(X, act_fmt, W, fmt, bias)
+    assert_within_bound(Y, Y_ref, bound, what)
+
+
+@pytest.mark.parametrize("act_fmt", ACT)
+@pytest.mark.parametrize("mask", [0x007, 0x1F8])
+def test_single_layer_w8a8_w4a8(cl, act_fmt, mask):
+    X, W, bias = WL.single_layer()
+    fmt, _, _ = SEL.select_formats(W, mask)
+    check(cl, X, W, fmt, act_fmt, bias, "act %d mask %#x" % (act_fmt, mask))
+
+
+def test_weight_only_fp16_activations(cl):
+    X, W, bias = WL.single_layer()
+    fmt, _, _ = SEL.select_formats(W, 0x1F8)
+    check(cl, X, W, fmt, F.A_FP16, bias, "W4A16")
+
+
+@pytest.mark.parametrize("M,K,N", [(1, 32, 1), (2, 96, 130), (17, 160, 129), (200, 64, 300),
+                                   (300, 320, 257), (130, 352, 64)])
+@pytest.mark.parametrize("bits", [8, 4])
+def test_ragged_shapes_every_format(cl, M, K, N, bits):
+    g = np.random.default_rng(M * 1000 + K + N)
+    X = WL.to_fp16(g.standard_t(4, (M, K)))
+    W = WL.weight_mix(g, N, K)
+    pal = F.W8_PALETTE if bits == 8 else F.W4_PALETTE
+    fmt = np.asarray(pal, np.uint8)[g.integers(0, len(pal), N)]
+    bias = g.normal(0, 0.02, N).astype(np.float32)
+    for act_fmt in ACT + [F.A_FP16]:
+        check(cl, X, W, fmt, act_fmt, bias if act_fmt % 2 else None,
+              "M%d K%d N%d bits %d act %d" % (M, K, N, bits, act_fmt))
+
+
+def test_exact_special_operands(cl):
+    """W = I in MXINT8 (DQ exactly I): Y equals DQ(A) exactly; zero rows give exactly the bias."""
+    K = 128
+    X = WL.to_fp16(np.random.default_rng(2).standard_t(3, (64, K)))
+    X[5] = 0
+    W = np.eye(K, dtype=np.float16)
+    fmt = np.full(K, F.W_MXINT8, np.uint8)
+    bias = np.random.default_rng(3).normal(0, 1, K).astype(np.float32)
+    for act_fmt in ACT:
+        Y = gpu_linear(cl, X, W, fmt, act_fmt, bias)
+        a = F.act_dequant(F.act_quant(X, act_fmt))
+        np.testing.assert_array_equal(Y, (a + bias[None, :]).astype(np.float32))
+
+
+def test_deterministic(cl):
+    X, W, bias = WL.single_layer()
+    fmt, _, _ = SEL.select_formats(W, 0x1F8)
+    Y1 = gpu_linear(cl, X, W, fmt, F.A_E4M3, bias)
+    Y2 = gpu_linear(cl, X, W, fmt, F.A_E4M3, bias)
+    assert Y1.tobytes() == Y2.tobytes()
+
+
+@pytest.mark.parametrize("layer", range(len(WL.SDXL_PROJ_LAYERS)))
+def test_full_size_sdxl_projection_sampled_rows(cl, layer):
+    """Full-size W8A8 SDXL projections in the launch configuration the benchmark uses; the fp64
+    reference is computed on 96 seeded rows."""
+    import torch
+    name, M, K, N = WL.SDXL_PROJ_LAYERS[layer]
+    W, bias = WL.sdxl_layer_weights(layer)
+    fmt_dev, _ = cl.select_weight_formats(cuda(W), 0x007)
+    fmt = host(fmt_dev)
+    for bucket, act_fmt in [(9, F.A_E5M2), (3, F.A_E4M3), (0, F.A_INT8_ASYM)]:
+        X = WL.sdxl_layer_activation(layer, bucket)
+        Y = gpu_linear(cl, X, W, fmt, act_fmt, bias)
+        rows = np.sort(np.random.default_rng(layer).choice(M, 96, replace=False))
+        a = F.act_dequant(F.act_quant(X, act_fmt))
+        w = SEL.dequant_selected(W, fmt)
+        y_ref, bound = G.linear_rows_reference(a, w, rows, bias)
+        assert_within_bound(Y[rows], y_ref, bound, "%s bucket %d" % (name, bucket))

@@ -1,0 +1,100 @@
+"""GPU weight-format selection (a5) and pack (a6) against the oracle."""
+import numpy as np
+import pytest
+
+from oracle import formats as F
+from oracle import select as SEL
+from paper_2609_33496_gb300 import workloads as WL
+from gpu_common import lib_module, cuda, host
+from blob import unpack
+
+pytestmark = pytest.mark.gpu
+TURBO = (1 << F.W_INT4_ASYM) | (1 << F.W_NF4) | (1 << F.W_E2M1) | (1 << F.W_MXINT4) | (1 << F.W_MXFP4)
+
+
+@pytest.fixture(scope="module")
+def cl():
+    return lib_module()
+
+
+def gpu_select(cl, W, mask):
+    import torch
+    fmt, sse = cl.select_weight_formats(cuda(W), mask, want_sse=True)
+    torch.cuda.synchronize()
+    return host(fmt), host(sse)
+
+
+def check_selection(cl, W, mask):
+    fmt_g, sse_g = gpu_select(cl, W, mask)
+    fmt_o, sse_o, pal = SEL.select_formats(W, mask)
+    for j, f in enumerate(pal):
+        np.testing.assert_allclose(sse_g[:, f], sse_o[:, j], rtol=1e-6, atol=1e-30)
+    nonmember = [f for f in range(9) if f not in pal]
+    assert np.all(np.isinf(sse_g[:, nonmember]))
+    diff = np.nonzero(fmt_g != fmt_o)[0]
+    for c in diff:   # a different choice only where the oracle's two best errors are a near-tie
+        assert SEL.near_tie(sse_o[c]), (c, fmt_g[c], fmt_o[c], sse_o[c])
+    return fmt_g, fmt_o
+
+
+@pytest.mark.parametrize("mask", [0x007, 0x1F8, TURBO])
+def test_select_single_layer(cl, mask):
+    _, W, _ = WL.single_layer()
+    check_selection(cl, W, mask)
+
+
+@pytest.mark.parametrize("mask", [0x007, 0x1F8])
+def test_select_mixed_distributions(cl, mask):
+    W = WL.weight_mix(np.random.default_rng(3), 300, 320)
+    fmt_g, _ = check_selection(cl, W, mask)
+    assert len(np.unique(fmt_g)) >= 2
+
+
+def test_select_constructed_channels(cl):
+    K = 64
+    ints = np.tile(np.arange(-7, 8), 5)[:K].astype(np.float64)
+    W = np.stack([ints * 2.0 ** -9, np.zeros(K), np.ones(K) * 0.01]).astype(np.float16)
+    fmt_g, fmt_o = check_selection(cl, W, 0x1F8)
+    assert fmt_g[0] == F.W_INT4_SYM and fmt_g[1] == F.W_INT4_SYM
+
+
+def unpack_blob(cl, W, fmt):
+    import torch
+    d = cl.pack_plan(W.shape[0], W.shape[1], fmt)
+    blob, st = cl.pack_weights(cuda(W), cuda(fmt), d)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    return unpack(host(blob).tobytes())
+
+
+@pytest.mark.parametrize("mask,K", [(0x007, 320), (0x1F8, 320), (0x1F8, 96), (0x007, 160)])
+def test_pack_matches_oracle_codes(cl, mask, K):
+    W = WL.weight_mix(np.random.default_rng(K), 261, K)
+    fmt_o, _, pal = SEL.select_formats(W, mask)
+    fmt = fmt_o.copy()
+    fmt[::7] = pal[-1]          # make sure every palette member appears
+    fmt[1::7] = pal[0]
+    desc, got = unpack_blob(cl, W, fmt)
+    ref = SEL.quantize_selected(W, fmt)
+    assert sorted(got) == list(range(W.shape[0]))
+    for c, r in enumerate(ref):
+        g = got[c]
+        assert g["fmt"] == r["fmt"]
+        np.testing.assert_array_equal(g["codes"], r["codes"], err_msg="channel %d fmt %d" % (c, r["fmt"]))
+        if F.W_IS_MX[r["fmt"]]:
+            np.testing.assert_array_equal(g["e8m0"], r["e8m0"])
+        else:
+            assert np.float32(g["s"]).tobytes() == np.float32(r["s"]).tobytes()
+            assert g["z"] == r["z"]
+
+
+def test_pack_permutation_groups_formats(cl):
+    W = WL.weight_mix(np.random.default_rng(9), 200, 64)
+    fmt = np.random.default_rng(1).choice(np.arange(3, 9), 200).astype(np.uint8)
+    desc, got = unpack_blob(cl, W, fmt)
+    slots = sorted((g["slot"], c, g["fmt"]) for c, g in got.items())
+    order = {3: 0, 4: 1, 6: 2, 7: 3, 8: 4, 5: 10}   # class 0 formats, then NF4 (class 1)
+    keys = [(order[f], c) for _, c, f in slots]
+    assert keys == sorted(keys)                      # format runs, original order inside a run
+    class1_first = min(g["slot"] for g in got.values() if g["fmt"] == F.W_NF4)
+    assert class1_first % 128 == 0
