@@ -100,15 +100,14 @@ def layer_flops(M, K, N):
     return 2.0 * M * K * N
 
 
-def host_inputs(WL):
+def host_inputs(WL, layer_ids, buckets):
     """Weights, biases and the activations of every (layer, bucket), generated once on the host."""
-    layers = WL.SDXL_PROJ_LAYERS
     Wn, bn, Xn = [], [], []
-    for li in range(len(layers)):
+    for li in layer_ids:
         w, b = WL.sdxl_layer_weights(li)
         Wn.append(w)
         bn.append(b)
-        Xn.append([WL.sdxl_layer_activation(li, bk) for bk in range(10)])
+        Xn.append([WL.sdxl_layer_activation(li, bk) for bk in buckets])
     return Wn, bn, Xn
 
 
@@ -120,17 +119,17 @@ def build_inputs(torch, host, device):
     return W, bias, X
 
 
-def calibrate_lut(torch, cl, X, device):
+def calibrate_lut(torch, cl, X, buckets):
     """Alg. 1 on the synthetic activations: power sums on the GPU, kappa, SNR at the bucket
     midpoint (scaled-linear schedule), Route -> F[l, b]."""
     snr = cl.snr(cl.SCHEDULE_SCALED_LINEAR, 1000)
-    lut = np.zeros((len(X), 10), dtype=np.int64)
-    kappa = np.zeros((len(X), 10))
+    lut = np.zeros((len(X), len(buckets)), dtype=np.int64)
+    kappa = np.zeros((len(X), len(buckets)))
     for li, xs in enumerate(X):
-        for bk, x in enumerate(xs):
+        for j, x in enumerate(xs):
             sums = cl.act_moments(x).cpu().numpy()
-            kappa[li, bk] = cl.kurtosis(sums[:5])
-            lut[li, bk] = cl.route(kappa[li, bk], snr[bk * 100 + 50], False)
+            kappa[li, j] = cl.kurtosis(sums[:5])
+            lut[li, j] = cl.route(kappa[li, j], snr[buckets[j] * 100 + 50], False)
     return lut, kappa
 
 
@@ -142,6 +141,8 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", default="all", help="comma-separated layer indices (smaller cases for profiling)")
+    ap.add_argument("--buckets", default="all", help="comma-separated timestep buckets")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -169,10 +170,14 @@ def main():
     if world > 1:
         dist.init_process_group("nccl", device_id=device)
 
-    layers = WL.SDXL_PROJ_LAYERS
-    host = host_inputs(WL)
+    layer_ids = list(range(len(WL.SDXL_PROJ_LAYERS))) if args.layers == "all" else [
+        int(v) for v in args.layers.split(",")]
+    buckets = list(range(10)) if args.buckets == "all" else [int(v) for v in args.buckets.split(",")]
+    layers = [WL.SDXL_PROJ_LAYERS[i] for i in layer_ids]
+    nb = len(buckets)
+    host = host_inputs(WL, layer_ids, buckets)
     W, bias, X = build_inputs(torch, host, device)
-    lut, kappa = calibrate_lut(torch, cl, X, device)
+    lut, kappa = calibrate_lut(torch, cl, X, buckets)
     st = torch.zeros(1, dtype=torch.int32, device=device)
     stream = torch.cuda.current_stream()
 
@@ -192,12 +197,12 @@ def main():
             blobs.append(blob)
         return descs, blobs, fmts_host
 
-    flops_step = 10 * sum(layer_flops(M, K, N) for (_, M, K, N) in layers)
+    flops_step = nb * sum(layer_flops(M, K, N) for (_, M, K, N) in layers)
     quant_bytes_step = 0.0
     gemm_bytes_step = 0.0
 
     def run_step(descs, blobs, ev):
-        for bk in range(10):
+        for bk in range(nb):
             for li, (_, M, K, N) in enumerate(layers):
                 f = int(lut[li, bk])
                 if ev is not None:
@@ -222,9 +227,9 @@ def main():
     # kernel launches per step: select 1 + pack 3 per layer; per linear 2 (per-tensor) or 1 (MX)
     # quantizer kernels + 1 GEMM
     launches = 4 * len(layers) + sum(
-        (2 if lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(10))
+        (2 if lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(nb))
     for li, (_, M, K, N) in enumerate(layers):
-        for bk in range(10):
+        for bk in range(nb):
             mx = lut[li, bk] >= 3
             quant_bytes_step += M * K * 2 + M * K * 2 + (M * K / 32 if mx else 0)
             gemm_bytes_step += M * K * 1 + N * K * 1 + N * (4 + 1) + 4 * N + M * N * 4
@@ -274,14 +279,16 @@ def main():
     t_roof = 0.0
     for li, (_, M, K, N) in enumerate(layers):
         b = M * K + N * K + 5 * N + 4 * N + 4 * M * N
-        t_roof += 10 * max(layer_flops(M, K, N) / (peak_tensor * 1e12), b / (pk["hbm_gbs"] * 1e9))
+        t_roof += nb * max(layer_flops(M, K, N) / (peak_tensor * 1e12), b / (pk["hbm_gbs"] * 1e9))
     clocks = clk.summary()
 
     result = {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
         "warmup": args.warmup, "ms_per_step": round(elapsed_ms / K_, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "layers": len(layers), "buckets": 10, "global_batch": 2 * world,
+        "config": {"workload": WORKLOAD if (args.layers, args.buckets) == ("all", "all") else
+                   WORKLOAD + " (subset: layers %s, buckets %s)" % (layer_ids, buckets),
+                   "layers": len(layers), "buckets": nb, "global_batch": 2 * world,
                    "tokens": [M for (_, M, _, _) in layers], "weight_palette": "W8 {INT8-sym, INT8-asym, MXINT8}",
                    "activation_formats_used": sorted(set(int(v) for v in lut.ravel())),
                    "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant + GEMM",
@@ -304,7 +311,7 @@ def main():
     }
     if not args.no_e2e:
         del X
-        result["e2e"] = e2e_leg(args, torch, cl, host, layers, lut, device, stream, world, flops_step)
+        result["e2e"] = e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops_step)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline()
     if rank == 0:
@@ -314,7 +321,7 @@ def main():
     return 0
 
 
-def e2e_leg(args, torch, cl, host, layers, lut, device, stream, world, flops_step):
+def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops_step):
     """Same step through the public calls with HOST buffers: the weights and every activation are
     copied host->device from pinned memory and every output device->host inside the timed
     region."""
@@ -332,7 +339,7 @@ def e2e_leg(args, torch, cl, host, layers, lut, device, stream, world, flops_ste
     ws = [torch.empty(max(cl.linear_workspace_size(M, cl.pack_plan(N, K, np.zeros(N, np.uint8)), f)
                           for f in range(6)), dtype=torch.uint8, device=device) for (_, M, K, N) in layers]
     h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + sum(x.numel() * 2 for xs in Xh for x in xs)
-    d2h = 10 * sum(M * N * 4 for (_, M, K, N) in layers)
+    d2h = nb * sum(M * N * 4 for (_, M, K, N) in layers)
 
     def step():
         fmts, descs, blobs = [], [], []
@@ -344,7 +351,7 @@ def e2e_leg(args, torch, cl, host, layers, lut, device, stream, world, flops_ste
             d = cl.pack_plan(N, K, fmts[li].cpu().numpy())
             descs.append(d)
             blobs.append(cl.pack_weights(Wd[li], fmts[li], d, dev_status=st)[0])
-        for bk in range(10):
+        for bk in range(nb):
             for li in range(len(layers)):
                 Xd[li].copy_(Xh[li][bk], non_blocking=True)
                 cl.linear(Xd[li], descs[li], blobs[li], int(lut[li, bk]), bias=bd[li], Y=Yd[li], ws=ws[li],
