@@ -209,6 +209,21 @@ cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d
                                   int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
                                   int* dev_status, void* stream);
 
+/* chameleon_act_quant without a caller-supplied workspace.  The paper has no counterpart: this
+ * entry point exists for callers that cannot allocate device memory when they quantize -- code
+ * embedded in a host application or inference runtime that owns every device buffer and hands
+ * its plugins only their inputs and outputs, or that forbids allocation once serving starts.
+ * Same arguments, output layout and results as chameleon_act_quant, minus ws / ws_bytes.  The
+ * per-tensor formats keep their range partials in a library-owned static device array of
+ * 1024 x 16 bytes (16 KiB, held on every GPU that loads the library until exit); this fits any
+ * M, K on GPUs with up to 256 SMs and returns CHAM_ERR_WORKSPACE (nothing launched) otherwise.
+ * It calls no allocator.  The first call on a device looks up the array's address with that
+ * device current: make it before any stream capture.  All calls share the array; calls whose
+ * kernels overlap on the GPU (e.g. concurrent streams) race on it and give wrong results.
+ * Errors are returned as status codes only (chameleon_last_error_detail is not updated). */
+cham_status chameleon_act_quant_noalloc(const void* X, int M, int K, int fmt, void* qact, size_t qact_bytes,
+                                        int* dev_status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

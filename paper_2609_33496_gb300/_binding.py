@@ -30,7 +30,7 @@ EXPORTS = [
     "chameleon_act_quant_size", "chameleon_act_quant",
     "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_weights",
     "chameleon_linear_workspace_size", "chameleon_linear", "chameleon_linear_prepare",
-    "chameleon_linear_gemm",
+    "chameleon_linear_gemm", "chameleon_act_quant_noalloc",
 ]
 
 
@@ -95,6 +95,7 @@ def lib():
         "chameleon_linear": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
         "chameleon_linear_prepare": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
         "chameleon_linear_gemm": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
+        "chameleon_act_quant_noalloc": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -257,3 +258,12 @@ def linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream=None):
     """Second half of linear: the tcgen05 GEMM on the prepared operand."""
     check(lib().chameleon_linear_gemm(_ptr(X), X.shape[0], ctypes.byref(desc), _ptr(blob), act_fmt, _ptr(bias),
                                       _ptr(Y), _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))
+
+
+def act_quant_noalloc(X, fmt, qact, dev_status, stream=None):
+    """chameleon_act_quant without a workspace, for callers that cannot allocate at call time:
+    the caller passes the output buffer `qact` (sized by act_quant_size) and the status word; the
+    range partials live in a static device array inside the library.  Returns the raw status."""
+    M, K = X.shape
+    return lib().chameleon_act_quant_noalloc(_ptr(X), M, K, fmt, _ptr(qact), qact.numel(), _ptr(dev_status),
+                                             _stream(stream))

@@ -13,7 +13,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libchameleon.so")
-SOURCES = ["act_quant.cu", "weights.cu", "gemm.cu", "api.cu"]
+SOURCES = ["act_quant.cu", "weights.cu", "gemm.cu", "api.cu", "noalloc.cu"]
 # translation units whose quantizer arithmetic must not be contracted into FMAs
 NO_FMAD = {"act_quant.cu", "weights.cu"}
 HEADERS = ["common.cuh", "act_quant.cuh", "weights.cuh", "gemm.cuh"]
