@@ -181,48 +181,74 @@ def main():
     st = torch.zeros(1, dtype=torch.int32, device=device)
     stream = torch.cuda.current_stream()
 
-    # buffers reused every step
+    # buffers reused every step (the packed weights are re-packed in place every step)
     Y = [torch.empty((M, N), dtype=torch.float32, device=device) for (_, M, K, N) in layers]
     ws = [torch.empty(max(cl.linear_workspace_size(M, cl.pack_plan(N, K, np.zeros(N, np.uint8)), f)
                           for f in range(6)), dtype=torch.uint8, device=device) for (_, M, K, N) in layers]
+    blobs, descs = [None] * len(layers), [None] * len(layers)
 
     def select_pack():
-        descs, blobs = [], []
+        """a5 + a6 for every layer: GPU selection, host plan from the selected formats (one
+        device->host copy of N bytes per layer), GPU pack into the layer's blob."""
         fmts = [cl.select_weight_formats(W[li], cl.PALETTE_W8)[0] for li in range(len(layers))]
-        fmts_host = [f.cpu().numpy() for f in fmts]           # the plan needs the counts on the host
+        fmts_host = [f.cpu().numpy() for f in fmts]
         for li, (_, M, K, N) in enumerate(layers):
             d = cl.pack_plan(N, K, fmts_host[li])
-            blob, _ = cl.pack_weights(W[li], fmts[li], d, dev_status=st)
-            descs.append(d)
-            blobs.append(blob)
-        return descs, blobs, fmts_host
+            if descs[li] is not None and bytes(d) != bytes(descs[li]):
+                raise RuntimeError("packed layout changed between steps")
+            blobs[li], _ = cl.pack_weights(W[li], fmts[li], d, dev_status=st, blob=blobs[li])
+            descs[li] = d
 
     flops_step = nb * sum(layer_flops(M, K, N) for (_, M, K, N) in layers)
     quant_bytes_step = 0.0
     gemm_bytes_step = 0.0
 
-    def run_step(descs, blobs, ev):
+    try:
+        torch.cuda.Event(enable_timing=True, external=True)
+        ext = {"external": True}
+    except TypeError:
+        ext = None
+    n_ev = 2 * nb * len(layers) + 1
+    events = [torch.cuda.Event(enable_timing=True, **(ext or {})) for _ in range(n_ev)]
+    kinds = []
+
+    def run_step(record):
+        """a2-a4 + a7 for every (bucket, layer): act-quant in F[l, b], then the GEMM."""
+        k = 0
         for bk in range(nb):
             for li, (_, M, K, N) in enumerate(layers):
                 f = int(lut[li, bk])
-                if ev is not None:
-                    ev.append(("q", li, bk, torch.cuda.Event(enable_timing=True)))
-                    ev[-1][3].record(stream)
+                if record:
+                    events[k].record()
+                    k += 1
                 cl.linear_prepare(X[li][bk], f, ws[li], st)
-                if ev is not None:
-                    ev.append(("g", li, bk, torch.cuda.Event(enable_timing=True)))
-                    ev[-1][3].record(stream)
+                if record:
+                    events[k].record()
+                    k += 1
                 cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
-        if ev is not None:
-            ev.append(("end", -1, -1, torch.cuda.Event(enable_timing=True)))
-            ev[-1][3].record(stream)
+        if record:
+            events[k].record()
 
-    # warm-up
+    for bk in range(nb):
+        for li in range(len(layers)):
+            kinds.extend(["q", "g"])
+
+    # warm-up (eager), then capture the quantize + GEMM sequence of one step in a CUDA graph with
+    # timing event nodes between the kernels; select + pack stay eager (they need a host plan)
     for _ in range(args.warmup):
-        descs, blobs, fmts_host = select_pack()
-        run_step(descs, blobs, None)
+        select_pack()
+        run_step(False)
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
+    graph = None
+    if ext is not None:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            run_step(True)
+        for _ in range(args.warmup):
+            select_pack()
+            graph.replay()
+        torch.cuda.synchronize()
 
     # kernel launches per step: select 1 + pack 3 per layer; per linear 2 (per-tensor) or 1 (MX)
     # quantizer kernels + 1 GEMM
@@ -234,7 +260,18 @@ def main():
             quant_bytes_step += M * K * 2 + M * K * 2 + (M * K / 32 if mx else 0)
             gemm_bytes_step += M * K * 1 + N * K * 1 + N * (4 + 1) + 4 * N + M * N * 4
     # ---------------------------------------------------------------- timed region (device)
-    all_ev = []
+    gemm_ms, quant_ms, gemm_launch_ms = 0.0, 0.0, []
+
+    def collect():
+        nonlocal gemm_ms, quant_ms
+        for i in range(n_ev - 1):
+            d = events[i].elapsed_time(events[i + 1])
+            if kinds[i] == "g":
+                gemm_ms += d
+                gemm_launch_ms.append(d)
+            else:
+                quant_ms += d
+
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -242,13 +279,17 @@ def main():
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record(stream)
-        for _ in range(args.steps):
-            descs, blobs, fmts_host = select_pack()
-            ev = []
-            run_step(descs, blobs, ev)
-            all_ev.append(ev)
+        for k in range(args.steps):
+            select_pack()                 # its host plan waits for the previous step's graph
+            if k > 0:
+                collect()                 # events of the previous replay are complete here
+            if graph is not None:
+                graph.replay()
+            else:
+                run_step(True)
         t1.record(stream)
         torch.cuda.synchronize()
+        collect()
     if world > 1:
         dist.barrier()
     elapsed_ms = t0.elapsed_time(t1)
@@ -258,17 +299,6 @@ def main():
         elapsed_ms = float(tt.item())
     assert int(st.item()) == 0, "device status %d" % int(st.item())
 
-    # per-kernel durations from the events
-    gemm_ms, quant_ms, gemm_launch_ms = 0.0, 0.0, []
-    for ev in all_ev:
-        for i in range(len(ev) - 1):
-            kind, li, bk, e = ev[i]
-            d = e.elapsed_time(ev[i + 1][3])
-            if kind == "g":
-                gemm_ms += d
-                gemm_launch_ms.append(d)
-            elif kind == "q":
-                quant_ms += d
     K_ = args.steps
     value = world * flops_step * K_ / (elapsed_ms * 1e-3) / 1e12
     pk, pk_kind = peaks()
@@ -302,7 +332,9 @@ def main():
                      "peak_source": "%s bf16_tflops_sustained (fp16 MMA rate = bf16 rate)" % pk_kind,
                      "roofline_time_frac": round(t_roof * K_ / (gemm_ms * 1e-3), 4),
                      "gemm_ms_per_step": round(gemm_ms / K_, 4),
-                     "gemm_launch_ms_mean": round(statistics.mean(gemm_launch_ms), 5)},
+                     "gemm_launch_ms_mean": round(statistics.mean(gemm_launch_ms), 5),
+                     "timing": "CUDA-graph replay of the quantize+GEMM sequence, event nodes between kernels"
+                               if graph is not None else "eager launches, events between kernels"},
         "act_quant": {"achieved_gbs": round(quant_gbs, 1), "peak_gbs": pk["hbm_gbs"],
                       "frac": round(quant_gbs / pk["hbm_gbs"], 4), "ms_per_step": round(quant_ms / K_, 4),
                       "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"},

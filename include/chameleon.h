@@ -144,8 +144,9 @@ cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_
  * channel permutation") into two MMA classes, each padded to 128-channel tiles:
  *   class 0 = 4-bit formats with an 8-bit tensor-core path (INT4-sym, INT4-asym, E2M1, MXINT4,
  *             MXFP4), class 1 = the rest (NF4, INT8-sym, INT8-asym, MXINT8);
- * inside a class by format in that order, then by original channel index.  Offsets are from the
- * blob base, 256-byte aligned.  Blob regions:
+ * inside a class in original channel order (a tile's output columns stay contiguous; the GEMM
+ * decodes each channel in its own format).  Offsets are from the blob base, 256-byte aligned.
+ * Blob regions:
  *   [0, 256)       a copy of this descriptor
  *   codes          per tile t (128 packed channels) and K-chunk c (64 elements): 128 * CB bytes,
  *                  CB = 64 (8-bit) or 32 (4-bit) bytes per channel, stored as CB/16 slabs of

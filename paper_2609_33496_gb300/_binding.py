@@ -214,12 +214,13 @@ def pack_plan(N, K, fmt_host):
     return d
 
 
-def pack_weights(W, fmt_dev, desc, dev_status=None, stream=None):
+def pack_weights(W, fmt_dev, desc, dev_status=None, stream=None, blob=None):
     import torch
-    blob = _bytes(desc.bytes, W.device)
+    if blob is None or blob.numel() < desc.bytes:
+        blob = _bytes(desc.bytes, W.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=W.device)
-    check(lib().chameleon_pack_weights(_ptr(W), _ptr(fmt_dev), ctypes.byref(desc), _ptr(blob), desc.bytes,
+    check(lib().chameleon_pack_weights(_ptr(W), _ptr(fmt_dev), ctypes.byref(desc), _ptr(blob), blob.numel(),
                                        _ptr(dev_status), _stream(stream)))
     return blob, dev_status
 

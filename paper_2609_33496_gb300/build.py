@@ -13,10 +13,12 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libchameleon.so")
+PROBE_LIB = os.path.join(HERE, "libchameleon_probe.so")   # tensor-core throughput probe (bench only)
 SOURCES = ["act_quant.cu", "weights.cu", "gemm.cu", "api.cu", "noalloc.cu"]
 # translation units whose quantizer arithmetic must not be contracted into FMAs
 NO_FMAD = {"act_quant.cu", "weights.cu"}
 HEADERS = ["common.cuh", "act_quant.cuh", "weights.cuh", "gemm.cuh"]
+PROBE_SOURCES = ["probe.cu"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
@@ -41,10 +43,11 @@ def _inputs():
 
 
 def up_to_date():
-    if not os.path.exists(LIB):
-        return False
-    t = os.path.getmtime(LIB)
-    return all(os.path.getmtime(f) <= t for f in _inputs())
+    for lib in (LIB, PROBE_LIB):
+        if not os.path.exists(lib):
+            return False
+    t = min(os.path.getmtime(LIB), os.path.getmtime(PROBE_LIB))
+    return all(os.path.getmtime(f) <= t for f in _inputs() + [os.path.join(CSRC, s) for s in PROBE_SOURCES])
 
 
 def _compile(src):
@@ -62,14 +65,15 @@ def build(force=False, verbose=False):
     if not force and up_to_date():
         return LIB
     os.makedirs(BUILD, exist_ok=True)
-    with concurrent.futures.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(_compile, SOURCES))
-    tmp = LIB + ".tmp"
-    cmd = [nvcc()] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs
-    r = subprocess.run(cmd, capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))
-    os.replace(tmp, LIB)
+    with concurrent.futures.ThreadPoolExecutor(max_workers=len(SOURCES) + len(PROBE_SOURCES)) as ex:
+        objs = list(ex.map(_compile, SOURCES + PROBE_SOURCES))
+    for lib, lib_objs in ((LIB, objs[:len(SOURCES)]), (PROBE_LIB, objs[len(SOURCES):])):
+        tmp = lib + ".tmp"
+        cmd = [nvcc()] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + lib_objs
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))
+        os.replace(tmp, lib)
     if verbose:
         print("built", LIB)
     return LIB

@@ -235,7 +235,7 @@ __global__ void __launch_bounds__(256)
         const int qb = min(max(__float2int_rn(__fmul_rn(b, 64.f)), -127), 127);
         pair = (static_cast<uint32_t>(qa) & 0xFFu) | ((static_cast<uint32_t>(qb) & 0xFFu) << 8);
         if constexpr (DEQ) {
-          const float up = exp2i_f32(Xe - 6);
+          const float up = exp2i_f32(max(Xe - 6, -126));  // zero block (Xe = -127): codes are 0
           const __half2 h = __floats2half2_rn(__fmul_rn(static_cast<float>(qa), up),
                                               __fmul_rn(static_cast<float>(qb), up));
           d[j] = *reinterpret_cast<const uint32_t*>(&h);

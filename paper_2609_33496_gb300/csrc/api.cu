@@ -168,7 +168,7 @@ cham_status check_act_args(const void* X, int M, int K, int fmt, bool allow_fp16
   return CHAM_OK;
 }
 
-// Per-format packing order inside each MMA class (R15).
+// Formats of each MMA class (R15).
 const int kClassOrder[2][5] = {{CHAM_W_INT4_SYM, CHAM_W_INT4_ASYM, CHAM_W_E2M1, CHAM_W_MXINT4, CHAM_W_MXFP4},
                                {CHAM_W_NF4, CHAM_W_INT8_SYM, CHAM_W_INT8_ASYM, CHAM_W_MXINT8, -1}};
 
@@ -423,17 +423,10 @@ cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const 
   a.bits = d->bits;
   a.n_chunks = d->Kp / 64;
   a.n_packed = 128 * (d->n_tiles[0] + d->n_tiles[1]);
-  for (int cls = 0, base = 0; cls < 2; ++cls) {
-    int slot = base;
-    for (int j = 0; j < 5; ++j) {
-      const int f = kClassOrder[cls][j];
-      if (f < 0) continue;
-      a.base[f] = slot;
-      a.count[f] = d->n_fmt[f];
-      slot += d->n_fmt[f];
-    }
-    base += 128 * d->n_tiles[cls];
-  }
+  a.cls_base[0] = 0;
+  a.cls_base[1] = 128 * d->n_tiles[0];
+  a.cls_count[0] = d->n_class[0];
+  a.cls_count[1] = d->n_class[1];
   a.codes = b + d->off_codes;
   a.scale = reinterpret_cast<float*>(b + d->off_scale);
   a.zero = b + d->off_zero;
@@ -531,7 +524,8 @@ cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d
   s = make_act_map(&map, operand, M, K, bn);
   if (s != CHAM_OK) return s;
   g.tile0 = 0;
-  const cudaError_t e = cham::launch_gemm_f16(map, g, tiles, bn, static_cast<cudaStream_t>(stream));
+  g.n_ch_tiles = tiles;
+  const cudaError_t e = cham::launch_gemm_f16(map, g, num_sms, bn, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "gemm launch");
 }
 

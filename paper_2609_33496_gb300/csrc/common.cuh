@@ -51,19 +51,48 @@ CHAM_DEV bool mbar_test(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Polls before a wait gives up.  try_wait itself suspends for a hardware time slice, and the
-// loop backs off with nanosleep after the first polls, so the limit is seconds of wall time --
-// far beyond any legitimate wait in these kernels.
-constexpr uint32_t kWaitPolls = 1u << 22;
+// Non-blocking test of the phase with the given parity (returns at once; try_wait, by contrast,
+// costs a suspend/resume of a few hundred cycles even when the phase has already completed).
+CHAM_DEV bool mbar_ready(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Suspending wait: the hardware parks the thread until the phase completes or `ns` nanoseconds
+// pass, so waiting warps do not poll (polling warps flood the barrier path and delay the
+// latency-critical MMA-issuing thread's own waits by hundreds of cycles).
+CHAM_DEV bool mbar_try_wait_for(uint64_t* bar, uint32_t parity, uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(ns)
+      : "memory");
+  return ok != 0;
+}
+
+// Rounds of 1 ms suspended waits before a wait gives up: about two seconds, far beyond any
+// legitimate wait in these kernels.
+constexpr uint32_t kWaitRounds = 2000;
+constexpr uint32_t kWaitRoundNs = 1000000;
+constexpr uint32_t kWaitPolls = 1u << 22;  // polls of the drain waits (mbar_test)
 
 // Wait for the phase with the given parity to complete.  Returns false (after recording
 // CHAM_ERR_TIMEOUT and raising the CTA's abort flag) when the limit is reached or another
 // thread of the CTA has already aborted.
 CHAM_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* dev_status) {
-  for (uint32_t i = 0; i < kWaitPolls; ++i) {
-    if (mbar_test(bar, parity)) return true;
+  for (uint32_t i = 0; i < kWaitRounds; ++i) {
+    if (mbar_try_wait_for(bar, parity, kWaitRoundNs)) return true;
     if (*abort_flag) return false;
-    if (i > 64) __nanosleep(128);
   }
   *abort_flag = 1;
   set_status(dev_status, CHAM_ERR_TIMEOUT);

@@ -3,43 +3,60 @@
 // Y[m, perm[p]] = s_a * s_w[p] * sum_k A^[m, k] * W^[p, k] + bias[perm[p]]   (Sec. 3.6, Alg. 2/3)
 //
 // Operand roles are swapped relative to the textbook layout so that the weight side -- the
-// operand that needs per-channel decoding -- never touches shared memory:
+// operand that needs per-channel decoding -- never has to be written to shared memory:
 //   * MMA "A" (M = 128 rows) = one tile of 128 packed weight channels.  Four decode warps own one
-//     channel per thread, read its codes with coalesced 16-byte loads, decode them in registers to
-//     exact fp16 operand values (the MX block exponent folded in, the per-channel scale kept for
-//     the epilogue) and write them straight into tensor memory with tcgen05.st.
+//     channel per thread, read its codes from a shared-memory stage that a bulk copy filled,
+//     decode them in registers to the exact fp16 operand values (MX block exponent folded in, the
+//     per-channel scale kept for the epilogue) and write them into tensor memory (tcgen05.st).
 //   * MMA "B" (N = BN tokens) = a tile of activation operand rows, brought into shared memory by
 //     TMA with 128-byte swizzling, K-major.
-//   * D (128 channels x BN tokens, fp32) accumulates in tensor memory; the same four warps read
-//     it back with tcgen05.ld, apply s_a * s_w and the bias, and store Y in original channel order.
-// A 4-stage ring over K-chunks of 64 couples them: TMA and decode fill stage s, one thread issues
-// four kind::f16 MMAs (K = 16 each) on it, and the MMA commit frees the stage for both producers.
-// Every wait is bounded (common.cuh); on a timeout the kernel records CHAM_ERR_TIMEOUT, drains
-// its own copies and MMAs, releases tensor memory and returns.
+//   * D (128 channels x BN tokens, fp32) accumulates in tensor memory, double buffered: four
+//     epilogue warps drain one buffer (tcgen05.ld, s_a * s_w, bias, coalesced stores of Y in
+//     original channel order) while the MMA fills the other with the next tile.
+// The kernel is persistent: each CTA walks tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of
+// the (channel tile, token tile) grid.  Two rings over K-chunks of 64 couple the roles: a 6-8
+// stage shared-memory ring (activation tile + raw weight codes + their E8M0 bytes, filled by TMA
+// and bulk copies, deep enough to cover the load round trip) and a 4-slot tensor-memory ring of
+// decoded weight operands; one thread issues four kind::f16 MMAs (K = 16 each) per chunk, and
+// MMA commits free both slots.  Every wait is bounded (common.cuh); on a timeout
+// the kernel records CHAM_ERR_TIMEOUT, drains its own copies and MMAs, releases tensor memory and
+// returns.
 #include "gemm.cuh"
 
 namespace cham {
 
-constexpr int kStages = 4;
 constexpr int kBK = 64;  // K elements per stage: 128 bytes of fp16 per activation row
-constexpr int kGemmThreads = 256;
+constexpr int kDecodeGroups = 2;  // decode warpgroups, taking alternate K-chunks
+constexpr int kGemmThreads = 128 * (2 + kDecodeGroups);
 
-template <int BN>
+template <int BN, int BITS>
 struct GemmCfg {
-  static constexpr int kBStage = BN * 128;
-  static constexpr int kData = kStages * kBStage;
-  static constexpr int kTmemCols = (BN + kStages * 32) <= 256 ? 256 : 512;
-  static constexpr int kACol = kTmemCols - kStages * 32;  // first TMEM column of the A stages
-  static constexpr int kMisc = 1024 /*NF4 pair table*/ + 8 * (3 * kStages + 1) + 16;
+  static constexpr int kBBytes = BN * 128;                        // activation tile
+  static constexpr int kWBytes = 128 * (BITS == 8 ? 64 : 32);     // raw codes of 128 channels
+  static constexpr int kEBytes = 256;                             // their E8M0 pairs
+  static constexpr int kStage = (kBBytes + kWBytes + kEBytes + 1023) / 1024 * 1024;
+  // shared-memory ring: as deep as fits in ~200 KiB, to cover the TMA round trip (~1000 cycles)
+  // plus decode and MMA time of the stages in flight
+  static constexpr int kStages = (200 * 1024) / kStage > 8 ? 8 : (200 * 1024) / kStage;
+  static constexpr int kData = kStages * kStage;
+  static constexpr int kAccCols = (BN + 31) / 32 * 32;
+  static constexpr int kACol = 2 * kAccCols;                      // first column of the A stages
+  // tensor-memory ring of decoded weight operands (32 columns per K-chunk) and the number of
+  // consecutive chunks one MMA-side wait covers: as many as the 512 columns allow next to the two
+  // accumulators (every wait of the MMA thread costs a few hundred cycles of drained pipe)
+  static constexpr int kAStages = (kACol + 8 * 32) <= 512 ? 8 : 4;
+  static constexpr int kGroup = kAStages / 2;
+  static constexpr int kNeedCols = kACol + kAStages * 32;
+  static constexpr int kTmemCols = kNeedCols <= 256 ? 256 : 512;
+  static constexpr int kMisc = 1024 /*NF4 pair table*/ + 8 * (2 * kStages + 2 * 8 + 4) + 16;
   static constexpr int kNeed = 1024 /*alignment slack*/ + kData + kMisc;
-  // Shared-memory request: at most two CTAs per SM when each holds 256 TMEM columns, one when it
-  // holds 512, so tensor-memory allocations never have to wait for each other.
-  static constexpr int kFloor = kTmemCols == 512 ? 120 * 1024 : 80 * 1024;
-  static constexpr int kSmem = kNeed > kFloor ? kNeed : kFloor;
+  // at least 116 KiB so that two CTAs (and two tensor-memory allocations) never share an SM
+  static constexpr int kSmem = kNeed > 116 * 1024 ? kNeed : 116 * 1024;
+  static_assert(kStages >= 4, "ring depth");
+  static_assert(kSmem <= 227 * 1024, "within the opt-in shared-memory limit");
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "MMA N for M = 128");
+  static_assert(kNeedCols <= 512, "tensor memory budget");
 };
-
-CHAM_DEV float exp2i_clamped(int e) { return exp2i_f32(e < -126 ? -126 : e); }
 
 CHAM_DEV bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* st) {
   const bool ok = mbar_wait(bar, parity, abort_flag, st);
@@ -54,88 +71,113 @@ CHAM_DEV void drain_wait(uint64_t* bar, uint32_t parity) {
   }
 }
 
-// 8-bit codes of one channel's 64-element chunk -> 32 fp16 pairs (element 2c, 2c+1 in column c).
-CHAM_DEV void decode_w8(const uint32_t (&w)[16], int f, int z, uint32_t e8, uint32_t (&out)[32]) {
-  if (f == CHAM_W_MXINT8) {
-    const float sc0 = exp2i_clamped(static_cast<int>(e8 & 0xFFu) - 127 - 6);
-    const float sc1 = exp2i_clamped(static_cast<int>((e8 >> 8) & 0xFFu) - 127 - 6);
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const float sc = i < 8 ? sc0 : sc1;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int b0 = static_cast<int>(static_cast<int8_t>((w[i] >> (16 * h)) & 0xFFu));
-        const int b1 = static_cast<int>(static_cast<int8_t>((w[i] >> (16 * h + 8)) & 0xFFu));
-        out[2 * i + h] = h2_as_u32(__floats2half2_rn(__fmul_rn(static_cast<float>(b0), sc),
-                                                     __fmul_rn(static_cast<float>(b1), sc)));
-      }
-    }
+CHAM_DEV void bulk_load(uint32_t smem_dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(smem_dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// 2^e as an fp16 bit pattern for e in [-24, 15] (0 below).
+CHAM_DEV uint32_t exp2_h(int e) {
+  if (e >= -14) return static_cast<uint32_t>(e + 15) << 10;
+  if (e >= -24) return 1u << (e + 24);
+  return 0u;
+}
+
+// Two fp16 factors (as half2 bit patterns) whose product is 2^e, each applied exactly: the first
+// keeps an integer or E2M1 code in the normal range, the second carries what is left (the
+// product is an exact fp16 value, which the packer checks for MX weights).
+CHAM_DEV void pow2_factors(int e, uint32_t& f1, uint32_t& f2) {
+  const int a = min(max(e, -14), 15);
+  const uint32_t h1 = exp2_h(a), h2 = exp2_h(e - a);
+  f1 = h1 | (h1 << 16);
+  f2 = h2 | (h2 << 16);
+}
+
+CHAM_DEV uint32_t hsub2u(uint32_t a, uint32_t b) { return h2_as_u32(__hsub2(u32_as_h2(a), u32_as_h2(b))); }
+CHAM_DEV uint32_t hmul2u(uint32_t a, uint32_t b) { return h2_as_u32(__hmul2(u32_as_h2(a), u32_as_h2(b))); }
+
+// Per-channel decode constants.
+struct ChanDecode {
+  int f;          // weight format
+  uint32_t flip;  // xor applied to the raw code word (two's complement -> biased)
+  uint32_t sub;   // half2 (1024 + offset) subtracted from the magic-number value
+  int e_off;      // MX: block exponent offset of the element scale (MXINT8 -6, MXINT4 -2, MXFP4 0)
+};
+
+CHAM_DEV ChanDecode chan_decode(int f, int z) {
+  ChanDecode c;
+  c.f = f;
+  const bool asym = f == CHAM_W_INT8_ASYM || f == CHAM_W_INT4_ASYM;
+  const int off = asym ? z : (wbits(f) == 8 ? 128 : 8);
+  c.flip = asym ? 0u : (wbits(f) == 8 ? 0x80808080u : 0x88888888u);
+  const uint32_t h = h2_as_u32(__float2half2_rn(1024.f + static_cast<float>(off))) & 0xFFFFu;
+  c.sub = h | (h << 16);
+  c.e_off = f == CHAM_W_MXINT8 ? -6 : (f == CHAM_W_MXINT4 ? -2 : 0);
+  return c;
+}
+
+// Block scale factors of one chunk (two 32-element blocks); 1.0 for non-MX channels.
+CHAM_DEV void chunk_factors(const ChanDecode& c, uint32_t e8, uint32_t (&f1)[2], uint32_t (&f2)[2]) {
+  if (w_is_mx(c.f)) {
+    pow2_factors(static_cast<int>(e8 & 0xFFu) - 127 + c.e_off, f1[0], f2[0]);
+    pow2_factors(static_cast<int>((e8 >> 8) & 0xFFu) - 127 + c.e_off, f1[1], f2[1]);
   } else {
-    // 0x64XX as fp16 is 1024 + XX: subtract 1024 + 128 (sym, codes biased by the xor) or 1024 + z
-    const uint32_t flip = f == CHAM_W_INT8_SYM ? 0x80808080u : 0u;
-    const __half2 sub = __float2half2_rn(f == CHAM_W_INT8_SYM ? 1152.f : 1024.f + static_cast<float>(z));
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const uint32_t v = w[i] ^ flip;
-      out[2 * i] = h2_as_u32(__hsub2(u32_as_h2(__byte_perm(v, 0x64646464u, 0x4140)), sub));
-      out[2 * i + 1] = h2_as_u32(__hsub2(u32_as_h2(__byte_perm(v, 0x64646464u, 0x4342)), sub));
-    }
+    f1[0] = f1[1] = f2[0] = f2[1] = 0x3C003C00u;  // 1.0
   }
 }
 
-// 4-bit codes of one channel's chunk -> 32 fp16 pairs.  Word i holds elements 8i..8i+7 with
-// nibble j = element 2j and nibble 4+j = element 2j+1, so (x >> 4j) & 0x000F000F isolates a pair.
-CHAM_DEV void decode_w4(const uint32_t (&w)[8], int f, int z, uint32_t e8, const uint32_t* lut,
+// 8-bit codes of one channel's 64-element chunk -> 32 fp16 pairs (element 2c, 2c+1 in column c).
+// One branch-free path for INT8-sym, INT8-asym and MXINT8: 0x64XX as fp16 is 1024 + XX.
+CHAM_DEV void decode_w8(const uint32_t (&w)[16], const ChanDecode& c, uint32_t e8, uint32_t (&out)[32]) {
+  uint32_t f1[2], f2[2];
+  chunk_factors(c, e8, f1, f2);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const uint32_t v = w[i] ^ c.flip;
+    const int b = i >> 3;
+    out[2 * i] = hmul2u(hsub2u(__byte_perm(v, 0x64646464u, 0x4140), c.sub), f1[b]);
+    out[2 * i + 1] = hmul2u(hsub2u(__byte_perm(v, 0x64646464u, 0x4342), c.sub), f1[b]);
+  }
+  // the second factor is 1 unless a block's scale is below 2^-14 (tiny MX blocks): skip it when
+  // no lane of the warp needs it
+  if (!__all_sync(0xffffffffu, f2[0] == 0x3C003C00u && f2[1] == 0x3C003C00u)) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) out[i] = hmul2u(out[i], f2[i >> 4]);
+  }
+}
+
+// 4-bit codes -> 32 fp16 pairs.  Word i holds elements 8i..8i+7 with nibble j = element 2j and
+// nibble 4+j = element 2j+1, so (x >> 4j) & 0x000F000F isolates a pair.
+CHAM_DEV void decode_w4(const uint32_t (&w)[8], const ChanDecode& c, uint32_t e8, const uint32_t* lut,
                         uint32_t (&out)[32]) {
-  if (f == CHAM_W_NF4) {
+  uint32_t f1[2], f2[2];
+  chunk_factors(c, e8, f1, f2);
+  if (c.f == CHAM_W_NF4) {
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) out[4 * i + j] = lut[((w[i] >> (4 * j)) & 0xFu) | ((w[i] >> (4 * j + 12)) & 0xF0u)];
-    return;
-  }
-  if (f == CHAM_W_E2M1 || f == CHAM_W_MXFP4) {
+  } else if (c.f == CHAM_W_E2M1 || c.f == CHAM_W_MXFP4) {
     // E2M1 s.e1e0.m placed at fp16 bits 15 and 11..9 is value * 2^-14: multiply back by 2^14
-    const __half2 k = __float2half2_rn(16384.f);
-    const float up0 = exp2i_clamped(static_cast<int>(e8 & 0xFFu) - 127);
-    const float up1 = exp2i_clamped(static_cast<int>((e8 >> 8) & 0xFFu) - 127);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < 8; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const uint32_t x = w[i] >> (4 * j);
         const uint32_t bits = ((x & 0x00070007u) << 9) | ((x & 0x00080008u) << 12);
-        const __half2 h = __hmul2(u32_as_h2(bits), k);
-        if (f == CHAM_W_E2M1) {
-          out[4 * i + j] = h2_as_u32(h);
-        } else {
-          const float up = i < 4 ? up0 : up1;
-          const float2 v = __half22float2(h);
-          out[4 * i + j] = h2_as_u32(__floats2half2_rn(__fmul_rn(v.x, up), __fmul_rn(v.y, up)));
-        }
+        out[4 * i + j] = hmul2u(hmul2u(hmul2u(bits, 0x74007400u), f1[i >> 2]), f2[i >> 2]);
       }
-    }
-    return;
-  }
-  // INT4-sym, INT4-asym, MXINT4: 0x640N as fp16 is 1024 + N
-  const bool sym = f != CHAM_W_INT4_ASYM;
-  const uint32_t flip = sym ? 0x88888888u : 0u;
-  const __half2 sub = __float2half2_rn(sym ? 1032.f : 1024.f + static_cast<float>(z));
-  const float up0 = exp2i_clamped(static_cast<int>(e8 & 0xFFu) - 127 - 2);
-  const float up1 = exp2i_clamped(static_cast<int>((e8 >> 8) & 0xFFu) - 127 - 2);
+  } else {
+    // INT4-sym, INT4-asym, MXINT4: 0x640N as fp16 is 1024 + N
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint32_t v = w[i] ^ flip;
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t v = w[i] ^ c.flip;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const __half2 h = __hsub2(u32_as_h2(((v >> (4 * j)) & 0x000F000Fu) | 0x64006400u), sub);
-      if (f != CHAM_W_MXINT4) {
-        out[4 * i + j] = h2_as_u32(h);
-      } else {
-        const float up = i < 4 ? up0 : up1;
-        const float2 q = __half22float2(h);
-        out[4 * i + j] = h2_as_u32(__floats2half2_rn(__fmul_rn(q.x, up), __fmul_rn(q.y, up)));
-      }
+      for (int j = 0; j < 4; ++j)
+        out[4 * i + j] =
+            hmul2u(hmul2u(hsub2u(((v >> (4 * j)) & 0x000F000Fu) | 0x64006400u, c.sub), f1[i >> 2]), f2[i >> 2]);
     }
   }
 }
@@ -150,46 +192,42 @@ CHAM_DEV void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)[16]) {
       : "memory");
 }
 
-template <int BITS>
-CHAM_DEV void load_raw(const uint8_t* chunk_base, uint32_t (&raw)[16]) {
-  // slab j of a chunk holds bytes [16j, 16j+16) of all 128 channels, 2048 bytes apart
-#pragma unroll
-  for (int j = 0; j < BITS / 2; ++j) {
-    const uint4 u = __ldg(reinterpret_cast<const uint4*>(chunk_base + j * 2048));
-    raw[4 * j] = u.x;
-    raw[4 * j + 1] = u.y;
-    raw[4 * j + 2] = u.z;
-    raw[4 * j + 3] = u.w;
-  }
-}
-
 template <int BN, int BITS>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm_ts_f16(const __grid_constant__ CUtensorMap act_map, const GemmArgs a) {
-  using C = GemmCfg<BN>;
+  using C = GemmCfg<BN, BITS>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sB = smem;
   uint32_t* lut = reinterpret_cast<uint32_t*>(smem + C::kData);
-  uint64_t* full_b = reinterpret_cast<uint64_t*>(lut + 256);
-  uint64_t* full_a = full_b + kStages;
-  uint64_t* empty = full_a + kStages;
-  uint64_t* accum = empty + kStages;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  constexpr int S = C::kStages;
+  constexpr int kAStages = C::kAStages, kGroup = C::kGroup, kAGroups = kAStages / kGroup;
+  uint64_t* full = reinterpret_cast<uint64_t*>(lut + 256);  // [S] producer -> decoders, MMA (tx bytes)
+  uint64_t* empty = full + S;                                // [S] MMA commit -> producer
+  uint64_t* afull = empty + S;                               // [kAGroups] decode warps -> MMA
+  uint64_t* aempty = afull + kAStages;                       // [kAStages] MMA commit -> decoders
+  uint64_t* accfull = aempty + kAStages;                     // [2] MMA commit -> epilogue
+  uint64_t* accempty = accfull + 2;                          // [2] epilogue warps (4) -> MMA
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tile = a.tile0 + blockIdx.x;
-  const int tok0 = blockIdx.y * BN;
   const int nk = a.n_chunks;
+  const int n_ch = a.n_ch_tiles;
+  const int n_tiles = n_ch * ((a.M + BN - 1) / BN);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&full_b[s], 1);
-      mbar_init(&full_a[s], 128);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(accum, 1);
+    for (int s = 0; s < kAStages; ++s) {
+      if (s < kAGroups) mbar_init(&afull[s], 4 * kGroup);  // one elected lane per warp and chunk
+      mbar_init(&aempty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accfull[b], 1);
+      mbar_init(&accempty[b], 4);  // one elected lane per epilogue warp
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -201,102 +239,156 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t d_tmem = tmem;               // columns [0, BN)
-  const uint32_t a_tmem = tmem + C::kACol;    // stage s at columns kACol + 32 s
 
   if (warp == 0) {
-    // ---------------- TMA producer: activation tiles
+    // ---------------- producer: activation tile (TMA), raw weight codes and E8M0 bytes (bulk)
     if (lane == 0) {
-      int issued = 0;
-      for (int kc = 0; kc < nk; ++kc) {
-        const int s = kc % kStages;
-        const uint32_t ph = (kc / kStages) & 1;
-        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, a.dev_status)) break;
-        mbar_arrive_expect_tx(&full_b[s], C::kBStage);
-        tma_load_2d(smem_u32(sB + s * C::kBStage), &act_map, &full_b[s], kc * kBK, tok0);
-        issued = kc + 1;
+      uint32_t it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+        const int ch = a.tile0 + t % n_ch, tok0 = (t / n_ch) * BN;
+        for (int kc = 0; kc < nk; ++kc, ++it) {
+          const int s = it % S;
+          const uint32_t ph = (it / S) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, a.dev_status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + s * C::kStage;
+          const size_t chunk = static_cast<size_t>(ch) * nk + kc;
+          mbar_arrive_expect_tx(&full[s], C::kBBytes + C::kWBytes + C::kEBytes);
+          tma_load_2d(smem_u32(st), &act_map, &full[s], kc * kBK, tok0);
+          bulk_load(smem_u32(st + C::kBBytes), a.codes + chunk * C::kWBytes, C::kWBytes, &full[s]);
+          bulk_load(smem_u32(st + C::kBBytes + C::kWBytes), a.we8m0 + chunk * C::kEBytes, C::kEBytes, &full[s]);
+        }
       }
-      for (int kc = issued > kStages ? issued - kStages : 0; kc < issued; ++kc)
-        drain_wait(&full_b[kc % kStages], (kc / kStages) & 1);
+      // every issued copy must have landed before the CTA may exit
+      const uint32_t first = it > S ? it - S : 0;
+      for (uint32_t j = first; j < it; ++j) drain_wait(&full[j % S], (j / S) & 1);
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16(128, BN);
-      for (int kc = 0; kc < nk; ++kc) {
-        const int s = kc % kStages;
-        const uint32_t ph = (kc / kStages) & 1;
-        if (!mbar_wait(&full_b[s], ph, abort_flag, a.dev_status)) break;
-        if (!mbar_wait(&full_a[s], ph, abort_flag, a.dev_status)) break;
+      uint32_t it = 0, acc_it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++acc_it) {
+        const int b = acc_it & 1;
+        if (!mbar_wait(&accempty[b], ((acc_it >> 1) & 1) ^ 1, abort_flag, a.dev_status)) break;
         tc_fence_after();
-        const uint32_t b0 = smem_u32(sB + s * C::kBStage);
+        const uint32_t d_tmem = tmem + b * C::kAccCols;
+        // One wait per group of kGroup consecutive K-chunks: every stall of this thread drains the
+        // tensor pipe's short instruction queue, so waits are amortised over 4 * kGroup MMAs.  Only
+        // the decoded-operand barrier is waited on: the decoders arrive on it after they have
+        // themselves observed the stage's TMA barrier, so the activation tile has landed too.  A
+        // group may straddle two tiles; its wait then also covers the next tile's first chunks.
+        for (int kc = 0; kc < nk; ++kc, ++it) {
+          if (it % kGroup == 0) {
+            if (!mbar_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+          }
+          const int s = it % S, sa = it % kAStages;
+          const uint32_t b0 = smem_u32(smem + s * C::kStage);
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk)
-          mma_f16_ts(d_tmem, a_tmem + s * 32 + kk * 8, smem_desc_sw128(b0 + kk * 32), idesc, (kc | kk) != 0);
-        mma_commit(&empty[s]);
+          for (int kk = 0; kk < kBK / 16; ++kk)
+            mma_f16_ts(d_tmem, tmem + C::kACol + sa * 32 + kk * 8, smem_desc_sw128(b0 + kk * 32), idesc,
+                       (kc | kk) != 0);
+          mma_commit(&empty[s]);
+          mma_commit(&aempty[sa]);
+        }
+        mma_commit(&accfull[b]);
       }
-      mma_commit(accum);
-      drain_wait(accum, 0);  // all issued MMAs have finished before tensor memory is released
+      // all issued MMAs have finished before tensor memory is released
+      if (acc_it > 0) drain_wait(&accfull[(acc_it - 1) & 1], ((acc_it - 1) >> 1) & 1);
     }
-  } else if (warp >= 4) {
-    // ---------------- weight decode (one channel per thread), then the epilogue
-    const int q = warp - 4;  // tensor-memory lane quadrant of this warp
+  } else if (warp >= 4 && warp < 4 + 4 * kDecodeGroups) {
+    // ---------------- weight decode: one channel per thread; group g takes chunks it % G == g
+    const int q = warp & 3;  // tensor-memory lane quadrant of this warp (warp % 4)
+    const int grp = (warp - 4) >> 2;
     const int r = q * 32 + lane;
-    const int p = tile * 128 + r;
-    const int f = a.wfmt[p];
-    const int z = a.wzero[p];
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    constexpr int kChunkBytes = BITS == 8 ? 8192 : 4096;
-    const uint8_t* cbase = a.codes + static_cast<size_t>(tile) * nk * kChunkBytes + r * 16;
-    const uint16_t* e8base = reinterpret_cast<const uint16_t*>(a.we8m0) + static_cast<size_t>(tile) * nk * 128 + r;
-    uint32_t raw[16];
-    load_raw<BITS>(cbase, raw);
-    uint32_t e8 = e8base[0];
+    uint32_t it = 0;
     bool ok = true;
-    for (int kc = 0; kc < nk; ++kc) {
-      const int s = kc % kStages;
-      const uint32_t ph = (kc / kStages) & 1;
-      uint32_t out[32];
-      if constexpr (BITS == 8) {
-        decode_w8(raw, f, z, e8, out);
-      } else {
-        const uint32_t (&r8)[8] = *reinterpret_cast<const uint32_t(*)[8]>(&raw[0]);
-        decode_w4(r8, f, z, e8, lut, out);
+    // chunks this CTA processes; the last one also arrives for the missing chunks of its group
+    const uint32_t total = static_cast<uint32_t>((n_tiles - static_cast<int>(blockIdx.x) + gridDim.x - 1) / gridDim.x) * nk;
+    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      const int p = (a.tile0 + t % n_ch) * 128 + r;
+      const ChanDecode cd = chan_decode(a.wfmt[p], a.wzero[p]);
+      for (int kc = 0; kc < nk; ++kc, ++it) {
+        if (static_cast<int>(it % kDecodeGroups) != grp) continue;
+        const int s = it % S, sa = it % kAStages;
+        const uint32_t ph = (it / S) & 1, pa = (it / kAStages) & 1;
+        if (!warp_wait(&full[s], ph, abort_flag, a.dev_status) ||
+            !warp_wait(&aempty[sa], pa ^ 1, abort_flag, a.dev_status)) {
+          ok = false;
+          break;
+        }
+        const uint8_t* st = smem + s * C::kStage;
+        const uint32_t e8 = reinterpret_cast<const uint16_t*>(st + C::kBBytes + C::kWBytes)[r];
+        uint32_t raw[16];
+#pragma unroll
+        for (int j = 0; j < BITS / 2; ++j) {  // slab j: bytes [16j, 16j+16) of every channel
+          const uint4 u = *reinterpret_cast<const uint4*>(st + C::kBBytes + j * 2048 + r * 16);
+          raw[4 * j] = u.x;
+          raw[4 * j + 1] = u.y;
+          raw[4 * j + 2] = u.z;
+          raw[4 * j + 3] = u.w;
+        }
+        uint32_t out[32];
+        if constexpr (BITS == 8) {
+          decode_w8(raw, cd, e8, out);
+        } else {
+          const uint32_t (&r8)[8] = *reinterpret_cast<const uint32_t(*)[8]>(&raw[0]);
+          decode_w4(r8, cd, e8, lut, out);
+        }
+        tc_fence_after();
+        tmem_st_32x32b_x32(tmem + C::kACol + lane_off + sa * 32, out);
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();  // 128 separate arrivals on one barrier word serialise: one per warp
+        if (lane == 0) {
+          const int missing = it + 1 == total ? kGroup - 1 - static_cast<int>(it % kGroup) : 0;
+          for (int m = 0; m <= missing; ++m) mbar_arrive(&afull[(it / kGroup) % kAGroups]);
+        }
       }
-      if (kc + 1 < nk) {
-        load_raw<BITS>(cbase + static_cast<size_t>(kc + 1) * kChunkBytes, raw);
-        e8 = e8base[static_cast<size_t>(kc + 1) * 128];
-      }
-      if (!warp_wait(&empty[s], ph ^ 1, abort_flag, a.dev_status)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      tmem_st_32x32b_x32(a_tmem + lane_off + s * 32, out);
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(&full_a[s]);
     }
-    if (ok && warp_wait(accum, 0, abort_flag, a.dev_status)) {
+  } else if (warp >= 4 + 4 * kDecodeGroups) {
+    // ---------------- epilogue: drain one accumulator buffer per tile
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const float sa = a.act_scale != nullptr ? *a.act_scale : 1.f;
+    uint32_t acc_it = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++acc_it) {
+      const int b = acc_it & 1;
+      if (!warp_wait(&accfull[b], (acc_it >> 1) & 1, abort_flag, a.dev_status)) break;
       tc_fence_after();
+      const int p = (a.tile0 + t % n_ch) * 128 + r;
+      const int tok0 = (t / n_ch) * BN;
       const int orig = a.perm[p];
-      const float sa = a.act_scale != nullptr ? *a.act_scale : 1.f;
       const float scale = __fmul_rn(sa, a.wscale[p]);
-      const float b = (a.bias != nullptr && orig >= 0) ? a.bias[orig] : 0.f;
+      const float bv = (a.bias != nullptr && orig >= 0) ? a.bias[orig] : 0.f;
       float* yc = a.Y + (orig >= 0 ? orig : 0);
+      const uint32_t d_tmem = tmem + b * C::kAccCols + lane_off;
 #pragma unroll 1
       for (int j = 0; j < BN / 16; ++j) {
         uint32_t v[16];
-        tmem_ld_32x32b_x16(d_tmem + lane_off + j * 16, v);
+        tmem_ld_32x32b_x16(d_tmem + j * 16, v);
         tmem_wait_ld();
         if (orig >= 0) {
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             const int tok = tok0 + j * 16 + i;
-            if (tok < a.M) yc[static_cast<size_t>(tok) * a.N] = fmaf(__uint_as_float(v[i]), scale, b);
+            if (tok < a.M) yc[static_cast<size_t>(tok) * a.N] = fmaf(__uint_as_float(v[i]), scale, bv);
           }
         }
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&accempty[b]);
     }
   }
   tc_fence_before();
@@ -308,18 +400,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 }
 
 int gemm_pick_bn(int M, int n_tiles, int num_sms) {
+  (void)n_tiles;
+  (void)num_sms;
   if (M <= 16) return 16;
   if (M <= 32) return 32;
   if (M <= 64) return 64;
   if (M <= 128) return 128;
-  const long ctas256 = static_cast<long>(n_tiles) * ((M + 255) / 256);
-  return ctas256 >= num_sms ? 256 : 128;
+  return 192;
 }
 
 template <int BN, int BITS>
-static cudaError_t launch_bn(const CUtensorMap& map, const GemmArgs& a, int n_tiles, cudaStream_t st) {
-  using C = GemmCfg<BN>;
-  static int configured_device = -1;  // attribute is per device; re-set when the device changes
+static cudaError_t launch_bn(const CUtensorMap& map, const GemmArgs& a, int num_sms, cudaStream_t st) {
+  using C = GemmCfg<BN, BITS>;
+  static int configured_device = -1;  // the attribute is per device; set again when it changes
   int dev = 0;
   cudaGetDevice(&dev);
   if (configured_device != dev) {
@@ -328,27 +421,28 @@ static cudaError_t launch_bn(const CUtensorMap& map, const GemmArgs& a, int n_ti
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
-  const dim3 grid(n_tiles, (a.M + BN - 1) / BN);
+  const long tiles = static_cast<long>(a.n_ch_tiles) * ((a.M + BN - 1) / BN);
+  const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
   k_gemm_ts_f16<BN, BITS><<<grid, kGemmThreads, C::kSmem, st>>>(map, a);
   return cudaGetLastError();
 }
 
-cudaError_t launch_gemm_f16(const CUtensorMap& map, const GemmArgs& a, int n_tiles, int bn, cudaStream_t st) {
+cudaError_t launch_gemm_f16(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
   if (a.bits == 8) {
     switch (bn) {
-      case 16: return launch_bn<16, 8>(map, a, n_tiles, st);
-      case 32: return launch_bn<32, 8>(map, a, n_tiles, st);
-      case 64: return launch_bn<64, 8>(map, a, n_tiles, st);
-      case 128: return launch_bn<128, 8>(map, a, n_tiles, st);
-      default: return launch_bn<256, 8>(map, a, n_tiles, st);
+      case 16: return launch_bn<16, 8>(map, a, num_sms, st);
+      case 32: return launch_bn<32, 8>(map, a, num_sms, st);
+      case 64: return launch_bn<64, 8>(map, a, num_sms, st);
+      case 128: return launch_bn<128, 8>(map, a, num_sms, st);
+      default: return launch_bn<192, 8>(map, a, num_sms, st);
     }
   }
   switch (bn) {
-    case 16: return launch_bn<16, 4>(map, a, n_tiles, st);
-    case 32: return launch_bn<32, 4>(map, a, n_tiles, st);
-    case 64: return launch_bn<64, 4>(map, a, n_tiles, st);
-    case 128: return launch_bn<128, 4>(map, a, n_tiles, st);
-    default: return launch_bn<256, 4>(map, a, n_tiles, st);
+    case 16: return launch_bn<16, 4>(map, a, num_sms, st);
+    case 32: return launch_bn<32, 4>(map, a, num_sms, st);
+    case 64: return launch_bn<64, 4>(map, a, num_sms, st);
+    case 128: return launch_bn<128, 4>(map, a, num_sms, st);
+    default: return launch_bn<192, 4>(map, a, num_sms, st);
   }
 }
 

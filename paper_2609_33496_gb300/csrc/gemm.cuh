@@ -19,13 +19,15 @@ struct GemmArgs {
   float* Y;                  // [M][N] fp32
   int M, N, n_chunks;        // n_chunks = Kp / 64
   int tile0;                 // first 128-channel tile of this launch
+  int n_ch_tiles;            // 128-channel tiles of this launch
   int bits;                  // 4 or 8
   int* dev_status;
   uint16_t nf4_level[16];    // NF4 levels as fp16 bit patterns
 };
 
-// Token-tile (MMA N) sizes the kernel is instantiated for.
+// Token-tile (MMA N) size for M tokens: 16, 32, 64, 128 or 192.
 int gemm_pick_bn(int M, int n_tiles, int num_sms);
-cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int n_tiles, int bn, cudaStream_t st);
+// Persistent launch: min(tiles, num_sms) CTAs walk the (channel tile, token tile) grid.
+cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
 
 }  // namespace cham

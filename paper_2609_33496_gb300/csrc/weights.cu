@@ -6,9 +6,9 @@
 // earlier palette member on ties (strict '<').  One CTA per channel: the row (at most 10 KB for
 // K = 5120) stays in L1 across the format passes.
 //
-// Pack: channels are permuted into format-homogeneous runs (Sec. 5: "same-format sub-GEMMs after
-// a channel permutation"), grouped by MMA class and padded to 128-channel tiles, and encoded in
-// the tiled layout the GEMM's decode warps read with coalesced 16-byte loads (include/chameleon.h).
+// Pack: channels are permuted (Sec. 5: "same-format sub-GEMMs after a channel permutation") into
+// the two MMA classes, each kept in original channel order and padded to 128-channel tiles, and
+// encoded in the tiled layout the GEMM reads with bulk copies (include/chameleon.h).
 #include "weights.cuh"
 
 namespace cham {
@@ -146,37 +146,40 @@ void launch_select(const __half* W, int N, int K, uint32_t mask, uint8_t* fmt_ou
 }
 
 // ------------------------------------------------------------------ a6: slot assignment
-// Packed slot of every channel: base[f] + (number of earlier channels with the same format).
-// One CTA walks the channels in chunks of 1024 with per-format warp ballots.
+// Packed slot of every channel: the first slot of its MMA class plus the number of earlier
+// channels of the same class (so each class keeps the original channel order, and a tile's Y
+// columns are contiguous).  One CTA walks the channels in chunks of 1024 with warp ballots.
 __global__ void __launch_bounds__(1024) k_w_slots(PackArgs a) {
-  __shared__ int warp_cnt[32][CHAM_W_NFORMATS];
-  __shared__ int running[CHAM_W_NFORMATS];
+  __shared__ int warp_cnt[32][2];
+  __shared__ int running[2];
   for (int p = threadIdx.x; p < a.n_packed; p += blockDim.x) {
     a.perm[p] = -1;
     a.fmtp[p] = 0xFF;
   }
-  if (threadIdx.x < CHAM_W_NFORMATS) running[threadIdx.x] = 0;
+  if (threadIdx.x < 2) running[threadIdx.x] = 0;
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int c0 = 0; c0 < a.N; c0 += blockDim.x) {
     const int c = c0 + threadIdx.x;
     const int f = c < a.N ? a.fmt_dev[c] : -1;
+    const bool valid = f >= 0 && f < CHAM_W_NFORMATS;
+    const int cls = valid ? w_class(f) : -1;
     int my_rank_in_warp = 0;
 #pragma unroll
-    for (int g = 0; g < CHAM_W_NFORMATS; ++g) {
-      const uint32_t m = __ballot_sync(0xffffffffu, f == g);
-      if (f == g) my_rank_in_warp = __popc(m & ((1u << lane) - 1u));
+    for (int g = 0; g < 2; ++g) {
+      const uint32_t m = __ballot_sync(0xffffffffu, cls == g);
+      if (cls == g) my_rank_in_warp = __popc(m & ((1u << lane) - 1u));
       if (lane == 0) warp_cnt[warp][g] = __popc(m);
     }
     __syncthreads();
     if (c < a.N) {
-      if (f < 0 || f >= CHAM_W_NFORMATS) {
+      if (!valid) {
         set_status(a.dev_status, CHAM_ERR_INVALID_ARG);
       } else {
-        int rank = running[f] + my_rank_in_warp;
-        for (int w = 0; w < warp; ++w) rank += warp_cnt[w][f];
-        if (rank < a.count[f]) {  // device formats must match the host plan
-          const int slot = a.base[f] + rank;
+        int rank = running[cls] + my_rank_in_warp;
+        for (int w = 0; w < warp; ++w) rank += warp_cnt[w][cls];
+        if (rank < a.cls_count[cls]) {  // device formats must match the host plan
+          const int slot = a.cls_base[cls] + rank;
           a.perm[slot] = c;
           a.fmtp[slot] = static_cast<uint8_t>(f);
         } else {
@@ -185,7 +188,7 @@ __global__ void __launch_bounds__(1024) k_w_slots(PackArgs a) {
       }
     }
     __syncthreads();
-    if (threadIdx.x < CHAM_W_NFORMATS) {
+    if (threadIdx.x < 2) {
       int t = 0;
       for (int w = 0; w < 32; ++w) t += warp_cnt[w][threadIdx.x];
       running[threadIdx.x] += t;

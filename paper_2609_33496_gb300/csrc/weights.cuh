@@ -133,19 +133,20 @@ CHAM_DEV int mx_exponent(int fmt, float amax) {
 // Encode one MX element given its block exponent; returns the code (two's complement byte /
 // nibble or E2M1 pattern) and the exact DQ value in fp32.
 CHAM_DEV int encode_mx(int fmt, float w, int X, float* dq) {
+  // an all-zero block has X = -127: its codes are 0 and its decode scale only needs to be finite
   const float v = __fmul_rn(w, exp2i_f32(-X));
   if (fmt == CHAM_W_MXINT8) {
     const int q = min(max(__float2int_rn(__fmul_rn(v, 64.f)), -127), 127);
-    *dq = __fmul_rn(static_cast<float>(q), exp2i_f32(X - 6));
+    *dq = __fmul_rn(static_cast<float>(q), exp2i_f32(max(X - 6, -126)));
     return q & 0xFF;
   }
   if (fmt == CHAM_W_MXINT4) {
     const int q = min(max(__float2int_rn(__fmul_rn(v, 4.f)), -7), 7);
-    *dq = __fmul_rn(static_cast<float>(q), exp2i_f32(X - 2));
+    *dq = __fmul_rn(static_cast<float>(q), exp2i_f32(max(X - 2, -126)));
     return q & 0xF;
   }
   const uint32_t n = cvt_e2m1x2(0.f, v) & 0xFu;
-  *dq = __fmul_rn(e2m1_value(n), exp2i_f32(X));
+  *dq = __fmul_rn(e2m1_value(n), exp2i_f32(max(X, -126)));
   return static_cast<int>(n);
 }
 
@@ -154,8 +155,8 @@ struct PackArgs {
   const uint8_t* fmt_dev;   // selected format of each original channel
   int N, K, Kp, bits, n_chunks;
   int n_packed;             // Np
-  int base[CHAM_W_NFORMATS];  // first packed slot of each format
-  int count[CHAM_W_NFORMATS];
+  int cls_base[2];          // first packed slot of each MMA class
+  int cls_count[2];         // channels of each class (from the host plan)
   uint8_t* codes;
   float* scale;
   uint8_t* zero;
