@@ -30,9 +30,11 @@ METRIC = "mixed-format linear TFLOP/s & % tensor peak; act-quant HBM GB/s"
 WORKLOAD = "SDXL-UNet attention/FFN projections, W8A8, batch 2 (CFG), 10 timestep buckets"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_BYTES = 126 * 2 ** 20
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of the dominant kernel from an ncu
-# capture (None until a capture of the current kernel exists)
-GEMM_TRAFFIC_PER_LAUNCH = None
+# dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant kernel, from an ncu
+# capture of the GEGLU-in projection (M 2048, K 1280, N 10240; profiles/gemm_ts_f16_sdxl_geglu_in.md).
+# Set to None whenever the kernel changes until it is captured again.
+GEMM_TRAFFIC_PER_LAUNCH = {"bytes": 44.22e6, "launch": "2048x1280x10240 (GEGLU-in)",
+                           "algorithmic_bytes": 99.8e6}
 
 
 def peaks():
@@ -311,6 +313,7 @@ def main():
         b = M * K + N * K + 5 * N + 4 * N + 4 * M * N
         t_roof += nb * max(layer_flops(M, K, N) / (peak_tensor * 1e12), b / (pk["hbm_gbs"] * 1e9))
     clocks = clk.summary()
+    probe = tensor_probe(torch, device)
 
     result = {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
@@ -333,6 +336,8 @@ def main():
                      "roofline_time_frac": round(t_roof * K_ / (gemm_ms * 1e-3), 4),
                      "gemm_ms_per_step": round(gemm_ms / K_, 4),
                      "gemm_launch_ms_mean": round(statistics.mean(gemm_launch_ms), 5),
+                     "probe_tflops": probe,
+                     "frac_of_probe_f16": round(gemm_tflops / probe["f16"], 4) if probe else None,
                      "timing": "CUDA-graph replay of the quantize+GEMM sequence, event nodes between kernels"
                                if graph is not None else "eager launches, events between kernels"},
         "act_quant": {"achieved_gbs": round(quant_gbs, 1), "peak_gbs": pk["hbm_gbs"],
@@ -439,6 +444,35 @@ def oracle_sample(layers_idx=(4,), buckets=(0, 9)):
     desc = "oracle select(W8)+act-quant+fp64 GEMM of layer(s) %s at buckets %s" % (
         [WL.SDXL_PROJ_LAYERS[i][0] for i in layers_idx], list(buckets))
     return flops, t, desc
+
+
+def tensor_probe(torch, device):
+    """Dense tcgen05 throughput this GPU sustains for the GEMM's instruction forms (the probe
+    library of the build): kind::f16 (fp16 operands, the W8A8 path) and kind::f8f6f4 (E4M3),
+    M = 128, N = 192, on seeded finite operands.  Returns TFLOP/s per kind."""
+    import ctypes
+    from paper_2609_33496_gb300 import build as B
+    L = ctypes.CDLL(B.PROBE_LIB)
+    L.chameleon_probe_mma.argtypes = [ctypes.c_int] * 4 + [ctypes.c_void_p] * 3
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    cyc = torch.zeros(1, dtype=torch.int64, device=device)
+    st = torch.zeros(1, dtype=torch.int32, device=device)
+    s = torch.cuda.current_stream()
+    out = {}
+    for kind, name, K in ((0, "f16", 16), (2, "f8f6f4", 32)):
+        iters, best = 4000, 0.0
+        for _ in range(3):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+            rc = L.chameleon_probe_mma(kind, 192, sms, iters, ctypes.c_void_p(cyc.data_ptr()),
+                                       ctypes.c_void_p(st.data_ptr()), ctypes.c_void_p(s.cuda_stream))
+            e1.record(s)
+            torch.cuda.synchronize()
+            if rc != 0 or int(st.item()) != 0:
+                return None
+            best = max(best, sms * iters * 4 * 2.0 * 128 * 192 * K / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+        out[name] = round(best, 1)
+    return out
 
 
 def cpu_baseline():
