@@ -2,9 +2,12 @@
 //
 // The dynamic path of Alg. 3: lo, hi = min x, max x over the tensor; ScaleZP (App. A.7); every
 // element encoded in the format the LUT picked.  Per-tensor formats need the range before any
-// element can be encoded, so they take two launches (range partials, then encode; the second
-// read of X mostly hits L2).  MX formats (32-element blocks along K, E8M0 exponent, Sec. 3.6 /
-// App. A.11) need only the block's own amax and run in one launch, four lanes per block.
+// element can be encoded, so they take two launches: range partials, then encode (the second
+// read of X mostly hits L2).  A single cooperative launch that stages X in shared memory across
+// a grid barrier was measured slower: the barrier costs as much as the load.
+// MX formats (32-element blocks along K, E8M0 exponent, Sec. 3.6 / App. A.11) need only the
+// block's own amax and run in one launch, four lanes per block.  Every kernel keeps several
+// 16-byte loads in flight per thread (HBM latency x bandwidth needs ~7 MB in flight).
 //
 // All scale arithmetic is IEEE fp32 with explicit round-to-nearest intrinsics (no contraction),
 // in the order of readings R4-R8: inv by one correctly rounded division, the product x * inv
@@ -14,64 +17,25 @@
 
 namespace cham {
 
-// ------------------------------------------------------------------ a2: range partials
-__global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, int64_t nvec,
-                                                  RangePartial* __restrict__ parts) {
-  __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
-  uint32_t nonfinite = 0;
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec; i += stride) {
-    const uint4 v = __ldg(X + i);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+constexpr int kUnroll = 4;  // independent 16-byte loads in flight per thread
+
+// min / max / non-finite flag of eight fp16 values packed in a uint4.
+CHAM_DEV void range8(const uint4& v, __half2& lo2, __half2& hi2, uint32_t& nonfinite) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      // exponent field all ones in either half: Inf or NaN
-      nonfinite |= (((w[j] & 0x7C00u) == 0x7C00u) | ((w[j] & 0x7C000000u) == 0x7C000000u));
-      const __half2 h = *reinterpret_cast<const __half2*>(&w[j]);
-      lo2 = __hmin2(lo2, h);
-      hi2 = __hmax2(hi2, h);
-    }
-  }
-  float lo = fminf(__low2float(lo2), __high2float(lo2));
-  float hi = fmaxf(__low2float(hi2), __high2float(hi2));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-    hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-    nonfinite |= __shfl_xor_sync(0xffffffffu, nonfinite, o);
-  }
-  __shared__ float s_lo[8], s_hi[8];
-  __shared__ uint32_t s_nf[8];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) {
-    s_lo[warp] = lo;
-    s_hi[warp] = hi;
-    s_nf[warp] = nonfinite;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int k = 1; k < static_cast<int>(blockDim.x >> 5); ++k) {
-      lo = fminf(lo, s_lo[k]);
-      hi = fmaxf(hi, s_hi[k]);
-      nonfinite |= s_nf[k];
-    }
-    parts[blockIdx.x] = RangePartial{lo, hi, static_cast<int>(nonfinite), 0};
+  for (int j = 0; j < 4; ++j) {
+    // exponent field all ones in either half: Inf or NaN
+    nonfinite |= (((w[j] & 0x7C00u) == 0x7C00u) | ((w[j] & 0x7C000000u) == 0x7C000000u));
+    const __half2 h = u32_as_h2(w[j]);
+    lo2 = __hmin2(lo2, h);
+    hi2 = __hmax2(hi2, h);
   }
 }
 
-// Reduce the range partials (identically in every CTA: min/max are exact and order-free) and
-// derive the per-tensor quantizer parameters.  Returns false for a non-finite tensor.
-__device__ bool tensor_params(const RangePartial* parts, int nparts, int fmt, TensorParams* out) {
+// CTA-wide reduction of (lo, hi, nonfinite); the result is valid in every thread.
+CHAM_DEV void block_range(float& lo, float& hi, uint32_t& nf) {
   __shared__ float s_lo[32], s_hi[32];
-  __shared__ int s_nf[32];
-  float lo = INFINITY, hi = -INFINITY;
-  int nf = 0;
-  for (int i = threadIdx.x; i < nparts; i += blockDim.x) {
-    const RangePartial p = parts[i];
-    lo = fminf(lo, p.lo);
-    hi = fmaxf(hi, p.hi);
-    nf |= p.nonfinite;
-  }
+  __shared__ uint32_t s_nf[32];
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
@@ -79,23 +43,28 @@ __device__ bool tensor_params(const RangePartial* parts, int nparts, int fmt, Te
     nf |= __shfl_xor_sync(0xffffffffu, nf, o);
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
   if (lane == 0) {
     s_lo[warp] = lo;
     s_hi[warp] = hi;
     s_nf[warp] = nf;
   }
   __syncthreads();
-  lo = INFINITY;
-  hi = -INFINITY;
-  nf = 0;
-  for (int k = 0; k < static_cast<int>(blockDim.x >> 5); ++k) {
+  lo = s_lo[0];
+  hi = s_hi[0];
+  nf = s_nf[0];
+  for (int k = 1; k < static_cast<int>(blockDim.x >> 5); ++k) {
     lo = fminf(lo, s_lo[k]);
     hi = fmaxf(hi, s_hi[k]);
     nf |= s_nf[k];
   }
+}
+
+// ScaleZP (App. A.7) of a per-tensor format from the tensor's range (readings R4-R8, R11).
+CHAM_DEV TensorParams scale_zp(int fmt, float lo, float hi) {
   TensorParams p;
   if (fmt == CHAM_A_INT8_ASYM) {
-    // ScaleZP: s = (hi - lo)/255, z = round(-lo/s), zero-inclusive range (R4), degenerate (R7)
+    // s = (hi - lo)/255, z = round(-lo/s), zero-inclusive range (R4), degenerate range (R7)
     const float lo_ = fminf(lo, 0.f), hi_ = fmaxf(hi, 0.f);
     const float d = __fsub_rn(hi_, lo_);
     if (d == 0.f) {
@@ -108,7 +77,7 @@ __device__ bool tensor_params(const RangePartial* parts, int nparts, int fmt, Te
       p.z = min(max(__float2int_rn(__fmul_rn(-lo_, p.inv)), 0), 255);
     }
   } else {
-    // FP8: s = amax / Fmax, inv = Fmax / amax (App. A.7, R11)
+    // FP8: s = amax / Fmax, inv = Fmax / amax
     const float fmax = (fmt == CHAM_A_E4M3) ? 448.f : 57344.f;
     const float amax = fmaxf(fabsf(lo), fabsf(hi));
     if (amax == 0.f) {
@@ -120,57 +89,112 @@ __device__ bool tensor_params(const RangePartial* parts, int nparts, int fmt, Te
     }
     p.z = 0;
   }
-  *out = p;
-  return nf == 0;
+  return p;
+}
+
+// Reduce `nparts` range partials (identically in every CTA: min/max are exact and order-free).
+CHAM_DEV void reduce_partials(const RangePartial* parts, int nparts, float& lo, float& hi, uint32_t& nf) {
+  lo = INFINITY;
+  hi = -INFINITY;
+  nf = 0;
+  for (int i = threadIdx.x; i < nparts; i += blockDim.x) {
+    const RangePartial p = parts[i];
+    lo = fminf(lo, p.lo);
+    hi = fmaxf(hi, p.hi);
+    nf |= static_cast<uint32_t>(p.nonfinite);
+  }
+  block_range(lo, hi, nf);
+}
+
+// Eight elements of a per-tensor format: code bytes (element 0 in the low byte) and the exact
+// fp16 operand values (q - z for INT8-asym, value(code) for FP8; the scale s stays outside).
+template <int FMT, bool DEQ>
+CHAM_DEV void encode8_tensor(const uint4& v, const TensorParams& p, uint2& code, uint4& deq) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t c[2] = {0, 0};
+  uint32_t d[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 f = __half22float2(u32_as_h2(w[j]));
+    const float a = __fmul_rn(f.x, p.inv), b = __fmul_rn(f.y, p.inv);
+    uint32_t pair;
+    if constexpr (FMT == CHAM_A_INT8_ASYM) {
+      const int qa = min(max(__float2int_rn(a) + p.z, 0), 255);
+      const int qb = min(max(__float2int_rn(b) + p.z, 0), 255);
+      pair = static_cast<uint32_t>(qa) | (static_cast<uint32_t>(qb) << 8);
+      if constexpr (DEQ) d[j] = h2_as_u32(__halves2half2(__int2half_rn(qa - p.z), __int2half_rn(qb - p.z)));
+    } else if constexpr (FMT == CHAM_A_E4M3) {
+      const uint16_t e = cvt_e4m3x2(b, a);
+      pair = e;
+      if constexpr (DEQ) d[j] = cvt_e4m3x2_to_f16x2(e);
+    } else {
+      const uint16_t e = cvt_e5m2x2(b, a);
+      pair = e;
+      if constexpr (DEQ) d[j] = cvt_e5m2x2_to_f16x2(e);
+    }
+    c[j >> 1] |= pair << (16 * (j & 1));
+  }
+  code = make_uint2(c[0], c[1]);
+  deq = make_uint4(d[0], d[1], d[2], d[3]);
+}
+
+// ------------------------------------------------------------------ a2: range partials
+__global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, int64_t nvec,
+                                                  RangePartial* __restrict__ parts) {
+  __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
+  uint32_t nonfinite = 0;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec; i0 += stride * kUnroll) {
+    uint4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = i0 + u * stride;
+      v[u] = i < nvec ? __ldg(X + i) : make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u)
+      if (i0 + u * stride < nvec) range8(v[u], lo2, hi2, nonfinite);
+  }
+  float lo = fminf(__low2float(lo2), __high2float(lo2));
+  float hi = fmaxf(__low2float(hi2), __high2float(hi2));
+  block_range(lo, hi, nonfinite);
+  if (threadIdx.x == 0) parts[blockIdx.x] = RangePartial{lo, hi, static_cast<int>(nonfinite), 0};
 }
 
 // ------------------------------------------------------------------ a3: per-tensor encode
-// Eight elements per thread per iteration (one 16-byte load): eight code bytes and/or eight exact
-// fp16 operand values (q - z for INT8-asym, value(code) for FP8; the scale s stays outside).
 template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_tensor(const uint4* __restrict__ X, int64_t nvec, const RangePartial* __restrict__ parts,
                         int nparts, uint2* __restrict__ codes, uint4* __restrict__ deq,
                         cham_qparams* __restrict__ params, float* __restrict__ scale_out, int* dev_status) {
-  TensorParams p;
-  const bool finite = tensor_params(parts, nparts, FMT, &p);
+  float lo, hi;
+  uint32_t nf;
+  reduce_partials(parts, nparts, lo, hi, nf);
+  const TensorParams p = scale_zp(FMT, lo, hi);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     if (params != nullptr) *params = cham_qparams{p.s, p.z, p.inv, FMT};
     if (scale_out != nullptr) *scale_out = p.s;
-    if (!finite) set_status(dev_status, CHAM_ERR_NONFINITE);
+    if (nf) set_status(dev_status, CHAM_ERR_NONFINITE);
   }
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nvec; i += stride) {
-    const uint4 v = __ldg(X + i);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-    uint32_t c[2] = {0, 0};
-    uint32_t d[4];
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec; i0 += stride * kUnroll) {
+    uint4 v[kUnroll];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
-      const float a = __fmul_rn(f.x, p.inv), b = __fmul_rn(f.y, p.inv);
-      uint32_t pair;  // two code bytes, element 2j in the low byte
-      if constexpr (FMT == CHAM_A_INT8_ASYM) {
-        const int qa = min(max(__float2int_rn(a) + p.z, 0), 255);
-        const int qb = min(max(__float2int_rn(b) + p.z, 0), 255);
-        pair = static_cast<uint32_t>(qa) | (static_cast<uint32_t>(qb) << 8);
-        if constexpr (DEQ) {
-          const __half2 h = __halves2half2(__int2half_rn(qa - p.z), __int2half_rn(qb - p.z));
-          d[j] = *reinterpret_cast<const uint32_t*>(&h);
-        }
-      } else if constexpr (FMT == CHAM_A_E4M3) {
-        const uint16_t e = cvt_e4m3x2(b, a);
-        pair = e;
-        if constexpr (DEQ) d[j] = cvt_e4m3x2_to_f16x2(e);
-      } else {
-        const uint16_t e = cvt_e5m2x2(b, a);
-        pair = e;
-        if constexpr (DEQ) d[j] = cvt_e5m2x2_to_f16x2(e);
-      }
-      c[j >> 1] |= pair << (16 * (j & 1));
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = i0 + u * stride;
+      v[u] = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
     }
-    if constexpr (CODES) codes[i] = make_uint2(c[0], c[1]);
-    if constexpr (DEQ) deq[i] = make_uint4(d[0], d[1], d[2], d[3]);
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = i0 + u * stride;
+      if (i < nvec) {
+        uint2 c;
+        uint4 d;
+        encode8_tensor<FMT, DEQ>(v[u], p, c, d);
+        if constexpr (CODES) codes[i] = c;
+        if constexpr (DEQ) deq[i] = d;
+      }
+    }
   }
 }
 
@@ -178,75 +202,93 @@ __global__ void __launch_bounds__(256)
 // Four consecutive lanes own one 32-element block (8 elements each).  Shared exponent
 // X = floor(log2 amax) - emax_elem (R1; 8 for the E4M3 body, 0 for the int8 body), element
 // v = x * 2^-X (exact), body code; all-zero block -> E8M0 byte 0 (R2).
+template <int FMT, bool DEQ>
+CHAM_DEV void encode8_mx(const uint4& v, int lane, uint2& code, uint4& deq, int& byte_out, uint32_t& nonfinite) {
+  constexpr int kOff = (FMT == CHAM_A_MXFP8) ? 8 : 0;
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  float f[8];
+  float amax = 0.f;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    nonfinite |= (((w[j] & 0x7C00u) == 0x7C00u) | ((w[j] & 0x7C000000u) == 0x7C000000u));
+    const float2 t = __half22float2(u32_as_h2(w[j]));
+    f[2 * j] = t.x;
+    f[2 * j + 1] = t.y;
+    amax = fmaxf(amax, fmaxf(fabsf(t.x), fabsf(t.y)));
+  }
+  amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));  // 4 lanes = one 32-element block
+  amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 2));
+  int Xe, byte;
+  if (amax == 0.f) {
+    Xe = -127;
+    byte = 0;
+  } else {
+    Xe = floor_log2_f32(amax) - kOff;
+    byte = min(max(Xe + 127, 0), 254);
+    Xe = byte - 127;
+  }
+  const float down = exp2i_f32(-Xe);  // 2^-X, exact scaling
+  uint32_t c[2] = {0, 0};
+  uint32_t d[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float a = __fmul_rn(f[2 * j], down), b = __fmul_rn(f[2 * j + 1], down);
+    uint32_t pair;
+    if constexpr (FMT == CHAM_A_MXFP8) {
+      const uint16_t e = cvt_e4m3x2(b, a);
+      pair = e;
+      if constexpr (DEQ) {
+        const float2 val = __half22float2(u32_as_h2(cvt_e4m3x2_to_f16x2(e)));
+        const float up = exp2i_f32(Xe);
+        d[j] = h2_as_u32(__floats2half2_rn(__fmul_rn(val.x, up), __fmul_rn(val.y, up)));
+      }
+    } else {
+      const int qa = min(max(__float2int_rn(__fmul_rn(a, 64.f)), -127), 127);
+      const int qb = min(max(__float2int_rn(__fmul_rn(b, 64.f)), -127), 127);
+      pair = (static_cast<uint32_t>(qa) & 0xFFu) | ((static_cast<uint32_t>(qb) & 0xFFu) << 8);
+      if constexpr (DEQ) {
+        const float up = exp2i_f32(max(Xe - 6, -126));  // zero block (Xe = -127): codes are 0
+        d[j] = h2_as_u32(__floats2half2_rn(__fmul_rn(static_cast<float>(qa), up),
+                                           __fmul_rn(static_cast<float>(qb), up)));
+      }
+    }
+    c[j >> 1] |= pair << (16 * (j & 1));
+  }
+  code = make_uint2(c[0], c[1]);
+  deq = make_uint4(d[0], d[1], d[2], d[3]);
+  byte_out = byte;
+  (void)lane;
+}
+
 template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_mx(const uint4* __restrict__ X, int64_t nvec, uint2* __restrict__ codes, uint4* __restrict__ deq,
                     uint8_t* __restrict__ e8m0, cham_qparams* __restrict__ params, int* dev_status) {
-  constexpr int kOff = (FMT == CHAM_A_MXFP8) ? 8 : 0;
   if (blockIdx.x == 0 && threadIdx.x == 0 && params != nullptr) *params = cham_qparams{1.f, 0, 1.f, FMT};
   const int lane = threadIdx.x & 31;
   const int64_t warp_global = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const int64_t warps_total = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  const int64_t span = (static_cast<int64_t>(gridDim.x) * blockDim.x);  // vectors per unrolled step
   uint32_t nonfinite = 0;
-  for (int64_t base = warp_global * 32; base < nvec; base += warps_total * 32) {
-    const int64_t i = base + lane;
-    const bool active = i < nvec;  // nvec is a multiple of 4: a block's lanes agree
-    const uint4 v = active ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-    float f[8];
-    float amax = 0.f;
+  // lanes of a warp cover 32 consecutive vectors (8 blocks); every lane runs the same trip count
+  for (int64_t base = warp_global * 32; base < nvec; base += span * kUnroll) {
+    uint4 v[kUnroll];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      nonfinite |= (((w[j] & 0x7C00u) == 0x7C00u) | ((w[j] & 0x7C000000u) == 0x7C000000u));
-      const float2 t = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
-      f[2 * j] = t.x;
-      f[2 * j + 1] = t.y;
-      amax = fmaxf(amax, fmaxf(fabsf(t.x), fabsf(t.y)));
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = base + u * span + lane;
+      v[u] = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
     }
-    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 1));
-    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, 2));
-    int Xe, byte;
-    if (amax == 0.f) {
-      Xe = -127;
-      byte = 0;
-    } else {
-      Xe = floor_log2_f32(amax) - kOff;
-      byte = min(max(Xe + 127, 0), 254);
-      Xe = byte - 127;
-    }
-    const float down = exp2i_f32(-Xe);  // 2^-X, exact scaling
-    uint32_t c[2] = {0, 0};
-    uint32_t d[4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float a = __fmul_rn(f[2 * j], down), b = __fmul_rn(f[2 * j + 1], down);
-      uint32_t pair;
-      if constexpr (FMT == CHAM_A_MXFP8) {
-        const uint16_t e = cvt_e4m3x2(b, a);
-        pair = e;
-        if constexpr (DEQ) {
-          const float2 val = __half22float2(u32_as_h2(cvt_e4m3x2_to_f16x2(e)));
-          const float up = exp2i_f32(Xe);
-          const __half2 h = __floats2half2_rn(__fmul_rn(val.x, up), __fmul_rn(val.y, up));
-          d[j] = *reinterpret_cast<const uint32_t*>(&h);
-        }
-      } else {
-        const int qa = min(max(__float2int_rn(__fmul_rn(a, 64.f)), -127), 127);
-        const int qb = min(max(__float2int_rn(__fmul_rn(b, 64.f)), -127), 127);
-        pair = (static_cast<uint32_t>(qa) & 0xFFu) | ((static_cast<uint32_t>(qb) & 0xFFu) << 8);
-        if constexpr (DEQ) {
-          const float up = exp2i_f32(max(Xe - 6, -126));  // zero block (Xe = -127): codes are 0
-          const __half2 h = __floats2half2_rn(__fmul_rn(static_cast<float>(qa), up),
-                                              __fmul_rn(static_cast<float>(qb), up));
-          d[j] = *reinterpret_cast<const uint32_t*>(&h);
-        }
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = base + u * span + lane;  // nvec is a multiple of 4: a block's lanes agree
+      uint2 c;
+      uint4 d;
+      int byte;
+      encode8_mx<FMT, DEQ>(v[u], lane, c, d, byte, nonfinite);
+      if (i < nvec) {
+        if constexpr (CODES) codes[i] = c;
+        if constexpr (DEQ) deq[i] = d;
+        if (e8m0 != nullptr && (lane & 3) == 0) e8m0[i >> 2] = static_cast<uint8_t>(byte);
       }
-      c[j >> 1] |= pair << (16 * (j & 1));
-    }
-    if (active) {
-      if constexpr (CODES) codes[i] = make_uint2(c[0], c[1]);
-      if constexpr (DEQ) deq[i] = make_uint4(d[0], d[1], d[2], d[3]);
-      if (e8m0 != nullptr && (lane & 3) == 0) e8m0[i >> 2] = static_cast<uint8_t>(byte);
     }
   }
   if (nonfinite) set_status(dev_status, CHAM_ERR_NONFINITE);
@@ -263,7 +305,7 @@ __global__ void __launch_bounds__(256) k_act_moments(const uint4* __restrict__ X
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[j]));
+      const float2 f = __half22float2(u32_as_h2(w[j]));
       lo = fminf(lo, fminf(f.x, f.y));
       hi = fmaxf(hi, fmaxf(f.x, f.y));
       const double a = f.x, b = f.y;
@@ -295,20 +337,36 @@ __global__ void __launch_bounds__(256) k_act_moments(const uint4* __restrict__ X
     parts[blockIdx.x] = MomentPartial{{sh[0][0], sh[1][0], sh[2][0], sh[3][0]}, sl[0], shh[0]};
 }
 
-__global__ void k_act_moments_finish(const MomentPartial* __restrict__ parts, int nparts, int64_t count,
-                                     double* __restrict__ out) {
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+// Sum the partials in a fixed order: 256 threads each add a strided subset, then a fixed tree.
+__global__ void __launch_bounds__(256) k_act_moments_finish(const MomentPartial* __restrict__ parts, int nparts,
+                                                           int64_t count, double* __restrict__ out) {
+  __shared__ double sh[4][256];
+  __shared__ float sl[256], shh[256];
   double s[4] = {0, 0, 0, 0};
   float lo = INFINITY, hi = -INFINITY;
-  for (int i = 0; i < nparts; ++i) {
+  for (int i = threadIdx.x; i < nparts; i += blockDim.x) {
     for (int k = 0; k < 4; ++k) s[k] += parts[i].s[k];
     lo = fminf(lo, parts[i].lo);
     hi = fmaxf(hi, parts[i].hi);
   }
-  out[0] += static_cast<double>(count);
-  for (int k = 0; k < 4; ++k) out[1 + k] += s[k];
-  out[5] = fmin(out[5], static_cast<double>(lo));
-  out[6] = fmax(out[6], static_cast<double>(hi));
+  for (int k = 0; k < 4; ++k) sh[k][threadIdx.x] = s[k];
+  sl[threadIdx.x] = lo;
+  shh[threadIdx.x] = hi;
+  __syncthreads();
+  for (int o = blockDim.x / 2; o > 0; o >>= 1) {
+    if (threadIdx.x < o) {
+      for (int k = 0; k < 4; ++k) sh[k][threadIdx.x] += sh[k][threadIdx.x + o];
+      sl[threadIdx.x] = fminf(sl[threadIdx.x], sl[threadIdx.x + o]);
+      shh[threadIdx.x] = fmaxf(shh[threadIdx.x], shh[threadIdx.x + o]);
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    out[0] += static_cast<double>(count);
+    for (int k = 0; k < 4; ++k) out[1 + k] += sh[k][0];
+    out[5] = fmin(out[5], static_cast<double>(sl[0]));
+    out[6] = fmax(out[6], static_cast<double>(shh[0]));
+  }
 }
 
 // ------------------------------------------------------------------ host-side launchers
@@ -320,10 +378,12 @@ int range_grid(int64_t nvec, int num_sms) {
 
 template <int FMT, bool CODES, bool DEQ>
 static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
+  k_act_range<<<a.nparts, 256, 0, st>>>(a.X, a.nvec, a.parts);
   const int g = range_grid(a.nvec, a.num_sms);
   k_act_encode_tensor<FMT, CODES, DEQ><<<g, 256, 0, st>>>(a.X, a.nvec, a.parts, a.nparts, a.codes, a.deq,
                                                           a.params, a.scale_out, a.dev_status);
 }
+
 template <int FMT, bool CODES, bool DEQ>
 static void launch_mx(const ActQuantArgs& a, cudaStream_t st) {
   const int64_t warps = (a.nvec + 31) / 32;
@@ -348,8 +408,6 @@ static void dispatch(int fmt, const ActQuantArgs& a, cudaStream_t st) {
 }
 
 void launch_act_quant(int fmt, const ActQuantArgs& a, bool codes, bool deq, cudaStream_t st) {
-  const bool per_tensor = fmt <= CHAM_A_E5M2;
-  if (per_tensor) k_act_range<<<a.nparts, 256, 0, st>>>(a.X, a.nvec, a.parts);
   if (codes && deq) dispatch<true, true>(fmt, a, st);
   else if (codes) dispatch<true, false>(fmt, a, st);
   else dispatch<false, true>(fmt, a, st);
@@ -358,7 +416,7 @@ void launch_act_quant(int fmt, const ActQuantArgs& a, bool codes, bool deq, cuda
 void launch_act_moments(const uint4* X, int64_t nvec, int64_t count, MomentPartial* parts, int nparts,
                         double* out, cudaStream_t st) {
   k_act_moments<<<nparts, 256, 0, st>>>(X, nvec, parts);
-  k_act_moments_finish<<<1, 32, 0, st>>>(parts, nparts, count, out);
+  k_act_moments_finish<<<1, 256, 0, st>>>(parts, nparts, count, out);
 }
 
 }  // namespace cham

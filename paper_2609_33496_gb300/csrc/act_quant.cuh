@@ -25,8 +25,8 @@ struct MomentPartial {  // one CTA's power sums (Alg. 1 accumulator)
 struct ActQuantArgs {
   const uint4* X;          // fp16 tensor, 8 elements per vector
   int64_t nvec;            // M*K/8
-  RangePartial* parts;     // per-tensor formats: nparts partials (scratch)
-  int nparts;
+  RangePartial* parts;     // per-tensor formats: range partials (scratch)
+  int nparts;              // CTAs of the two-launch range kernel (range_grid)
   uint2* codes;            // 8 code bytes per vector, or null
   uint4* deq;              // 8 exact fp16 operand values per vector, or null
   uint8_t* e8m0;           // MX formats: one byte per 4 vectors, or null

@@ -314,9 +314,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     bool ok = true;
     // chunks this CTA processes; the last one also arrives for the missing chunks of its group
     const uint32_t total = static_cast<uint32_t>((n_tiles - static_cast<int>(blockIdx.x) + gridDim.x - 1) / gridDim.x) * nk;
+    // the channel's format and zero point for the next tile are loaded one tile ahead
+    int nf = 0, nz = 0;
+    if (static_cast<int>(blockIdx.x) < n_tiles) {
+      const int p0 = (a.tile0 + static_cast<int>(blockIdx.x) % n_ch) * 128 + r;
+      nf = a.wfmt[p0];
+      nz = a.wzero[p0];
+    }
     for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
-      const int p = (a.tile0 + t % n_ch) * 128 + r;
-      const ChanDecode cd = chan_decode(a.wfmt[p], a.wzero[p]);
+      const ChanDecode cd = chan_decode(nf, nz);
+      if (t + static_cast<int>(gridDim.x) < n_tiles) {
+        const int pn = (a.tile0 + (t + static_cast<int>(gridDim.x)) % n_ch) * 128 + r;
+        nf = a.wfmt[pn];
+        nz = a.wzero[pn];
+      }
       for (int kc = 0; kc < nk; ++kc, ++it) {
         if (static_cast<int>(it % kDecodeGroups) != grp) continue;
         const int s = it % S, sa = it % kAStages;
@@ -364,20 +375,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint32_t acc_it = 0;
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++acc_it) {
       const int b = acc_it & 1;
-      if (!warp_wait(&accfull[b], (acc_it >> 1) & 1, abort_flag, a.dev_status)) break;
-      tc_fence_after();
+      // per-channel constants first: their (dependent) loads overlap the wait for the accumulator
       const int p = (a.tile0 + t % n_ch) * 128 + r;
       const int tok0 = (t / n_ch) * BN;
       const int orig = a.perm[p];
       const float scale = __fmul_rn(sa, a.wscale[p]);
       const float bv = (a.bias != nullptr && orig >= 0) ? a.bias[orig] : 0.f;
+      if (!warp_wait(&accfull[b], (acc_it >> 1) & 1, abort_flag, a.dev_status)) break;
+      tc_fence_after();
       float* yc = a.Y + (orig >= 0 ? orig : 0);
       const uint32_t d_tmem = tmem + b * C::kAccCols + lane_off;
-#pragma unroll 1
-      for (int j = 0; j < BN / 16; ++j) {
-        uint32_t v[16];
-        tmem_ld_32x32b_x16(d_tmem + j * 16, v);
-        tmem_wait_ld();
+      // 16 token columns per tcgen05.ld; the load of the next 16 is in flight while the current
+      // ones are scaled and stored (a wait per load would serialise its latency 12 times per tile)
+      auto store16 = [&](const uint32_t (&v)[16], int j) {
         if (orig >= 0) {
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
@@ -385,6 +395,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (tok < a.M) yc[static_cast<size_t>(tok) * a.N] = fmaf(__uint_as_float(v[i]), scale, bv);
           }
         }
+      };
+      constexpr int kLoads = BN / 16;
+      uint32_t va[16], vb[16];
+      tmem_ld_32x32b_x16(d_tmem, va);
+      tmem_wait_ld();
+#pragma unroll 1
+      for (int j = 0; j < kLoads; j += 2) {
+        if (j + 1 < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + 1) * 16, vb);
+        store16(va, j);
+        tmem_wait_ld();
+        if (j + 2 < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + 2) * 16, va);
+        if (j + 1 < kLoads) store16(vb, j + 1);
+        tmem_wait_ld();
       }
       tc_fence_before();
       __syncwarp();
