@@ -151,11 +151,13 @@ cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_
  *   codes          per tile t (128 packed channels) and K-chunk c (64 elements): 128 * CB bytes,
  *                  CB = 64 (8-bit) or 32 (4-bit) bytes per channel, stored as CB/16 slabs of
  *                  128 x 16 bytes: slab j holds bytes [16j, 16j+16) of every channel's CB bytes.
- *                  8-bit: byte i = element i of the chunk (int8 two's complement for INT8-sym and
- *                  MXINT8, uint8 q for INT8-asym).  4-bit: each 32-bit word holds 8 elements
+ *                  8-bit: byte i = element i of the chunk (offset binary q + 128 for INT8-sym
+ *                  and MXINT8, uint8 q for INT8-asym).  4-bit: each 32-bit word holds 8 elements
  *                  e0..e7, nibble j (bits 4j..4j+3) = e_{2j} for j < 4 and e_{2(j-4)+1} for j >= 4;
- *                  INT4-sym/MXINT4 two's complement, INT4-asym q, NF4 level index, E2M1/MXFP4
- *                  bit pattern.  Elements k >= K are code 0.
+ *                  INT4-sym/MXINT4 offset binary q + 8, INT4-asym q, NF4 level index, E2M1/MXFP4
+ *                  bit pattern.  Elements k >= K hold the code of the value 0.  (Offset binary
+ *                  lets the GEMM turn a code into its fp16 value with one byte permute and one
+ *                  subtraction.)
  *   scale          float [Np]: per-channel scale s (1 for MX and padding)
  *   zero           uint8 [Np]: zero point z (asym formats, else 0)
  *   e8m0           uint8 [tiles][Kp/64][128][2]: the two E8M0 exponents of each channel's chunk

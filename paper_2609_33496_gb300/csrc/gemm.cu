@@ -16,9 +16,9 @@
 // The kernel is persistent: each CTA walks tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of
 // the (channel tile, token tile) grid.  Two rings over K-chunks of 64 couple the roles: a 6-8
 // stage shared-memory ring (activation tile + raw weight codes + their E8M0 bytes, filled by TMA
-// and bulk copies, deep enough to cover the load round trip) and a 4-slot tensor-memory ring of
-// decoded weight operands; one thread issues four kind::f16 MMAs (K = 16 each) per chunk, and
-// MMA commits free both slots.  Every wait is bounded (common.cuh); on a timeout
+// and bulk copies, deep enough to cover the load round trip) and a 4-8 slot tensor-memory ring of
+// decoded weight operands in two commit groups; one thread issues four kind::f16 MMAs (K = 16
+// each) per chunk and one commit per group, which frees the group's slots in both rings.  Every wait is bounded (common.cuh); on a timeout
 // the kernel records CHAM_ERR_TIMEOUT, drains its own copies and MMAs, releases tensor memory and
 // returns.
 #include "gemm.cuh"
@@ -41,21 +41,28 @@ struct GemmCfg {
   static constexpr int kData = kStages * kStage;
   static constexpr int kAccCols = (BN + 31) / 32 * 32;
   static constexpr int kACol = 2 * kAccCols;                      // first column of the A stages
-  // tensor-memory ring of decoded weight operands (32 columns per K-chunk) and the number of
-  // consecutive chunks one MMA-side wait covers: as many as the 512 columns allow next to the two
-  // accumulators (every wait of the MMA thread costs a few hundred cycles of drained pipe)
-  static constexpr int kAStages = (kACol + 8 * 32) <= 512 ? 8 : 4;
+  // Tensor-memory ring of decoded weight operands (32 columns per K-chunk), as deep as the 512
+  // columns allow next to the two accumulators, split into two commit groups of kGroup chunks.
+  // The MMA thread commits once per group, and that one barrier frees both the group's
+  // shared-memory stages and its tensor-memory stages: every commit another warp waits on costs
+  // the tensor pipe a fixed round trip of several hundred cycles, so it must cover many MMAs.
+  static constexpr int kAFit = (512 - kACol) / 32;
+  static constexpr int kAStages = (kAFit > 8 ? 8 : kAFit) / 2 * 2;
   static constexpr int kGroup = kAStages / 2;
+  static constexpr int kDone = 8;                                 // group-completion barriers
   static constexpr int kNeedCols = kACol + kAStages * 32;
   static constexpr int kTmemCols = kNeedCols <= 256 ? 256 : 512;
-  static constexpr int kMisc = 1024 /*NF4 pair table*/ + 8 * (2 * kStages + 2 * 8 + 4) + 16;
+  static constexpr int kMisc = 1024 /*NF4 pair table*/ + 8 * (kStages + kDone + 2 + 4) + 16;
   static constexpr int kNeed = 1024 /*alignment slack*/ + kData + kMisc;
   // at least 116 KiB so that two CTAs (and two tensor-memory allocations) never share an SM
   static constexpr int kSmem = kNeed > 116 * 1024 ? kNeed : 116 * 1024;
   static_assert(kStages >= 4, "ring depth");
   static_assert(kSmem <= 227 * 1024, "within the opt-in shared-memory limit");
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "MMA N for M = 128");
-  static_assert(kNeedCols <= 512, "tensor memory budget");
+  static_assert(kNeedCols <= 512 && kAStages >= 4, "tensor memory budget");
+  // a shared-memory stage is refilled only after the group holding its previous chunk completed;
+  // kDone barriers in rotation keep a waiter from missing a phase
+  static_assert(kDone * kGroup > kStages + kGroup, "group barrier rotation");
 };
 
 CHAM_DEV bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* st) {
@@ -101,84 +108,137 @@ CHAM_DEV uint32_t hmul2u(uint32_t a, uint32_t b) { return h2_as_u32(__hmul2(u32_
 // Per-channel decode constants.
 struct ChanDecode {
   int f;          // weight format
-  uint32_t flip;  // xor applied to the raw code word (two's complement -> biased)
-  uint32_t sub;   // half2 (1024 + offset) subtracted from the magic-number value
+  int off;        // stored code of the value 0: zero point (asym) or the offset-binary bias
   int e_off;      // MX: block exponent offset of the element scale (MXINT8 -6, MXINT4 -2, MXFP4 0)
+  bool mx;
 };
 
 CHAM_DEV ChanDecode chan_decode(int f, int z) {
   ChanDecode c;
   c.f = f;
   const bool asym = f == CHAM_W_INT8_ASYM || f == CHAM_W_INT4_ASYM;
-  const int off = asym ? z : (wbits(f) == 8 ? 128 : 8);
-  c.flip = asym ? 0u : (wbits(f) == 8 ? 0x80808080u : 0x88888888u);
-  const uint32_t h = h2_as_u32(__float2half2_rn(1024.f + static_cast<float>(off))) & 0xFFFFu;
-  c.sub = h | (h << 16);
+  c.off = asym ? z : (wbits(f) == 8 ? 128 : 8);
   c.e_off = f == CHAM_W_MXINT8 ? -6 : (f == CHAM_W_MXINT4 ? -2 : 0);
+  c.mx = w_is_mx(f);
   return c;
 }
 
-// Block scale factors of one chunk (two 32-element blocks); 1.0 for non-MX channels.
-CHAM_DEV void chunk_factors(const ChanDecode& c, uint32_t e8, uint32_t (&f1)[2], uint32_t (&f2)[2]) {
-  if (w_is_mx(c.f)) {
-    pow2_factors(static_cast<int>(e8 & 0xFFu) - 127 + c.e_off, f1[0], f2[0]);
-    pow2_factors(static_cast<int>((e8 >> 8) & 0xFFu) - 127 + c.e_off, f1[1], f2[1]);
-  } else {
-    f1[0] = f1[1] = f2[0] = f2[1] = 0x3C003C00u;  // 1.0
-  }
+// Element-scale exponent of block b (0 or 1) of a chunk: 0 for per-channel formats.
+CHAM_DEV int block_exp(const ChanDecode& c, uint32_t e8, int b) {
+  return c.mx ? static_cast<int>((e8 >> (8 * b)) & 0xFFu) - 127 + c.e_off : 0;
 }
 
+// Magic-number decode of integer codes.  An fp16 whose exponent field is E and whose low
+// mantissa bits hold the code u (shifted left by t bits) has the value 2^(E-25) * (1024 + u * 2^t);
+// subtracting the same construction with u = off leaves (u - off) * 2^(E-25+t) exactly (both
+// operands lie in one binade).  Choosing E = e + 25 - t puts the block's power-of-two element
+// scale 2^e into the same two instructions (PRMT or LOP3, then HSUB2), for every e that keeps E
+// in [1, 30].
+CHAM_DEV uint32_t dup16(uint32_t h) { return h | (h << 16); }
+
 // 8-bit codes of one channel's 64-element chunk -> 32 fp16 pairs (element 2c, 2c+1 in column c).
-// One branch-free path for INT8-sym, INT8-asym and MXINT8: 0x64XX as fp16 is 1024 + XX.
+// Called by whole warps (the vote below needs every lane).
 CHAM_DEV void decode_w8(const uint32_t (&w)[16], const ChanDecode& c, uint32_t e8, uint32_t (&out)[32]) {
-  uint32_t f1[2], f2[2];
-  chunk_factors(c, e8, f1, f2);
+  const int e0 = block_exp(c, e8, 0), e1 = block_exp(c, e8, 1);
+  // a block decodes on the fast path when its exponent fits; an all-zero MX block (E8M0 byte 0)
+  // decodes to zeros whatever exponent is used
+  const bool z0 = c.mx && (e8 & 0xFFu) == 0, z1 = c.mx && ((e8 >> 8) & 0xFFu) == 0;
+  const bool fast = (z0 || (e0 >= -24 && e0 <= 5)) && (z1 || (e1 >= -24 && e1 <= 5));
+  if (__all_sync(0xffffffffu, fast)) {
+    const int E0 = min(max(e0, -24), 5) + 25, E1 = min(max(e1, -24), 5) + 25;
+    const uint32_t hi[2] = {static_cast<uint32_t>(E0) << 2, static_cast<uint32_t>(E1) << 2};
+    const uint32_t sub[2] = {dup16((static_cast<uint32_t>(E0) << 10) | static_cast<uint32_t>(c.off)),
+                             dup16((static_cast<uint32_t>(E1) << 10) | static_cast<uint32_t>(c.off))};
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const uint32_t v = w[i] ^ c.flip;
-    const int b = i >> 3;
-    out[2 * i] = hmul2u(hsub2u(__byte_perm(v, 0x64646464u, 0x4140), c.sub), f1[b]);
-    out[2 * i + 1] = hmul2u(hsub2u(__byte_perm(v, 0x64646464u, 0x4342), c.sub), f1[b]);
-  }
-  // the second factor is 1 unless a block's scale is below 2^-14 (tiny MX blocks): skip it when
-  // no lane of the warp needs it
-  if (!__all_sync(0xffffffffu, f2[0] == 0x3C003C00u && f2[1] == 0x3C003C00u)) {
+    for (int i = 0; i < 16; ++i) {
+      const int b = i >> 3;
+      out[2 * i] = hsub2u(__byte_perm(w[i], hi[b], 0x4140), sub[b]);
+      out[2 * i + 1] = hsub2u(__byte_perm(w[i], hi[b], 0x4342), sub[b]);
+    }
+  } else {
+    // general path: unscaled integers, then the block scale as two exact power-of-two factors
+    uint32_t f1[2], f2[2];
+    pow2_factors(e0, f1[0], f2[0]);
+    pow2_factors(e1, f1[1], f2[1]);
+    const uint32_t sub = dup16((25u << 10) | static_cast<uint32_t>(c.off));
 #pragma unroll
-    for (int i = 0; i < 32; ++i) out[i] = hmul2u(out[i], f2[i >> 4]);
+    for (int i = 0; i < 16; ++i) {
+      const int b = i >> 3;
+      out[2 * i] = hmul2u(hmul2u(hsub2u(__byte_perm(w[i], 0x64u, 0x4140), sub), f1[b]), f2[b]);
+      out[2 * i + 1] = hmul2u(hmul2u(hsub2u(__byte_perm(w[i], 0x64u, 0x4342), sub), f1[b]), f2[b]);
+    }
   }
 }
 
 // 4-bit codes -> 32 fp16 pairs.  Word i holds elements 8i..8i+7 with nibble j = element 2j and
-// nibble 4+j = element 2j+1, so (x >> 4j) & 0x000F000F isolates a pair.
+// nibble 4+j = element 2j+1, so a mask of 0x000F000F << 4j isolates a pair.  The lanes of a warp
+// hold channels of different formats: every warp vote is taken before the per-format branches.
 CHAM_DEV void decode_w4(const uint32_t (&w)[8], const ChanDecode& c, uint32_t e8, const uint32_t* lut,
                         uint32_t (&out)[32]) {
+  const int e0 = block_exp(c, e8, 0), e1 = block_exp(c, e8, 1);
+  const bool is_nf4 = c.f == CHAM_W_NF4;
+  const bool is_fp4 = c.f == CHAM_W_E2M1 || c.f == CHAM_W_MXFP4;
+  // E2M1 s.e1e0.m placed at fp16 bits 15 and 11..9 is value * 2^-14: multiply back by 2^(14 + e);
+  // integer codes use the unscaled magic-number construction on the general path
   uint32_t f1[2], f2[2];
-  chunk_factors(c, e8, f1, f2);
-  if (c.f == CHAM_W_NF4) {
+  pow2_factors(is_fp4 ? e0 + 14 : e0, f1[0], f2[0]);
+  pow2_factors(is_fp4 ? e1 + 14 : e1, f1[1], f2[1]);
+  // INT4-sym, INT4-asym, MXINT4 fast path: nibble at bit 0 of a half uses E = e + 25, nibble at
+  // bit 4 uses E = e + 21, so both pairs of a byte need no shift; all-zero MX blocks decode to 0
+  const bool z0 = c.mx && (e8 & 0xFFu) == 0, z1 = c.mx && ((e8 >> 8) & 0xFFu) == 0;
+  const bool int_fast = (z0 || (e0 >= -20 && e0 <= 5)) && (z1 || (e1 >= -20 && e1 <= 5));
+  const bool fp4_fast = f2[0] == 0x3C003C00u && f2[1] == 0x3C003C00u;
+  const bool all_int_fast = __all_sync(0xffffffffu, is_nf4 || is_fp4 || int_fast);
+  const bool all_fp4_fast = __all_sync(0xffffffffu, !is_fp4 || fp4_fast);
+  if (is_nf4) {
+    // level table of nibble pairs (per-channel scale in the epilogue)
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) out[4 * i + j] = lut[((w[i] >> (4 * j)) & 0xFu) | ((w[i] >> (4 * j + 12)) & 0xF0u)];
-  } else if (c.f == CHAM_W_E2M1 || c.f == CHAM_W_MXFP4) {
-    // E2M1 s.e1e0.m placed at fp16 bits 15 and 11..9 is value * 2^-14: multiply back by 2^14
+  } else if (is_fp4) {
+    if (all_fp4_fast) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t x = w[i] >> (4 * j);
+          out[4 * i + j] = hmul2u(((x & 0x00070007u) << 9) | ((x & 0x00080008u) << 12), f1[i >> 2]);
+        }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t x = w[i] >> (4 * j);
+          out[4 * i + j] =
+              hmul2u(hmul2u(((x & 0x00070007u) << 9) | ((x & 0x00080008u) << 12), f1[i >> 2]), f2[i >> 2]);
+        }
+    }
+  } else if (all_int_fast) {
+    const int c0 = min(max(e0, -20), 5), c1 = min(max(e1, -20), 5);
+    const uint32_t m0[2] = {dup16(static_cast<uint32_t>(c0 + 25) << 10), dup16(static_cast<uint32_t>(c1 + 25) << 10)};
+    const uint32_t m1[2] = {dup16(static_cast<uint32_t>(c0 + 21) << 10), dup16(static_cast<uint32_t>(c1 + 21) << 10)};
+    const uint32_t o = static_cast<uint32_t>(c.off);
+    const uint32_t s0[2] = {m0[0] | dup16(o), m0[1] | dup16(o)};
+    const uint32_t s1[2] = {m1[0] | dup16(o << 4), m1[1] | dup16(o << 4)};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int b = i >> 2;
+      const uint32_t v = w[i], t = w[i] >> 8;
+      out[4 * i + 0] = hsub2u((v & 0x000F000Fu) | m0[b], s0[b]);
+      out[4 * i + 1] = hsub2u((v & 0x00F000F0u) | m1[b], s1[b]);
+      out[4 * i + 2] = hsub2u((t & 0x000F000Fu) | m0[b], s0[b]);
+      out[4 * i + 3] = hsub2u((t & 0x00F000F0u) | m1[b], s1[b]);
+    }
+  } else {
+    const uint32_t sub = dup16((25u << 10) | static_cast<uint32_t>(c.off));
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const uint32_t x = w[i] >> (4 * j);
-        const uint32_t bits = ((x & 0x00070007u) << 9) | ((x & 0x00080008u) << 12);
-        out[4 * i + j] = hmul2u(hmul2u(hmul2u(bits, 0x74007400u), f1[i >> 2]), f2[i >> 2]);
-      }
-  } else {
-    // INT4-sym, INT4-asym, MXINT4: 0x640N as fp16 is 1024 + N
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const uint32_t v = w[i] ^ c.flip;
-#pragma unroll
       for (int j = 0; j < 4; ++j)
         out[4 * i + j] =
-            hmul2u(hmul2u(hsub2u(((v >> (4 * j)) & 0x000F000Fu) | 0x64006400u, c.sub), f1[i >> 2]), f2[i >> 2]);
-    }
+            hmul2u(hmul2u(hsub2u(((w[i] >> (4 * j)) & 0x000F000Fu) | 0x64006400u, sub), f1[i >> 2]), f2[i >> 2]);
   }
 }
 
@@ -201,11 +261,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint32_t* lut = reinterpret_cast<uint32_t*>(smem + C::kData);
   constexpr int S = C::kStages;
   constexpr int kAStages = C::kAStages, kGroup = C::kGroup, kAGroups = kAStages / kGroup;
+  constexpr int kDone = C::kDone;
   uint64_t* full = reinterpret_cast<uint64_t*>(lut + 256);  // [S] producer -> decoders, MMA (tx bytes)
-  uint64_t* empty = full + S;                                // [S] MMA commit -> producer
-  uint64_t* afull = empty + S;                               // [kAGroups] decode warps -> MMA
-  uint64_t* aempty = afull + kAStages;                       // [kAStages] MMA commit -> decoders
-  uint64_t* accfull = aempty + kAStages;                     // [2] MMA commit -> epilogue
+  uint64_t* done = full + S;                                 // [kDone] MMA group commit -> producer, decoders
+  uint64_t* afull = done + kDone;                            // [kAGroups] decode warps -> MMA
+  uint64_t* accfull = afull + kAGroups;                      // [2] MMA commit -> epilogue
   uint64_t* accempty = accfull + 2;                          // [2] epilogue warps (4) -> MMA
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -214,16 +274,21 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const int nk = a.n_chunks;
   const int n_ch = a.n_ch_tiles;
   const int n_tiles = n_ch * ((a.M + BN - 1) / BN);
+  // K-chunks this CTA processes (its tiles x nk); the last commit group may be partial
+  const uint32_t total =
+      static_cast<int>(blockIdx.x) < n_tiles
+          ? static_cast<uint32_t>((n_tiles - static_cast<int>(blockIdx.x) + gridDim.x - 1) / gridDim.x) * nk
+          : 0u;
+  // wait until the MMAs of chunk j have completed (the commit of its group)
+  auto wait_done = [&](uint32_t j) {
+    const uint32_t g = j / kGroup;
+    return mbar_wait(&done[g % kDone], (g / kDone) & 1, abort_flag, a.dev_status);
+  };
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < S; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
-    }
-    for (int s = 0; s < kAStages; ++s) {
-      if (s < kAGroups) mbar_init(&afull[s], 4 * kGroup);  // one elected lane per warp and chunk
-      mbar_init(&aempty[s], 1);
-    }
+    for (int s = 0; s < S; ++s) mbar_init(&full[s], 1);
+    for (int g = 0; g < kDone; ++g) mbar_init(&done[g], 1);
+    for (int g = 0; g < kAGroups; ++g) mbar_init(&afull[g], 4 * kGroup);  // one elected lane per warp and chunk
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accfull[b], 1);
       mbar_init(&accempty[b], 4);  // one elected lane per epilogue warp
@@ -249,8 +314,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int ch = a.tile0 + t % n_ch, tok0 = (t / n_ch) * BN;
         for (int kc = 0; kc < nk; ++kc, ++it) {
           const int s = it % S;
-          const uint32_t ph = (it / S) & 1;
-          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, a.dev_status)) {
+          if (it >= static_cast<uint32_t>(S) && !wait_done(it - S)) {  // the stage's previous chunk is consumed
             ok = false;
             break;
           }
@@ -270,34 +334,40 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ---------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_f16(128, BN);
-      uint32_t it = 0, acc_it = 0;
+      // operand addresses advance incrementally: the activation stage's descriptor (start address
+      // in 16-byte units in the low bits) and the decoded-weight stage's tensor-memory column
+      const uint64_t desc0 = smem_desc_sw128(smem_u32(smem));
+      constexpr uint32_t kStageDesc = C::kStage >> 4;
+      uint32_t it = 0, acc_it = 0, s = 0, sa = 0, gi = 0;  // s = it % S, sa = it % kAStages, gi = it % kGroup
       bool ok = true;
       for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++acc_it) {
         const int b = acc_it & 1;
         if (!mbar_wait(&accempty[b], ((acc_it >> 1) & 1) ^ 1, abort_flag, a.dev_status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem + b * C::kAccCols;
-        // One wait per group of kGroup consecutive K-chunks: every stall of this thread drains the
-        // tensor pipe's short instruction queue, so waits are amortised over 4 * kGroup MMAs.  Only
-        // the decoded-operand barrier is waited on: the decoders arrive on it after they have
-        // themselves observed the stage's TMA barrier, so the activation tile has landed too.  A
-        // group may straddle two tiles; its wait then also covers the next tile's first chunks.
+        // One wait per group of kGroup consecutive K-chunks, on the decoded-operand barrier only:
+        // the decoders arrive on it after they have themselves observed the stage's TMA barrier,
+        // so the activation tile has landed too.  A group may straddle two tiles.
         for (int kc = 0; kc < nk; ++kc, ++it) {
-          if (it % kGroup == 0) {
+          if (gi == 0) {
             if (!mbar_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
               ok = false;
               break;
             }
             tc_fence_after();
           }
-          const int s = it % S, sa = it % kAStages;
-          const uint32_t b0 = smem_u32(smem + s * C::kStage);
-#pragma unroll
-          for (int kk = 0; kk < kBK / 16; ++kk)
-            mma_f16_ts(d_tmem, tmem + C::kACol + sa * 32 + kk * 8, smem_desc_sw128(b0 + kk * 32), idesc,
-                       (kc | kk) != 0);
-          mma_commit(&empty[s]);
-          mma_commit(&aempty[sa]);
+          const uint64_t bd = desc0 + s * kStageDesc;
+          const uint32_t ad = tmem + C::kACol + sa * 32;
+          mma_f16_ts(d_tmem, ad, bd, idesc, kc != 0);
+          mma_f16_ts(d_tmem, ad + 8, bd + 2, idesc, 1u);
+          mma_f16_ts(d_tmem, ad + 16, bd + 4, idesc, 1u);
+          mma_f16_ts(d_tmem, ad + 24, bd + 6, idesc, 1u);
+          if (++gi == kGroup || it + 1 == total) {
+            mma_commit(&done[(it / kGroup) % kDone]);
+            gi = gi == kGroup ? 0 : gi;
+          }
+          s = s + 1 == static_cast<uint32_t>(S) ? 0 : s + 1;
+          sa = sa + 1 == static_cast<uint32_t>(kAStages) ? 0 : sa + 1;
         }
         mma_commit(&accfull[b]);
       }
@@ -312,8 +382,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     uint32_t it = 0;
     bool ok = true;
-    // chunks this CTA processes; the last one also arrives for the missing chunks of its group
-    const uint32_t total = static_cast<uint32_t>((n_tiles - static_cast<int>(blockIdx.x) + gridDim.x - 1) / gridDim.x) * nk;
+    // the last chunk of this CTA also arrives for the missing chunks of its group
     // the channel's format and zero point for the next tile are loaded one tile ahead
     int nf = 0, nz = 0;
     if (static_cast<int>(blockIdx.x) < n_tiles) {
@@ -331,9 +400,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       for (int kc = 0; kc < nk; ++kc, ++it) {
         if (static_cast<int>(it % kDecodeGroups) != grp) continue;
         const int s = it % S, sa = it % kAStages;
-        const uint32_t ph = (it / S) & 1, pa = (it / kAStages) & 1;
-        if (!warp_wait(&full[s], ph, abort_flag, a.dev_status) ||
-            !warp_wait(&aempty[sa], pa ^ 1, abort_flag, a.dev_status)) {
+        const uint32_t ph = (it / S) & 1;
+        // the tensor-memory stage's previous chunk (it - kAStages, two groups back) is consumed
+        const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
+        if (!__all_sync(0xffffffffu, free_ok) || !warp_wait(&full[s], ph, abort_flag, a.dev_status)) {
           ok = false;
           break;
         }
@@ -355,6 +425,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           const uint32_t (&r8)[8] = *reinterpret_cast<const uint32_t(*)[8]>(&raw[0]);
           decode_w4(r8, cd, e8, lut, out);
         }
+        __syncwarp();  // the per-format decode branches reconverge before the warp-wide store
         tc_fence_after();
         tmem_st_32x32b_x32(tmem + C::kACol + lane_off + sa * 32, out);
         tmem_wait_st();

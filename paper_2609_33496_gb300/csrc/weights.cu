@@ -266,10 +266,15 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
       }
     }
     if (v >= nvec_p) continue;
-    if (v >= nvec) {  // K padding up to a multiple of 64: code 0
+    if (v >= nvec) {  // K padding up to a multiple of 64: the value 0
 #pragma unroll
-      for (int i = 0; i < 8; ++i) code[i] = 0;
+      for (int i = 0; i < 8; ++i) code[i] = f == CHAM_W_INT8_ASYM || f == CHAM_W_INT4_ASYM ? cs.z : 0;
     }
+    // symmetric integer codes are stored in offset binary (q + 128, q + 8)
+    const int bias = (f == CHAM_W_INT8_SYM || f == CHAM_W_MXINT8) ? 0x80
+                     : ((f == CHAM_W_INT4_SYM || f == CHAM_W_MXINT4) ? 0x8 : 0);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) code[i] = (code[i] & (a.bits == 8 ? 0xFF : 0xF)) ^ bias;
     const size_t off = code_offset(p, v * 8, a.n_chunks, a.bits);
     if (a.bits == 8) {
       uint32_t lo = 0, hi = 0;

@@ -53,10 +53,16 @@ def unpack(blob_bytes):
         f = int(fmt[p])
         t, r = divmod(p, 128)
         e8c = e8[t, :, r, :].reshape(-1)[:K // 32]
-        if f == 0:                      # INT8-sym: two's complement byte
-            vals = np.where(vals >= 128, vals - 256, vals)
-        elif f == 3:                    # INT4-sym: two's complement nibble
-            vals = np.where(vals >= 8, vals - 16, vals)
+        # symmetric integer codes are stored in offset binary; the oracle keeps INT8/INT4-sym
+        # signed and MXINT8/MXINT4 as two's-complement bytes / nibbles
+        if f == 0:                      # INT8-sym: q + 128
+            vals = vals - 128
+        elif f == 2:                    # MXINT8: (q + 128) -> q & 0xFF
+            vals = vals ^ 0x80
+        elif f == 3:                    # INT4-sym: q + 8
+            vals = vals - 8
+        elif f == 7:                    # MXINT4: (q + 8) -> q & 0xF
+            vals = vals ^ 0x8
         out[c] = {"fmt": f, "codes": vals, "s": np.float32(scale[p]), "z": int(zero[p]), "e8m0": e8c,
                   "slot": p}
     return d, out
