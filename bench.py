@@ -204,57 +204,46 @@ def main():
     quant_bytes_step = 0.0
     gemm_bytes_step = 0.0
 
-    try:
-        torch.cuda.Event(enable_timing=True, external=True)
-        ext = {"external": True}
-    except TypeError:
-        ext = None
-    n_ev = 2 * nb * len(layers) + 1
-    events = [torch.cuda.Event(enable_timing=True, **(ext or {})) for _ in range(n_ev)]
-    kinds = []
-
-    def run_step(record):
-        """a2-a4 + a7 for every (bucket, layer): act-quant in F[l, b], then the GEMM."""
-        k = 0
+    def run_step(parts="qg"):
+        """a2-a4 + a7 for every (bucket, layer): act-quant in F[l, b] ("q"), then the GEMM ("g")."""
         for bk in range(nb):
             for li, (_, M, K, N) in enumerate(layers):
                 f = int(lut[li, bk])
-                if record:
-                    events[k].record()
-                    k += 1
-                cl.linear_prepare(X[li][bk], f, ws[li], st)
-                if record:
-                    events[k].record()
-                    k += 1
-                cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
-        if record:
-            events[k].record()
+                if "q" in parts:
+                    cl.linear_prepare(X[li][bk], f, ws[li], st)
+                if "g" in parts:
+                    cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
 
-    for bk in range(nb):
-        for li in range(len(layers)):
-            kinds.extend(["q", "g"])
-
-    # warm-up (eager), then capture the quantize + GEMM sequence of one step in a CUDA graph with
-    # timing event nodes between the kernels; select + pack stay eager (they need a host plan)
+    # warm-up (eager), then capture the quantize + GEMM sequence of one step in a CUDA graph (no
+    # event nodes inside: each costs about 5 us of serialisation), plus two graphs holding only
+    # the quantizer launches and only the GEMM launches of the step, which time those kernel
+    # classes; select + pack stay eager (they need a host plan)
     for _ in range(args.warmup):
         select_pack()
-        run_step(False)
+        run_step()
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
-    graph = None
-    if ext is not None:
-        try:
+    graphs = {}
+    try:
+        for key in ("qg", "q", "g"):
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
-                run_step(True)
-            for _ in range(args.warmup):
-                select_pack()
-                g.replay()
-            torch.cuda.synchronize()
-            graph = g
-        except RuntimeError as exc:  # a launch that cannot be captured: time eager launches
-            print("bench: CUDA-graph capture failed (%s); timing eager launches" % exc, file=sys.stderr)
-            torch.cuda.synchronize()
+                run_step(key)
+            graphs[key] = g
+        for _ in range(args.warmup):
+            select_pack()
+            graphs["qg"].replay()
+        torch.cuda.synchronize()
+    except RuntimeError as exc:  # a launch that cannot be captured: time eager launches
+        print("bench: CUDA-graph capture failed (%s); timing eager launches" % exc, file=sys.stderr)
+        graphs = {}
+        torch.cuda.synchronize()
+
+    def replay(key):
+        if key in graphs:
+            graphs[key].replay()
+        else:
+            run_step(key)
 
     # kernel launches per step: select 1 + pack 3 per layer; per linear 2 (per-tensor) or 1 (MX)
     # quantizer kernels + 1 GEMM
@@ -266,18 +255,6 @@ def main():
             quant_bytes_step += M * K * 2 + M * K * 2 + (M * K / 32 if mx else 0)
             gemm_bytes_step += M * K * 1 + N * K * 1 + N * (4 + 1) + 4 * N + M * N * 4
     # ---------------------------------------------------------------- timed region (device)
-    gemm_ms, quant_ms, gemm_launch_ms = 0.0, 0.0, []
-
-    def collect():
-        nonlocal gemm_ms, quant_ms
-        for i in range(n_ev - 1):
-            d = events[i].elapsed_time(events[i + 1])
-            if kinds[i] == "g":
-                gemm_ms += d
-                gemm_launch_ms.append(d)
-            else:
-                quant_ms += d
-
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -287,15 +264,23 @@ def main():
         t0.record(stream)
         for k in range(args.steps):
             select_pack()                 # its host plan waits for the previous step's graph
-            if k > 0:
-                collect()                 # events of the previous replay are complete here
-            if graph is not None:
-                graph.replay()
-            else:
-                run_step(True)
+            replay("qg")
         t1.record(stream)
         torch.cuda.synchronize()
-        collect()
+        # kernel classes, each alone: the step's 100 quantizer (or GEMM) launches back to back,
+        # replayed as many times as the timed steps, two events around them
+        class_ms = {}
+        for key in ("g", "q"):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for k in range(args.steps):
+                replay(key)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            class_ms[key] = e0.elapsed_time(e1)
+    gemm_ms, quant_ms = class_ms["g"], class_ms["q"]
+    n_linear = nb * len(layers)
     if world > 1:
         dist.barrier()
     elapsed_ms = t0.elapsed_time(t1)
@@ -339,11 +324,13 @@ def main():
                      "peak_source": "%s bf16_tflops_sustained (fp16 MMA rate = bf16 rate)" % pk_kind,
                      "roofline_time_frac": round(t_roof * K_ / (gemm_ms * 1e-3), 4),
                      "gemm_ms_per_step": round(gemm_ms / K_, 4),
-                     "gemm_launch_ms_mean": round(statistics.mean(gemm_launch_ms), 5),
+                     "gemm_launch_ms_mean": round(gemm_ms / (args.steps * n_linear), 5),
                      "probe_tflops": probe,
                      "frac_of_probe_f16": round(gemm_tflops / probe["f16"], 4) if probe else None,
-                     "timing": "CUDA-graph replay of the quantize+GEMM sequence, event nodes between kernels"
-                               if graph is not None else "eager launches, events between kernels"},
+                     "timing": ("value: CUDA-graph replay of each step's quantize+GEMM sequence, no event "
+                                "nodes inside; kernel classes: the step's GEMM (quantizer) launches alone, "
+                                "graph-replayed once per timed step between two events")
+                               if graphs else "eager launches"},
         "act_quant": {"achieved_gbs": round(quant_gbs, 1), "peak_gbs": pk["hbm_gbs"],
                       "frac": round(quant_gbs / pk["hbm_gbs"], 4), "ms_per_step": round(quant_ms / K_, 4),
                       "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"},

@@ -10,8 +10,8 @@
 //     per-channel scale kept for the epilogue) and write them into tensor memory (tcgen05.st).
 //   * MMA "B" (N = BN tokens) = a tile of activation operand rows, brought into shared memory by
 //     TMA with 128-byte swizzling, K-major.
-//   * D (128 channels x BN tokens, fp32) accumulates in tensor memory, double buffered: four
-//     epilogue warps drain one buffer (tcgen05.ld, s_a * s_w, bias, coalesced stores of Y in
+//   * D (128 channels x BN tokens, fp32) accumulates in tensor memory, double buffered: eight
+//     epilogue warps (two per lane quadrant, alternate 16-column slices) drain one buffer (tcgen05.ld, s_a * s_w, bias, coalesced stores of Y in
 //     original channel order) while the MMA fills the other with the next tile.
 // The kernel is persistent: each CTA walks tiles t = blockIdx.x, blockIdx.x + gridDim.x, ... of
 // the (channel tile, token tile) grid.  Two rings over K-chunks of 64 couple the roles: a 6-8
@@ -27,7 +27,8 @@ namespace cham {
 
 constexpr int kBK = 64;  // K elements per stage: 128 bytes of fp16 per activation row
 constexpr int kDecodeGroups = 2;  // decode warpgroups, taking alternate K-chunks
-constexpr int kGemmThreads = 128 * (2 + kDecodeGroups);
+constexpr int kEpiGroups = 2;     // epilogue warpgroups, taking alternate 16-column slices
+constexpr int kGemmThreads = 128 * (1 + kDecodeGroups + kEpiGroups);
 
 template <int BN, int BITS>
 struct GemmCfg {
@@ -266,7 +267,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   uint64_t* done = full + S;                                 // [kDone] MMA group commit -> producer, decoders
   uint64_t* afull = done + kDone;                            // [kAGroups] decode warps -> MMA
   uint64_t* accfull = afull + kAGroups;                      // [2] MMA commit -> epilogue
-  uint64_t* accempty = accfull + 2;                          // [2] epilogue warps (4) -> MMA
+  uint64_t* accempty = accfull + 2;                          // [2] epilogue warps (8) -> MMA
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accempty + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -291,7 +292,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     for (int g = 0; g < kAGroups; ++g) mbar_init(&afull[g], 4 * kGroup);  // one elected lane per warp and chunk
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accfull[b], 1);
-      mbar_init(&accempty[b], 4);  // one elected lane per epilogue warp
+      mbar_init(&accempty[b], 4 * kEpiGroups);  // one elected lane per epilogue warp
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -438,8 +439,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
     }
   } else if (warp >= 4 + 4 * kDecodeGroups) {
-    // ---------------- epilogue: drain one accumulator buffer per tile
+    // ---------------- epilogue: drain one accumulator buffer per tile; warpgroup h takes the
+    // 16-column slices j = h, h + kEpiGroups, ...
     const int q = warp & 3;
+    const int h = (warp - (4 + 4 * kDecodeGroups)) >> 2;
     const int r = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const float sa = a.act_scale != nullptr ? *a.act_scale : 1.f;
@@ -456,8 +459,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       tc_fence_after();
       float* yc = a.Y + (orig >= 0 ? orig : 0);
       const uint32_t d_tmem = tmem + b * C::kAccCols + lane_off;
-      // 16 token columns per tcgen05.ld; the load of the next 16 is in flight while the current
-      // ones are scaled and stored (a wait per load would serialise its latency 12 times per tile)
+      // 16 token columns per tcgen05.ld; the load of the warp's next slice is in flight while the
+      // current one is scaled and stored (a wait per load would serialise its latency)
       auto store16 = [&](const uint32_t (&v)[16], int j) {
         if (orig >= 0) {
 #pragma unroll
@@ -467,17 +470,19 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
         }
       };
-      constexpr int kLoads = BN / 16;
+      constexpr int kLoads = BN / 16, kE = kEpiGroups;
       uint32_t va[16], vb[16];
-      tmem_ld_32x32b_x16(d_tmem, va);
-      tmem_wait_ld();
+      if (h < kLoads) {
+        tmem_ld_32x32b_x16(d_tmem + h * 16, va);
+        tmem_wait_ld();
+      }
 #pragma unroll 1
-      for (int j = 0; j < kLoads; j += 2) {
-        if (j + 1 < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + 1) * 16, vb);
+      for (int j = h; j < kLoads; j += 2 * kE) {
+        if (j + kE < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + kE) * 16, vb);
         store16(va, j);
         tmem_wait_ld();
-        if (j + 2 < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + 2) * 16, va);
-        if (j + 1 < kLoads) store16(vb, j + 1);
+        if (j + 2 * kE < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + 2 * kE) * 16, va);
+        if (j + kE < kLoads) store16(vb, j + kE);
         tmem_wait_ld();
       }
       tc_fence_before();
@@ -528,6 +533,7 @@ cudaError_t launch_gemm_f16(const CUtensorMap& map, const GemmArgs& a, int num_s
       case 32: return launch_bn<32, 8>(map, a, num_sms, st);
       case 64: return launch_bn<64, 8>(map, a, num_sms, st);
       case 128: return launch_bn<128, 8>(map, a, num_sms, st);
+      case 144: return launch_bn<144, 8>(map, a, num_sms, st);
       default: return launch_bn<192, 8>(map, a, num_sms, st);
     }
   }
@@ -536,6 +542,7 @@ cudaError_t launch_gemm_f16(const CUtensorMap& map, const GemmArgs& a, int num_s
     case 32: return launch_bn<32, 4>(map, a, num_sms, st);
     case 64: return launch_bn<64, 4>(map, a, num_sms, st);
     case 128: return launch_bn<128, 4>(map, a, num_sms, st);
+    case 144: return launch_bn<144, 4>(map, a, num_sms, st);
     default: return launch_bn<192, 4>(map, a, num_sms, st);
   }
 }
