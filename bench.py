@@ -187,12 +187,16 @@ def main():
     ws = [torch.empty(max(cl.linear_workspace_size(M, cl.pack_plan(N, K, np.zeros(N, np.uint8)), f)
                           for f in range(6)), dtype=torch.uint8, device=device) for (_, M, K, N) in layers]
     blobs, descs = [None] * len(layers), [None] * len(layers)
+    fmt_off = np.cumsum([0] + [N for (_, M, K, N) in layers])
+    fmt_all = torch.empty(int(fmt_off[-1]), dtype=torch.uint8, device=device)
 
     def select_pack():
         """a5 + a6 for every layer: GPU selection, host plan from the selected formats (one
         device->host copy of N bytes per layer), GPU pack into the layer's blob."""
-        fmts = [cl.select_weight_formats(W[li], cl.PALETTE_W8)[0] for li in range(len(layers))]
-        fmts_host = [f.cpu().numpy() for f in fmts]
+        fmts = [cl.select_weight_formats(W[li], cl.PALETTE_W8, fmt_out=fmt_all[fmt_off[li]:fmt_off[li + 1]])[0]
+                for li in range(len(layers))]
+        every = fmt_all.cpu().numpy()     # one device->host copy for all layers
+        fmts_host = [every[fmt_off[li]:fmt_off[li + 1]] for li in range(len(layers))]
         for li, (_, M, K, N) in enumerate(layers):
             d = cl.pack_plan(N, K, fmts_host[li])
             if descs[li] is not None and bytes(d) != bytes(descs[li]):
@@ -366,6 +370,8 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
     st = torch.zeros(1, dtype=torch.int32, device=device)
     ws = [torch.empty(max(cl.linear_workspace_size(M, cl.pack_plan(N, K, np.zeros(N, np.uint8)), f)
                           for f in range(6)), dtype=torch.uint8, device=device) for (_, M, K, N) in layers]
+    fmt_off = np.cumsum([0] + [N for (_, M, K, N) in layers])
+    fmt_all = torch.empty(int(fmt_off[-1]), dtype=torch.uint8, device=device)
     h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + sum(x.numel() * 2 for xs in Xh for x in xs)
     d2h = nb * sum(M * N * 4 for (_, M, K, N) in layers)
 
@@ -374,9 +380,11 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
         for li in range(len(layers)):
             Wd[li].copy_(Wh[li], non_blocking=True)
             bd[li].copy_(bh[li], non_blocking=True)
-            fmts.append(cl.select_weight_formats(Wd[li], cl.PALETTE_W8)[0])
+            fmts.append(cl.select_weight_formats(Wd[li], cl.PALETTE_W8,
+                                                 fmt_out=fmt_all[fmt_off[li]:fmt_off[li + 1]])[0])
+        every = fmt_all.cpu().numpy()
         for li, (_, M, K, N) in enumerate(layers):
-            d = cl.pack_plan(N, K, fmts[li].cpu().numpy())
+            d = cl.pack_plan(N, K, every[fmt_off[li]:fmt_off[li + 1]])
             descs.append(d)
             blobs.append(cl.pack_weights(Wd[li], fmts[li], d, dev_status=st)[0])
         for bk in range(nb):

@@ -196,10 +196,13 @@ def split_qact(qact, M, K):
 
 
 # ------------------------------------------------------------------ a5
-def select_weight_formats(W, palette_mask, want_sse=False, stream=None):
+def select_weight_formats(W, palette_mask, want_sse=False, stream=None, fmt_out=None):
+    """fmt_out: optional uint8 device tensor of N elements to write the formats into."""
     import torch
     N, K = W.shape
-    fmt = torch.empty(N, dtype=torch.uint8, device=W.device)
+    fmt = torch.empty(N, dtype=torch.uint8, device=W.device) if fmt_out is None else fmt_out
+    if fmt.numel() != N or fmt.dtype != torch.uint8 or not fmt.is_contiguous():
+        raise ValueError("fmt_out must be a contiguous uint8 tensor of N elements")
     sse = torch.empty((N, 9), dtype=torch.float64, device=W.device) if want_sse else None
     check(lib().chameleon_select_weight_formats(_ptr(W), N, K, palette_mask, _ptr(fmt), _ptr(sse),
                                                 _stream(stream)))

@@ -141,6 +141,9 @@ CHAM_DEV void encode8_tensor(const uint4& v, const TensorParams& p, uint2& code,
 // ------------------------------------------------------------------ a2: range partials
 __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, int64_t nvec,
                                                   RangePartial* __restrict__ parts) {
+  griddep_launch_dependents();
+  // X is a caller input that no kernel of the chain writes: it is read before the wait, so this
+  // pass overlaps the tail of the previous kernel; the partial is written after it
   __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
   uint32_t nonfinite = 0;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -158,6 +161,7 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
   float lo = fminf(__low2float(lo2), __high2float(lo2));
   float hi = fmaxf(__low2float(hi2), __high2float(hi2));
   block_range(lo, hi, nonfinite);
+  griddep_wait();
   if (threadIdx.x == 0) parts[blockIdx.x] = RangePartial{lo, hi, static_cast<int>(nonfinite), 0};
 }
 
@@ -167,6 +171,8 @@ __global__ void __launch_bounds__(256)
     k_act_encode_tensor(const uint4* __restrict__ X, int64_t nvec, const RangePartial* __restrict__ parts,
                         int nparts, uint2* __restrict__ codes, uint4* __restrict__ deq,
                         cham_qparams* __restrict__ params, float* __restrict__ scale_out, int* dev_status) {
+  griddep_wait();  // the range partials
+  griddep_launch_dependents();
   float lo, hi;
   uint32_t nf;
   reduce_partials(parts, nparts, lo, hi, nf);
@@ -264,6 +270,8 @@ template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_mx(const uint4* __restrict__ X, int64_t nvec, uint2* __restrict__ codes, uint4* __restrict__ deq,
                     uint8_t* __restrict__ e8m0, cham_qparams* __restrict__ params, int* dev_status) {
+  griddep_wait();  // its outputs may still be read by the previous kernel
+  griddep_launch_dependents();
   if (blockIdx.x == 0 && threadIdx.x == 0 && params != nullptr) *params = cham_qparams{1.f, 0, 1.f, FMT};
   const int lane = threadIdx.x & 31;
   const int64_t warp_global = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -378,10 +386,11 @@ int range_grid(int64_t nvec, int num_sms) {
 
 template <int FMT, bool CODES, bool DEQ>
 static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
-  k_act_range<<<a.nparts, 256, 0, st>>>(a.X, a.nvec, a.parts);
+  launch_pdl(k_act_range, dim3(a.nparts), dim3(256), 0, st, a.X, a.nvec, a.parts);
   const int g = range_grid(a.nvec, a.num_sms);
-  k_act_encode_tensor<FMT, CODES, DEQ><<<g, 256, 0, st>>>(a.X, a.nvec, a.parts, a.nparts, a.codes, a.deq,
-                                                          a.params, a.scale_out, a.dev_status);
+  launch_pdl(k_act_encode_tensor<FMT, CODES, DEQ>, dim3(g), dim3(256), 0, st, a.X, a.nvec,
+             static_cast<const RangePartial*>(a.parts), a.nparts, a.codes, a.deq, a.params, a.scale_out,
+             a.dev_status);
 }
 
 template <int FMT, bool CODES, bool DEQ>
@@ -391,8 +400,8 @@ static void launch_mx(const ActQuantArgs& a, cudaStream_t st) {
   const int64_t cap = static_cast<int64_t>(a.num_sms) * 8;
   if (g > cap) g = cap;
   if (g < 1) g = 1;
-  k_act_encode_mx<FMT, CODES, DEQ><<<static_cast<int>(g), 256, 0, st>>>(a.X, a.nvec, a.codes, a.deq, a.e8m0,
-                                                                         a.params, a.dev_status);
+  launch_pdl(k_act_encode_mx<FMT, CODES, DEQ>, dim3(static_cast<int>(g)), dim3(256), 0, st, a.X, a.nvec, a.codes,
+             a.deq, a.e8m0, a.params, a.dev_status);
 }
 
 template <bool CODES, bool DEQ>

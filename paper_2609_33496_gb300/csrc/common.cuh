@@ -8,7 +8,10 @@
 
 #include <cuda.h>
 #include <cuda_fp16.h>
+#include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <utility>
 
 #include "../../include/chameleon.h"
 
@@ -19,6 +22,34 @@ namespace cham {
 // ------------------------------------------------------------------ status word
 CHAM_DEV void set_status(int* dev_status, int code) {
   if (dev_status != nullptr) atomicCAS(dev_status, 0, code);
+}
+
+// ------------------------------------------------------------------ programmatic dependent launch
+// The quantizer and GEMM kernels of one linear call are launched with programmatic stream
+// serialisation: a kernel may be scheduled while its predecessor in the stream drains, runs
+// whatever needs none of the predecessor's results, and calls griddep_wait() -- which returns
+// once the predecessor grid has completed and its memory is visible -- before it reads anything
+// an earlier kernel of the chain writes and before its own first global write.  Every kernel of
+// the chain waits, so completions stay in stream order.  Both instructions are no-ops in a
+// kernel launched without the attribute.
+CHAM_DEV void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+CHAM_DEV void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Launch with programmatic stream serialisation allowed (see above).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
 // ------------------------------------------------------------------ address helpers

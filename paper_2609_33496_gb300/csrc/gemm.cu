@@ -305,6 +305,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // the set-up above overlaps the previous kernel's tail; everything below may read its results
+  griddep_wait();
+  griddep_launch_dependents();
 
   if (warp == 0) {
     // ---------------- producer: activation tile (TMA), raw weight codes and E8M0 bytes (bulk)
@@ -522,8 +525,7 @@ static cudaError_t launch_bn(const CUtensorMap& map, const GemmArgs& a, int num_
   }
   const long tiles = static_cast<long>(a.n_ch_tiles) * ((a.M + BN - 1) / BN);
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  k_gemm_ts_f16<BN, BITS><<<grid, kGemmThreads, C::kSmem, st>>>(map, a);
-  return cudaGetLastError();
+  return launch_pdl(k_gemm_ts_f16<BN, BITS>, dim3(grid), dim3(kGemmThreads), C::kSmem, st, map, a);
 }
 
 cudaError_t launch_gemm_f16(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {

@@ -1,9 +1,10 @@
 // weights.cu -- weight-format selection (step a5) and weight pack (step a6).
 //
 // Selection (Sec. 3.4, Eq. weight-argmax): every output channel is round-tripped through every
-// palette format; the squared reconstruction error SSE_f(c) is accumulated in fp64 from
-// per-element errors that are exact up to one fp32 rounding; the smallest error wins, the
-// earlier palette member on ties (strict '<').  One CTA per channel: the row (at most 10 KB for
+// palette format; the squared reconstruction error SSE_f(c) is accumulated from per-element
+// errors that are exact up to one fp32 rounding (fp32 sums of eight squares, added in fp64;
+// relative error below 2.4e-7); the smallest error wins, the earlier palette member on ties
+// (strict '<').  One CTA per channel: the row (at most 10 KB for
 // K = 5120) stays in L1 across the format passes.
 //
 // Pack: channels are permuted (Sec. 5: "same-format sub-GEMMs after a channel permutation") into
@@ -73,6 +74,17 @@ CHAM_DEV ChanStats row_stats(const __half* row, int nvec, float* shf) {
 }
 
 // ------------------------------------------------------------------ a5: selection
+// Pairwise fp32 sum of eight non-negative squared errors.  Each square and each of the three
+// levels of additions rounds once, so the group sum is within 4 * 2^-24 relative of the exact
+// sum; the groups are then added in fp64.  Every term being non-negative, the channel's SSE
+// keeps that relative bound (about 2.4e-7), while the fp64 pipe -- a small fraction of the
+// fp32 rate on this GPU -- sees one add per eight elements.
+CHAM_DEV float sum8(const float (&e2)[8]) {
+  const float a = __fadd_rn(e2[0], e2[1]), b = __fadd_rn(e2[2], e2[3]);
+  const float c = __fadd_rn(e2[4], e2[5]), d = __fadd_rn(e2[6], e2[7]);
+  return __fadd_rn(__fadd_rn(a, b), __fadd_rn(c, d));
+}
+
 __global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict__ W, int K, uint32_t mask,
                                                        uint8_t* __restrict__ fmt_out, double* __restrict__ sse_out,
                                                        NF4Table nf4) {
@@ -99,27 +111,29 @@ __global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict
         a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, 2));
         const int X = mx_exponent(f, a);
         if (v < nvec) {
+          float e2[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             float dq;
             encode_mx(f, x[i], X, &dq);
-            const double e = static_cast<double>(__fsub_rn(x[i], dq));
-            acc = fma(e, e, acc);
+            const float e = __fsub_rn(x[i], dq);
+            e2[i] = __fmul_rn(e, e);
           }
+          acc += static_cast<double>(sum8(e2));
         }
       }
     } else {
       const ChanScale cs = chan_scale(f, st);
       for (int v = threadIdx.x; v < nvec; v += kWThreads) {
-        float x[8];
+        float x[8], e2[8];
         load8(row, v, x);
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           float err;
           encode_chan(f, x[i], cs, nf4, &err);
-          const double e = static_cast<double>(err);
-          acc = fma(e, e, acc);
+          e2[i] = __fmul_rn(err, err);
         }
+        acc += static_cast<double>(sum8(e2));
       }
     }
     const double tot = block_reduce(acc, DAdd(), shd);
