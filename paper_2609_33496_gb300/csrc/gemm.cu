@@ -43,13 +43,13 @@ struct GemmCfg {
   static constexpr int kAccCols = (BN + 31) / 32 * 32;
   static constexpr int kACol = 2 * kAccCols;                      // first column of the A stages
   // Tensor-memory ring of decoded weight operands (32 columns per K-chunk), as deep as the 512
-  // columns allow next to the two accumulators, split into two commit groups of kGroup chunks.
+  // columns allow next to the two accumulators, split into commit groups of kGroup chunks.
   // The MMA thread commits once per group, and that one barrier frees both the group's
   // shared-memory stages and its tensor-memory stages: every commit another warp waits on costs
   // the tensor pipe a fixed round trip of several hundred cycles, so it must cover many MMAs.
   static constexpr int kAFit = (512 - kACol) / 32;
   static constexpr int kAStages = (kAFit > 8 ? 8 : kAFit) / 2 * 2;
-  static constexpr int kGroup = kAStages / 2;
+  static constexpr int kGroup = 2;  // chunks per commit group: kAStages / 2 groups in flight
   static constexpr int kDone = 8;                                 // group-completion barriers
   static constexpr int kNeedCols = kACol + kAStages * 32;
   static constexpr int kTmemCols = kNeedCols <= 256 ? 256 : 512;
@@ -405,7 +405,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         if (static_cast<int>(it % kDecodeGroups) != grp) continue;
         const int s = it % S, sa = it % kAStages;
         const uint32_t ph = (it / S) & 1;
-        // the tensor-memory stage's previous chunk (it - kAStages, two groups back) is consumed
+        // the tensor-memory stage's previous chunk (it - kAStages) is consumed
         const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
         if (!__all_sync(0xffffffffu, free_ok) || !warp_wait(&full[s], ph, abort_flag, a.dev_status)) {
           ok = false;
@@ -536,6 +536,7 @@ cudaError_t launch_gemm_f16(const CUtensorMap& map, const GemmArgs& a, int num_s
       case 64: return launch_bn<64, 8>(map, a, num_sms, st);
       case 128: return launch_bn<128, 8>(map, a, num_sms, st);
       case 144: return launch_bn<144, 8>(map, a, num_sms, st);
+      case 160: return launch_bn<160, 8>(map, a, num_sms, st);
       default: return launch_bn<192, 8>(map, a, num_sms, st);
     }
   }
@@ -545,6 +546,7 @@ cudaError_t launch_gemm_f16(const CUtensorMap& map, const GemmArgs& a, int num_s
     case 64: return launch_bn<64, 4>(map, a, num_sms, st);
     case 128: return launch_bn<128, 4>(map, a, num_sms, st);
     case 144: return launch_bn<144, 4>(map, a, num_sms, st);
+    case 160: return launch_bn<160, 4>(map, a, num_sms, st);
     default: return launch_bn<192, 4>(map, a, num_sms, st);
   }
 }
