@@ -143,6 +143,7 @@ def main():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-variants", action="store_true", help="skip the per-variant matrix")
     ap.add_argument("--layers", default="all", help="comma-separated layer indices (smaller cases for profiling)")
     ap.add_argument("--buckets", default="all", help="comma-separated timestep buckets")
     args = ap.parse_args()
@@ -308,6 +309,7 @@ def main():
         t_roof += nb * max(layer_flops(M, K, N) / (peak_tensor * 1e12), b / (pk["hbm_gbs"] * 1e9))
     clocks = clk.summary()
     probe = tensor_probe(torch, device)
+    variants = None if args.no_variants else variant_matrix(torch, cl, W, bias, X, layers, st, pk, probe)
 
     result = {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
@@ -339,6 +341,7 @@ def main():
         "act_quant": {"achieved_gbs": round(quant_gbs, 1), "peak_gbs": pk["hbm_gbs"],
                       "frac": round(quant_gbs / pk["hbm_gbs"], 4), "ms_per_step": round(quant_ms / K_, 4),
                       "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"},
+        "variants": variants,
         "gpu_launches": launches * K_,
         "clocks": clocks,
     }
@@ -444,6 +447,77 @@ def oracle_sample(layers_idx=(4,), buckets=(0, 9)):
     desc = "oracle select(W8)+act-quant+fp64 GEMM of layer(s) %s at buckets %s" % (
         [WL.SDXL_PROJ_LAYERS[i][0] for i in layers_idx], list(buckets))
     return flops, t, desc
+
+
+def variant_matrix(torch, cl, W, bias, X, layers, st, pk, probe, reps=20):
+    """Every activation-format x weight-palette variant of the GEMM (plus W4A16) on the largest
+    layer of the step, and the quantizer per activation format, the selection and the pack per
+    palette on the same tensors.  Each figure is `reps` launches captured in one CUDA graph and
+    timed between two events after a warm replay (kernel timed alone: burst peaks apply)."""
+    li = max(range(len(layers)), key=lambda i: layer_flops(*layers[i][1:]))
+    name, M, K, N = layers[li]
+    x = X[li][-1]
+    dev = x.device
+    Y = torch.empty((M, N), dtype=torch.float32, device=dev)
+    hbm = pk["hbm_gbs"] * 1e9
+    p16 = (probe or {}).get("f16", pk.get("bf16_tflops", 1900.0)) * 1e12
+    p8 = (probe or {}).get("f8f6f4", 2 * p16 / 1e12) * 1e12
+
+    def timed(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for _ in range(reps):
+                fn()
+        g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps  # ms per launch
+
+    out = {"layer": name, "M": M, "K": K, "N": N, "reps": reps, "gemm": [], "quant": [], "weights": [],
+           "peaks": {"f16_tflops": round(p16 / 1e12, 1), "f8_tflops": round(p8 / 1e12, 1),
+                     "hbm_gbs": pk["hbm_gbs"], "source": "tensor-core probe of this run; measured HBM copy"}}
+    flops = layer_flops(M, K, N)
+    for pal_name, mask, bits in (("W8", cl.PALETTE_W8, 8), ("W4", cl.PALETTE_W4, 4)):
+        fmt = torch.empty(N, dtype=torch.uint8, device=dev)
+        t_sel = timed(lambda: cl.select_weight_formats(W[li], mask, fmt_out=fmt))
+        desc = cl.pack_plan(N, K, fmt.cpu().numpy())
+        blob, _ = cl.pack_weights(W[li], fmt, desc, dev_status=st)
+        t_pack = timed(lambda: cl.pack_weights(W[li], fmt, desc, dev_status=st, blob=blob))
+        pack_bytes = 2 * N * K + N * K * bits / 8 + 10 * N
+        out["weights"].append({"palette": pal_name, "select_us": round(t_sel * 1e3, 2),
+                               "pack_us": round(t_pack * 1e3, 2),
+                               "pack_gbs": round(pack_bytes / (t_pack * 1e-3) / 1e9, 1),
+                               "pack_frac_hbm": round(pack_bytes / (t_pack * 1e-3) / hbm, 4),
+                               "formats": {int(f): int(c) for f, c in zip(*np.unique(fmt.cpu().numpy(),
+                                                                                       return_counts=True))}})
+        ws = torch.empty(max(cl.linear_workspace_size(M, desc, f) for f in range(6)), dtype=torch.uint8, device=dev)
+        for af in ([0, 1, 2, 3, 4] + ([5] if bits == 4 else [])):
+            if af != 5:
+                cl.linear_prepare(x, af, ws, st)
+            t = timed(lambda: cl.linear_gemm(x, desc, blob, af, bias[li], Y, ws, st))
+            a_bytes = M * K * (2 if af == 5 else 1) + (M * K / 32 if af in (3, 4) else 0)
+            byts = a_bytes + N * K * bits / 8 + 9 * N + 4 * M * N
+            t_s = t * 1e-3
+            row = {"act_fmt": af, "weights": pal_name, "tflops": round(flops / t_s / 1e12, 1),
+                   "us": round(t * 1e3, 2),
+                   "frac_f16_roofline": round(max(flops / p16, byts / hbm) / t_s, 4)}
+            if af != 5:
+                row["frac_fp8_roofline"] = round(max(flops / p8, byts / hbm) / t_s, 4)
+            out["gemm"].append(row)
+            if bits == 8 and af != 5:
+                tq = timed(lambda: cl.linear_prepare(x, af, ws, st))
+                qb = 4 * M * K + (M * K / 32 if af in (3, 4) else 0)
+                out["quant"].append({"act_fmt": af, "us": round(tq * 1e3, 2),
+                                     "gbs": round(qb / (tq * 1e-3) / 1e9, 1),
+                                     "frac_hbm": round(qb / (tq * 1e-3) / hbm, 4),
+                                     "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"})
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0, "device status %d" % int(st.item())
+    return out
 
 
 def tensor_probe(torch, device):

@@ -405,9 +405,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         if (static_cast<int>(it % kDecodeGroups) != grp) continue;
         const int s = it % S, sa = it % kAStages;
         const uint32_t ph = (it / S) & 1;
-        // the tensor-memory stage's previous chunk (it - kAStages) is consumed
-        const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
-        if (!__all_sync(0xffffffffu, free_ok) || !warp_wait(&full[s], ph, abort_flag, a.dev_status)) {
+        // decode as soon as the codes have landed; the tensor-memory slot (its previous chunk,
+        // it - kAStages, must be consumed by the MMAs) is waited for only before the store, so
+        // the decode stays off the MMA-completion -> store -> MMA-issue loop
+        if (!warp_wait(&full[s], ph, abort_flag, a.dev_status)) {
           ok = false;
           break;
         }
@@ -428,6 +429,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         } else {
           const uint32_t (&r8)[8] = *reinterpret_cast<const uint32_t(*)[8]>(&raw[0]);
           decode_w4(r8, cd, e8, lut, out);
+        }
+        const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
+        if (!__all_sync(0xffffffffu, free_ok)) {
+          ok = false;
+          break;
         }
         __syncwarp();  // the per-format decode branches reconverge before the warp-wide store
         tc_fence_after();
