@@ -4,8 +4,8 @@
 // palette format; the squared reconstruction error SSE_f(c) is accumulated from per-element
 // errors that are exact up to one fp32 rounding (fp32 sums of eight squares, added in fp64;
 // relative error below 2.4e-7); the smallest error wins, the earlier palette member on ties
-// (strict '<').  One CTA per channel: the row (at most 10 KB for
-// K = 5120) stays in L1 across the format passes.
+// (strict '<').  One warp per channel: the row (at most 10 KB for K = 5120) stays in L1 across
+// the format passes, and every reduction is a warp shuffle tree.
 //
 // Pack: channels are permuted (Sec. 5: "same-format sub-GEMMs after a channel permutation") into
 // the two MMA classes, each kept in original channel order and padded to 128-channel tiles, and
@@ -14,21 +14,16 @@
 
 namespace cham {
 
-constexpr int kWThreads = 128;
+// One warp per channel (shuffle reductions only, no block barriers), kWWarps channels per CTA.
+constexpr int kWWarps = 8;
+constexpr int kWThreads = 32 * kWWarps;
 
-// Block-wide reductions for 128 threads.
+// Warp-wide reduction in a fixed xor-tree order; the result is valid in every lane.
 template <typename T, typename Op>
-CHAM_DEV T block_reduce(T v, Op op, T* sh) {
+CHAM_DEV T warp_reduce(T v, Op op) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v = op(v, __shfl_xor_sync(0xffffffffu, v, o));
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __syncthreads();
-  if (lane == 0) sh[warp] = v;
-  __syncthreads();
-  T r = sh[0];
-#pragma unroll
-  for (int k = 1; k < kWThreads / 32; ++k) r = op(r, sh[k]);
-  return r;
+  return v;
 }
 
 struct FMin {
@@ -53,10 +48,10 @@ CHAM_DEV void load8(const __half* row, int v, float (&x)[8]) {
   }
 }
 
-// Channel statistics (amax, lo, hi) of one row, reduced over the CTA.
-CHAM_DEV ChanStats row_stats(const __half* row, int nvec, float* shf) {
+// Channel statistics (amax, lo, hi) of one row, reduced over the warp.
+CHAM_DEV ChanStats row_stats(const __half* row, int nvec, int lane) {
   float amax = 0.f, lo = INFINITY, hi = -INFINITY;
-  for (int v = threadIdx.x; v < nvec; v += kWThreads) {
+  for (int v = lane; v < nvec; v += 32) {
     float x[8];
     load8(row, v, x);
 #pragma unroll
@@ -67,9 +62,9 @@ CHAM_DEV ChanStats row_stats(const __half* row, int nvec, float* shf) {
     }
   }
   ChanStats s;
-  s.amax = block_reduce(amax, FMax(), shf);
-  s.lo = block_reduce(lo, FMin(), shf);
-  s.hi = block_reduce(hi, FMax(), shf);
+  s.amax = warp_reduce(amax, FMax());
+  s.lo = warp_reduce(lo, FMin());
+  s.hi = warp_reduce(hi, FMax());
   return s;
 }
 
@@ -85,23 +80,24 @@ CHAM_DEV float sum8(const float (&e2)[8]) {
   return __fadd_rn(__fadd_rn(a, b), __fadd_rn(c, d));
 }
 
-__global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict__ W, int K, uint32_t mask,
+__global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict__ W, int N, int K, uint32_t mask,
                                                        uint8_t* __restrict__ fmt_out, double* __restrict__ sse_out,
                                                        NF4Table nf4) {
-  __shared__ float shf[kWThreads / 32];
-  __shared__ double shd[kWThreads / 32];
-  __shared__ double sse[CHAM_W_NFORMATS];
-  const int c = blockIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int c = blockIdx.x * kWWarps + (threadIdx.x >> 5);
+  if (c >= N) return;  // whole warps: no block-wide barrier follows
   const __half* row = W + static_cast<size_t>(c) * K;
   const int nvec = K / 8;
-  const ChanStats st = row_stats(row, nvec, shf);
-  const int iters = (nvec + kWThreads - 1) / kWThreads;  // same trip count in every lane (shuffles)
+  const ChanStats st = row_stats(row, nvec, lane);
+  const int iters = (nvec + 31) / 32;  // same trip count in every lane (shuffles)
+  int best = -1;
+  double best_e = 0.0;
   for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
     if (!((mask >> f) & 1u)) continue;
     double acc = 0.0;
     if (w_is_mx(f)) {
       for (int it = 0; it < iters; ++it) {
-        const int v = it * kWThreads + threadIdx.x;
+        const int v = it * 32 + lane;
         float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
         if (v < nvec) load8(row, v, x);
         float a = 0.f;
@@ -124,7 +120,7 @@ __global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict
       }
     } else {
       const ChanScale cs = chan_scale(f, st);
-      for (int v = threadIdx.x; v < nvec; v += kWThreads) {
+      for (int v = lane; v < nvec; v += 32) {
         float x[8], e2[8];
         load8(row, v, x);
 #pragma unroll
@@ -136,27 +132,24 @@ __global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict
         acc += static_cast<double>(sum8(e2));
       }
     }
-    const double tot = block_reduce(acc, DAdd(), shd);
-    if (threadIdx.x == 0) sse[f] = tot;
-  }
-  if (threadIdx.x == 0) {
-    int best = -1;
-    double best_e = 0.0;
-    for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
-      const bool member = (mask >> f) & 1u;
-      if (member && (best < 0 || sse[f] < best_e)) {
-        best = f;
-        best_e = sse[f];
-      }
-      if (sse_out != nullptr) sse_out[static_cast<size_t>(c) * CHAM_W_NFORMATS + f] = member ? sse[f] : INFINITY;
+    const double tot = warp_reduce(acc, DAdd());
+    if (best < 0 || tot < best_e) {  // palette order: the earlier member wins a tie
+      best = f;
+      best_e = tot;
     }
+    if (lane == 0 && sse_out != nullptr) sse_out[static_cast<size_t>(c) * CHAM_W_NFORMATS + f] = tot;
+  }
+  if (lane == 0) {
+    if (sse_out != nullptr)
+      for (int f = 0; f < CHAM_W_NFORMATS; ++f)
+        if (!((mask >> f) & 1u)) sse_out[static_cast<size_t>(c) * CHAM_W_NFORMATS + f] = INFINITY;
     fmt_out[c] = static_cast<uint8_t>(best);
   }
 }
 
 void launch_select(const __half* W, int N, int K, uint32_t mask, uint8_t* fmt_out, double* sse_out,
                    const NF4Table& nf4, cudaStream_t st) {
-  k_w_select<<<N, kWThreads, 0, st>>>(W, K, mask, fmt_out, sse_out, nf4);
+  k_w_select<<<(N + kWWarps - 1) / kWWarps, kWThreads, 0, st>>>(W, N, K, mask, fmt_out, sse_out, nf4);
 }
 
 // ------------------------------------------------------------------ a6: slot assignment
@@ -222,23 +215,24 @@ CHAM_DEV size_t code_offset(int p, int k0, int n_chunks, int bits) {
 }
 
 __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) {
-  __shared__ float shf[kWThreads / 32];
-  const int p = blockIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int p = blockIdx.x * kWWarps + (threadIdx.x >> 5);  // one warp per packed slot
+  if (p >= a.n_packed) return;
   const int c = a.perm[p];
   const int nvec_p = a.Kp / 8;
   const int tile = p >> 7, r = p & 127;
   if (c < 0) {  // padding slot: zero codes, unit scale
-    for (int v = threadIdx.x; v < nvec_p; v += kWThreads) {
+    for (int v = lane; v < nvec_p; v += 32) {
       const size_t off = code_offset(p, v * 8, a.n_chunks, a.bits);
       if (a.bits == 8) *reinterpret_cast<uint2*>(a.codes + off) = make_uint2(0, 0);
       else *reinterpret_cast<uint32_t*>(a.codes + off) = 0u;
     }
-    for (int ch = threadIdx.x; ch < a.n_chunks; ch += kWThreads) {
+    for (int ch = lane; ch < a.n_chunks; ch += 32) {
       const size_t e = ((static_cast<size_t>(tile) * a.n_chunks + ch) * 128 + r) * 2;
       a.e8m0[e] = 127;
       a.e8m0[e + 1] = 127;
     }
-    if (threadIdx.x == 0) {
+    if (lane == 0) {
       a.scale[p] = 1.f;
       a.zero[p] = 0;
     }
@@ -247,13 +241,13 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
   const int f = a.fmtp[p];
   const __half* row = a.W + static_cast<size_t>(c) * a.K;
   const int nvec = a.K / 8;
-  const ChanStats st = row_stats(row, nvec, shf);
+  const ChanStats st = row_stats(row, nvec, lane);
   const ChanScale cs = chan_scale(f, st);
   const bool mx = w_is_mx(f);
-  const int iters = (nvec_p + kWThreads - 1) / kWThreads;
+  const int iters = (nvec_p + 31) / 32;
   bool range_ok = true;
   for (int it = 0; it < iters; ++it) {
-    const int v = it * kWThreads + threadIdx.x;
+    const int v = it * 32 + lane;
     float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     if (v < nvec) load8(row, v, x);
     int code[8];
@@ -308,14 +302,14 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
       }
       *reinterpret_cast<uint32_t*>(a.codes + off) = w;
     }
-    if ((threadIdx.x & 3) == 0) {  // one E8M0 byte per 32-element block
+    if ((lane & 3) == 0) {  // one E8M0 byte per 32-element block
       const int k0 = v * 8;
       const size_t e = ((static_cast<size_t>(tile) * a.n_chunks + (k0 >> 6)) * 128 + r) * 2 + ((k0 & 63) >> 5);
       a.e8m0[e] = mx ? static_cast<uint8_t>(X + 127) : 127;
     }
   }
   if (mx && !range_ok) set_status(a.dev_status, CHAM_ERR_RANGE);
-  if (threadIdx.x == 0) {
+  if (lane == 0) {
     a.scale[p] = mx ? 1.f : cs.s;
     a.zero[p] = static_cast<uint8_t>(cs.z);
   }
@@ -323,7 +317,7 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
 
 void launch_pack(const PackArgs& a, const NF4Table& nf4, cudaStream_t st) {
   k_w_slots<<<1, 1024, 0, st>>>(a);
-  k_w_pack<<<a.n_packed, kWThreads, 0, st>>>(a, nf4);
+  k_w_pack<<<(a.n_packed + kWWarps - 1) / kWWarps, kWThreads, 0, st>>>(a, nf4);
 }
 
 }  // namespace cham
