@@ -192,26 +192,29 @@ def main():
     fmt_off = np.cumsum([0] + [N for (_, M, K, N) in layers])
     fmt_all = torch.empty(int(fmt_off[-1]), dtype=torch.uint8, device=device)
 
+    # the W8 palette's formats share one MMA class, so the packed layout follows from N, K and
+    # the palette: selection and pack need no host round trip and run inside the step's graph
+    for li, (_, M, K, N) in enumerate(layers):
+        descs[li] = cl.pack_plan_palette(N, K, cl.PALETTE_W8)
+        blobs[li] = torch.empty(descs[li].bytes, dtype=torch.uint8, device=device)
+
     def select_pack():
-        """a5 + a6 for every layer: GPU selection, host plan from the selected formats (one
-        device->host copy of N bytes per layer), GPU pack into the layer's blob."""
-        fmts = [cl.select_weight_formats(W[li], cl.PALETTE_W8, fmt_out=fmt_all[fmt_off[li]:fmt_off[li + 1]])[0]
-                for li in range(len(layers))]
-        every = fmt_all.cpu().numpy()     # one device->host copy for all layers
-        fmts_host = [every[fmt_off[li]:fmt_off[li + 1]] for li in range(len(layers))]
-        for li, (_, M, K, N) in enumerate(layers):
-            d = cl.pack_plan(N, K, fmts_host[li])
-            if descs[li] is not None and bytes(d) != bytes(descs[li]):
-                raise RuntimeError("packed layout changed between steps")
-            blobs[li], _ = cl.pack_weights(W[li], fmts[li], d, dev_status=st, blob=blobs[li])
-            descs[li] = d
+        """a5 + a6 for every layer: GPU selection into the layer's slice of one format buffer,
+        GPU pack into the layer's blob."""
+        for li in range(len(layers)):
+            f = fmt_all[fmt_off[li]:fmt_off[li + 1]]
+            cl.select_weight_formats(W[li], cl.PALETTE_W8, fmt_out=f)
+            cl.pack_weights(W[li], f, descs[li], dev_status=st, blob=blobs[li])
 
     flops_step = nb * sum(layer_flops(M, K, N) for (_, M, K, N) in layers)
     quant_bytes_step = 0.0
     gemm_bytes_step = 0.0
 
-    def run_step(parts="qg"):
-        """a2-a4 + a7 for every (bucket, layer): act-quant in F[l, b] ("q"), then the GEMM ("g")."""
+    def run_step(parts="wqg"):
+        """a5 + a6 for every layer ("w"), then a2-a4 + a7 for every (bucket, layer): act-quant in
+        F[l, b] ("q") and the GEMM ("g")."""
+        if "w" in parts:
+            select_pack()
         for bk in range(nb):
             for li, (_, M, K, N) in enumerate(layers):
                 f = int(lut[li, bk])
@@ -220,25 +223,22 @@ def main():
                 if "g" in parts:
                     cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
 
-    # warm-up (eager), then capture the quantize + GEMM sequence of one step in a CUDA graph (no
-    # event nodes inside: each costs about 5 us of serialisation), plus two graphs holding only
-    # the quantizer launches and only the GEMM launches of the step, which time those kernel
-    # classes; select + pack stay eager (they need a host plan)
+    # warm-up (eager), then capture one whole step in a CUDA graph (no event nodes inside: each
+    # costs about 5 us of serialisation), plus graphs holding only the selection + pack, only the
+    # quantizer and only the GEMM launches of the step, which time those kernel classes
     for _ in range(args.warmup):
-        select_pack()
         run_step()
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
     graphs = {}
     try:
-        for key in ("qg", "q", "g"):
+        for key in ("wqg", "w", "q", "g"):
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
                 run_step(key)
             graphs[key] = g
         for _ in range(args.warmup):
-            select_pack()
-            graphs["qg"].replay()
+            graphs["wqg"].replay()
         torch.cuda.synchronize()
     except RuntimeError as exc:  # a launch that cannot be captured: time eager launches
         print("bench: CUDA-graph capture failed (%s); timing eager launches" % exc, file=sys.stderr)
@@ -269,14 +269,13 @@ def main():
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record(stream)
         for k in range(args.steps):
-            select_pack()                 # its host plan waits for the previous step's graph
-            replay("qg")
+            replay("wqg")
         t1.record(stream)
         torch.cuda.synchronize()
         # kernel classes, each alone: the step's 100 quantizer (or GEMM) launches back to back,
         # replayed as many times as the timed steps, two events around them
         class_ms = {}
-        for key in ("g", "q"):
+        for key in ("g", "q", "w"):
             e0 = torch.cuda.Event(enable_timing=True)
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record(stream)
@@ -285,7 +284,7 @@ def main():
             e1.record(stream)
             torch.cuda.synchronize()
             class_ms[key] = e0.elapsed_time(e1)
-    gemm_ms, quant_ms = class_ms["g"], class_ms["q"]
+    gemm_ms, quant_ms, weights_ms = class_ms["g"], class_ms["q"], class_ms["w"]
     n_linear = nb * len(layers)
     if world > 1:
         dist.barrier()
@@ -320,7 +319,7 @@ def main():
                    "layers": len(layers), "buckets": nb, "global_batch": 2 * world,
                    "tokens": [M for (_, M, _, _) in layers], "weight_palette": "W8 {INT8-sym, INT8-asym, MXINT8}",
                    "activation_formats_used": sorted(set(int(v) for v in lut.ravel())),
-                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant + GEMM",
+                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant + GEMM, one CUDA graph",
                    "l2": "inputs larger than L2 (%.0f MB of activations per step)" %
                          (sum(x.numel() * 2 for xs in X for x in xs) / 1e6),
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
@@ -334,10 +333,12 @@ def main():
                      "gemm_launch_ms_mean": round(gemm_ms / (args.steps * n_linear), 5),
                      "probe_tflops": probe,
                      "frac_of_probe_f16": round(gemm_tflops / probe["f16"], 4) if probe else None,
-                     "timing": ("value: CUDA-graph replay of each step's quantize+GEMM sequence, no event "
-                                "nodes inside; kernel classes: the step's GEMM (quantizer) launches alone, "
-                                "graph-replayed once per timed step between two events")
+                     "timing": ("value: one CUDA-graph replay per step (selection, pack, quantizer, GEMM), "
+                                "no event nodes inside; kernel classes: the step's GEMM (quantizer, "
+                                "selection + pack) launches alone, graph-replayed once per timed step "
+                                "between two events")
                                if graphs else "eager launches"},
+        "weights_select_pack_ms_per_step": round(weights_ms / K_, 4),
         "act_quant": {"achieved_gbs": round(quant_gbs, 1), "peak_gbs": pk["hbm_gbs"],
                       "frac": round(quant_gbs / pk["hbm_gbs"], 4), "ms_per_step": round(quant_ms / K_, 4),
                       "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"},
@@ -376,21 +377,18 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
                           for f in range(6)), dtype=torch.uint8, device=device) for (_, M, K, N) in layers]
     fmt_off = np.cumsum([0] + [N for (_, M, K, N) in layers])
     fmt_all = torch.empty(int(fmt_off[-1]), dtype=torch.uint8, device=device)
+    descs = [cl.pack_plan_palette(N, K, cl.PALETTE_W8) for (_, M, K, N) in layers]
+    blobs = [torch.empty(d.bytes, dtype=torch.uint8, device=device) for d in descs]
     h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + sum(x.numel() * 2 for xs in Xh for x in xs)
     d2h = nb * sum(M * N * 4 for (_, M, K, N) in layers)
 
     def step():
-        fmts, descs, blobs = [], [], []
         for li in range(len(layers)):
             Wd[li].copy_(Wh[li], non_blocking=True)
             bd[li].copy_(bh[li], non_blocking=True)
-            fmts.append(cl.select_weight_formats(Wd[li], cl.PALETTE_W8,
-                                                 fmt_out=fmt_all[fmt_off[li]:fmt_off[li + 1]])[0])
-        every = fmt_all.cpu().numpy()
-        for li, (_, M, K, N) in enumerate(layers):
-            d = cl.pack_plan(N, K, every[fmt_off[li]:fmt_off[li + 1]])
-            descs.append(d)
-            blobs.append(cl.pack_weights(Wd[li], fmts[li], d, dev_status=st)[0])
+            f = fmt_all[fmt_off[li]:fmt_off[li + 1]]
+            cl.select_weight_formats(Wd[li], cl.PALETTE_W8, fmt_out=f)
+            cl.pack_weights(Wd[li], f, descs[li], dev_status=st, blob=blobs[li])
         for bk in range(nb):
             for li in range(len(layers)):
                 Xd[li].copy_(Xh[li][bk], non_blocking=True)

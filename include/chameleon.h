@@ -181,6 +181,15 @@ typedef struct {
  * bit width).  desc->bytes is the blob size. */
 cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* desc);
 
+/* The same plan from the palette alone, for palettes whose members all share one MMA class (every
+ * 8-bit palette; 4-bit palettes without NF4, or NF4 alone): the layout then depends only on N, K
+ * and the bit width, so the selected formats need not be copied to the host and selection, pack
+ * and the linear calls can run back to back on the stream (Sec. 5's permutation is the identity
+ * up to padding).  desc->n_fmt[f] is -1 for every member (counts unknown on the host).  Returns
+ * CHAM_ERR_UNSUPPORTED for a palette that spans both classes; CHAM_ERR_INVALID_ARG for an empty
+ * mask, bits outside the 9 formats, mixed bit widths, or N, K <= 0 / K % 32 != 0.  Host-only. */
+cham_status chameleon_pack_plan_palette(int N, int K, uint32_t palette_mask, cham_wpack_desc* desc);
+
 /* Encode W (device, fp16 N x K) with each channel in fmt_dev[c] (device copy of the formats the
  * plan was made from) into blob (device, >= desc->bytes).  An MX channel whose dequantized values
  * are not all exact fp16 values sets *dev_status = CHAM_ERR_RANGE. */

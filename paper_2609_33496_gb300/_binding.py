@@ -28,7 +28,7 @@ EXPORTS = [
     "chameleon_bucket", "chameleon_snr", "chameleon_kurtosis", "chameleon_route",
     "chameleon_act_moments_workspace_size", "chameleon_act_moments",
     "chameleon_act_quant_size", "chameleon_act_quant",
-    "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_weights",
+    "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_plan_palette", "chameleon_pack_weights",
     "chameleon_linear_workspace_size", "chameleon_linear", "chameleon_linear_prepare",
     "chameleon_linear_gemm", "chameleon_act_quant_noalloc",
 ]
@@ -90,6 +90,7 @@ def lib():
         "chameleon_act_quant": (i32, [vp, i32, i32, i32, vp, sz, vp, sz, vp, vp]),
         "chameleon_select_weight_formats": (i32, [vp, i32, i32, u32, vp, vp, vp]),
         "chameleon_pack_plan": (i32, [i32, i32, vp, pdesc]),
+        "chameleon_pack_plan_palette": (i32, [i32, i32, ctypes.c_uint32, pdesc]),
         "chameleon_pack_weights": (i32, [vp, vp, pdesc, vp, sz, vp, vp]),
         "chameleon_linear_workspace_size": (i32, [i32, pdesc, i32, psz]),
         "chameleon_linear": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
@@ -210,6 +211,12 @@ def select_weight_formats(W, palette_mask, want_sse=False, stream=None, fmt_out=
 
 
 # ------------------------------------------------------------------ a6
+def pack_plan_palette(N, K, palette_mask):
+    d = WPackDesc()
+    check(lib().chameleon_pack_plan_palette(N, K, palette_mask, ctypes.byref(d)))
+    return d
+
+
 def pack_plan(N, K, fmt_host):
     f = np.ascontiguousarray(np.asarray(fmt_host, dtype=np.uint8))
     d = WPackDesc()

@@ -349,6 +349,12 @@ cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_
 }
 
 // ---------------------------------------------------------------- a6
+}  // extern "C"
+namespace {
+void finish_plan(cham_wpack_desc* d, int N, int K, int bits);
+}  // namespace
+extern "C" {
+
 cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* d) {
   if (N <= 0 || K <= 0 || K % 32 != 0 || fmt_host == nullptr || d == nullptr)
     return fail(CHAM_ERR_INVALID_ARG, "N=%d K=%d (K must be a multiple of 32)", N, K);
@@ -362,17 +368,47 @@ cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpac
     bits = b;
     d->n_fmt[f] += 1;
   }
+  for (int cls = 0; cls < 2; ++cls)
+    for (int j = 0; j < 5; ++j)
+      if (kClassOrder[cls][j] >= 0) d->n_class[cls] += d->n_fmt[kClassOrder[cls][j]];
+  finish_plan(d, N, K, bits);
+  return CHAM_OK;
+}
+
+// A plan from the palette alone: when every member shares one MMA class, the packed layout
+// depends only on N, K and the bit width (no device -> host copy of the selected formats).
+cham_status chameleon_pack_plan_palette(int N, int K, uint32_t palette_mask, cham_wpack_desc* d) {
+  if (N <= 0 || K <= 0 || K % 32 != 0 || d == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "N=%d K=%d (K must be a multiple of 32)", N, K);
+  if (palette_mask == 0 || (palette_mask & ~0x1FFu) != 0) return fail(CHAM_ERR_INVALID_ARG, "palette mask 0x%x", palette_mask);
+  int bits = 0, cls = -1;
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
+    if (!((palette_mask >> f) & 1u)) continue;
+    if (bits != 0 && cham::wbits(f) != bits) return fail(CHAM_ERR_INVALID_ARG, "palette mixes 8-bit and 4-bit formats");
+    bits = cham::wbits(f);
+    if (cls >= 0 && cham::w_class(f) != cls)
+      return fail(CHAM_ERR_UNSUPPORTED, "palette 0x%x spans both MMA classes: plan from the selected formats", palette_mask);
+    cls = cham::w_class(f);
+  }
+  std::memset(d, 0, sizeof(*d));
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f)
+    if ((palette_mask >> f) & 1u) d->n_fmt[f] = -1;  // per-format counts are not known on the host
+  d->n_class[cls] = N;
+  finish_plan(d, N, K, bits);
+  return CHAM_OK;
+}
+
+}  // extern "C"
+
+namespace {
+void finish_plan(cham_wpack_desc* d, int N, int K, int bits) {
   d->magic = 0x574D4843u;
   d->version = 1;
   d->N = N;
   d->K = K;
   d->Kp = static_cast<int>(round_up(K, 64));
   d->bits = bits;
-  for (int cls = 0; cls < 2; ++cls) {
-    for (int j = 0; j < 5; ++j)
-      if (kClassOrder[cls][j] >= 0) d->n_class[cls] += d->n_fmt[kClassOrder[cls][j]];
-    d->n_tiles[cls] = (d->n_class[cls] + 127) / 128;
-  }
+  for (int cls = 0; cls < 2; ++cls) d->n_tiles[cls] = (d->n_class[cls] + 127) / 128;
   const size_t tiles = static_cast<size_t>(d->n_tiles[0] + d->n_tiles[1]);
   const size_t np = tiles * 128, chunks = d->Kp / 64;
   size_t off = 256;
@@ -389,10 +425,8 @@ cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpac
   d->off_perm = off;
   off = round_up(off + np * 4, 256);
   d->bytes = off;
-  return CHAM_OK;
 }
-
-}  // extern "C"
+}  // namespace
 
 namespace cham {
 __global__ void k_write_desc(cham_wpack_desc d, cham_wpack_desc* out) {

@@ -75,6 +75,30 @@ def test_pack_plan_layout(cl):
     assert d.off_scale - d.off_codes >= 3 * 5 * 128 * 32
 
 
+def test_pack_plan_palette_matches_format_plan(cl):
+    """A one-class palette gives the layout the selected formats would give, whatever they are."""
+    rng = np.random.default_rng(5)
+    fields = lambda d: (d.N, d.K, d.Kp, d.bits, list(d.n_class), list(d.n_tiles), d.off_codes, d.off_scale,
+                        d.off_zero, d.off_e8m0, d.off_fmt, d.off_perm, d.bytes)
+    cases = [(cl.PALETTE_W8, [F.W_INT8_SYM, F.W_INT8_ASYM, F.W_MXINT8], 300, 320),
+             ((1 << F.W_INT4_ASYM) | (1 << F.W_E2M1) | (1 << F.W_MXINT4) | (1 << F.W_MXFP4),
+              [F.W_INT4_ASYM, F.W_E2M1, F.W_MXINT4, F.W_MXFP4], 129, 96),
+             (1 << F.W_NF4, [F.W_NF4], 1, 32)]
+    for mask, members, N, K in cases:
+        dp = cl.pack_plan_palette(N, K, mask)
+        for _ in range(3):
+            fmt = np.asarray(members, np.uint8)[rng.integers(0, len(members), N)]
+            assert fields(dp) == fields(cl.pack_plan(N, K, fmt))
+        assert [dp.n_fmt[f] for f in members] == [-1] * len(members)
+    with pytest.raises(cl.ChameleonError) as e:
+        cl.pack_plan_palette(64, 64, cl.PALETTE_W4)                # NF4 with class-0 formats
+    assert e.value.status == cl.ERR_UNSUPPORTED
+    for bad in (0, 0x200, 0x009):                                  # empty, out of range, mixed widths
+        with pytest.raises(cl.ChameleonError) as e:
+            cl.pack_plan_palette(64, 64, bad)
+        assert e.value.status == cl.ERR_INVALID_ARG
+
+
 def test_host_validation_errors(cl):
     with pytest.raises(cl.ChameleonError) as e:
         cl.pack_plan(4, 320, np.array([0, 0, 3, 3], np.uint8))     # mixed bit widths

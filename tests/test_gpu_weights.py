@@ -97,3 +97,31 @@ def test_pack_permutation_groups_classes(cl):
     assert keys == sorted(keys)                      # class 0 first, original order inside a class
     class1_first = min(g["slot"] for g in got.values() if g["fmt"] == F.W_NF4)
     assert class1_first == 128 * desc["n_tiles"][0]
+
+
+@pytest.mark.parametrize("mask,K", [(0x007, 320), ((1 << F.W_INT4_ASYM) | (1 << F.W_E2M1) | (1 << F.W_MXINT4) | (1 << F.W_MXFP4), 96)])
+def test_palette_plan_packs_the_same_blob(cl, mask, K):
+    """A blob packed from the palette-only plan equals the one packed from the host plan of the
+    selected formats, except for the per-format counts in its header copy."""
+    import torch
+    W = WL.weight_mix(np.random.default_rng(11), 260, K)
+    Wd = cuda(W)
+    fmt, _ = cl.select_weight_formats(Wd, mask)
+    d_host = cl.pack_plan(W.shape[0], K, host(fmt))
+    d_pal = cl.pack_plan_palette(W.shape[0], K, mask)
+    assert d_host.bytes == d_pal.bytes
+    b_host, st1 = cl.pack_weights(Wd, fmt, d_host)
+    b_pal, st2 = cl.pack_weights(Wd, fmt, d_pal)
+    torch.cuda.synchronize()
+    assert int(st1.item()) == 0 and int(st2.item()) == 0
+    a, b = host(b_host), host(b_pal)
+    d = d_host
+    tiles = d.n_tiles[0] + d.n_tiles[1]
+    np_, chunks, cb = 128 * tiles, d.Kp // 64, 64 if d.bits == 8 else 32
+    regions = [(d.off_codes, tiles * chunks * 128 * cb), (d.off_scale, 4 * np_), (d.off_zero, np_),
+               (d.off_e8m0, tiles * chunks * 256), (d.off_fmt, np_), (d.off_perm, 4 * np_)]
+    for off, n in regions:                             # the bytes the pack defines (gaps are not written)
+        assert np.array_equal(a[off:off + n], b[off:off + n]), off
+    assert np.array_equal(a[:40], b[:40]) and np.array_equal(a[76:256], b[76:256])
+    n_fmt = slice(40, 40 + 4 * 9)                      # int32 n_fmt[9] in the descriptor copy
+    assert np.all(b[n_fmt].view(np.int32)[[f for f in range(9) if (mask >> f) & 1]] == -1)
