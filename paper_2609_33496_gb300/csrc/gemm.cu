@@ -53,7 +53,9 @@ struct GemmCfg {
   static constexpr int kDone = 8;                                 // group-completion barriers
   static constexpr int kNeedCols = kACol + kAStages * 32;
   static constexpr int kTmemCols = kNeedCols <= 256 ? 256 : 512;
-  static constexpr int kMisc = 1024 /*NF4 pair table*/ + 8 * (kStages + kDone + 2 + 4) + 16;
+  // NF4 pair table, then the mbarriers (full[S], done[kDone], afull[kAStages / kGroup],
+  // accfull[2], accempty[2]), the TMEM address slot and the abort flag
+  static constexpr int kMisc = 1024 + 8 * (kStages + kDone + kAStages / kGroup + 4) + 16;
   static constexpr int kNeed = 1024 /*alignment slack*/ + kData + kMisc;
   // at least 116 KiB so that two CTAs (and two tensor-memory allocations) never share an SM
   static constexpr int kSmem = kNeed > 116 * 1024 ? kNeed : 116 * 1024;
