@@ -121,6 +121,7 @@ constexpr uint32_t kWaitPolls = 1u << 22;  // polls of the drain waits (mbar_tes
 // CHAM_ERR_TIMEOUT and raising the CTA's abort flag) when the limit is reached or another
 // thread of the CTA has already aborted.
 CHAM_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* dev_status) {
+  if (mbar_ready(bar, parity)) return true;  // an already-completed phase costs no suspend / resume
   for (uint32_t i = 0; i < kWaitRounds; ++i) {
     if (mbar_try_wait_for(bar, parity, kWaitRoundNs)) return true;
     if (*abort_flag) return false;

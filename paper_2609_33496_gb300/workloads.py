@@ -90,3 +90,25 @@ def weight_mix(g, N, K, scale=0.02):
             idx = g.choice(K, max(1, K // 64), replace=False)
             W[n, idx] *= 12.0
     return to_fp16(W)
+
+
+# Representative layer shapes (M, K, N) of the wider workloads, batch 2 unless stated:
+# * SDXL UNet step at 1024^2 (latent 128^2): time embedding (M = 2), text cross-attention K/V
+#   (M = 2 x 77), the 1280-wide transformer stage, a 640-wide 1x1 conv and the 32768-token stage;
+# * PixArt-alpha DiT (hidden 1152, MLP 4608, 4096 tokens, 120 caption tokens);
+# * SDXL-Turbo weight-only at batch 1 / 8 / 16: M = b, 77 b and b x HW rows.
+UNET_W4A8_SHAPES = ((2, 320, 1280), (154, 2048, 1280), (2048, 5120, 1280), (8192, 1920, 640),
+                    (32768, 960, 320))
+PIXART_W4A8_SHAPES = ((240, 1152, 1152), (8192, 1152, 4608), (8192, 4608, 1152), (240, 4096, 1152))
+TURBO_W4A16_SHAPES = ((1, 320, 1280), (16, 1280, 1280), (616, 2048, 640), (8192, 640, 640))
+
+
+def config_layer(config, index, M, K, N, nu=7):
+    """X fp16 M x K = StudentT(nu) * c_k (config 2's mid-bucket distribution with channel
+    jitter), weights with per-channel distribution diversity, bias N(0, 0.02^2)."""
+    g = rng(config, index)
+    c = channel_jitter(g, K)
+    X = to_fp16(student_t(g, nu, (M, K)) * c[None, :])
+    W = weight_mix(g, N, K)
+    bias = g.normal(0.0, 0.02, N).astype(np.float32)
+    return X, W, bias

@@ -102,3 +102,27 @@ def test_full_size_sdxl_projection_sampled_rows(cl, layer):
         w = SEL.dequant_selected(W, fmt)
         y_ref, bound = G.linear_rows_reference(a, w, rows, bias)
         assert_within_bound(Y[rows], y_ref, bound, "%s bucket %d" % (name, bucket))
+
+
+W4_TURBO = (1 << F.W_INT4_ASYM) | (1 << F.W_NF4) | (1 << F.W_E2M1) | (1 << F.W_MXINT4) | (1 << F.W_MXFP4)
+WIDE_CASES = ([(3, i, shp, [F.A_E4M3, F.A_E5M2]) for i, shp in enumerate(WL.UNET_W4A8_SHAPES)]
+              + [(4, i, shp, [F.A_E4M3, F.A_MXFP8]) for i, shp in enumerate(WL.PIXART_W4A8_SHAPES)]
+              + [(5, i, shp, [F.A_FP16]) for i, shp in enumerate(WL.TURBO_W4A16_SHAPES)])
+
+
+@pytest.mark.parametrize("config,index,shape,act_fmts", WIDE_CASES)
+def test_wider_workload_shapes_sampled_rows(cl, config, index, shape, act_fmts):
+    """SDXL-UNet and PixArt-alpha W4A8 layers and SDXL-Turbo W4A16 layers (M from 1 to 32768)
+    with the 4-bit palette of those workloads selected on the GPU; the fp64 reference is computed
+    on up to 64 seeded rows."""
+    M, K, N = shape
+    X, W, bias = WL.config_layer(config, index, M, K, N)
+    fmt_dev, _ = cl.select_weight_formats(cuda(W), W4_TURBO)
+    fmt = host(fmt_dev)
+    w = SEL.dequant_selected(W, fmt)
+    rows = np.arange(M) if M <= 64 else np.sort(np.random.default_rng(index).choice(M, 64, replace=False))
+    for act_fmt in act_fmts:
+        Y = gpu_linear(cl, X, W, fmt, act_fmt, bias)
+        a = X.astype(np.float64) if act_fmt == F.A_FP16 else F.act_dequant(F.act_quant(X, act_fmt))
+        y_ref, bound = G.linear_rows_reference(a, w, rows, bias)
+        assert_within_bound(Y[rows], y_ref, bound, "config %d %s act %d" % (config, shape, act_fmt))
