@@ -153,9 +153,9 @@ cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_
  *                  128 x 16 bytes: slab j holds bytes [16j, 16j+16) of every channel's CB bytes.
  *                  8-bit: byte i = element i of the chunk (offset binary q + 128 for INT8-sym
  *                  and MXINT8, uint8 q for INT8-asym).  4-bit: each 32-bit word holds 8 elements
- *                  e0..e7, nibble j (bits 4j..4j+3) = e_{2j} for j < 4 and e_{2(j-4)+1} for j >= 4;
- *                  INT4-sym/MXINT4 offset binary q + 8, INT4-asym q, NF4 level index, E2M1/MXFP4
- *                  bit pattern.  Elements k >= K hold the code of the value 0.  (Offset binary
+ *                  e0..e7, nibble j (bits 4j..4j+3) = e_{2j} for j < 4 and e_{2(j-4)+1} for j >= 4
+ *                  (NF4 channels: nibble j = e_j); INT4-sym/MXINT4 offset binary q + 8, INT4-asym
+ *                  q, NF4 level index, E2M1/MXFP4 bit pattern.  Elements k >= K hold the code of the value 0.  (Offset binary
  *                  lets the GEMM turn a code into its fp16 value with one byte permute and one
  *                  subtraction.)
  *   scale          float [Np]: per-channel scale s (1 for MX and padding)

@@ -550,7 +550,13 @@ cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d
   g.bits = d->bits;
   g.dev_status = dev_status;
   const cham::NF4Table& nf4 = nf4_table();
-  for (int i = 0; i < 16; ++i) g.nf4_level[i] = nf4.level[i];
+  for (int r = 0; r < 4; ++r) {
+    g.nf4_lo[r] = g.nf4_hi[r] = 0;
+    for (int k = 0; k < 4; ++k) {
+      g.nf4_lo[r] |= static_cast<uint32_t>(nf4.level[4 * r + k] & 0xFFu) << (8 * k);
+      g.nf4_hi[r] |= static_cast<uint32_t>(nf4.level[4 * r + k] >> 8) << (8 * k);
+    }
+  }
   const int num_sms = num_sms_current();
   const int tiles = d->n_tiles[0] + d->n_tiles[1];
   const int bn = cham::gemm_pick_bn(M, tiles, num_sms);

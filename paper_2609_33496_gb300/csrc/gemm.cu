@@ -53,9 +53,9 @@ struct GemmCfg {
   static constexpr int kDone = 8;                                 // group-completion barriers
   static constexpr int kNeedCols = kACol + kAStages * 32;
   static constexpr int kTmemCols = kNeedCols <= 256 ? 256 : 512;
-  // NF4 pair table, then the mbarriers (full[S], done[kDone], afull[kAStages / kGroup],
-  // accfull[2], accempty[2]), the TMEM address slot and the abort flag
-  static constexpr int kMisc = 1024 + 8 * (kStages + kDone + kAStages / kGroup + 4) + 16;
+  // the mbarriers (full[S], done[kDone], afull[kAStages / kGroup], accfull[2], accempty[2]),
+  // the TMEM address slot and the abort flag
+  static constexpr int kMisc = 8 * (kStages + kDone + kAStages / kGroup + 4) + 16;
   static constexpr int kNeed = 1024 /*alignment slack*/ + kData + kMisc;
   // at least 116 KiB so that two CTAs (and two tensor-memory allocations) never share an SM
   static constexpr int kSmem = kNeed > 116 * 1024 ? kNeed : 116 * 1024;
@@ -176,8 +176,26 @@ CHAM_DEV void decode_w8(const uint32_t (&w)[16], const ChanDecode& c, uint32_t e
 // 4-bit codes -> 32 fp16 pairs.  Word i holds elements 8i..8i+7 with nibble j = element 2j and
 // nibble 4+j = element 2j+1, so a mask of 0x000F000F << 4j isolates a pair.  The lanes of a warp
 // hold channels of different formats: every warp vote is taken before the per-format branches.
-CHAM_DEV void decode_w4(const uint32_t (&w)[8], const ChanDecode& c, uint32_t e8, const uint32_t* lut,
-                        uint32_t (&out)[32]) {
+CHAM_DEV uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));  // selector bit 3: sign replicate
+  return d;
+}
+
+// Four NF4 level indices (nibbles of the low 16 bits of h, element order) -> two fp16 pairs, from
+// byte tables in registers: PRMT picks the low and the high byte of each level among entries
+// 0..7 and 8..15, and a per-byte mask built from each index's bit 3 chooses between the two.
+CHAM_DEV void nf4_lookup4(uint32_t h, const uint32_t (&lo)[4], const uint32_t (&hi)[4], uint32_t& p01, uint32_t& p23) {
+  const uint32_t sel = h & 0x7777u;
+  const uint32_t m = prmt(h << 4, h, 0xD9C8u);  // byte k = 0xFF where index k >= 8
+  const uint32_t l = (prmt(lo[0], lo[1], sel) & ~m) | (prmt(lo[2], lo[3], sel) & m);
+  const uint32_t u = (prmt(hi[0], hi[1], sel) & ~m) | (prmt(hi[2], hi[3], sel) & m);
+  p01 = prmt(l, u, 0x5140u);
+  p23 = prmt(l, u, 0x7362u);
+}
+
+CHAM_DEV void decode_w4(const uint32_t (&w)[8], const ChanDecode& c, uint32_t e8, const uint32_t (&nlo)[4],
+                        const uint32_t (&nhi)[4], uint32_t (&out)[32]) {
   const int e0 = block_exp(c, e8, 0), e1 = block_exp(c, e8, 1);
   const bool is_nf4 = c.f == CHAM_W_NF4;
   const bool is_fp4 = c.f == CHAM_W_E2M1 || c.f == CHAM_W_MXFP4;
@@ -194,11 +212,13 @@ CHAM_DEV void decode_w4(const uint32_t (&w)[8], const ChanDecode& c, uint32_t e8
   const bool all_int_fast = __all_sync(0xffffffffu, is_nf4 || is_fp4 || int_fast);
   const bool all_fp4_fast = __all_sync(0xffffffffu, !is_fp4 || fp4_fast);
   if (is_nf4) {
-    // level table of nibble pairs (per-channel scale in the epilogue)
+    // NF4 codes are stored in element order (nibble j of word i = element 8i + j); levels from
+    // the register tables (per-channel scale in the epilogue)
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) out[4 * i + j] = lut[((w[i] >> (4 * j)) & 0xFu) | ((w[i] >> (4 * j + 12)) & 0xF0u)];
+    for (int i = 0; i < 8; ++i) {
+      nf4_lookup4(w[i] & 0xFFFFu, nlo, nhi, out[4 * i], out[4 * i + 1]);
+      nf4_lookup4(w[i] >> 16, nlo, nhi, out[4 * i + 2], out[4 * i + 3]);
+    }
   } else if (is_fp4) {
     if (all_fp4_fast) {
 #pragma unroll
@@ -261,11 +281,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   using C = GemmCfg<BN, BITS>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint32_t* lut = reinterpret_cast<uint32_t*>(smem + C::kData);
+  uint32_t* misc = reinterpret_cast<uint32_t*>(smem + C::kData);
   constexpr int S = C::kStages;
   constexpr int kAStages = C::kAStages, kGroup = C::kGroup, kAGroups = kAStages / kGroup;
   constexpr int kDone = C::kDone;
-  uint64_t* full = reinterpret_cast<uint64_t*>(lut + 256);  // [S] producer -> decoders, MMA (tx bytes)
+  uint64_t* full = reinterpret_cast<uint64_t*>(misc);       // [S] producer -> decoders, MMA (tx bytes)
   uint64_t* done = full + S;                                 // [kDone] MMA group commit -> producer, decoders
   uint64_t* afull = done + kDone;                            // [kAGroups] decode warps -> MMA
   uint64_t* accfull = afull + kAGroups;                      // [2] MMA commit -> epilogue
@@ -299,8 +319,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
-  for (int i = threadIdx.x; i < 256; i += kGemmThreads)  // NF4 pair table (low half = even element)
-    lut[i] = static_cast<uint32_t>(a.nf4_level[i & 15]) | (static_cast<uint32_t>(a.nf4_level[i >> 4]) << 16);
   if (warp == 0 && lane == 0) tma_prefetch_desc(&act_map);
   if (warp == 2) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
@@ -430,7 +448,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           decode_w8(raw, cd, e8, out);
         } else {
           const uint32_t (&r8)[8] = *reinterpret_cast<const uint32_t(*)[8]>(&raw[0]);
-          decode_w4(r8, cd, e8, lut, out);
+          decode_w4(r8, cd, e8, a.nf4_lo, a.nf4_hi, out);
         }
         const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
         if (!__all_sync(0xffffffffu, free_ok)) {

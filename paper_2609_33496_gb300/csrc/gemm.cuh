@@ -22,7 +22,8 @@ struct GemmArgs {
   int n_ch_tiles;            // 128-channel tiles of this launch
   int bits;                  // 4 or 8
   int* dev_status;
-  uint16_t nf4_level[16];    // NF4 levels as fp16 bit patterns
+  uint32_t nf4_lo[4];        // NF4 levels as fp16: low bytes of levels 4r..4r+3 in word r
+  uint32_t nf4_hi[4];        // high bytes, same layout
 };
 
 // Token-tile (MMA N) size for M tokens: 16, 32, 64, 128 or 192.

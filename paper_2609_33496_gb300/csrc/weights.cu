@@ -293,12 +293,18 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
       }
       *reinterpret_cast<uint2*>(a.codes + off) = make_uint2(lo, hi);
     } else {
-      // nibble j (j < 4) = element 2j, nibble 4 + j = element 2j + 1
+      // nibble j (j < 4) = element 2j, nibble 4 + j = element 2j + 1 (the integer and E2M1 decodes
+      // isolate a pair with one mask); NF4: nibble j = element j (the register-table decode)
       uint32_t w = 0;
+      if (f == CHAM_W_NF4) {
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        w |= (static_cast<uint32_t>(code[2 * j]) & 0xFu) << (4 * j);
-        w |= (static_cast<uint32_t>(code[2 * j + 1]) & 0xFu) << (4 * (j + 4));
+        for (int j = 0; j < 8; ++j) w |= (static_cast<uint32_t>(code[j]) & 0xFu) << (4 * j);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          w |= (static_cast<uint32_t>(code[2 * j]) & 0xFu) << (4 * j);
+          w |= (static_cast<uint32_t>(code[2 * j + 1]) & 0xFu) << (4 * (j + 4));
+        }
       }
       *reinterpret_cast<uint32_t*>(a.codes + off) = w;
     }

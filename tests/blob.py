@@ -46,9 +46,13 @@ def unpack(blob_bytes):
             words = raw.view(np.uint32)
             vals = np.zeros(Kp, dtype=np.int64)
             nib = [(words >> (4 * j)) & 0xF for j in range(8)]
-            for j in range(4):
-                vals[2 * j::8] = nib[j]
-                vals[2 * j + 1::8] = nib[4 + j]
+            if int(fmt[p]) == 5:            # NF4: nibble j = element j
+                for j in range(8):
+                    vals[j::8] = nib[j]
+            else:
+                for j in range(4):
+                    vals[2 * j::8] = nib[j]
+                    vals[2 * j + 1::8] = nib[4 + j]
             vals = vals[:K]
         f = int(fmt[p])
         t, r = divmod(p, 128)
