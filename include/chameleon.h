@@ -221,6 +221,14 @@ cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d
                                   int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
                                   int* dev_status, void* stream);
 
+/* Test hook, not part of the method: the next chameleon_linear_gemm (or chameleon_linear) launch
+ * on this host thread's library instance has the producer of its first CTA withhold the copies of
+ * that CTA's K-chunk number `chunk` (0-based over its work), so the decoders' bounded wait for it
+ * runs out: the kernel records CHAM_ERR_TIMEOUT in the call's device status word, drains its own
+ * copies and MMAs, releases tensor memory and returns within a few seconds, leaving the context
+ * usable (the output of that call is undefined).  chunk = -1 cancels.  Host-only, no GPU work. */
+cham_status chameleon_debug_stall_next_gemm(int chunk);
+
 /* chameleon_act_quant without a caller-supplied workspace.  The paper has no counterpart: this
  * entry point exists for callers that cannot allocate device memory when they quantize -- code
  * embedded in a host application or inference runtime that owns every device buffer and hands

@@ -30,7 +30,7 @@ EXPORTS = [
     "chameleon_act_quant_size", "chameleon_act_quant",
     "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_plan_palette", "chameleon_pack_weights",
     "chameleon_linear_workspace_size", "chameleon_linear", "chameleon_linear_prepare",
-    "chameleon_linear_gemm", "chameleon_act_quant_noalloc",
+    "chameleon_linear_gemm", "chameleon_act_quant_noalloc", "chameleon_debug_stall_next_gemm",
 ]
 
 
@@ -97,6 +97,7 @@ def lib():
         "chameleon_linear_prepare": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
         "chameleon_linear_gemm": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
         "chameleon_act_quant_noalloc": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
+        "chameleon_debug_stall_next_gemm": (i32, [i32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -256,6 +257,11 @@ def linear(X, desc, blob, act_fmt, bias=None, Y=None, ws=None, dev_status=None, 
     check(lib().chameleon_linear(_ptr(X), M, ctypes.byref(desc), _ptr(blob), act_fmt, _ptr(bias), _ptr(Y),
                                  _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))
     return Y, dev_status
+
+
+def debug_stall_next_gemm(chunk):
+    """Test hook: the next GEMM launch withholds one K-chunk so its bounded waits run out."""
+    check(lib().chameleon_debug_stall_next_gemm(chunk))
 
 
 def linear_prepare(X, act_fmt, ws, dev_status, stream=None):

@@ -517,6 +517,16 @@ cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, v
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "linear_prepare launch");
 }
 
+namespace {
+int g_stall_next_gemm = -1;  // set by chameleon_debug_stall_next_gemm, consumed by the next launch
+}  // namespace
+
+cham_status chameleon_debug_stall_next_gemm(int chunk) {
+  if (chunk < -1) return fail(CHAM_ERR_INVALID_ARG, "chunk %d", chunk);
+  g_stall_next_gemm = chunk;
+  return CHAM_OK;
+}
+
 cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d, const void* blob, int act_fmt,
                                   const float* bias, float* Y, void* ws, size_t ws_bytes, int* dev_status,
                                   void* stream) {
@@ -548,6 +558,8 @@ cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d
   g.N = d->N;
   g.n_chunks = d->Kp / 64;
   g.bits = d->bits;
+  g.stall_chunk = g_stall_next_gemm;
+  g_stall_next_gemm = -1;
   g.dev_status = dev_status;
   const cham::NF4Table& nf4 = nf4_table();
   for (int r = 0; r < 4; ++r) {

@@ -70,18 +70,6 @@ CHAM_DEV void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
                "r"(bytes)
                : "memory");
 }
-CHAM_DEV bool mbar_test(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}\n"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
 // Non-blocking test of the phase with the given parity (returns at once; try_wait, by contrast,
 // costs a suspend/resume of a few hundred cycles even when the phase has already completed).
 CHAM_DEV bool mbar_ready(uint64_t* bar, uint32_t parity) {
@@ -115,7 +103,6 @@ CHAM_DEV bool mbar_try_wait_for(uint64_t* bar, uint32_t parity, uint32_t ns) {
 // legitimate wait in these kernels.
 constexpr uint32_t kWaitRounds = 2000;
 constexpr uint32_t kWaitRoundNs = 1000000;
-constexpr uint32_t kWaitPolls = 1u << 22;  // polls of the drain waits (mbar_test)
 
 // Wait for the phase with the given parity to complete.  Returns false (after recording
 // CHAM_ERR_TIMEOUT and raising the CTA's abort flag) when the limit is reached or another

@@ -21,6 +21,7 @@ struct GemmArgs {
   int tile0;                 // first 128-channel tile of this launch
   int n_ch_tiles;            // 128-channel tiles of this launch
   int bits;                  // 4 or 8
+  int stall_chunk;           // test hook: CTA 0's producer withholds this K-chunk's copies (-1: off)
   int* dev_status;
   uint32_t nf4_lo[4];        // NF4 levels as fp16: low bytes of levels 4r..4r+3 in word r
   uint32_t nf4_hi[4];        // high bytes, same layout
