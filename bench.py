@@ -97,6 +97,21 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+# ------------------------------------------------------------------ replicas (N > 1)
+def max_over_ranks(ms, device=None):
+    """The slowest rank's time: every rank gets the maximum (the job ends with its last rank)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tflops(flops_step, steps, world, max_ms):
+    """Whole-job throughput: every rank runs the full step (weak scaling, independent replicas)."""
+    return world * flops_step * steps / (max_ms * 1e-3) / 1e12
+
+
 # ------------------------------------------------------------------ workload
 def layer_flops(M, K, N):
     return 2.0 * M * K * N
@@ -290,13 +305,11 @@ def main():
         dist.barrier()
     elapsed_ms = t0.elapsed_time(t1)
     if world > 1:
-        tt = torch.tensor([elapsed_ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(tt.item())
+        elapsed_ms = max_over_ranks(elapsed_ms, device)
     assert int(st.item()) == 0, "device status %d" % int(st.item())
 
     K_ = args.steps
-    value = world * flops_step * K_ / (elapsed_ms * 1e-3) / 1e12
+    value = job_tflops(flops_step, K_, world, elapsed_ms)
     pk, pk_kind = peaks()
     peak_tensor = pk.get("bf16_tflops_sustained", pk.get("bf16_tflops"))
     gemm_tflops = flops_step * K_ / (gemm_ms * 1e-3) / 1e12
@@ -410,11 +423,9 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
     torch.cuda.synchronize()
     ms = t0.elapsed_time(t1)
     if world > 1:
-        tt = torch.tensor([ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+        ms = max_over_ranks(ms, device)
     assert int(st.item()) == 0
-    return {"value": round(world * flops_step * args.steps / (ms * 1e-3) / 1e12, 3), "unit": "TFLOP/s",
+    return {"value": round(job_tflops(flops_step, args.steps, world, ms), 3), "unit": "TFLOP/s",
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
             "ms_per_step": round(ms / args.steps, 3)}
 
