@@ -395,20 +395,48 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
     h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + sum(x.numel() * 2 for xs in Xh for x in xs)
     d2h = nb * sum(M * N * 4 for (_, M, K, N) in layers)
 
+    # three streams: host->device copies, the library calls, device->host copies; per-layer events
+    # keep each layer's input and output buffers from being overwritten while still in use, so
+    # one layer's upload and download overlap the other layers' compute
+    s_h2d, s_d2h = torch.cuda.Stream(device), torch.cuda.Stream(device)
+    ev = lambda: [torch.cuda.Event() for _ in layers]
+    x_ready, x_free, y_ready, y_free = ev(), ev(), ev(), ev()
+    w_ready = torch.cuda.Event()
+
     def step():
+        with torch.cuda.stream(s_h2d):
+            for li in range(len(layers)):
+                Wd[li].copy_(Wh[li], non_blocking=True)
+                bd[li].copy_(bh[li], non_blocking=True)
+            w_ready.record(s_h2d)
+        stream.wait_event(w_ready)
         for li in range(len(layers)):
-            Wd[li].copy_(Wh[li], non_blocking=True)
-            bd[li].copy_(bh[li], non_blocking=True)
             f = fmt_all[fmt_off[li]:fmt_off[li + 1]]
-            cl.select_weight_formats(Wd[li], cl.PALETTE_W8, fmt_out=f)
-            cl.pack_weights(Wd[li], f, descs[li], dev_status=st, blob=blobs[li])
+            cl.select_weight_formats(Wd[li], cl.PALETTE_W8, fmt_out=f, stream=stream)
+            cl.pack_weights(Wd[li], f, descs[li], dev_status=st, blob=blobs[li], stream=stream)
         for bk in range(nb):
             for li in range(len(layers)):
-                Xd[li].copy_(Xh[li][bk], non_blocking=True)
+                with torch.cuda.stream(s_h2d):
+                    s_h2d.wait_event(x_free[li])
+                    Xd[li].copy_(Xh[li][bk], non_blocking=True)
+                    x_ready[li].record(s_h2d)
+                stream.wait_event(x_ready[li])
+                stream.wait_event(y_free[li])
                 cl.linear(Xd[li], descs[li], blobs[li], int(lut[li, bk]), bias=bd[li], Y=Yd[li], ws=ws[li],
-                          dev_status=st)
-                Yh[li].copy_(Yd[li], non_blocking=True)
+                          dev_status=st, stream=stream)
+                x_free[li].record(stream)
+                y_ready[li].record(stream)
+                with torch.cuda.stream(s_d2h):
+                    s_d2h.wait_event(y_ready[li])
+                    Yh[li].copy_(Yd[li], non_blocking=True)
+                    y_free[li].record(s_d2h)
+        for li in range(len(layers)):      # the step ends when its last download has landed
+            stream.wait_event(y_free[li])
+        # the next step's weight upload must not overwrite weights still read by this step
+        s_h2d.wait_stream(stream)
 
+    for e in x_free + y_free:             # a fresh event: waiting on it is a no-op
+        e.record(stream)
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
