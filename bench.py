@@ -395,10 +395,11 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
     h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + sum(x.numel() * 2 for xs in Xh for x in xs)
     d2h = nb * sum(M * N * 4 for (_, M, K, N) in layers)
 
-    # three streams: host->device copies, the library calls, device->host copies; per-layer events
+    # streams for host->device copies, the library calls and (two) device->host copies; per-layer events
     # keep each layer's input and output buffers from being overwritten while still in use, so
     # one layer's upload and download overlap the other layers' compute
-    s_h2d, s_d2h = torch.cuda.Stream(device), torch.cuda.Stream(device)
+    s_h2d = torch.cuda.Stream(device)
+    s_d2h_all = [torch.cuda.Stream(device) for _ in range(2)]  # one download stream reached ~0.8x
     ev = lambda: [torch.cuda.Event() for _ in layers]
     x_ready, x_free, y_ready, y_free = ev(), ev(), ev(), ev()
     w_ready = torch.cuda.Event()
@@ -426,6 +427,7 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
                           dev_status=st, stream=stream)
                 x_free[li].record(stream)
                 y_ready[li].record(stream)
+                s_d2h = s_d2h_all[li % len(s_d2h_all)]
                 with torch.cuda.stream(s_d2h):
                     s_d2h.wait_event(y_ready[li])
                     Yh[li].copy_(Yd[li], non_blocking=True)
