@@ -266,9 +266,9 @@ def main():
         else:
             run_step(key)
 
-    # kernel launches per step: select 1 + pack 3 per layer; per linear 2 (per-tensor) or 1 (MX)
-    # quantizer kernels + 1 GEMM
-    launches = 4 * len(layers) + sum(
+    # kernel launches per step: select 1 + pack 1 per layer (one MMA class: no slot ranking);
+    # per linear 2 (per-tensor) or 1 (MX) quantizer kernels + 1 GEMM
+    launches = 2 * len(layers) + sum(
         (2 if lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(nb))
     for li, (_, M, K, N) in enumerate(layers):
         for bk in range(nb):

@@ -428,13 +428,6 @@ void finish_plan(cham_wpack_desc* d, int N, int K, int bits) {
 }
 }  // namespace
 
-namespace cham {
-__global__ void k_write_desc(cham_wpack_desc d, cham_wpack_desc* out) {
-  const uint32_t* src = reinterpret_cast<const uint32_t*>(&d);
-  uint32_t* dst = reinterpret_cast<uint32_t*>(out);
-  for (int i = threadIdx.x; i < 64; i += blockDim.x) dst[i] = src[i];
-}
-}  // namespace cham
 
 extern "C" {
 
@@ -468,7 +461,9 @@ cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const 
   a.fmtp = b + d->off_fmt;
   a.perm = reinterpret_cast<int32_t*>(b + d->off_perm);
   a.dev_status = dev_status;
-  cham::k_write_desc<<<1, 64, 0, st>>>(*d, reinterpret_cast<cham_wpack_desc*>(b));
+  a.one_class = d->n_class[0] == 0 ? 1 : (d->n_class[1] == 0 ? 0 : -1);
+  a.desc = *d;
+  a.desc_out = reinterpret_cast<cham_wpack_desc*>(b);
   cham::launch_pack(a, nf4_table(), st);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "pack launch");

@@ -215,10 +215,28 @@ CHAM_DEV size_t code_offset(int p, int k0, int n_chunks, int bits) {
 }
 
 __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) {
+  if (blockIdx.x == 0 && threadIdx.x < 64)  // the blob's header: a copy of the descriptor
+    reinterpret_cast<uint32_t*>(a.desc_out)[threadIdx.x] = reinterpret_cast<const uint32_t*>(&a.desc)[threadIdx.x];
   const int lane = threadIdx.x & 31;
   const int p = blockIdx.x * kWWarps + (threadIdx.x >> 5);  // one warp per packed slot
   if (p >= a.n_packed) return;
-  const int c = a.perm[p];
+  int c;
+  if (a.one_class >= 0) {
+    // one MMA class: slot p holds channel p - base in original order, the rest is padding
+    const int rank = p - a.cls_base[a.one_class];
+    c = (rank >= 0 && rank < a.cls_count[a.one_class]) ? rank : -1;
+    if (lane == 0) {
+      const int f = c >= 0 ? a.fmt_dev[c] : -1;
+      const bool valid = f >= 0 && f < CHAM_W_NFORMATS && w_class(f) == a.one_class;
+      if (c >= 0 && !valid) set_status(a.dev_status, CHAM_ERR_INVALID_ARG);  // formats must match the plan
+      a.perm[p] = c;
+      a.fmtp[p] = c >= 0 ? static_cast<uint8_t>(valid ? f : 0xFF) : static_cast<uint8_t>(0xFF);
+    }
+    __syncwarp();
+    if (c >= 0 && (a.fmtp[p] == 0xFF)) return;  // invalid format: nothing to encode
+  } else {
+    c = a.perm[p];
+  }
   const int nvec_p = a.Kp / 8;
   const int tile = p >> 7, r = p & 127;
   if (c < 0) {  // padding slot: zero codes, unit scale
@@ -322,7 +340,7 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
 }
 
 void launch_pack(const PackArgs& a, const NF4Table& nf4, cudaStream_t st) {
-  k_w_slots<<<1, 1024, 0, st>>>(a);
+  if (a.one_class < 0) k_w_slots<<<1, 1024, 0, st>>>(a);  // two classes: rank the channels of each
   k_w_pack<<<(a.n_packed + kWWarps - 1) / kWWarps, kWThreads, 0, st>>>(a, nf4);
 }
 

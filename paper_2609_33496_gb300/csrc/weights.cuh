@@ -157,6 +157,9 @@ struct PackArgs {
   int n_packed;             // Np
   int cls_base[2];          // first packed slot of each MMA class
   int cls_count[2];         // channels of each class (from the host plan)
+  int one_class;            // the class of every channel when the plan has one (slot = channel), else -1
+  cham_wpack_desc desc;     // copied to desc_out (the blob header) by the pack kernel
+  cham_wpack_desc* desc_out;
   uint8_t* codes;
   float* scale;
   uint8_t* zero;
