@@ -321,7 +321,7 @@ def main():
         t_roof += nb * max(layer_flops(M, K, N) / (peak_tensor * 1e12), b / (pk["hbm_gbs"] * 1e9))
     clocks = clk.summary()
     probe = tensor_probe(torch, device)
-    variants = None if args.no_variants else variant_matrix(torch, cl, W, bias, X, layers, st, pk, probe)
+    variants = None if args.no_variants else variant_matrix(torch, cl, W, bias, X, layers, lut, st, pk, probe)
 
     result = {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
@@ -488,7 +488,7 @@ def oracle_sample(layers_idx=(4,), buckets=(0, 9)):
     return flops, t, desc
 
 
-def variant_matrix(torch, cl, W, bias, X, layers, st, pk, probe, reps=20):
+def variant_matrix(torch, cl, W, bias, X, layers, lut, st, pk, probe, reps=20):
     """Every activation-format x weight-palette variant of the GEMM (plus W4A16) on the largest
     layer of the step, and the quantizer per activation format, the selection and the pack per
     palette on the same tensors.  Each figure is `reps` launches captured in one CUDA graph and
@@ -554,6 +554,26 @@ def variant_matrix(torch, cl, W, bias, X, layers, st, pk, probe, reps=20):
                                      "gbs": round(qb / (tq * 1e-3) / 1e9, 1),
                                      "frac_hbm": round(qb / (tq * 1e-3) / hbm, 4),
                                      "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"})
+    # every layer of the step: its GEMM alone in the LUT format of bucket 9, f16 roofline
+    # (max(flops / f16 peak, bytes / HBM)) and whether it is tensor- or HBM-bound
+    out["layers"] = []
+    for lj, (lname, Ml, Kl, Nl) in enumerate(layers):
+        af = int(lut[lj, -1])
+        desc_l = cl.pack_plan_palette(Nl, Kl, cl.PALETTE_W8)
+        fmt_l = torch.empty(Nl, dtype=torch.uint8, device=dev)
+        cl.select_weight_formats(W[lj], cl.PALETTE_W8, fmt_out=fmt_l)
+        blob_l = torch.empty(desc_l.bytes, dtype=torch.uint8, device=dev)
+        cl.pack_weights(W[lj], fmt_l, desc_l, dev_status=st, blob=blob_l)
+        ws_l = torch.zeros(cl.linear_workspace_size(Ml, desc_l, af), dtype=torch.uint8, device=dev)
+        Y_l = torch.empty((Ml, Nl), dtype=torch.float32, device=dev)
+        cl.linear_prepare(X[lj][-1], af, ws_l, st)
+        t = timed(lambda: cl.linear_gemm(X[lj][-1], desc_l, blob_l, af, bias[lj], Y_l, ws_l, st)) * 1e-3
+        fl = layer_flops(Ml, Kl, Nl)
+        byts = Ml * Kl + Nl * Kl + 9 * Nl + 4 * Ml * Nl
+        t_f, t_b = fl / p16, byts / hbm
+        out["layers"].append({"layer": lname, "M": Ml, "K": Kl, "N": Nl, "act_fmt": af, "us": round(t * 1e6, 2),
+                              "tflops": round(fl / t / 1e12, 1), "bound": "tensor" if t_f >= t_b else "hbm",
+                              "frac_f16_roofline": round(max(t_f, t_b) / t, 4)})
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
     return out
