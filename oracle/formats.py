@@ -156,11 +156,26 @@ def scale_sym(amax, fmax):
     return np.float32(amax / np.float32(fmax)), np.float32(np.float32(fmax) / amax)
 
 
+def scale_zp(fmt, lo, hi):
+    """ScaleZP of a per-tensor activation format from an observed range (App. A.7; the helper of
+    Alg. 1 and Alg. 3): INT8-asym by scale_zp_asym, E4M3 / E5M2 by scale_sym of max(|lo|, |hi|).
+    Returns fp32 (s, inv) and int z."""
+    if fmt == A_INT8_ASYM:
+        return scale_zp_asym(lo, hi, 255)
+    if fmt in (A_E4M3, A_E5M2):
+        amax = max(abs(np.float32(lo)), abs(np.float32(hi)))
+        s, inv = scale_sym(amax, 448.0 if fmt == A_E4M3 else 57344.0)
+        return s, inv, 0
+    raise ValueError("ScaleZP is defined for the per-tensor formats 0..2, not %r" % (fmt,))
+
+
 # ---------------------------------------------------------------- activation quantizer
-def act_quant(X, fmt):
-    """Quantize one activation tensor X (fp16, M x K, K contiguous) in activation format `fmt`
-    with a scale computed from X's own range -- the dynamic path of Alg. 3 (lo, hi = min, max
-    of the tensor; ScaleZP; fq_f).  Returns a dict:
+def act_quant(X, fmt, lo=None, hi=None):
+    """Quantize one activation tensor X (fp16, M x K, K contiguous) in activation format `fmt`.
+    Per-tensor formats take ScaleZP of a range: by default X's own range -- the dynamic path of
+    Alg. 3 (lo, hi = min, max of the tensor); with `lo`, `hi` given, that range -- the UNet /
+    few-step path of Alg. 2, whose (s, z) are ScaleZP of the calibration range stored by Alg. 1
+    (values outside it clamp to the extreme codes).  MX formats ignore lo, hi.  Returns a dict:
       codes  uint8 M x K  (INT8-asym: q; E4M3/E5M2/MXFP8: FP8 bit pattern; MXINT8: int8 byte)
       s, z   per-tensor fp32 scale and integer zero point (MX: s = 1, z = 0, App. A.7)
       e8m0   uint8 M x K/32 for the MX formats, else None
@@ -169,16 +184,16 @@ def act_quant(X, fmt):
     x = X.astype(np.float32)
     M, K = x.shape
     out = {"fmt": fmt, "e8m0": None, "s": np.float32(1.0), "z": 0}
-    if fmt == A_INT8_ASYM:
+    if fmt in (A_INT8_ASYM, A_E4M3, A_E5M2) and lo is None:
         lo = x.min() if x.size else np.float32(0)
         hi = x.max() if x.size else np.float32(0)
-        s, inv, z = scale_zp_asym(lo, hi, 255)
+    if fmt == A_INT8_ASYM:
+        s, inv, z = scale_zp(fmt, lo, hi)
         q = rne(_f32(x * inv)) + z
         out.update(codes=np.clip(q, 0, 255).astype(np.uint8), s=s, z=z, inv=inv)
     elif fmt in (A_E4M3, A_E5M2):
-        name, fmax = ("e4m3", 448.0) if fmt == A_E4M3 else ("e5m2", 57344.0)
-        amax = np.abs(x).max() if x.size else np.float32(0)
-        s, inv = scale_sym(amax, fmax)
+        name = "e4m3" if fmt == A_E4M3 else "e5m2"
+        s, inv, _ = scale_zp(fmt, lo, hi)
         out.update(codes=fp_quantize(_f32(x * inv), name).astype(np.uint8), s=s, z=0, inv=inv)
     elif fmt in (A_MXFP8, A_MXINT8):
         assert K % MX_BLOCK == 0

@@ -225,3 +225,36 @@ def test_weight_e2m1_grid_channel_is_exact():
     w = (np.tile(np.concatenate([g, -g]), 2) * 2.0 ** -7).astype(np.float16).reshape(1, -1)
     q = F.weight_quant(w, F.W_E2M1)
     np.testing.assert_array_equal(F.weight_dequant(q), w.astype(np.float64))
+
+
+# ---------------------------------------------------------------- static scales (Alg. 1 / Alg. 2)
+@pytest.mark.parametrize("fmt", [F.A_INT8_ASYM, F.A_E4M3, F.A_E5M2])
+def test_static_range_equal_to_own_range_is_the_dynamic_path(fmt):
+    """Alg. 2 with the calibration range equal to the tensor's own range reduces to Alg. 3."""
+    X = (np.random.default_rng(7).standard_t(3, (64, 96)) * 0.7).astype(np.float16)
+    x = X.astype(np.float32)
+    dyn = F.act_quant(X, fmt)
+    sta = F.act_quant(X, fmt, lo=x.min(), hi=x.max())
+    assert np.array_equal(dyn["codes"], sta["codes"]) and dyn["s"] == sta["s"] and dyn["z"] == sta["z"]
+
+
+def test_static_int8_asym_closed_form_and_clamping():
+    """Range [-1, 1]: s = 2/255, inv = 127.5, z = RNE(127.5) = 128; 0.5 -> RNE(63.75) + 128 = 192;
+    values beyond the calibration range clamp to codes 0 and 255."""
+    s, inv, z = F.scale_zp(F.A_INT8_ASYM, -1.0, 1.0)
+    assert s == np.float32(2.0 / 255.0) and inv == np.float32(127.5) and z == 128
+    X = np.array([[0.5, -0.5, 3.0, -3.0, 0.0]], np.float16)
+    q = F.act_quant(X, F.A_INT8_ASYM, lo=-1.0, hi=1.0)
+    assert list(q["codes"][0]) == [192, 64, 255, 0, 128]
+
+
+@pytest.mark.parametrize("fmt,fmax", [(F.A_E4M3, 448.0), (F.A_E5M2, 57344.0)])
+def test_static_fp8_scale_and_saturation(fmt, fmax):
+    """Range [-2, 1]: amax = 2, s = 2/Fmax, inv = Fmax/2; x = 1 lands on Fmax/2 exactly; x = 3
+    is beyond the range and saturates to Fmax (never NaN, note (ii))."""
+    s, inv, z = F.scale_zp(fmt, -2.0, 1.0)
+    assert s == np.float32(2.0 / fmax) and inv == np.float32(fmax / 2.0) and z == 0
+    name = "e4m3" if fmt == F.A_E4M3 else "e5m2"
+    q = F.act_quant(np.array([[1.0, 3.0, -3.0]], np.float16), fmt, lo=-2.0, hi=1.0)
+    vals = F.fp_decode(q["codes"][0], name)
+    assert list(vals) == [fmax / 2.0, fmax, -fmax]
