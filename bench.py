@@ -137,17 +137,22 @@ def build_inputs(torch, host, device):
 
 
 def calibrate_lut(torch, cl, X, buckets):
-    """Alg. 1 on the synthetic activations: power sums on the GPU, kappa, SNR at the bucket
-    midpoint (scaled-linear schedule), Route -> F[l, b]."""
+    """Alg. 1 on the synthetic activations (the calibration set is the step's own activations):
+    power sums and range on the GPU, kappa, SNR at the bucket midpoint (scaled-linear schedule),
+    Route -> F[l, b], and the static ScaleZP(F[l, b], lo[l, b], hi[l, b]) that the UNet path
+    quantizes with (Alg. 2; None for the MX formats, which carry block exponents instead)."""
     snr = cl.snr(cl.SCHEDULE_SCALED_LINEAR, 1000)
     lut = np.zeros((len(X), len(buckets)), dtype=np.int64)
     kappa = np.zeros((len(X), len(buckets)))
+    qp = [[None] * len(buckets) for _ in X]
     for li, xs in enumerate(X):
         for j, x in enumerate(xs):
             sums = cl.act_moments(x).cpu().numpy()
             kappa[li, j] = cl.kurtosis(sums[:5])
             lut[li, j] = cl.route(kappa[li, j], snr[buckets[j] * 100 + 50], False)
-    return lut, kappa
+            if lut[li, j] <= 2:
+                qp[li][j] = cl.scale_zp(int(lut[li, j]), float(sums[5]), float(sums[6]))
+    return lut, kappa, qp
 
 
 def main():
@@ -195,7 +200,7 @@ def main():
     nb = len(buckets)
     host = host_inputs(WL, layer_ids, buckets)
     W, bias, X = build_inputs(torch, host, device)
-    lut, kappa = calibrate_lut(torch, cl, X, buckets)
+    lut, kappa, qp = calibrate_lut(torch, cl, X, buckets)
     st = torch.zeros(1, dtype=torch.int32, device=device)
     stream = torch.cuda.current_stream()
 
@@ -227,14 +232,14 @@ def main():
 
     def run_step(parts="wqg"):
         """a5 + a6 for every layer ("w"), then a2-a4 + a7 for every (bucket, layer): act-quant in
-        F[l, b] ("q") and the GEMM ("g")."""
+        F[l, b] with the calibrated static (S, Z)[l, b] of the UNet path ("q") and the GEMM ("g")."""
         if "w" in parts:
             select_pack()
         for bk in range(nb):
             for li, (_, M, K, N) in enumerate(layers):
                 f = int(lut[li, bk])
                 if "q" in parts:
-                    cl.linear_prepare(X[li][bk], f, ws[li], st)
+                    cl.linear_prepare_static(X[li][bk], f, qp[li][bk], ws[li], st)
                 if "g" in parts:
                     cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
 
@@ -267,9 +272,8 @@ def main():
             run_step(key)
 
     # kernel launches per step: select 1 + pack 1 per layer (one MMA class: no slot ranking);
-    # per linear 2 (per-tensor) or 1 (MX) quantizer kernels + 1 GEMM
-    launches = 2 * len(layers) + sum(
-        (2 if lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(nb))
+    # per linear 1 quantizer kernel (static scales or MX) + 1 GEMM
+    launches = 2 * len(layers) + 2 * len(layers) * nb
     for li, (_, M, K, N) in enumerate(layers):
         for bk in range(nb):
             mx = lut[li, bk] >= 3
@@ -321,7 +325,7 @@ def main():
         t_roof += nb * max(layer_flops(M, K, N) / (peak_tensor * 1e12), b / (pk["hbm_gbs"] * 1e9))
     clocks = clk.summary()
     probe = tensor_probe(torch, device)
-    variants = None if args.no_variants else variant_matrix(torch, cl, W, bias, X, layers, lut, st, pk, probe)
+    variants = None if args.no_variants else variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe)
 
     result = {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
@@ -332,7 +336,8 @@ def main():
                    "layers": len(layers), "buckets": nb, "global_batch": 2 * world,
                    "tokens": [M for (_, M, _, _) in layers], "weight_palette": "W8 {INT8-sym, INT8-asym, MXINT8}",
                    "activation_formats_used": sorted(set(int(v) for v in lut.ravel())),
-                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant + GEMM, one CUDA graph",
+                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant (static calibrated "
+                           "per-(layer, bucket) scales, Alg. 2) + GEMM, one CUDA graph",
                    "l2": "inputs larger than L2 (%.0f MB of activations per step)" %
                          (sum(x.numel() * 2 for xs in X for x in xs) / 1e6),
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
@@ -361,7 +366,7 @@ def main():
     }
     if not args.no_e2e:
         del X
-        result["e2e"] = e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops_step)
+        result["e2e"] = e2e_leg(args, torch, cl, host, layers, nb, lut, qp, device, stream, world, flops_step)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline()
     if rank == 0:
@@ -371,7 +376,7 @@ def main():
     return 0
 
 
-def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops_step):
+def e2e_leg(args, torch, cl, host, layers, nb, lut, qp, device, stream, world, flops_step):
     """Same step through the public calls with HOST buffers: the weights and every activation are
     copied host->device from pinned memory and every output device->host inside the timed
     region."""
@@ -423,8 +428,8 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, device, stream, world, flops
                     x_ready[li].record(s_h2d)
                 stream.wait_event(x_ready[li])
                 stream.wait_event(y_free[li])
-                cl.linear(Xd[li], descs[li], blobs[li], int(lut[li, bk]), bias=bd[li], Y=Yd[li], ws=ws[li],
-                          dev_status=st, stream=stream)
+                cl.linear_static(Xd[li], descs[li], blobs[li], int(lut[li, bk]), qp[li][bk], bias=bd[li], Y=Yd[li],
+                                 ws=ws[li], dev_status=st, stream=stream)
                 x_free[li].record(stream)
                 y_ready[li].record(stream)
                 s_d2h = s_d2h_all[li % len(s_d2h_all)]
@@ -480,15 +485,16 @@ def oracle_sample(layers_idx=(4,), buckets=(0, 9)):
             t0 = time.perf_counter()
             fmt, _, _ = SEL.select_formats(W, 0x007)
             f = S.route(S.kurtosis(X), snr[int(S.bucket_midpoint(bk))])
-            G.linear_reference(X, f, W, fmt, bias)
+            x = X.astype(np.float32)          # Alg. 1's range on this sample, then Alg. 2's static scale
+            G.linear_reference(X, f, W, fmt, bias, float(x.min()), float(x.max()))
             t += time.perf_counter() - t0
             flops += layer_flops(M, K, N)
-    desc = "oracle select(W8)+act-quant+fp64 GEMM of layer(s) %s at buckets %s" % (
+    desc = "oracle select(W8)+static act-quant+fp64 GEMM of layer(s) %s at buckets %s" % (
         [WL.SDXL_PROJ_LAYERS[i][0] for i in layers_idx], list(buckets))
     return flops, t, desc
 
 
-def variant_matrix(torch, cl, W, bias, X, layers, lut, st, pk, probe, reps=20):
+def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=20):
     """Every activation-format x weight-palette variant of the GEMM (plus W4A16) on the largest
     layer of the step, and the quantizer per activation format, the selection and the pack per
     palette on the same tensors.  Each figure is `reps` launches captured in one CUDA graph and
@@ -549,9 +555,13 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, st, pk, probe, reps=20):
             out["gemm"].append(row)
             if bits == 8 and af != 5:
                 tq = timed(lambda: cl.linear_prepare(x, af, ws, st))
+                xf = x.float()
+                p_af = cl.scale_zp(af, float(xf.min()), float(xf.max())) if af <= 2 else None
+                tqs = timed(lambda: cl.linear_prepare_static(x, af, p_af, ws, st))
                 qb = 4 * M * K + (M * K / 32 if af in (3, 4) else 0)
-                out["quant"].append({"act_fmt": af, "us": round(tq * 1e3, 2),
+                out["quant"].append({"act_fmt": af, "us": round(tq * 1e3, 2), "static_us": round(tqs * 1e3, 2),
                                      "gbs": round(qb / (tq * 1e-3) / 1e9, 1),
+                                     "static_gbs": round(qb / (tqs * 1e-3) / 1e9, 1),
                                      "frac_hbm": round(qb / (tq * 1e-3) / hbm, 4),
                                      "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"})
     # every layer of the step: its GEMM alone in the LUT format of bucket 9, f16 roofline
@@ -566,7 +576,7 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, st, pk, probe, reps=20):
         cl.pack_weights(W[lj], fmt_l, desc_l, dev_status=st, blob=blob_l)
         ws_l = torch.zeros(cl.linear_workspace_size(Ml, desc_l, af), dtype=torch.uint8, device=dev)
         Y_l = torch.empty((Ml, Nl), dtype=torch.float32, device=dev)
-        cl.linear_prepare(X[lj][-1], af, ws_l, st)
+        cl.linear_prepare_static(X[lj][-1], af, qp[lj][-1], ws_l, st)
         t = timed(lambda: cl.linear_gemm(X[lj][-1], desc_l, blob_l, af, bias[lj], Y_l, ws_l, st)) * 1e-3
         fl = layer_flops(Ml, Kl, Nl)
         byts = Ml * Kl + Nl * Kl + 9 * Nl + 4 * Ml * Nl

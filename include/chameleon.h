@@ -111,7 +111,8 @@ cham_status chameleon_act_moments(const void* X, int64_t count, double* out, voi
  *                           (per-tensor formats; MX formats store s = 1, z = 0, inv = 1)
  *   [P+256, P+256+M*K/32)   E8M0 block exponents, uint8 M x (K/32) row-major (MX formats only)
  * Dequantized value: INT8-asym (q - z) * s; E4M3/E5M2 value(code) * s; MXFP8 value(code) * 2^(e-127);
- * MXINT8 code * 2^-6 * 2^(e-127)  (App. A.7 ScaleZP, App. A.11; readings R1-R8 in the design doc). */
+ * MXINT8 code * 2^-6 * 2^(e-127)  (App. A.7 ScaleZP, App. A.11).  MX shared exponent floor(log2 amax) - emax
+ * of the element body (8 for E4M3, 0 for the int8 body); an all-zero block has E8M0 byte 0. */
 typedef struct {
   float s;
   int32_t z;
@@ -127,6 +128,29 @@ cham_status chameleon_act_quant_size(int M, int K, int fmt, size_t* qact_bytes, 
  * unspecified). */
 cham_status chameleon_act_quant(const void* X, int M, int K, int fmt, void* qact, size_t qact_bytes,
                                 void* ws, size_t ws_bytes, int* dev_status, void* stream);
+
+/* ScaleZP of a per-tensor format (0..2) from a range [lo, hi] (App. A.7; the helper Alg. 1 uses
+ * when it stores the scale of each layer and bucket from the calibration range, and the one the
+ * quantizer applies to a tensor's own range in Alg. 3).  INT8-asym: s = (hi' - lo')/255,
+ * inv = 255/(hi' - lo'), z = round_half_even(-lo' * inv) clamped to [0, 255], where lo' = min(lo, 0),
+ * hi' = max(hi, 0); E4M3 / E5M2: s = amax/Fmax, inv = Fmax/amax, z = 0 (amax = max(|lo|, |hi|),
+ * Fmax 448 / 57344); a degenerate range gives s = inv = 1, z = 0.  Each step is one fp32 operation
+ * rounded to nearest, as the device quantizer computes it, so the same range gives the same bits.
+ * Host only (out is host memory).  CHAM_ERR_INVALID_ARG for another format, a non-finite or
+ * reversed range (lo > hi), or a range whose width overflows fp32. */
+cham_status chameleon_scale_zp(int fmt, float lo, float hi, cham_qparams* out);
+
+/* The static path of Alg. 2: quantize X (device, fp16 M x K) with the per-tensor parameters
+ * *params (host; made by chameleon_scale_zp from the calibration range of this layer and bucket)
+ * instead of X's own range: one pass, no workspace.  Values outside that range clamp to codes 0 /
+ * 255 (INT8-asym) or saturate to +-Fmax (FP8).  The qact layout and the stored cham_qparams are
+ * those of chameleon_act_quant.  MX formats (3, 4) have no per-tensor parameters: params is
+ * ignored (may be NULL) and the result equals chameleon_act_quant's.  CHAM_ERR_INVALID_ARG when
+ * params is NULL for fmt 0..2, its fmt field differs, s or inv is not finite and positive, or z is
+ * outside the format's range (0..255 for INT8-asym, 0 for FP8).  Non-finite input sets
+ * *dev_status = CHAM_ERR_NONFINITE (codes then unspecified). */
+cham_status chameleon_act_quant_static(const void* X, int M, int K, int fmt, const cham_qparams* params,
+                                       void* qact, size_t qact_bytes, int* dev_status, void* stream);
 
 /* ------------------------------------------------------------------ a5: weight-format selection */
 
@@ -217,6 +241,11 @@ cham_status chameleon_linear(const void* X, int M, const cham_wpack_desc* desc, 
  * otherwise) with the packed weights.  Same arguments, workspace and errors as chameleon_linear. */
 cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, void* ws, size_t ws_bytes,
                                      int* dev_status, void* stream);
+/* chameleon_linear_prepare on the static path of Alg. 2: the operand is quantized with *params
+ * (host; see chameleon_act_quant_static for its checks and for MX / FP16, which ignore it) in
+ * one pass.  Same workspace as chameleon_linear_prepare; chameleon_linear_gemm then multiplies it. */
+cham_status chameleon_linear_prepare_static(const void* X, int M, int K, int act_fmt, const cham_qparams* params,
+                                            void* ws, size_t ws_bytes, int* dev_status, void* stream);
 cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* desc, const void* blob,
                                   int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
                                   int* dev_status, void* stream);

@@ -8,7 +8,7 @@ Test infrastructure (see ``oracle/__init__``).  Passages followed:
   * clamp before the FP8 cast -- App. A.7, implementation note (ii);
   * MX shared exponent floor(log2 max|x|) with an E8M0 byte -- Sec. 3.6, App. A.11, App. A.12.
 
-Readings of passages the paper leaves open (each one also listed in the design doc):
+Readings of passages the paper leaves open (numbered R1..R17 across the project):
   R1  MX shared exponent: X = floor(log2 amax) - emax_elem with emax_elem = 8 (E4M3 body),
       2 (E2M1 body), 0 (integer bodies) -- the OCP rule the paper says it follows exactly.
   R2  all-zero MX block: E8M0 byte 0; the element codes are the encodings of the zero elements

@@ -17,13 +17,15 @@ from .select import dequant_selected
 TOL_REL = 2.0 ** -10
 
 
-def linear_reference(X, act_fmt, W, wfmt, bias=None):
-    """Returns (Y_ref float64 M x N, bound float64 M x N, A_dq, W_dq)."""
+def linear_reference(X, act_fmt, W, wfmt, bias=None, lo=None, hi=None):
+    """Returns (Y_ref float64 M x N, bound float64 M x N, A_dq, W_dq).  With lo, hi given, X is
+    quantized with the static ScaleZP of that calibration range (Alg. 2), else with its own range
+    (Alg. 3)."""
     X = np.asarray(X)
     if act_fmt == F.A_FP16:
         a = X.astype(np.float64)                      # weight-only fork (Sec. 3.5, SDXL-Turbo)
     else:
-        a = F.act_dequant(F.act_quant(X, act_fmt))
+        a = F.act_dequant(F.act_quant(X, act_fmt, lo, hi))
     w = dequant_selected(W, np.asarray(wfmt))
     y = a @ w.T
     if bias is not None:

@@ -10,7 +10,7 @@ dropping the zero); one zero is added; all 16 values are divided by the largest,
 so they span [-1, 1].  The outermost probability delta is the mean of 1 - 1/(2*15) and
 1 - 1/(2*16), the offsets of a 15- and a 16-level quantile grid.
 
-The levels are then frozen as fp16 values (R9 in the design doc): the codec, the selector and the
+The levels are then frozen as fp16 values (reading R9): the codec, the selector and the
 GEMM all use the fp16-rounded levels, so an NF4 weight decodes exactly in fp16.
 
 Parity unpinned beyond: 16 sorted values, exactly one zero, L0 = -1, L15 = 1, 7 negative and

@@ -10,7 +10,7 @@ Test infrastructure (see ``oracle/__init__``).  Passages followed:
   * routing rule -- Sec. 3.3 (shortcut -> MXFP8; kappa > 5 or SNR < 0.2 -> E5M2;
     kappa <= 3 and SNR > 2 -> INT8-asym; otherwise E4M3).
 
-Readings (DESIGN.md): timesteps are integers 0..T-1 with alpha_bar_t including beta_t (R17);
+Readings of passages the paper leaves open: timesteps are integers 0..T-1 with alpha_bar_t including beta_t (R17);
 the scaled-linear betas interpolate linearly in sqrt(beta) (Stable-Diffusion schedule named by
 App. A.11 "scaled-linear"), the linear betas linearly in beta; kappa := 0 when the variance is 0.
 """

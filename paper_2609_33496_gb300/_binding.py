@@ -31,6 +31,7 @@ EXPORTS = [
     "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_plan_palette", "chameleon_pack_weights",
     "chameleon_linear_workspace_size", "chameleon_linear", "chameleon_linear_prepare",
     "chameleon_linear_gemm", "chameleon_act_quant_noalloc", "chameleon_debug_stall_next_gemm",
+    "chameleon_scale_zp", "chameleon_act_quant_static", "chameleon_linear_prepare_static",
 ]
 
 
@@ -48,6 +49,14 @@ class WPackDesc(ctypes.Structure):
 
 
 assert ctypes.sizeof(WPackDesc) == 256
+
+
+class QParams(ctypes.Structure):
+    """cham_qparams: per-tensor scale s, zero point z, 1/s as the quantizer multiplies, format."""
+    _fields_ = [("s", ctypes.c_float), ("z", ctypes.c_int32), ("inv", ctypes.c_float), ("fmt", ctypes.c_int32)]
+
+
+assert ctypes.sizeof(QParams) == 16
 
 _lib = None
 
@@ -98,6 +107,9 @@ def lib():
         "chameleon_linear_gemm": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
         "chameleon_act_quant_noalloc": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
         "chameleon_debug_stall_next_gemm": (i32, [i32]),
+        "chameleon_scale_zp": (i32, [i32, ctypes.c_float, ctypes.c_float, ctypes.POINTER(QParams)]),
+        "chameleon_act_quant_static": (i32, [vp, i32, i32, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
+        "chameleon_linear_prepare_static": (i32, [vp, i32, i32, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -184,6 +196,31 @@ def act_quant(X, fmt, dev_status=None, stream=None):
     return qact, dev_status
 
 
+def scale_zp(fmt, lo, hi):
+    """ScaleZP of a per-tensor activation format from the range [lo, hi] (host only)."""
+    p = QParams()
+    check(lib().chameleon_scale_zp(fmt, lo, hi, ctypes.byref(p)))
+    return p
+
+
+def _pref(params):
+    return None if params is None else ctypes.byref(params)
+
+
+def act_quant_static(X, fmt, params, dev_status=None, stream=None):
+    """Quantize fp16 X with fixed per-tensor parameters (a QParams from scale_zp of a calibration
+    range); MX formats ignore params.  Returns the qact byte buffer and the device status word."""
+    import torch
+    M, K = X.shape
+    qb, _ = act_quant_size(M, K, fmt)
+    qact = _bytes(qb, X.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
+    check(lib().chameleon_act_quant_static(_ptr(X), M, K, fmt, _pref(params), _ptr(qact), qb, _ptr(dev_status),
+                                           _stream(stream)))
+    return qact, dev_status
+
+
 def split_qact(qact, M, K):
     """Views of a qact buffer: codes (M x K uint8), params (s, z, inv, fmt), e8m0 (M x K/32)."""
     import torch
@@ -259,6 +296,23 @@ def linear(X, desc, blob, act_fmt, bias=None, Y=None, ws=None, dev_status=None, 
     return Y, dev_status
 
 
+def linear_static(X, desc, blob, act_fmt, params, bias=None, Y=None, ws=None, dev_status=None, stream=None):
+    """linear with the activation quantized by fixed parameters (linear_prepare_static, then
+    linear_gemm on the same stream)."""
+    import torch
+    M = X.shape[0]
+    need = linear_workspace_size(M, desc, act_fmt)
+    if ws is None or ws.numel() < need:
+        ws = _bytes(need, X.device)
+    if Y is None:
+        Y = torch.empty((M, desc.N), dtype=torch.float32, device=X.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
+    linear_prepare_static(X, act_fmt, params, ws, dev_status, stream)
+    linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream)
+    return Y, dev_status
+
+
 def debug_stall_next_gemm(chunk):
     """Test hook: the next GEMM launch withholds one K-chunk so its bounded waits run out."""
     check(lib().chameleon_debug_stall_next_gemm(chunk))
@@ -269,6 +323,13 @@ def linear_prepare(X, act_fmt, ws, dev_status, stream=None):
     M, K = X.shape
     check(lib().chameleon_linear_prepare(_ptr(X), M, K, act_fmt, _ptr(ws), ws.numel(), _ptr(dev_status),
                                          _stream(stream)))
+
+
+def linear_prepare_static(X, act_fmt, params, ws, dev_status, stream=None):
+    """First half of linear on the static path: quantize X with fixed parameters (QParams)."""
+    M, K = X.shape
+    check(lib().chameleon_linear_prepare_static(_ptr(X), M, K, act_fmt, _pref(params), _ptr(ws), ws.numel(),
+                                                _ptr(dev_status), _stream(stream)))
 
 
 def linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream=None):

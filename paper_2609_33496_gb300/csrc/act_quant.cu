@@ -166,6 +166,46 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
 }
 
 // ------------------------------------------------------------------ a3: per-tensor encode
+// Non-finite fp16 lanes of one 16-byte vector (exponent field all ones), as a 0/1 flag.
+CHAM_DEV uint32_t nonfinite8(const uint4& v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t nf = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) nf |= ((w[j] & 0x7C00u) == 0x7C00u) | ((w[j] & 0x7C000000u) == 0x7C000000u);
+  return nf;
+}
+
+// Grid-stride encode of the whole tensor with parameters p; CHECK also returns whether any input
+// lane was non-finite (the static path has no range pass to find out).
+template <int FMT, bool CODES, bool DEQ, bool CHECK>
+CHAM_DEV uint32_t encode_tensor_body(const uint4* __restrict__ X, int64_t nvec, const TensorParams& p,
+                                     uint2* __restrict__ codes, uint4* __restrict__ deq) {
+  uint32_t nf = 0;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec; i0 += stride * kUnroll) {
+    uint4 v[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = i0 + u * stride;
+      v[u] = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = i0 + u * stride;
+      if (i < nvec) {
+        if constexpr (CHECK) nf |= nonfinite8(v[u]);
+        uint2 c;
+        uint4 d;
+        encode8_tensor<FMT, DEQ>(v[u], p, c, d);
+        if constexpr (CODES) codes[i] = c;
+        if constexpr (DEQ) deq[i] = d;
+      }
+    }
+  }
+  return nf;
+}
+
+// Dynamic path (Alg. 3): ScaleZP of the tensor's own range, reduced from the range partials.
 template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_tensor(const uint4* __restrict__ X, int64_t nvec, const RangePartial* __restrict__ parts,
@@ -182,26 +222,25 @@ __global__ void __launch_bounds__(256)
     if (scale_out != nullptr) *scale_out = p.s;
     if (nf) set_status(dev_status, CHAM_ERR_NONFINITE);
   }
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec; i0 += stride * kUnroll) {
-    uint4 v[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t i = i0 + u * stride;
-      v[u] = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t i = i0 + u * stride;
-      if (i < nvec) {
-        uint2 c;
-        uint4 d;
-        encode8_tensor<FMT, DEQ>(v[u], p, c, d);
-        if constexpr (CODES) codes[i] = c;
-        if constexpr (DEQ) deq[i] = d;
-      }
-    }
+  encode_tensor_body<FMT, CODES, DEQ, false>(X, nvec, p, codes, deq);
+}
+
+// Static path (Alg. 2): (s, z) fixed beforehand -- ScaleZP of the calibration range that Alg. 1
+// stored for this layer and bucket -- so one pass encodes; values outside that range clamp to the
+// extreme codes (INT8) or saturate (FP8).  Non-finite inputs are flagged on the fly.
+template <int FMT, bool CODES, bool DEQ>
+__global__ void __launch_bounds__(256)
+    k_act_encode_static(const uint4* __restrict__ X, int64_t nvec, TensorParams p, uint2* __restrict__ codes,
+                        uint4* __restrict__ deq, cham_qparams* __restrict__ params, float* __restrict__ scale_out,
+                        int* dev_status) {
+  griddep_wait();  // X may be the previous kernel's output; the outputs may still be read by it
+  griddep_launch_dependents();
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    if (params != nullptr) *params = cham_qparams{p.s, p.z, p.inv, FMT};
+    if (scale_out != nullptr) *scale_out = p.s;
   }
+  const uint32_t nf = encode_tensor_body<FMT, CODES, DEQ, true>(X, nvec, p, codes, deq);
+  if (__any_sync(0xffffffffu, nf != 0) && (threadIdx.x & 31) == 0) set_status(dev_status, CHAM_ERR_NONFINITE);
 }
 
 // ------------------------------------------------------------------ a4: MX encode
@@ -386,6 +425,11 @@ int range_grid(int64_t nvec, int num_sms) {
 
 template <int FMT, bool CODES, bool DEQ>
 static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
+  if (a.use_static) {
+    launch_pdl(k_act_encode_static<FMT, CODES, DEQ>, dim3(range_grid(a.nvec, a.num_sms)), dim3(256), 0, st, a.X,
+               a.nvec, a.stat, a.codes, a.deq, a.params, a.scale_out, a.dev_status);
+    return;
+  }
   launch_pdl(k_act_range, dim3(a.nparts), dim3(256), 0, st, a.X, a.nvec, a.parts);
   const int g = range_grid(a.nvec, a.num_sms);
   launch_pdl(k_act_encode_tensor<FMT, CODES, DEQ>, dim3(g), dim3(256), 0, st, a.X, a.nvec,

@@ -34,6 +34,8 @@ struct ActQuantArgs {
   float* scale_out;        // the per-tensor scale s as a bare float (GEMM epilogue), or null
   int* dev_status;
   int num_sms;
+  bool use_static;         // per-tensor formats: encode with `stat` (Alg. 2), no range pass
+  TensorParams stat;
 };
 
 int range_grid(int64_t nvec, int num_sms);

@@ -168,6 +168,25 @@ cham_status check_act_args(const void* X, int M, int K, int fmt, bool allow_fp16
   return CHAM_OK;
 }
 
+// Parameters a caller hands to the static path (Alg. 2) must be those ScaleZP gives for that
+// format: finite positive s and 1/s, z in the format's code range.
+cham_status check_static_params(int fmt, const cham_qparams* p) {
+  if (fmt > CHAM_A_E5M2) return CHAM_OK;  // MX formats and FP16 carry no per-tensor parameters
+  if (p == nullptr) return fail(CHAM_ERR_INVALID_ARG, "static parameters are required for format %d", fmt);
+  if (p->fmt != fmt) return fail(CHAM_ERR_INVALID_ARG, "parameters of format %d given for format %d", p->fmt, fmt);
+  if (!std::isfinite(p->s) || !std::isfinite(p->inv) || !(p->s > 0.f) || !(p->inv > 0.f))
+    return fail(CHAM_ERR_INVALID_ARG, "static scale s=%g inv=%g", p->s, p->inv);
+  if (p->z < 0 || p->z > (fmt == CHAM_A_INT8_ASYM ? 255 : 0))
+    return fail(CHAM_ERR_INVALID_ARG, "zero point %d out of range for format %d", p->z, fmt);
+  return CHAM_OK;
+}
+
+cham::TensorParams tensor_params(const cham_qparams* p) {
+  cham::TensorParams t{1.f, 1.f, 0};
+  if (p != nullptr) t = cham::TensorParams{p->s, p->inv, p->z};
+  return t;
+}
+
 // Formats of each MMA class (R15).
 const int kClassOrder[2][5] = {{CHAM_W_INT4_SYM, CHAM_W_INT4_ASYM, CHAM_W_E2M1, CHAM_W_MXINT4, CHAM_W_MXFP4},
                                {CHAM_W_NF4, CHAM_W_INT8_SYM, CHAM_W_INT8_ASYM, CHAM_W_MXINT8, -1}};
@@ -332,6 +351,62 @@ cham_status chameleon_act_quant(const void* X, int M, int K, int fmt, void* qact
   cham::launch_act_quant(fmt, a, true, false, static_cast<cudaStream_t>(stream));
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "act_quant launch");
+}
+
+cham_status chameleon_scale_zp(int fmt, float lo, float hi, cham_qparams* out) {
+  if (out == nullptr) return fail(CHAM_ERR_INVALID_ARG, "out is NULL");
+  if (fmt < 0 || fmt > CHAM_A_E5M2) return fail(CHAM_ERR_INVALID_ARG, "ScaleZP is per-tensor: format %d", fmt);
+  if (!std::isfinite(lo) || !std::isfinite(hi) || lo > hi)
+    return fail(CHAM_ERR_INVALID_ARG, "range [%g, %g] must be finite and ordered", lo, hi);
+  // The arithmetic of the quantizer's own ScaleZP, in the same fp32 operations and rounding.
+  cham_qparams p{1.f, 0, 1.f, fmt};
+  if (fmt == CHAM_A_INT8_ASYM) {
+    const float lo_ = std::fmin(lo, 0.f), hi_ = std::fmax(hi, 0.f);
+    const float d = hi_ - lo_;
+    if (d != 0.f) {
+      p.s = d / 255.f;
+      p.inv = 255.f / d;
+      const float zf = std::nearbyint(-lo_ * p.inv);
+      p.z = zf < 0.f ? 0 : (zf > 255.f ? 255 : static_cast<int32_t>(zf));
+    }
+  } else {
+    const float fmax = fmt == CHAM_A_E4M3 ? 448.f : 57344.f;
+    const float amax = std::fmax(std::fabs(lo), std::fabs(hi));
+    if (amax != 0.f) {
+      p.s = amax / fmax;
+      p.inv = fmax / amax;
+    }
+  }
+  if (!std::isfinite(p.s) || !(p.inv > 0.f)) return fail(CHAM_ERR_INVALID_ARG, "range [%g, %g] too wide", lo, hi);
+  *out = p;
+  return CHAM_OK;
+}
+
+cham_status chameleon_act_quant_static(const void* X, int M, int K, int fmt, const cham_qparams* params, void* qact,
+                                       size_t qact_bytes, int* dev_status, void* stream) {
+  cham_status s = check_act_args(X, M, K, fmt, false);
+  if (s != CHAM_OK) return s;
+  s = check_static_params(fmt, params);
+  if (s != CHAM_OK) return s;
+  size_t need_q = 0;
+  chameleon_act_quant_size(M, K, fmt, &need_q, nullptr);
+  if (qact == nullptr || !aligned16(qact)) return fail(CHAM_ERR_INVALID_ARG, "qact must be 16-byte aligned");
+  if (qact_bytes < need_q) return fail(CHAM_ERR_WORKSPACE, "qact %zu < %zu bytes", qact_bytes, need_q);
+  const ActLayout L = act_layout(M, K);
+  uint8_t* q = static_cast<uint8_t*>(qact);
+  cham::ActQuantArgs a{};
+  a.X = static_cast<const uint4*>(X);
+  a.nvec = static_cast<int64_t>(M) * K / 8;
+  a.num_sms = num_sms_current();
+  a.codes = reinterpret_cast<uint2*>(q + L.codes);
+  a.e8m0 = fmt >= CHAM_A_MXFP8 ? q + L.e8m0 : nullptr;
+  a.params = reinterpret_cast<cham_qparams*>(q + L.params);
+  a.dev_status = dev_status;
+  a.use_static = true;
+  a.stat = tensor_params(params);
+  cham::launch_act_quant(fmt, a, true, false, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "act_quant_static launch");
 }
 
 // ---------------------------------------------------------------- a5
@@ -510,6 +585,31 @@ cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, v
   cham::launch_act_quant(act_fmt, a, false, true, static_cast<cudaStream_t>(stream));
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "linear_prepare launch");
+}
+
+cham_status chameleon_linear_prepare_static(const void* X, int M, int K, int act_fmt, const cham_qparams* params,
+                                            void* ws, size_t ws_bytes, int* dev_status, void* stream) {
+  cham_status s = check_act_args(X, M, K, act_fmt, true);
+  if (s != CHAM_OK) return s;
+  s = check_static_params(act_fmt, params);
+  if (s != CHAM_OK) return s;
+  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
+  if (s != CHAM_OK) return s;
+  if (act_fmt == CHAM_A_FP16) return CHAM_OK;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  const LinearWs L = linear_ws(M, K);
+  cham::ActQuantArgs a{};
+  a.X = static_cast<const uint4*>(X);
+  a.nvec = static_cast<int64_t>(M) * K / 8;
+  a.num_sms = num_sms_current();
+  a.deq = reinterpret_cast<uint4*>(w + L.operand);
+  a.scale_out = act_fmt <= CHAM_A_E5M2 ? reinterpret_cast<float*>(w + L.scale) : nullptr;
+  a.dev_status = dev_status;
+  a.use_static = true;
+  a.stat = tensor_params(params);
+  cham::launch_act_quant(act_fmt, a, false, true, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "linear_prepare_static launch");
 }
 
 namespace {

@@ -111,3 +111,44 @@ def test_host_validation_errors(cl):
         cl.act_quant_size(16, 64, 7)
     q, w = cl.act_quant_size(256, 320, 3)
     assert q >= 256 * 320 + 256 + 256 * 10 and w == 0
+
+
+def test_scale_zp_host_matches_oracle_bit_for_bit(cl):
+    """The host ScaleZP (the static path's parameters, Alg. 1 / Alg. 2) gives the oracle's fp32 s,
+    1/s and z for random, tiny, one-sided, degenerate and fp16-extreme ranges."""
+    rng = np.random.default_rng(11)
+    ranges = [(0.0, 0.0), (-1.0, -1.0), (2.0, 2.0), (-65504.0, 65504.0), (-1e-7, 3e-8), (0.0, 6.0),
+              (-6.0, 0.0), (-0.5, 0.5), (-1.0, 254.0), (-254.0, 1.0), (-1.0 / 255, 1.0)]
+    for _ in range(300):
+        lo, hi = np.sort(rng.standard_normal(2) * 10.0 ** rng.uniform(-4, 4, 2))
+        ranges.append((float(np.float32(lo)), float(np.float32(hi))))
+    for fmt in (F.A_INT8_ASYM, F.A_E4M3, F.A_E5M2):
+        for lo, hi in ranges:
+            p = cl.scale_zp(fmt, lo, hi)
+            s, inv, z = F.scale_zp(fmt, lo, hi)
+            assert (np.float32(p.s), np.float32(p.inv), p.z, p.fmt) == (s, inv, z, fmt), (fmt, lo, hi)
+
+
+def test_scale_zp_and_static_entry_points_reject_bad_arguments(cl):
+    for fmt, lo, hi in [(3, -1.0, 1.0), (5, -1.0, 1.0), (-1, 0.0, 1.0), (0, 1.0, -1.0),
+                        (1, float("nan"), 1.0), (2, 0.0, float("inf")), (0, -3e38, 3e38)]:
+        with pytest.raises(cl.ChameleonError) as e:
+            cl.scale_zp(fmt, lo, hi)
+        assert e.value.status == cl.ERR_INVALID_ARG
+    L = cl.lib()
+    buf = ctypes.create_string_buffer(1 << 16)
+    x = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
+    good = cl.scale_zp(F.A_INT8_ASYM, -1.0, 3.0)
+    bad = [None, cl.QParams(good.s, good.z, good.inv, F.A_E4M3), cl.QParams(0.0, 0, 1.0, 0),
+           cl.QParams(1.0, 256, 1.0, 0), cl.QParams(float("inf"), 0, 1.0, 0), cl.QParams(1.0, -1, 1.0, 0)]
+    for p in bad:
+        ref = None if p is None else ctypes.byref(p)
+        assert L.chameleon_act_quant_static(x, 16, 64, F.A_INT8_ASYM, ref, x, 1 << 15, x, None) == cl.ERR_INVALID_ARG
+        assert L.chameleon_linear_prepare_static(x, 16, 64, F.A_INT8_ASYM, ref, x, 1 << 15, x,
+                                                 None) == cl.ERR_INVALID_ARG
+    fp8 = cl.scale_zp(F.A_E4M3, -1.0, 3.0)
+    fp8.z = 1
+    assert L.chameleon_act_quant_static(x, 16, 64, F.A_E4M3, ctypes.byref(fp8), x, 1 << 15, x,
+                                        None) == cl.ERR_INVALID_ARG
+    assert L.chameleon_act_quant_static(x, 16, 48, F.A_INT8_ASYM, ctypes.byref(good), x, 1 << 15, x,
+                                        None) == cl.ERR_INVALID_ARG      # K not a multiple of 32
