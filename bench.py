@@ -564,6 +564,32 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
                                      "static_gbs": round(qb / (tqs * 1e-3) / 1e9, 1),
                                      "frac_hbm": round(qb / (tq * 1e-3) / hbm, 4),
                                      "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"})
+    # output type and scale granularity of the epilogue on the largest layer and on the first
+    # layer with a large fp32 output (8192 x 640 x 640): f32 / f16 / bf16 Y, one tensor scale or
+    # two per-sample scales (the DiT path's), E4M3 activations, W8 weights
+    out["epilogue"] = []
+    tdt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}
+    hbm_layer = next((j for j, l in enumerate(layers) if l[1] >= 8192), None)
+    for lj in sorted({li} | ({hbm_layer} if hbm_layer is not None else set())):
+        lname, Ml, Kl, Nl = layers[lj]
+        desc_l = cl.pack_plan_palette(Nl, Kl, cl.PALETTE_W8)
+        fmt_l = torch.empty(Nl, dtype=torch.uint8, device=dev)
+        cl.select_weight_formats(W[lj], cl.PALETTE_W8, fmt_out=fmt_l)
+        blob_l = torch.empty(desc_l.bytes, dtype=torch.uint8, device=dev)
+        cl.pack_weights(W[lj], fmt_l, desc_l, dev_status=st, blob=blob_l)
+        ws_l = torch.zeros(cl.linear_workspace_size(Ml, desc_l, 1), dtype=torch.uint8, device=dev)
+        fl = layer_flops(Ml, Kl, Nl)
+        for groups in (1, 2):
+            cl.linear_prepare_groups(X[lj][-1], 1, groups, ws_l, st)
+            for yn in ("f32", "f16", "bf16"):
+                Y_l = torch.empty((Ml, Nl), dtype=tdt[yn], device=dev)
+                t = timed(lambda: cl.linear_gemm_ex(X[lj][-1], desc_l, blob_l, 1, groups, bias[lj], Y_l, ws_l,
+                                                    st)) * 1e-3
+                byts = Ml * Kl + Nl * Kl + 9 * Nl + Y_l.element_size() * Ml * Nl
+                out["epilogue"].append({"layer": lname, "y": yn, "groups": groups, "us": round(t * 1e6, 2),
+                                        "tflops": round(fl / t / 1e12, 1),
+                                        "frac_f16_roofline": round(max(fl / p16, byts / hbm) / t, 4)})
+            del Y_l
     # every layer of the step: its GEMM alone in the LUT format of bucket 9, f16 roofline
     # (max(flops / f16 peak, bytes / HBM)) and whether it is tensor- or HBM-bound
     out["layers"] = []

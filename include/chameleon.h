@@ -64,6 +64,13 @@ typedef int cham_status;
 #define CHAM_PALETTE_W8 0x007u   /* INT8-sym, INT8-asym, MXINT8 */
 #define CHAM_PALETTE_W4 0x1F8u   /* INT4-sym, INT4-asym, NF4, E2M1, MXINT4, MXFP4 */
 
+/* Output element types of chameleon_linear_gemm_ex. */
+#define CHAM_Y_F32 0
+#define CHAM_Y_F16 1
+#define CHAM_Y_BF16 2
+/* Most row groups (samples) of chameleon_linear_prepare_groups. */
+#define CHAM_MAX_GROUPS 64
+
 /* Noise schedules for chameleon_snr (App. A.1, A.11): scaled-linear (SDXL, beta 0.00085 -> 0.012)
  * and linear (PixArt-alpha, beta 1e-4 -> 0.02). */
 #define CHAM_SCHEDULE_SCALED_LINEAR 0
@@ -249,6 +256,27 @@ cham_status chameleon_linear_prepare_static(const void* X, int M, int K, int act
 cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* desc, const void* blob,
                                   int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
                                   int* dev_status, void* stream);
+
+/* Per-sample dynamic scales (the DiT path scales each sample by its own range, Alg. 3): the M rows
+ * of X form n_groups equal groups of M / n_groups consecutive rows (one sample each, e.g. its
+ * tokens, or one half of a classifier-free-guidance pair), and each group of a per-tensor format
+ * (0..2) is quantized with ScaleZP of its own range.  n_groups = 1 is chameleon_linear_prepare.
+ * MX formats and FP16 have no per-tensor scale: for them n_groups is only checked.
+ * CHAM_ERR_INVALID_ARG unless 1 <= n_groups <= CHAM_MAX_GROUPS and n_groups divides M; otherwise
+ * as chameleon_linear_prepare (same workspace). */
+cham_status chameleon_linear_prepare_groups(const void* X, int M, int K, int act_fmt, int n_groups, void* ws,
+                                            size_t ws_bytes, int* dev_status, void* stream);
+
+/* chameleon_linear_gemm with the operand's row groups and a choice of output type.  n_groups must
+ * be the one the operand was prepared with (1 after chameleon_linear_prepare or
+ * chameleon_linear_prepare_static); row m uses the scale of group m / (M / n_groups).  y_type:
+ * CHAM_Y_F32 (as chameleon_linear_gemm), CHAM_Y_F16 or CHAM_Y_BF16 -- the fp32 value
+ * acc * (s_a * s_w) + bias rounded to nearest even into that type (beyond its range: +-Inf).
+ * Y (device, M x desc->N of y_type, 16-byte aligned).  CHAM_ERR_INVALID_ARG for another y_type or
+ * an n_groups that chameleon_linear_prepare_groups would reject. */
+cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc* desc, const void* blob,
+                                     int act_fmt, int n_groups, const float* bias, void* Y, int y_type, void* ws,
+                                     size_t ws_bytes, int* dev_status, void* stream);
 
 /* Test hook, not part of the method: the next chameleon_linear_gemm (or chameleon_linear) launch
  * on this host thread's library instance has the producer of its first CTA withhold the copies of

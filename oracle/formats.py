@@ -221,6 +221,23 @@ def act_dequant(q):
     raise ValueError(fmt)
 
 
+def act_quant_per_sample(X, fmt, n_groups):
+    """Per-sample dynamic scaling of the DiT path (Alg. 3 with min/max taken over one sample): the
+    M rows of X form n_groups equal groups of consecutive rows, and each group is quantized by
+    act_quant with its own range.  Returns the list of the groups' act_quant outputs."""
+    X = np.asarray(X)
+    M = X.shape[0]
+    if n_groups < 1 or M % n_groups:
+        raise ValueError("n_groups must divide M")
+    R = M // n_groups
+    return [act_quant(X[g * R:(g + 1) * R], fmt) for g in range(n_groups)]
+
+
+def act_dequant_per_sample(qs):
+    """DQ of act_quant_per_sample's output: the groups' dequantized rows stacked in order."""
+    return np.vstack([act_dequant(q) for q in qs])
+
+
 # ---------------------------------------------------------------- MX blocks (App. A.11/A.12)
 # element body: (emax_elem used by R1, integer scale exponent of the body)
 MX_BODIES = {"e4m3": 8, "e2m1": 2, "int8": 0, "int4": 0}

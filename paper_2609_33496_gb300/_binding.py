@@ -22,6 +22,8 @@ A_INT8_ASYM, A_E4M3, A_E5M2, A_MXFP8, A_MXINT8, A_FP16 = range(6)
 PALETTE_W8 = 0x007
 PALETTE_W4 = 0x1F8
 SCHEDULE_SCALED_LINEAR, SCHEDULE_LINEAR = 0, 1
+Y_F32, Y_F16, Y_BF16 = 0, 1, 2
+MAX_GROUPS = 64
 
 EXPORTS = [
     "chameleon_status_string", "chameleon_last_error_detail", "chameleon_version",
@@ -32,6 +34,7 @@ EXPORTS = [
     "chameleon_linear_workspace_size", "chameleon_linear", "chameleon_linear_prepare",
     "chameleon_linear_gemm", "chameleon_act_quant_noalloc", "chameleon_debug_stall_next_gemm",
     "chameleon_scale_zp", "chameleon_act_quant_static", "chameleon_linear_prepare_static",
+    "chameleon_linear_prepare_groups", "chameleon_linear_gemm_ex",
 ]
 
 
@@ -110,6 +113,8 @@ def lib():
         "chameleon_scale_zp": (i32, [i32, ctypes.c_float, ctypes.c_float, ctypes.POINTER(QParams)]),
         "chameleon_act_quant_static": (i32, [vp, i32, i32, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
         "chameleon_linear_prepare_static": (i32, [vp, i32, i32, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
+        "chameleon_linear_prepare_groups": (i32, [vp, i32, i32, i32, i32, vp, sz, vp, vp]),
+        "chameleon_linear_gemm_ex": (i32, [vp, i32, pdesc, vp, i32, i32, vp, vp, i32, vp, sz, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -310,6 +315,46 @@ def linear_static(X, desc, blob, act_fmt, params, bias=None, Y=None, ws=None, de
         dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
     linear_prepare_static(X, act_fmt, params, ws, dev_status, stream)
     linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream)
+    return Y, dev_status
+
+
+def _y_type(Y):
+    import torch
+    t = {torch.float32: Y_F32, torch.float16: Y_F16, torch.bfloat16: Y_BF16}.get(Y.dtype)
+    if t is None:
+        raise ValueError("Y must be float32, float16 or bfloat16")
+    return t
+
+
+def linear_prepare_groups(X, act_fmt, n_groups, ws, dev_status, stream=None):
+    """First half of linear with per-sample scales: rows in n_groups equal groups, each quantized
+    with the ScaleZP of its own range."""
+    M, K = X.shape
+    check(lib().chameleon_linear_prepare_groups(_ptr(X), M, K, act_fmt, n_groups, _ptr(ws), ws.numel(),
+                                                _ptr(dev_status), _stream(stream)))
+
+
+def linear_gemm_ex(X, desc, blob, act_fmt, n_groups, bias, Y, ws, dev_status, stream=None):
+    """Second half of linear with the operand's row groups; the output type is Y's dtype."""
+    check(lib().chameleon_linear_gemm_ex(_ptr(X), X.shape[0], ctypes.byref(desc), _ptr(blob), act_fmt, n_groups,
+                                         _ptr(bias), _ptr(Y), _y_type(Y), _ptr(ws), ws.numel(), _ptr(dev_status),
+                                         _stream(stream)))
+
+
+def linear_ex(X, desc, blob, act_fmt, n_groups=1, y_dtype=None, bias=None, Y=None, ws=None, dev_status=None,
+              stream=None):
+    """linear with per-sample activation scales (n_groups) and an fp32 / fp16 / bf16 output."""
+    import torch
+    M = X.shape[0]
+    need = linear_workspace_size(M, desc, act_fmt)
+    if ws is None or ws.numel() < need:
+        ws = _bytes(need, X.device)
+    if Y is None:
+        Y = torch.empty((M, desc.N), dtype=y_dtype or torch.float32, device=X.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
+    linear_prepare_groups(X, act_fmt, n_groups, ws, dev_status, stream)
+    linear_gemm_ex(X, desc, blob, act_fmt, n_groups, bias, Y, ws, dev_status, stream)
     return Y, dev_status
 
 

@@ -139,9 +139,13 @@ CHAM_DEV void encode8_tensor(const uint4& v, const TensorParams& p, uint2& code,
 }
 
 // ------------------------------------------------------------------ a2: range partials
+// Group blockIdx.y (rows split into gridDim.y equal groups, nvec vectors each; one group for a
+// per-tensor range) writes its gridDim.x partials at parts[blockIdx.y * gridDim.x ...].
 __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, int64_t nvec,
                                                   RangePartial* __restrict__ parts) {
   griddep_launch_dependents();
+  X += static_cast<int64_t>(blockIdx.y) * nvec;
+  parts += static_cast<int64_t>(blockIdx.y) * gridDim.x;
   // X is a caller input that no kernel of the chain writes: it is read before the wait, so this
   // pass overlaps the tail of the previous kernel; the partial is written after it
   __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
@@ -206,6 +210,8 @@ CHAM_DEV uint32_t encode_tensor_body(const uint4* __restrict__ X, int64_t nvec, 
 }
 
 // Dynamic path (Alg. 3): ScaleZP of the tensor's own range, reduced from the range partials.
+// Per-sample scales: group blockIdx.y (nvec vectors) uses the range of its own nparts partials
+// and stores its scale at scale_out[blockIdx.y] (params, of the public call, has one slot).
 template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_tensor(const uint4* __restrict__ X, int64_t nvec, const RangePartial* __restrict__ parts,
@@ -213,16 +219,18 @@ __global__ void __launch_bounds__(256)
                         cham_qparams* __restrict__ params, float* __restrict__ scale_out, int* dev_status) {
   griddep_wait();  // the range partials
   griddep_launch_dependents();
+  const int64_t g = blockIdx.y;
   float lo, hi;
   uint32_t nf;
-  reduce_partials(parts, nparts, lo, hi, nf);
+  reduce_partials(parts + g * nparts, nparts, lo, hi, nf);
   const TensorParams p = scale_zp(FMT, lo, hi);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
-    if (params != nullptr) *params = cham_qparams{p.s, p.z, p.inv, FMT};
-    if (scale_out != nullptr) *scale_out = p.s;
+    if (params != nullptr && g == 0) *params = cham_qparams{p.s, p.z, p.inv, FMT};
+    if (scale_out != nullptr) scale_out[g] = p.s;
     if (nf) set_status(dev_status, CHAM_ERR_NONFINITE);
   }
-  encode_tensor_body<FMT, CODES, DEQ, false>(X, nvec, p, codes, deq);
+  encode_tensor_body<FMT, CODES, DEQ, false>(X + g * nvec, nvec, p, codes == nullptr ? nullptr : codes + g * nvec,
+                                             deq == nullptr ? nullptr : deq + g * nvec);
 }
 
 // Static path (Alg. 2): (s, z) fixed beforehand -- ScaleZP of the calibration range that Alg. 1
@@ -423,6 +431,11 @@ int range_grid(int64_t nvec, int num_sms) {
   return static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
 }
 
+int group_grid(int64_t nvec, int n_groups, int num_sms) {
+  const int g = range_grid(nvec, num_sms) / (n_groups > 1 ? n_groups : 1);
+  return g < 1 ? 1 : g;
+}
+
 template <int FMT, bool CODES, bool DEQ>
 static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
   if (a.use_static) {
@@ -430,9 +443,12 @@ static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
                a.nvec, a.stat, a.codes, a.deq, a.params, a.scale_out, a.dev_status);
     return;
   }
-  launch_pdl(k_act_range, dim3(a.nparts), dim3(256), 0, st, a.X, a.nvec, a.parts);
-  const int g = range_grid(a.nvec, a.num_sms);
-  launch_pdl(k_act_encode_tensor<FMT, CODES, DEQ>, dim3(g), dim3(256), 0, st, a.X, a.nvec,
+  // per-sample groups: each group's range and encode grids are the per-tensor ones split evenly
+  const int G = a.n_groups > 1 ? a.n_groups : 1;
+  const int64_t nvg = a.nvec / G;
+  launch_pdl(k_act_range, dim3(a.nparts, G), dim3(256), 0, st, a.X, nvg, a.parts);
+  const int eg = group_grid(a.nvec, G, a.num_sms);
+  launch_pdl(k_act_encode_tensor<FMT, CODES, DEQ>, dim3(eg, G), dim3(256), 0, st, a.X, nvg,
              static_cast<const RangePartial*>(a.parts), a.nparts, a.codes, a.deq, a.params, a.scale_out,
              a.dev_status);
 }

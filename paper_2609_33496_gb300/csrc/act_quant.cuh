@@ -25,13 +25,14 @@ struct MomentPartial {  // one CTA's power sums (Alg. 1 accumulator)
 struct ActQuantArgs {
   const uint4* X;          // fp16 tensor, 8 elements per vector
   int64_t nvec;            // M*K/8
-  RangePartial* parts;     // per-tensor formats: range partials (scratch)
-  int nparts;              // CTAs of the two-launch range kernel (range_grid)
+  RangePartial* parts;     // per-tensor formats: range partials (scratch), nparts per group
+  int nparts;              // range CTAs per group: range_grid (one group) or group_grid
+  int n_groups;            // per-sample scales: rows in n_groups equal groups (0 or 1: per tensor)
   uint2* codes;            // 8 code bytes per vector, or null
   uint4* deq;              // 8 exact fp16 operand values per vector, or null
   uint8_t* e8m0;           // MX formats: one byte per 4 vectors, or null
   cham_qparams* params;    // per-tensor parameters, or null
-  float* scale_out;        // the per-tensor scale s as a bare float (GEMM epilogue), or null
+  float* scale_out;        // the per-tensor (per-group) scale s as bare floats (GEMM epilogue), or null
   int* dev_status;
   int num_sms;
   bool use_static;         // per-tensor formats: encode with `stat` (Alg. 2), no range pass
@@ -39,6 +40,9 @@ struct ActQuantArgs {
 };
 
 int range_grid(int64_t nvec, int num_sms);
+// CTAs per group when nvec vectors are split into n_groups groups (at least 1)
+int group_grid(int64_t nvec, int n_groups, int num_sms);
+constexpr int kMaxGroups = 64;  // per-sample groups: the scale slots of the linear workspace
 void launch_act_quant(int fmt, const ActQuantArgs& a, bool codes, bool deq, cudaStream_t st);
 void launch_act_moments(const uint4* X, int64_t nvec, int64_t count, MomentPartial* parts, int nparts,
                         double* out, cudaStream_t st);

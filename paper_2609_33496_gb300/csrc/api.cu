@@ -5,6 +5,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -204,9 +205,18 @@ cham_status check_desc(const cham_wpack_desc* d) {
 struct LinearWs {
   size_t scale, parts, operand;
 };
+// scale: one float per row group (kMaxGroups); parts: the range partials of every group
 LinearWs linear_ws(int M, int K) {
+  static_assert(cham::kMaxGroups == CHAM_MAX_GROUPS && cham::kMaxGroups * sizeof(float) <= 256, "scale slots");
   const int64_t nvec = static_cast<int64_t>(M) * K / 8;
-  return LinearWs{0, 256, 256 + range_ws_bytes(nvec)};
+  const int parts = std::max(cham::range_grid(nvec, num_sms_current()), cham::kMaxGroups);
+  return LinearWs{0, 256, 256 + round_up(static_cast<size_t>(parts) * sizeof(cham::RangePartial), 256)};
+}
+
+cham_status check_groups(int M, int n_groups) {
+  if (n_groups < 1 || n_groups > CHAM_MAX_GROUPS || M % n_groups != 0)
+    return fail(CHAM_ERR_INVALID_ARG, "n_groups=%d must be in 1..%d and divide M=%d", n_groups, CHAM_MAX_GROUPS, M);
+  return CHAM_OK;
 }
 
 cham_status check_linear_common(int M, int K, int act_fmt, void* ws, size_t ws_bytes, size_t need) {
@@ -563,7 +573,14 @@ extern "C" {
 
 cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, void* ws, size_t ws_bytes,
                                      int* dev_status, void* stream) {
+  return chameleon_linear_prepare_groups(X, M, K, act_fmt, 1, ws, ws_bytes, dev_status, stream);
+}
+
+cham_status chameleon_linear_prepare_groups(const void* X, int M, int K, int act_fmt, int n_groups, void* ws,
+                                            size_t ws_bytes, int* dev_status, void* stream) {
   cham_status s = check_act_args(X, M, K, act_fmt, true);
+  if (s != CHAM_OK) return s;
+  s = check_groups(M, n_groups);
   if (s != CHAM_OK) return s;
   s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
   if (s != CHAM_OK) return s;
@@ -575,7 +592,8 @@ cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, v
   a.nvec = static_cast<int64_t>(M) * K / 8;
   a.num_sms = num_sms_current();
   a.parts = reinterpret_cast<cham::RangePartial*>(w + L.parts);
-  a.nparts = cham::range_grid(a.nvec, a.num_sms);
+  a.n_groups = act_fmt <= CHAM_A_E5M2 ? n_groups : 1;
+  a.nparts = cham::group_grid(a.nvec, a.n_groups, a.num_sms);
   a.codes = nullptr;
   a.deq = reinterpret_cast<uint4*>(w + L.operand);
   a.e8m0 = nullptr;
@@ -625,7 +643,16 @@ cham_status chameleon_debug_stall_next_gemm(int chunk) {
 cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d, const void* blob, int act_fmt,
                                   const float* bias, float* Y, void* ws, size_t ws_bytes, int* dev_status,
                                   void* stream) {
+  return chameleon_linear_gemm_ex(X, M, d, blob, act_fmt, 1, bias, Y, CHAM_Y_F32, ws, ws_bytes, dev_status, stream);
+}
+
+cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc* d, const void* blob, int act_fmt,
+                                     int n_groups, const float* bias, void* Y, int y_type, void* ws,
+                                     size_t ws_bytes, int* dev_status, void* stream) {
   cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  if (y_type < CHAM_Y_F32 || y_type > CHAM_Y_BF16) return fail(CHAM_ERR_INVALID_ARG, "y_type %d", y_type);
+  s = check_groups(M, n_groups);
   if (s != CHAM_OK) return s;
   const int K = d->K;
   s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
@@ -649,6 +676,8 @@ cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d
   g.bias = bias;
   g.act_scale = act_scale;
   g.Y = Y;
+  g.y_type = y_type;
+  g.rows_per_group = act_fmt <= CHAM_A_E5M2 ? M / n_groups : M;
   g.M = M;
   g.N = d->N;
   g.n_chunks = d->Kp / 64;

@@ -15,8 +15,10 @@ struct GemmArgs {
   const uint8_t* wfmt;       // [Np]
   const int32_t* perm;       // [Np]
   const float* bias;         // [N] in original order, or null
-  const float* act_scale;    // device scalar s_a (per-tensor activation formats), or null for 1
-  float* Y;                  // [M][N] fp32
+  const float* act_scale;    // device s_a per row group (per-tensor formats: one group), or null for 1
+  void* Y;                   // [M][N] of y_type
+  int y_type;                // CHAM_Y_F32, CHAM_Y_F16 or CHAM_Y_BF16
+  int rows_per_group;        // rows sharing one act_scale entry (per-sample scales); >= M: one
   int M, N, n_chunks;        // n_chunks = Kp / 64
   int tile0;                 // first 128-channel tile of this launch
   int n_ch_tiles;            // 128-channel tiles of this launch
@@ -31,5 +33,11 @@ struct GemmArgs {
 int gemm_pick_bn(int M, int n_tiles, int num_sms);
 // Persistent launch: min(tiles, num_sms) CTAs walk the (channel tile, token tile) grid.
 cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
+// The launches of one output type (instantiated in gemm.cu, gemm_f16.cu, gemm_bf16.cu).
+template <int YT>
+cudaError_t launch_gemm_yt(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
+extern template cudaError_t launch_gemm_yt<CHAM_Y_F32>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_yt<CHAM_Y_F16>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_yt<CHAM_Y_BF16>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
 
 }  // namespace cham

@@ -152,3 +152,18 @@ def test_scale_zp_and_static_entry_points_reject_bad_arguments(cl):
                                         None) == cl.ERR_INVALID_ARG
     assert L.chameleon_act_quant_static(x, 16, 48, F.A_INT8_ASYM, ctypes.byref(good), x, 1 << 15, x,
                                         None) == cl.ERR_INVALID_ARG      # K not a multiple of 32
+
+
+def test_groups_and_output_type_argument_checks(cl):
+    """Per-sample groups must divide M and number 1..CHAM_MAX_GROUPS; y_type is one of three.
+    Every rejection happens on the host, before any launch."""
+    L = cl.lib()
+    buf = ctypes.create_string_buffer(1 << 20)
+    x = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
+    for M, n in [(64, 0), (64, 65), (64, 3), (60, -1), (128, 128)]:
+        assert L.chameleon_linear_prepare_groups(x, M, 64, F.A_E4M3, n, x, 1 << 19, x, None) == cl.ERR_INVALID_ARG
+    d = cl.pack_plan(64, 64, np.zeros(64, np.uint8))
+    for n, yt in [(3, cl.Y_F32), (0, cl.Y_F16), (1, 3), (1, -1), (65, cl.Y_BF16)]:
+        assert L.chameleon_linear_gemm_ex(x, 64, ctypes.byref(d), x, F.A_E4M3, n, None, x, yt, x, 1 << 19, x,
+                                          None) == cl.ERR_INVALID_ARG
+    assert cl.MAX_GROUPS == 64

@@ -258,3 +258,50 @@ def test_static_fp8_scale_and_saturation(fmt, fmax):
     q = F.act_quant(np.array([[1.0, 3.0, -3.0]], np.float16), fmt, lo=-2.0, hi=1.0)
     vals = F.fp_decode(q["codes"][0], name)
     assert list(vals) == [fmax / 2.0, fmax, -fmax]
+
+
+# ---------------------------------------------------------------- per-sample scales (Alg. 3 per sample)
+@pytest.mark.parametrize("fmt", F.ACT_FORMATS)
+def test_per_sample_with_one_group_is_the_per_tensor_path(fmt):
+    X = (np.random.default_rng(8).standard_t(3, (48, 64)) * 0.7).astype(np.float16)
+    (q,) = F.act_quant_per_sample(X, fmt, 1)
+    ref = F.act_quant(X, fmt)
+    assert np.array_equal(q["codes"], ref["codes"]) and q["s"] == ref["s"] and q["z"] == ref["z"]
+
+
+@pytest.mark.parametrize("fmt", F.ACT_FORMATS)
+@pytest.mark.parametrize("k", [-3, 2, 5])
+def test_per_sample_power_of_two_equivariance(fmt, k):
+    """A sample that is another sample times 2^k gets the same codes and a scale 2^k times as
+    large (the zero point unchanged; MX: block exponents shifted by k), whatever the other
+    samples hold -- a per-tensor scale would couple them."""
+    g = np.random.default_rng(9 + k)
+    Y = (g.standard_t(4, (16, 64)) * 0.5).astype(np.float16)
+    other = (g.standard_normal((16, 64)) * 40.0).astype(np.float16)
+    X = np.vstack([Y, (Y.astype(np.float64) * 2.0 ** k).astype(np.float16), other])
+    qs = F.act_quant_per_sample(X, fmt, 3)
+    assert np.array_equal(qs[0]["codes"], qs[1]["codes"])
+    if fmt in (F.A_MXFP8, F.A_MXINT8):
+        nz = Y.reshape(16, 2, 32).astype(np.float32).any(axis=2)
+        d = qs[1]["e8m0"].astype(int) - qs[0]["e8m0"].astype(int)
+        assert np.all(d[nz] == k)
+    else:
+        assert np.float32(qs[1]["s"]) == np.float32(np.float32(qs[0]["s"]) * np.float32(2.0 ** k))
+        assert qs[1]["z"] == qs[0]["z"]
+    np.testing.assert_array_equal(F.act_dequant_per_sample(qs)[16:32], F.act_dequant(qs[0]) * 2.0 ** k)
+
+
+def test_per_sample_zero_sample_is_degenerate_and_isolated():
+    """An all-zero sample takes the degenerate parameters (s = 1, z = 0, R7) and dequantizes to
+    exactly zero; its neighbours keep the parameters of their own ranges."""
+    X = np.zeros((12, 32), np.float16)
+    X[:4] = 0.25
+    X[:4, 0] = -0.75
+    X[8:] = np.linspace(-2, 6, 4 * 32).reshape(4, 32)
+    qs = F.act_quant_per_sample(X, F.A_INT8_ASYM, 3)
+    assert qs[1]["s"] == np.float32(1.0) and qs[1]["z"] == 0 and not qs[1]["codes"].any()
+    assert qs[0]["s"] == F.act_quant(X[:4], F.A_INT8_ASYM)["s"] == np.float32(1.0 / 255.0)
+    assert qs[2]["s"] == np.float32(8.0 / 255.0)
+    assert not F.act_dequant_per_sample(qs)[4:8].any()
+    with pytest.raises(ValueError):
+        F.act_quant_per_sample(X, F.A_E4M3, 5)
