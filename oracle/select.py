@@ -75,3 +75,25 @@ def dequant_selected(W, fmt):
         q = F.weight_quant(W[rows], int(f), nf4_levels=L)
         out[rows] = F.weight_dequant(q, nf4_levels=L)
     return out
+
+
+# ---------------------------------------------------------------- activation-format argmin (Eq. format-argmin)
+def act_format_sse(X):
+    """Squared quantization error of one activation tensor X (fp16, M x K) under every activation
+    format at its native granularity (Sec. 3.1 and 3.2: the per-tensor formats with the ScaleZP
+    of X's own range, the MX formats per 32-element block): SSE_f = sum (x - DQ_f(Q_f(x)))^2 in
+    fp64, f = 0..4 in palette order.  Summing it over the calibration tensors of one (layer,
+    bucket) gives the objective of Eq. format-argmin times their element count."""
+    x64 = np.asarray(X).astype(np.float64)
+    return np.array([((x64 - F.act_dequant(F.act_quant(X, f))) ** 2).sum() for f in F.ACT_FORMATS])
+
+
+def act_format_argmin(sse):
+    """f* = the first format of the activation palette with the least accumulated error (ties go
+    to the earlier format, as in the weight selection)."""
+    sse = np.asarray(sse, dtype=np.float64)
+    best = 0
+    for f in range(1, len(sse)):
+        if sse[f] < sse[best]:
+            best = f
+    return best

@@ -163,3 +163,120 @@ def test_nf4_quantiles_by_bisection():
     v = np.sort(np.array(pos + [0.0] + neg)) / max(pos)
     np.testing.assert_allclose(nf4.nf4_levels_exact(), v, atol=1e-12)
     assert np.all(v.astype(np.float16).astype(np.float64) == nf4.nf4_levels_fp16())
+
+
+# ---------------------------------------------------------------- activation-format argmin (Eq. format-argmin)
+def fp8_grid(ebits, mbits, bias, skip):
+    """(value, mantissa-is-even) of every non-negative finite value, from the bit definition."""
+    out = []
+    for E in range(1 << ebits):
+        for M in range(1 << mbits):
+            if skip(E, M):
+                continue
+            v = (M / (1 << mbits)) * 2.0 ** (1 - bias) if E == 0 else (1 + M / (1 << mbits)) * 2.0 ** (E - bias)
+            out.append((v, M % 2 == 0))
+    return sorted(out)
+
+
+E4M3 = fp8_grid(4, 3, 7, lambda E, M: E == 15 and M == 7)
+E5M2 = fp8_grid(5, 2, 15, lambda E, M: E == 31)
+
+
+def naive_fp8(v, grid):
+    """Nearest grid value to v (ties to the even mantissa), saturating beyond the largest."""
+    a = abs(v)
+    if a >= grid[-1][0]:
+        return math.copysign(grid[-1][0], v)
+    vals = [g for g, _ in grid]
+    r = nearest(a, vals, lambda c: [g for g, e in grid if g in c and e][0])
+    return math.copysign(r, v)
+
+
+def f32(v):
+    return float(np.float32(v))
+
+
+def naive_act_dq(X, fmt):
+    """An independent restatement of the five activation codecs, element by element: ScaleZP of
+    the tensor's range (App. A.7) with x/s as a rounded product by the reciprocal, nearest code by
+    search, and the MX shared exponent from frexp (OCP rule, body emax 8 for E4M3, 0 for int8)."""
+    x = np.asarray(X).astype(np.float64)
+    out = np.zeros_like(x)
+    if fmt in (F.A_INT8_ASYM, F.A_E4M3, F.A_E5M2):
+        lo, hi = float(x.min()), float(x.max())
+        if fmt == F.A_INT8_ASYM:
+            lo_, hi_ = min(lo, 0.0), max(hi, 0.0)
+            d = f32(hi_ - lo_)
+            s, inv = (1.0, 1.0) if d == 0 else (f32(d / 255), f32(255 / d))
+            z = 0 if d == 0 else min(max(nearest(f32(-lo_ * inv), range(-1, 257), even_int), 0), 255)
+            for i, v in np.ndenumerate(x):
+                t = f32(v * inv)
+                q = min(max(nearest(t, range(math.floor(t) - 1, math.floor(t) + 3), even_int) + z, 0), 255)
+                out[i] = (q - z) * s
+        else:
+            fmax, grid = (448.0, E4M3) if fmt == F.A_E4M3 else (57344.0, E5M2)
+            amax = max(abs(lo), abs(hi))
+            s, inv = (1.0, 1.0) if amax == 0 else (f32(amax / fmax), f32(fmax / amax))
+            for i, v in np.ndenumerate(x):
+                out[i] = naive_fp8(f32(v * inv), grid) * s
+        return out
+    for r in range(x.shape[0]):
+        for b0 in range(0, x.shape[1], 32):
+            blk = x[r, b0:b0 + 32]
+            amax = float(np.abs(blk).max())
+            if amax == 0:
+                continue
+            e = math.frexp(amax)[1] - 1                    # floor(log2 amax)
+            if fmt == F.A_MXFP8:
+                X_ = e - 8
+                out[r, b0:b0 + 32] = [naive_fp8(v * 2.0 ** -X_, E4M3) * 2.0 ** X_ for v in blk]
+            else:
+                X_ = e
+                out[r, b0:b0 + 32] = [min(max(nearest(v * 2.0 ** -X_ * 64, range(-128, 129), even_int), -127), 127)
+                                      * 2.0 ** -6 * 2.0 ** X_ for v in blk]
+    return out
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_act_format_sse_against_naive_codecs(seed):
+    g = np.random.default_rng(300 + seed)
+    X = (g.standard_t(3 + seed, (3, 64)) * 2.0 ** (seed - 1)).astype(np.float16)
+    x = X.astype(np.float64)
+    sse = SEL.act_format_sse(X)
+    naive = [((x - naive_act_dq(X, f)) ** 2).sum() for f in F.ACT_FORMATS]
+    np.testing.assert_allclose(sse, naive, rtol=1e-12, atol=0)
+    assert SEL.act_format_argmin(sse) == int(np.argmin(naive))
+
+
+def test_act_format_sse_zero_on_the_e4m3_grid():
+    """A tensor of E4M3 grid values whose largest magnitude is 448: per-tensor E4M3 reproduces it
+    exactly (s = 1), and so does MXFP8 (power-of-two block scaling keeps grid values on the grid);
+    INT8-asym and E5M2 cannot.  The argmin is E4M3, the earlier of the two exact formats."""
+    vals = np.array([g for g, _ in E4M3 if g >= 2.0 ** -6], np.float64)
+    g = np.random.default_rng(5)
+    x = g.choice(vals, (4, 96)) * g.choice([-1.0, 1.0], (4, 96))
+    x[0, 0] = 448.0
+    X = x.astype(np.float16)
+    assert np.array_equal(X.astype(np.float64), x)
+    sse = SEL.act_format_sse(X)
+    assert sse[F.A_E4M3] == 0 and sse[F.A_MXFP8] == 0
+    assert sse[F.A_INT8_ASYM] > 0 and sse[F.A_E5M2] > 0
+    assert SEL.act_format_argmin(sse) == F.A_E4M3
+
+
+@pytest.mark.parametrize("k", [-2, 3])
+def test_act_format_sse_power_of_two_scaling(k):
+    """Scaling X by 2^k scales every format's error by exactly 4^k (all five scale rules are
+    power-of-two equivariant away from fp16 subnormals), so the argmin does not move."""
+    X = (np.random.default_rng(6).standard_t(4, (8, 64)) * 4.0).astype(np.float16)
+    X2 = (X.astype(np.float64) * 2.0 ** k).astype(np.float16)
+    assert np.array_equal(X2.astype(np.float64), X.astype(np.float64) * 2.0 ** k)
+    a, b = SEL.act_format_sse(X), SEL.act_format_sse(X2)
+    np.testing.assert_array_equal(b, a * 4.0 ** k)
+    assert SEL.act_format_argmin(a) == SEL.act_format_argmin(b)
+
+
+def test_act_format_argmin_ties_and_zero_tensor():
+    assert SEL.act_format_argmin([1.0, 1.0, 0.5, 0.5, 2.0]) == 2
+    sse = SEL.act_format_sse(np.zeros((2, 32), np.float16))
+    assert not sse.any() and SEL.act_format_argmin(sse) == 0
