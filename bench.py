@@ -33,7 +33,7 @@ L2_BYTES = 126 * 2 ** 20
 # dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant kernel, from an ncu
 # capture of the GEGLU-in projection (M 2048, K 1280, N 10240; profiles/gemm_ts_f16_sdxl_geglu_in.md).
 # Set to None whenever the kernel changes until it is captured again.
-GEMM_TRAFFIC_PER_LAUNCH = {"bytes": 44.28e6, "launch": "2048x1280x10240 (GEGLU-in)",
+GEMM_TRAFFIC_PER_LAUNCH = {"bytes": 43.68e6, "launch": "2048x1280x10240 (GEGLU-in)",
                            "algorithmic_bytes": 99.8e6}
 
 
@@ -145,6 +145,7 @@ def calibrate_lut(torch, cl, X, buckets):
     lut = np.zeros((len(X), len(buckets)), dtype=np.int64)
     kappa = np.zeros((len(X), len(buckets)))
     qp = [[None] * len(buckets) for _ in X]
+    sse = np.zeros((len(X), len(buckets), 5))
     for li, xs in enumerate(X):
         for j, x in enumerate(xs):
             sums = cl.act_moments(x).cpu().numpy()
@@ -152,7 +153,31 @@ def calibrate_lut(torch, cl, X, buckets):
             lut[li, j] = cl.route(kappa[li, j], snr[buckets[j] * 100 + 50], False)
             if lut[li, j] <= 2:
                 qp[li][j] = cl.scale_zp(int(lut[li, j]), float(sums[5]), float(sums[6]))
-    return lut, kappa, qp
+            sse[li, j] = cl.act_format_sse(x)[0].cpu().numpy()   # Eq. format-argmin, for comparison
+    return lut, kappa, qp, sse
+
+
+def route_vs_argmin(cl, lut, sse):
+    """How the kappa / SNR route (Sec. 3.3) compares with the exhaustive argmin of Eq.
+    format-argmin on the same calibration tensors."""
+    best = np.array([[cl.act_format_argmin(sse[i, j]) for j in range(sse.shape[1])] for i in range(sse.shape[0])])
+    picked = np.take_along_axis(sse, lut[..., None], axis=2)[..., 0]
+    opt = np.take_along_axis(sse, best[..., None], axis=2)[..., 0]
+    ratio = picked / np.maximum(opt, 1e-300)
+    # the same over the per-tensor formats (0..2), the only ones the route picks off the shortcut layers
+    best3 = np.array([[cl.act_format_argmin(list(sse[i, j, :3]) + [np.inf, np.inf]) for j in range(sse.shape[1])]
+                      for i in range(sse.shape[0])])
+    opt3 = np.take_along_axis(sse, best3[..., None], axis=2)[..., 0]
+    ratio3 = picked / np.maximum(opt3, 1e-300)
+    return {"agree": round(float((best == lut).mean()), 3),
+            "sse_ratio_route_over_argmin": {"median": round(float(np.median(ratio)), 3),
+                                            "max": round(float(ratio.max()), 3)},
+            "agree_per_tensor_formats": round(float((best3 == lut).mean()), 3),
+            "sse_ratio_route_over_per_tensor_argmin": {"median": round(float(np.median(ratio3)), 3),
+                                                       "max": round(float(ratio3.max()), 3)},
+            "per_tensor_argmin_formats": {int(f): int(c) for f, c in zip(*np.unique(best3, return_counts=True))},
+            "argmin_formats": {int(f): int(c) for f, c in zip(*np.unique(best, return_counts=True))},
+            "route_formats": {int(f): int(c) for f, c in zip(*np.unique(lut, return_counts=True))}}
 
 
 def main():
@@ -164,6 +189,9 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-variants", action="store_true", help="skip the per-variant matrix")
+    ap.add_argument("--dynamic-scales", action="store_true",
+                    help="quantize with each tensor's own range (Alg. 3, the DiT path) instead of the "
+                         "calibrated static scales of the UNet path (Alg. 2)")
     ap.add_argument("--layers", default="all", help="comma-separated layer indices (smaller cases for profiling)")
     ap.add_argument("--buckets", default="all", help="comma-separated timestep buckets")
     args = ap.parse_args()
@@ -200,7 +228,7 @@ def main():
     nb = len(buckets)
     host = host_inputs(WL, layer_ids, buckets)
     W, bias, X = build_inputs(torch, host, device)
-    lut, kappa, qp = calibrate_lut(torch, cl, X, buckets)
+    lut, kappa, qp, cal_sse = calibrate_lut(torch, cl, X, buckets)
     st = torch.zeros(1, dtype=torch.int32, device=device)
     stream = torch.cuda.current_stream()
 
@@ -239,7 +267,10 @@ def main():
             for li, (_, M, K, N) in enumerate(layers):
                 f = int(lut[li, bk])
                 if "q" in parts:
-                    cl.linear_prepare_static(X[li][bk], f, qp[li][bk], ws[li], st)
+                    if args.dynamic_scales:
+                        cl.linear_prepare(X[li][bk], f, ws[li], st)
+                    else:
+                        cl.linear_prepare_static(X[li][bk], f, qp[li][bk], ws[li], st)
                 if "g" in parts:
                     cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
 
@@ -272,8 +303,9 @@ def main():
             run_step(key)
 
     # kernel launches per step: select 1 + pack 1 per layer (one MMA class: no slot ranking);
-    # per linear 1 quantizer kernel (static scales or MX) + 1 GEMM
-    launches = 2 * len(layers) + 2 * len(layers) * nb
+    # per linear 1 quantizer kernel (static scales or MX; 2 with dynamic per-tensor scales) + 1 GEMM
+    launches = 2 * len(layers) + sum(
+        (2 if args.dynamic_scales and lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(nb))
     for li, (_, M, K, N) in enumerate(layers):
         for bk in range(nb):
             mx = lut[li, bk] >= 3
@@ -336,8 +368,9 @@ def main():
                    "layers": len(layers), "buckets": nb, "global_batch": 2 * world,
                    "tokens": [M for (_, M, _, _) in layers], "weight_palette": "W8 {INT8-sym, INT8-asym, MXINT8}",
                    "activation_formats_used": sorted(set(int(v) for v in lut.ravel())),
-                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant (static calibrated "
-                           "per-(layer, bucket) scales, Alg. 2) + GEMM, one CUDA graph",
+                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant (%s) + GEMM, one "
+                           "CUDA graph" % ("dynamic per-tensor scales, Alg. 3" if args.dynamic_scales else
+                                           "static calibrated per-(layer, bucket) scales, Alg. 2"),
                    "l2": "inputs larger than L2 (%.0f MB of activations per step)" %
                          (sum(x.numel() * 2 for xs in X for x in xs) / 1e6),
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
@@ -361,6 +394,7 @@ def main():
                       "frac": round(quant_gbs / pk["hbm_gbs"], 4), "ms_per_step": round(quant_ms / K_, 4),
                       "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"},
         "variants": variants,
+        "calibration": route_vs_argmin(cl, lut, cal_sse),
         "gpu_launches": launches * K_,
         "clocks": clocks,
     }

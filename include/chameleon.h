@@ -159,6 +159,24 @@ cham_status chameleon_scale_zp(int fmt, float lo, float hi, cham_qparams* out);
 cham_status chameleon_act_quant_static(const void* X, int M, int K, int fmt, const cham_qparams* params,
                                        void* qact, size_t qact_bytes, int* dev_status, void* stream);
 
+/* ------------------------------------------------------------------ Eq. format-argmin */
+
+/* The exhaustive activation-format choice of Eq. format-argmin (Sec. 3.1), the objective that the
+ * kappa / SNR route approximates: for one activation tensor X (device, fp16 M x K, K a multiple of
+ * 32), SSE_f = sum over the elements of (x - DQ_f(Q_f(x)))^2 for the five activation formats f =
+ * 0..4 at their native granularity -- INT8-asym, E4M3, E5M2 with ScaleZP of X's own range (as
+ * chameleon_act_quant), MXFP8 and MXINT8 per 32-element block -- ADDED to sse (device, 5 doubles),
+ * so that calls accumulate over the calibration tensors of one (layer, bucket).  Each element's
+ * error is one fp32 fused multiply-add, squared and summed in fp32 over 8 elements, then in fp64
+ * in a fixed order (deterministic).  ws (device) >= the size query.  Non-finite input sets
+ * *dev_status = CHAM_ERR_NONFINITE (sums then unspecified). */
+cham_status chameleon_act_format_sse_workspace_size(int M, int K, size_t* ws_bytes);
+cham_status chameleon_act_format_sse(const void* X, int M, int K, double* sse, void* ws, size_t ws_bytes,
+                                     int* dev_status, void* stream);
+/* f* = the first format with the least accumulated error (host, sse = 5 doubles; ties go to the
+ * earlier format in palette order); -1 when sse is NULL. */
+int chameleon_act_format_argmin(const double* sse);
+
 /* ------------------------------------------------------------------ a5: weight-format selection */
 
 /* Per output channel c of W (device, fp16 N x K): SSE_f(c) = sum_k (w - DQ_f(Q_f(w)))^2 for every

@@ -35,6 +35,7 @@ EXPORTS = [
     "chameleon_linear_gemm", "chameleon_act_quant_noalloc", "chameleon_debug_stall_next_gemm",
     "chameleon_scale_zp", "chameleon_act_quant_static", "chameleon_linear_prepare_static",
     "chameleon_linear_prepare_groups", "chameleon_linear_gemm_ex",
+    "chameleon_act_format_sse_workspace_size", "chameleon_act_format_sse", "chameleon_act_format_argmin",
 ]
 
 
@@ -115,6 +116,9 @@ def lib():
         "chameleon_linear_prepare_static": (i32, [vp, i32, i32, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
         "chameleon_linear_prepare_groups": (i32, [vp, i32, i32, i32, i32, vp, sz, vp, vp]),
         "chameleon_linear_gemm_ex": (i32, [vp, i32, pdesc, vp, i32, i32, vp, vp, i32, vp, sz, vp, vp]),
+        "chameleon_act_format_sse_workspace_size": (i32, [i32, i32, psz]),
+        "chameleon_act_format_sse": (i32, [vp, i32, i32, vp, vp, sz, vp, vp]),
+        "chameleon_act_format_argmin": (i32, [ctypes.POINTER(ctypes.c_double)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -237,6 +241,30 @@ def split_qact(qact, M, K):
     z, fmt = int(np.frombuffer(pbytes[4:8], np.int32)[0]), int(np.frombuffer(pbytes[12:16], np.int32)[0])
     e8 = qact[P + 256:P + 256 + n // 32].view(M, K // 32)
     return codes, {"s": s, "z": z, "inv": inv, "fmt": fmt}, e8
+
+
+# ------------------------------------------------------------------ Eq. format-argmin
+def act_format_sse(X, out=None, dev_status=None, stream=None):
+    """SSE of the five activation formats on fp16 X (M x K, CUDA), added to `out` (5 float64 on the
+    device; zeros when not given).  Returns (out, dev_status)."""
+    import torch
+    M, K = X.shape
+    if out is None:
+        out = torch.zeros(5, dtype=torch.float64, device=X.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
+    w = ctypes.c_size_t()
+    check(lib().chameleon_act_format_sse_workspace_size(M, K, ctypes.byref(w)))
+    ws = _bytes(w.value, X.device)
+    check(lib().chameleon_act_format_sse(_ptr(X), M, K, _ptr(out), _ptr(ws), w.value, _ptr(dev_status),
+                                         _stream(stream)))
+    return out, dev_status
+
+
+def act_format_argmin(sse_host):
+    """First format of the activation palette with the least error (host)."""
+    a = (ctypes.c_double * 5)(*[float(v) for v in sse_host])
+    return lib().chameleon_act_format_argmin(a)
 
 
 # ------------------------------------------------------------------ a5

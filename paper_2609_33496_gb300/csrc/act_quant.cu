@@ -349,6 +349,99 @@ __global__ void __launch_bounds__(256)
   if (nonfinite) set_status(dev_status, CHAM_ERR_NONFINITE);
 }
 
+// ------------------------------------------------------------------ activation-format argmin (Eq. format-argmin)
+// Sum over 8 elements of (x - s * deq)^2: the error of each element rounded once (fma), squared
+// and summed in fp32 (a fixed order).  s = 1 for the MX formats, whose deq is the full value.
+CHAM_DEV float sq_err8(const float (&x)[8], const uint4& deq, float s) {
+  const uint32_t d[4] = {deq.x, deq.y, deq.z, deq.w};
+  float acc = 0.f;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const float2 q = __half22float2(u32_as_h2(d[j]));
+    const float ea = fmaf(-q.x, s, x[2 * j]), eb = fmaf(-q.y, s, x[2 * j + 1]);
+    acc = __fadd_rn(acc, __fadd_rn(__fmul_rn(ea, ea), __fmul_rn(eb, eb)));
+  }
+  return acc;
+}
+
+// Per CTA: SSE_f for the five activation formats over its vectors, f = 0..4 (Sec. 3.1): the
+// per-tensor formats with ScaleZP of the tensor's range (reduced from the range partials), the
+// MX formats per 32-element block (four consecutive lanes per block, as in the MX encoder).
+__global__ void __launch_bounds__(256)
+    k_act_format_sse(const uint4* __restrict__ X, int64_t nvec, const RangePartial* __restrict__ parts, int nparts,
+                     double* __restrict__ sse_parts, int* dev_status) {
+  griddep_wait();  // the range partials
+  griddep_launch_dependents();
+  float lo, hi;
+  uint32_t nf;
+  reduce_partials(parts, nparts, lo, hi, nf);
+  const TensorParams p0 = scale_zp(CHAM_A_INT8_ASYM, lo, hi);
+  const TensorParams p1 = scale_zp(CHAM_A_E4M3, lo, hi);
+  const TensorParams p2 = scale_zp(CHAM_A_E5M2, lo, hi);
+  if (blockIdx.x == 0 && threadIdx.x == 0 && nf) set_status(dev_status, CHAM_ERR_NONFINITE);
+  double acc[5] = {0, 0, 0, 0, 0};
+  const int lane = threadIdx.x & 31;
+  const int64_t warp_global = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t span = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t base = warp_global * 32; base < nvec; base += span) {
+    const int64_t i = base + lane;  // nvec is a multiple of 4: the lanes of one block agree
+    const uint4 v = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    float x[8];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 t = __half22float2(u32_as_h2(w[j]));
+      x[2 * j] = t.x;
+      x[2 * j + 1] = t.y;
+    }
+    uint2 c;
+    uint4 d;
+    int byte;
+    uint32_t nfx = 0;
+    float e[5];
+    encode8_tensor<CHAM_A_INT8_ASYM, true>(v, p0, c, d);
+    e[0] = sq_err8(x, d, p0.s);
+    encode8_tensor<CHAM_A_E4M3, true>(v, p1, c, d);
+    e[1] = sq_err8(x, d, p1.s);
+    encode8_tensor<CHAM_A_E5M2, true>(v, p2, c, d);
+    e[2] = sq_err8(x, d, p2.s);
+    encode8_mx<CHAM_A_MXFP8, true>(v, lane, c, d, byte, nfx);
+    e[3] = sq_err8(x, d, 1.f);
+    encode8_mx<CHAM_A_MXINT8, true>(v, lane, c, d, byte, nfx);
+    e[4] = sq_err8(x, d, 1.f);
+    if (i < nvec) {
+#pragma unroll
+      for (int f = 0; f < 5; ++f) acc[f] += static_cast<double>(e[f]);
+    }
+  }
+  __shared__ double sh[5][8];
+#pragma unroll
+  for (int f = 0; f < 5; ++f) {
+    double a = acc[f];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
+    if (lane == 0) sh[f][threadIdx.x >> 5] = a;
+  }
+  __syncthreads();
+  if (threadIdx.x < 5) {
+    double a = 0;
+    for (int k = 0; k < static_cast<int>(blockDim.x >> 5); ++k) a += sh[threadIdx.x][k];
+    sse_parts[static_cast<int64_t>(blockIdx.x) * 5 + threadIdx.x] = a;
+  }
+}
+
+// Adds the CTAs' sums, in CTA order, to out[0..4] (so that calls accumulate over the
+// calibration tensors of one layer and bucket).
+__global__ void __launch_bounds__(32) k_act_format_sse_finish(const double* __restrict__ sse_parts, int nparts,
+                                                             double* __restrict__ out) {
+  griddep_wait();
+  if (threadIdx.x < 5) {
+    double a = 0;
+    for (int k = 0; k < nparts; ++k) a += sse_parts[static_cast<int64_t>(k) * 5 + threadIdx.x];
+    out[threadIdx.x] += a;
+  }
+}
+
 // ------------------------------------------------------------------ calibration power sums (Alg. 1)
 __global__ void __launch_bounds__(256) k_act_moments(const uint4* __restrict__ X, int64_t nvec,
                                                     MomentPartial* __restrict__ parts) {
@@ -480,6 +573,14 @@ void launch_act_quant(int fmt, const ActQuantArgs& a, bool codes, bool deq, cuda
   if (codes && deq) dispatch<true, true>(fmt, a, st);
   else if (codes) dispatch<true, false>(fmt, a, st);
   else dispatch<false, true>(fmt, a, st);
+}
+
+void launch_act_format_sse(const uint4* X, int64_t nvec, RangePartial* parts, int nparts, double* sse_parts,
+                           double* out, int* dev_status, cudaStream_t st) {
+  launch_pdl(k_act_range, dim3(nparts), dim3(256), 0, st, X, nvec, parts);
+  launch_pdl(k_act_format_sse, dim3(nparts), dim3(256), 0, st, X, nvec, static_cast<const RangePartial*>(parts),
+             nparts, sse_parts, dev_status);
+  launch_pdl(k_act_format_sse_finish, dim3(1), dim3(32), 0, st, static_cast<const double*>(sse_parts), nparts, out);
 }
 
 void launch_act_moments(const uint4* X, int64_t nvec, int64_t count, MomentPartial* parts, int nparts,

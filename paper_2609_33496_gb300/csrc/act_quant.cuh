@@ -44,6 +44,10 @@ int range_grid(int64_t nvec, int num_sms);
 int group_grid(int64_t nvec, int n_groups, int num_sms);
 constexpr int kMaxGroups = 64;  // per-sample groups: the scale slots of the linear workspace
 void launch_act_quant(int fmt, const ActQuantArgs& a, bool codes, bool deq, cudaStream_t st);
+// Eq. format-argmin: range pass, per-CTA SSE of the five activation formats (nparts CTAs, 5
+// doubles each in sse_parts), then a one-CTA sum added to out[0..4].
+void launch_act_format_sse(const uint4* X, int64_t nvec, RangePartial* parts, int nparts, double* sse_parts,
+                           double* out, int* dev_status, cudaStream_t st);
 void launch_act_moments(const uint4* X, int64_t nvec, int64_t count, MomentPartial* parts, int nparts,
                         double* out, cudaStream_t st);
 

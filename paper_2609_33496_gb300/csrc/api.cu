@@ -419,6 +419,55 @@ cham_status chameleon_act_quant_static(const void* X, int M, int K, int fmt, con
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "act_quant_static launch");
 }
 
+// ---------------------------------------------------------------- Eq. format-argmin (calibration)
+namespace {
+struct SseWs {
+  size_t parts, sse;
+  size_t total;
+};
+SseWs sse_ws(int64_t nvec) {
+  const size_t n = static_cast<size_t>(cham::range_grid(nvec, num_sms_current()));
+  SseWs L;
+  L.parts = 0;
+  L.sse = round_up(n * sizeof(cham::RangePartial), 256);
+  L.total = L.sse + round_up(n * 5 * sizeof(double), 256);
+  return L;
+}
+}  // namespace
+
+cham_status chameleon_act_format_sse_workspace_size(int M, int K, size_t* ws_bytes) {
+  if (M <= 0 || K <= 0 || K % 32 != 0 || ws_bytes == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "M=%d K=%d (K must be a multiple of 32)", M, K);
+  *ws_bytes = sse_ws(static_cast<int64_t>(M) * K / 8).total;
+  return CHAM_OK;
+}
+
+cham_status chameleon_act_format_sse(const void* X, int M, int K, double* sse, void* ws, size_t ws_bytes,
+                                     int* dev_status, void* stream) {
+  cham_status s = check_act_args(X, M, K, CHAM_A_INT8_ASYM, false);
+  if (s != CHAM_OK) return s;
+  if (sse == nullptr || reinterpret_cast<uintptr_t>(sse) % 8 != 0)
+    return fail(CHAM_ERR_INVALID_ARG, "sse must be an 8-byte aligned device pointer");
+  const int64_t nvec = static_cast<int64_t>(M) * K / 8;
+  const SseWs L = sse_ws(nvec);
+  if (ws == nullptr || !aligned16(ws)) return fail(CHAM_ERR_INVALID_ARG, "ws must be 16-byte aligned");
+  if (ws_bytes < L.total) return fail(CHAM_ERR_WORKSPACE, "ws %zu < %zu bytes", ws_bytes, L.total);
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  cham::launch_act_format_sse(static_cast<const uint4*>(X), nvec, reinterpret_cast<cham::RangePartial*>(w + L.parts),
+                              cham::range_grid(nvec, num_sms_current()), reinterpret_cast<double*>(w + L.sse), sse,
+                              dev_status, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "act_format_sse launch");
+}
+
+int chameleon_act_format_argmin(const double* sse) {
+  if (sse == nullptr) return -1;
+  int best = 0;
+  for (int f = 1; f < 5; ++f)
+    if (sse[f] < sse[best]) best = f;
+  return best;
+}
+
 // ---------------------------------------------------------------- a5
 cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_t palette_mask, uint8_t* fmt_out,
                                             double* sse_out, void* stream) {

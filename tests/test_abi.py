@@ -10,6 +10,7 @@ import pytest
 
 from oracle import schedule as S
 from oracle import formats as F
+from oracle import select as SEL
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "chameleon.h")
@@ -167,3 +168,12 @@ def test_groups_and_output_type_argument_checks(cl):
         assert L.chameleon_linear_gemm_ex(x, 64, ctypes.byref(d), x, F.A_E4M3, n, None, x, yt, x, 1 << 19, x,
                                           None) == cl.ERR_INVALID_ARG
     assert cl.MAX_GROUPS == 64
+
+
+def test_act_format_argmin_host_helper(cl):
+    for sse in ([3.0, 2.0, 2.0, 5.0, 1.0], [0.0] * 5, [1.0, 0.5, 0.25, 0.25, 0.5], [7, 7, 7, 7, 6.999]):
+        assert cl.act_format_argmin(sse) == SEL.act_format_argmin(sse)
+    assert cl.lib().chameleon_act_format_argmin(None) == -1
+    w = ctypes.c_size_t()
+    assert cl.lib().chameleon_act_format_sse_workspace_size(16, 48, ctypes.byref(w)) == cl.ERR_INVALID_ARG
+    assert cl.lib().chameleon_act_format_sse_workspace_size(16, 64, ctypes.byref(w)) == cl.OK and w.value >= 256

@@ -249,13 +249,15 @@ def test_act_format_sse_against_naive_codecs(seed):
 
 
 def test_act_format_sse_zero_on_the_e4m3_grid():
-    """A tensor of E4M3 grid values whose largest magnitude is 448: per-tensor E4M3 reproduces it
-    exactly (s = 1), and so does MXFP8 (power-of-two block scaling keeps grid values on the grid);
-    INT8-asym and E5M2 cannot.  The argmin is E4M3, the earlier of the two exact formats."""
+    """A tensor of E4M3 grid values with 448 in every 32-element block: per-tensor E4M3 reproduces
+    it exactly (s = 1), and so does MXFP8 (every block's shared exponent is 0); INT8-asym and E5M2
+    cannot.  The argmin is E4M3, the earlier of the two exact formats.  (A block whose largest
+    value is 1.875 * 2^e would not be exact under MXFP8: the OCP exponent maps it to 480, which
+    saturates to 448.)"""
     vals = np.array([g for g, _ in E4M3 if g >= 2.0 ** -6], np.float64)
     g = np.random.default_rng(5)
     x = g.choice(vals, (4, 96)) * g.choice([-1.0, 1.0], (4, 96))
-    x[0, 0] = 448.0
+    x[:, ::32] = 448.0
     X = x.astype(np.float16)
     assert np.array_equal(X.astype(np.float64), x)
     sse = SEL.act_format_sse(X)
