@@ -368,3 +368,38 @@ def weight_dequant(q, nf4_levels=None):
         return L[c] * s
     body = {W_MXINT8: "int8", W_MXINT4: "int4", W_MXFP4: "e2m1"}[fmt]
     return mx_dequant_rows(c.astype(np.uint8), q["e8m0"], body)
+
+
+# ---------------------------------------------------------------- group-wise weight formats (Sec. 3.5 forks)
+GROUP_SIZES = (32, 64, 128, 192, 288)
+
+
+def group_bounds(K, g):
+    """[k0, k1) of each group of one row: runs of g consecutive input channels, the last one
+    shorter when g does not divide K (reading R24)."""
+    return [(k0, min(k0 + g, K)) for k0 in range(0, K, g)]
+
+
+def weight_quant_grouped(W, fmt, g, nf4_levels=None):
+    """Group-wise quantization of a non-MX weight format (the DiT and few-step forks, Sec. 3.5):
+    every run of g input channels of every output channel is quantized by the format's own rule
+    (weight_quant applied to that slice: its scale, and zero point for asym, from the group's
+    statistics).  Returns {"fmt", "g", "groups": [(k0, k1, weight_quant dict)]}."""
+    if W_IS_MX[fmt]:
+        raise ValueError("MX formats carry their own 32-element blocks")
+    W = np.asarray(W)
+    return {"fmt": fmt, "g": g,
+            "groups": [(k0, k1, weight_quant(W[:, k0:k1], fmt, nf4_levels)) for k0, k1 in group_bounds(W.shape[1], g)]}
+
+
+def weight_dequant_grouped(q, nf4_levels=None):
+    """DQ of weight_quant_grouped's output (R24): the code's value times the group scale stored as
+    fp16 (the weights' own type), the product rounded once to fp16.  float64 N x K."""
+    N = q["groups"][0][2]["codes"].shape[0]
+    K = q["groups"][-1][1]
+    out = np.zeros((N, K))
+    for k0, k1, qq in q["groups"]:
+        s16 = qq["s"].astype(np.float16).astype(np.float64)
+        v = weight_dequant(dict(qq, s=np.ones_like(qq["s"])), nf4_levels)  # the codes' values
+        out[:, k0:k1] = (v * s16[:, None]).astype(np.float16)    # exact product, one rounding
+    return out

@@ -97,3 +97,47 @@ def act_format_argmin(sse):
         if sse[f] < sse[best]:
             best = f
     return best
+
+
+# ---------------------------------------------------------------- per-linear (g, f) search (Sec. 3.5 forks)
+def input_energy(X):
+    """Activation energy of each input channel, sum_m x[m, k]^2 in fp64 (the input-aware SQNR of
+    the DiT fork weights channel k's error by E[x_k^2]; the sum over the calibration rows is that
+    expectation times their number, which leaves the argmax unchanged)."""
+    x = np.asarray(X).astype(np.float64)
+    return (x * x).sum(axis=0)
+
+
+def group_candidates(palette, groups=F.GROUP_SIZES):
+    """The (g, f) tuples searched, in order (ties go to the earlier one): g-major; at every g the
+    non-MX members of the palette in palette order, and at g = 32 the MX members too (their block
+    is 32 whatever g is searched)."""
+    out = []
+    for g in groups:
+        for f in palette:
+            if not F.W_IS_MX[f] or g == 32:
+                out.append((g, f))
+    return out
+
+
+def grouped_dequant(W, g, f):
+    """DQ of W in format f at group size g (MX formats: their own 32-element blocks)."""
+    L = nf4_levels_fp16()
+    if F.W_IS_MX[f]:
+        return F.weight_dequant(F.weight_quant(W, f))
+    return F.weight_dequant_grouped(F.weight_quant_grouped(W, f, g, nf4_levels=L), nf4_levels=L)
+
+
+def select_grouped(W, palette, groups=F.GROUP_SIZES, energy=None):
+    """Per-linear (g, f) choice: the candidate with the highest SQNR, i.e. the least weighted
+    squared error sum_{c,k} e_k (w - DQ(w))^2 (the signal term sum e_k w^2 is the same for every
+    candidate); e_k = 1 without activation energies.  Returns ((g, f), scores fp64, candidates)."""
+    w64 = np.asarray(W).astype(np.float64)
+    e = np.ones(w64.shape[1]) if energy is None else np.asarray(energy, dtype=np.float64)
+    cands = group_candidates(palette, groups)
+    scores = np.array([(((w64 - grouped_dequant(W, g, f)) ** 2) * e[None, :]).sum() for g, f in cands])
+    best = 0
+    for i in range(1, len(cands)):
+        if scores[i] < scores[best]:
+            best = i
+    return cands[best], scores, cands

@@ -282,3 +282,109 @@ def test_act_format_argmin_ties_and_zero_tensor():
     assert SEL.act_format_argmin([1.0, 1.0, 0.5, 0.5, 2.0]) == 2
     sse = SEL.act_format_sse(np.zeros((2, 32), np.float16))
     assert not sse.any() and SEL.act_format_argmin(sse) == 0
+
+
+# ---------------------------------------------------------------- group-wise formats and the (g, f) search
+GROUPED_W4 = [F.W_INT4_ASYM, F.W_NF4, F.W_E2M1]
+
+
+def test_group_bounds_ragged_tail():
+    assert F.group_bounds(320, 192) == [(0, 192), (192, 320)]
+    assert F.group_bounds(320, 288) == [(0, 288), (288, 320)]
+    assert F.group_bounds(1152, 288) == [(0, 288), (288, 576), (576, 864), (864, 1152)]
+    assert F.group_bounds(64, 128) == [(0, 64)]
+
+
+@pytest.mark.parametrize("fmt", [F.W_INT8_SYM, F.W_INT8_ASYM, F.W_INT4_SYM, F.W_INT4_ASYM, F.W_NF4, F.W_E2M1])
+def test_one_group_is_the_per_channel_code(fmt):
+    """A group as long as the row has the per-channel format's codes, scale and zero point."""
+    W = (RNG.standard_normal((5, 96)) * 0.05).astype(np.float16)
+    L = nf4.nf4_levels_fp16()
+    (k0, k1, q), = F.weight_quant_grouped(W, fmt, 128, nf4_levels=L)["groups"]
+    ref = F.weight_quant(W, fmt, nf4_levels=L)
+    assert (k0, k1) == (0, 96)
+    assert np.array_equal(q["codes"], ref["codes"]) and np.array_equal(q["s"], ref["s"])
+    assert np.array_equal(q["z"], ref["z"])
+
+
+def naive_grouped_dq(W, fmt, g):
+    """Independent restatement: per group, the scale rule of Sec. 3.2 / App. A.7 in fp32, nearest
+    code by search, then value x fp16(scale) rounded to fp16."""
+    L = [float(v) for v in nf4.nf4_levels_fp16()]
+    e2m1 = sorted(set(E2M1_POS + [-v for v in E2M1_POS]))
+    w = np.asarray(W).astype(np.float64)
+    out = np.zeros_like(w)
+    for c in range(w.shape[0]):
+        for k0, k1 in F.group_bounds(w.shape[1], g):
+            seg = w[c, k0:k1]
+            amax = float(np.abs(seg).max())
+            if fmt == F.W_INT4_ASYM:
+                lo, hi = min(float(seg.min()), 0.0), max(float(seg.max()), 0.0)
+                d = f32(hi - lo)
+                s, inv = (1.0, 1.0) if d == 0 else (f32(d / 15), f32(15 / d))
+                z = 0 if d == 0 else min(max(nearest(f32(-lo * inv), range(-1, 17), even_int), 0), 15)
+                vals = [min(max(nearest(f32(v * inv), range(-40, 41), even_int) + z, 0), 15) - z for v in seg]
+            elif fmt == F.W_E2M1:
+                s, inv = (1.0, 1.0) if amax == 0 else (f32(amax / 6), f32(6 / amax))
+                even = (0.0, 1.0, 2.0, 4.0, -1.0, -2.0, -4.0)     # the values with an even mantissa bit
+                vals = [nearest(f32(v * inv), e2m1, lambda cc: [x for x in cc if x in even][0]) for v in seg]
+            else:
+                s = amax if amax != 0 else 1.0
+                vals = [nearest(f32(v / s), L, lambda cc: min(cc)) for v in seg]
+            s16 = float(np.float16(s))
+            out[c, k0:k1] = [float(np.float16(v * s16)) for v in vals]
+    return out
+
+
+@pytest.mark.parametrize("fmt", GROUPED_W4)
+@pytest.mark.parametrize("g", [32, 64, 192])
+def test_grouped_dq_against_naive(fmt, g):
+    W = (RNG.standard_t(4, (3, 320)) * 0.03).astype(np.float16)
+    L = nf4.nf4_levels_fp16()
+    dq = F.weight_dequant_grouped(F.weight_quant_grouped(W, fmt, g, nf4_levels=L), nf4_levels=L)
+    np.testing.assert_array_equal(dq, naive_grouped_dq(W, fmt, g))
+
+
+def test_grouped_search_finds_the_exact_grid():
+    """Rows built on an INT4-asym grid per 64-channel group, with power-of-two scales that differ
+    between groups: (64, INT4-asym) reproduces them exactly and wins; 128 and coarser mix two
+    scales in one group and do not."""
+    g = np.random.default_rng(12)
+    N, K = 4, 256
+    W = np.zeros((N, K))
+    for c in range(N):
+        for k0 in range(0, K, 64):
+            s = 2.0 ** g.integers(-9, -4)
+            q = g.integers(0, 16, 64)
+            q[0], q[1] = 0, 15                      # the group's range spans the whole grid
+            W[c, k0:k0 + 64] = (q - 5) * s          # zero point 5: lo = -5 s, hi = 10 s
+    W16 = W.astype(np.float16)
+    assert np.array_equal(W16.astype(np.float64), W)
+    (gb, fb), scores, cands = SEL.select_grouped(W16, GROUPED_W4)
+    assert (gb, fb) == (32, F.W_INT4_ASYM) or (gb, fb) == (64, F.W_INT4_ASYM)
+    assert scores[cands.index((64, F.W_INT4_ASYM))] == 0
+    assert scores[cands.index((128, F.W_INT4_ASYM))] > 0
+
+
+def test_energy_weighting():
+    W = (RNG.standard_normal((6, 128)) * 0.02).astype(np.float16)
+    pal = [F.W_INT4_ASYM, F.W_NF4]
+    _, plain, cands = SEL.select_grouped(W, pal)
+    _, const, _ = SEL.select_grouped(W, pal, energy=np.full(128, 3.0))
+    np.testing.assert_allclose(const, 3.0 * plain, rtol=1e-13)
+    e = np.zeros(128)
+    e[77] = 2.5
+    _, one, _ = SEL.select_grouped(W, pal, energy=e)
+    for i, (g, f) in enumerate(cands):
+        err = W.astype(np.float64)[:, 77] - SEL.grouped_dequant(W, g, f)[:, 77]
+        assert one[i] == pytest.approx(2.5 * (err ** 2).sum(), rel=1e-13)
+    X = np.array([[1.0, -2.0], [3.0, 0.5]], np.float16)
+    np.testing.assert_array_equal(SEL.input_energy(X), [10.0, 4.25])
+
+
+def test_candidate_order():
+    c = SEL.group_candidates([F.W_INT4_ASYM, F.W_NF4, F.W_E2M1, F.W_MXINT4, F.W_MXFP4])
+    assert c[:5] == [(32, 4), (32, 5), (32, 6), (32, 7), (32, 8)]
+    assert c[5:8] == [(64, 4), (64, 5), (64, 6)] and len(c) == 5 + 4 * 3
+    assert SEL.group_candidates([F.W_INT8_SYM, F.W_INT8_ASYM, F.W_MXINT8], (32, 64)) == [
+        (32, 0), (32, 1), (32, 2), (64, 0), (64, 1)]
