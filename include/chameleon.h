@@ -187,6 +187,33 @@ int chameleon_act_format_argmin(const double* sse);
 cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_t palette_mask,
                                             uint8_t* fmt_out, double* sse_out, void* stream);
 
+/* The per-linear (g, f) search of the DiT and few-step forks (Sec. 3.5).  Candidates, in search
+ * order (ties go to the earlier): for each group size g of group_mask (bit i = g_i of {32, 64,
+ * 128, 192, 288}, ascending), the non-MX members of palette_mask in palette order, and at g = 32
+ * the MX members too (their own 32-element blocks); chameleon_group_candidates lists them.
+ * scores (device, double [n_candidates]) = sum over channels c and input channels k of
+ * e_k * (w - DQ(w))^2 with DQ the group-wise decode (fp16 scale, product rounded to fp16) or the
+ * MX decode, e_k = energy[k] (device, double [K], e.g. chameleon_act_channel_energy sums over
+ * calibration activations: the input-aware SQNR) or 1 when energy is NULL.  The SQNR argmax is
+ * the score argmin (the signal term is the same for all candidates): chameleon_candidate_argmin.
+ * Each element error is one fp32 fma, weighted and squared in fp32, summed in fp32 over 8
+ * elements, then in fp64 in a fixed order.  K a multiple of 32, at most 256 groups per row.
+ * ws (device) >= the size query. */
+cham_status chameleon_group_candidates(uint32_t palette_mask, uint32_t group_mask, int* g_out, int* fmt_out,
+                                       int cap, int* n_out);
+cham_status chameleon_select_weight_groups_workspace_size(int N, int K, uint32_t palette_mask, uint32_t group_mask,
+                                                          size_t* ws_bytes);
+cham_status chameleon_select_weight_groups(const void* W, int N, int K, uint32_t palette_mask, uint32_t group_mask,
+                                           const double* energy, double* scores, void* ws, size_t ws_bytes,
+                                           void* stream);
+/* Index of the first smallest of n scores (host); -1 when n <= 0 or scores is NULL. */
+int chameleon_candidate_argmin(const double* scores, int n);
+
+/* Activation energy per input channel for the input-aware SQNR: energy[k] += sum_m x[m, k]^2
+ * (device, double [K]) over X (device, fp16 M x K, K a multiple of 8), so calls accumulate over
+ * calibration tensors.  Deterministic (fixed summation order). */
+cham_status chameleon_act_channel_energy(const void* X, int M, int K, double* energy, void* stream);
+
 /* ------------------------------------------------------------------ a6: weight pack */
 
 /* Packed-weight descriptor.  Channels are permuted (Sec. 5: "same-format sub-GEMMs after a
@@ -210,25 +237,39 @@ cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_
  *   scale          float [Np]: per-channel scale s (1 for MX and padding)
  *   zero           uint8 [Np]: zero point z (asym formats, else 0)
  *   e8m0           uint8 [tiles][Kp/64][128][2]: the two E8M0 exponents of each channel's chunk
- *                  (MX formats; 127 otherwise)
+ *                  (MX formats; 127 otherwise).  Group-wise blobs (group > 0): the zero points
+ *                  of the chunk's two 32-element blocks (asym formats, else 0)
  *   fmt            uint8 [Np]: format of each packed channel, 255 for padding
  *   perm           int32 [Np]: original channel of each packed channel, -1 for padding
- * with Np = 128 * (n_tiles[0] + n_tiles[1]) and Kp = K rounded up to 64. */
+ *   gscale         (group > 0 only) uint32 [tiles][Kp/64][128]: the fp16 scales of the chunk's
+ *                  two 32-element blocks (block 0 in the low half), each its group's scale
+ *                  rounded to fp16 (0 beyond K); the per-channel scale region then holds 1
+ * with Np = 128 * (n_tiles[0] + n_tiles[1]) and Kp = K rounded up to 64.  A group-wise blob has
+ * one non-MX format for every channel and a scale per run of `group` input channels (Sec. 3.5
+ * forks); its weights decode to fp16(value(code) * scale16), the product rounded once. */
 typedef struct {
   uint32_t magic;    /* 0x574D4843 ("CHMW") */
-  uint32_t version;  /* 1 */
+  uint32_t version;  /* 2 */
   int32_t N, K, Kp, bits;
   int32_t n_class[2];
   int32_t n_tiles[2];
   int32_t n_fmt[CHAM_W_NFORMATS];
-  int32_t reserved0;
+  int32_t group;              /* 0: per-channel (or MX) formats; g > 0: group-wise, g input channels */
   uint64_t off_codes, off_scale, off_zero, off_e8m0, off_fmt, off_perm, bytes;
-  uint8_t reserved[120];      /* pads the descriptor to 256 bytes */
+  uint64_t off_gscale;        /* group-wise blobs: the gscale region, else 0 */
+  uint8_t reserved[112];      /* pads the descriptor to 256 bytes */
 } cham_wpack_desc;
 
 /* Fill *desc for N x K weights whose selected formats are fmt_host (host, uint8 [N], all of one
  * bit width).  desc->bytes is the blob size. */
 cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* desc);
+
+/* A group-wise plan (the DiT and few-step forks, Sec. 3.5): every channel in format fmt (a non-MX
+ * format: INT8-sym, INT8-asym, INT4-sym, INT4-asym, NF4 or E2M1), one scale (and zero point) per
+ * run of `group` input channels along K -- group a multiple of 32 with at most 256 groups per row
+ * (the last group of a row is shorter when group does not divide K).  chameleon_pack_weights then
+ * takes a device format array holding fmt for every channel.  CHAM_ERR_INVALID_ARG otherwise. */
+cham_status chameleon_pack_plan_grouped(int N, int K, int fmt, int group, cham_wpack_desc* desc);
 
 /* The same plan from the palette alone, for palettes whose members all share one MMA class (every
  * 8-bit palette; 4-bit palettes without NF4, or NF4 alone): the layout then depends only on N, K

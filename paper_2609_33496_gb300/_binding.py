@@ -36,6 +36,8 @@ EXPORTS = [
     "chameleon_scale_zp", "chameleon_act_quant_static", "chameleon_linear_prepare_static",
     "chameleon_linear_prepare_groups", "chameleon_linear_gemm_ex",
     "chameleon_act_format_sse_workspace_size", "chameleon_act_format_sse", "chameleon_act_format_argmin",
+    "chameleon_pack_plan_grouped", "chameleon_group_candidates", "chameleon_select_weight_groups_workspace_size",
+    "chameleon_select_weight_groups", "chameleon_candidate_argmin", "chameleon_act_channel_energy",
 ]
 
 
@@ -45,11 +47,12 @@ class WPackDesc(ctypes.Structure):
                 ("N", ctypes.c_int32), ("K", ctypes.c_int32), ("Kp", ctypes.c_int32),
                 ("bits", ctypes.c_int32), ("n_class", ctypes.c_int32 * 2),
                 ("n_tiles", ctypes.c_int32 * 2), ("n_fmt", ctypes.c_int32 * 9),
-                ("reserved0", ctypes.c_int32),
+                ("group", ctypes.c_int32),
                 ("off_codes", ctypes.c_uint64), ("off_scale", ctypes.c_uint64),
                 ("off_zero", ctypes.c_uint64), ("off_e8m0", ctypes.c_uint64),
                 ("off_fmt", ctypes.c_uint64), ("off_perm", ctypes.c_uint64),
-                ("bytes", ctypes.c_uint64), ("reserved", ctypes.c_uint8 * 120)]
+                ("bytes", ctypes.c_uint64), ("off_gscale", ctypes.c_uint64),
+                ("reserved", ctypes.c_uint8 * 112)]
 
 
 assert ctypes.sizeof(WPackDesc) == 256
@@ -119,6 +122,12 @@ def lib():
         "chameleon_act_format_sse_workspace_size": (i32, [i32, i32, psz]),
         "chameleon_act_format_sse": (i32, [vp, i32, i32, vp, vp, sz, vp, vp]),
         "chameleon_act_format_argmin": (i32, [ctypes.POINTER(ctypes.c_double)]),
+        "chameleon_pack_plan_grouped": (i32, [i32, i32, i32, i32, pdesc]),
+        "chameleon_group_candidates": (i32, [u32, u32, vp, vp, i32, ctypes.POINTER(ctypes.c_int)]),
+        "chameleon_select_weight_groups_workspace_size": (i32, [i32, i32, u32, u32, psz]),
+        "chameleon_select_weight_groups": (i32, [vp, i32, i32, u32, u32, vp, vp, vp, sz, vp]),
+        "chameleon_candidate_argmin": (i32, [ctypes.POINTER(ctypes.c_double), i32]),
+        "chameleon_act_channel_energy": (i32, [vp, i32, i32, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -286,6 +295,58 @@ def pack_plan_palette(N, K, palette_mask):
     d = WPackDesc()
     check(lib().chameleon_pack_plan_palette(N, K, palette_mask, ctypes.byref(d)))
     return d
+
+
+GROUP_SIZES = (32, 64, 128, 192, 288)
+
+
+def group_mask(groups):
+    """Bit mask of group sizes (bit i = GROUP_SIZES[i])."""
+    return sum(1 << GROUP_SIZES.index(g) for g in groups)
+
+
+def pack_plan_grouped(N, K, fmt, group):
+    """Plan of a group-wise blob: every channel in fmt, one scale per `group` input channels."""
+    d = WPackDesc()
+    check(lib().chameleon_pack_plan_grouped(N, K, fmt, group, ctypes.byref(d)))
+    return d
+
+
+def group_candidates(palette_mask, gmask):
+    """The (g, f) candidates of a search, in search order."""
+    n = ctypes.c_int()
+    g = (ctypes.c_int * 64)()
+    f = (ctypes.c_int * 64)()
+    check(lib().chameleon_group_candidates(palette_mask, gmask, g, f, 64, ctypes.byref(n)))
+    return [(g[i], f[i]) for i in range(n.value)]
+
+
+def select_weight_groups(W, palette_mask, gmask, energy=None, stream=None):
+    """Scores (device float64, one per candidate) of the per-linear (g, f) search."""
+    import torch
+    N, K = W.shape
+    w = ctypes.c_size_t()
+    check(lib().chameleon_select_weight_groups_workspace_size(N, K, palette_mask, gmask, ctypes.byref(w)))
+    ws = _bytes(w.value, W.device)
+    scores = torch.empty(len(group_candidates(palette_mask, gmask)), dtype=torch.float64, device=W.device)
+    check(lib().chameleon_select_weight_groups(_ptr(W), N, K, palette_mask, gmask, _ptr(energy), _ptr(scores),
+                                               _ptr(ws), w.value, _stream(stream)))
+    return scores
+
+
+def candidate_argmin(scores_host):
+    a = (ctypes.c_double * len(scores_host))(*[float(v) for v in scores_host])
+    return lib().chameleon_candidate_argmin(a, len(scores_host))
+
+
+def act_channel_energy(X, energy=None, stream=None):
+    """energy[k] += sum_m X[m, k]^2 (device float64 [K], zeros when not given)."""
+    import torch
+    M, K = X.shape
+    if energy is None:
+        energy = torch.zeros(K, dtype=torch.float64, device=X.device)
+    check(lib().chameleon_act_channel_energy(_ptr(X), M, K, _ptr(energy), _stream(stream)))
+    return energy
 
 
 def pack_plan(N, K, fmt_host):

@@ -194,9 +194,11 @@ const int kClassOrder[2][5] = {{CHAM_W_INT4_SYM, CHAM_W_INT4_ASYM, CHAM_W_E2M1, 
 
 cham_status check_desc(const cham_wpack_desc* d) {
   if (d == nullptr) return fail(CHAM_ERR_INVALID_ARG, "descriptor is NULL");
-  if (d->magic != 0x574D4843u || d->version != 1) return fail(CHAM_ERR_INVALID_ARG, "not a packed-weight descriptor");
+  if (d->magic != 0x574D4843u || d->version != 2) return fail(CHAM_ERR_INVALID_ARG, "not a packed-weight descriptor");
   if (d->N <= 0 || d->K <= 0 || d->K % 32 != 0 || (d->bits != 4 && d->bits != 8))
     return fail(CHAM_ERR_INVALID_ARG, "descriptor sizes are invalid");
+  if (d->group < 0 || d->group % 32 != 0 || (d->group > 0 && (d->K + d->group - 1) / d->group > cham::kMaxRowGroups))
+    return fail(CHAM_ERR_INVALID_ARG, "descriptor group size %d", d->group);
   return CHAM_OK;
 }
 
@@ -252,7 +254,7 @@ const char* chameleon_status_string(cham_status s) {
 
 const char* chameleon_last_error_detail(void) { return g_detail; }
 
-int chameleon_version(void) { return 1; }
+int chameleon_version(void) { return 2; }
 
 // ---------------------------------------------------------------- a1 and the LUT builder
 int chameleon_bucket(int t, int T, int B) {
@@ -482,6 +484,108 @@ cham_status chameleon_select_weight_formats(const void* W, int N, int K, uint32_
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "select launch");
 }
 
+// ---------------------------------------------------------------- (g, f) search (Sec. 3.5 forks)
+namespace {
+const int kGroupSizes[5] = {32, 64, 128, 192, 288};
+
+int group_candidates(uint32_t palette_mask, uint32_t group_mask, cham::GroupCand* out, int cap) {
+  int n = 0;
+  for (int i = 0; i < 5; ++i) {
+    if (!((group_mask >> i) & 1u)) continue;
+    for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
+      if (!((palette_mask >> f) & 1u)) continue;
+      if (cham::w_is_mx(f) && kGroupSizes[i] != 32) continue;
+      if (n < cap) out[n] = cham::GroupCand{kGroupSizes[i], f};
+      ++n;
+    }
+  }
+  return n;
+}
+
+cham_status check_group_search(int N, int K, uint32_t palette_mask, uint32_t group_mask) {
+  if (N <= 0 || K <= 0 || K % 32 != 0) return fail(CHAM_ERR_INVALID_ARG, "N=%d K=%d (K must be a multiple of 32)", N, K);
+  if (palette_mask == 0 || (palette_mask & ~0x1FFu) != 0) return fail(CHAM_ERR_INVALID_ARG, "palette mask 0x%x", palette_mask);
+  if ((palette_mask & CHAM_PALETTE_W8) && (palette_mask & CHAM_PALETTE_W4))
+    return fail(CHAM_ERR_INVALID_ARG, "palette mixes 8-bit and 4-bit formats");
+  if (group_mask == 0 || (group_mask & ~0x1Fu) != 0) return fail(CHAM_ERR_INVALID_ARG, "group mask 0x%x", group_mask);
+  for (int i = 0; i < 5; ++i)
+    if (((group_mask >> i) & 1u) && (K + kGroupSizes[i] - 1) / kGroupSizes[i] > cham::kMaxRowGroups)
+      return fail(CHAM_ERR_INVALID_ARG, "K=%d has more than %d groups of %d", K, cham::kMaxRowGroups, kGroupSizes[i]);
+  cham::GroupCand c[cham::kMaxCands];
+  if (group_candidates(palette_mask, group_mask, c, cham::kMaxCands) == 0)
+    return fail(CHAM_ERR_INVALID_ARG, "no (g, f) candidate: palette 0x%x, groups 0x%x", palette_mask, group_mask);
+  return CHAM_OK;
+}
+
+size_t group_search_ws(int N, int K, int n_cand) {
+  return round_up(static_cast<size_t>(K) * 4, 256) + round_up(static_cast<size_t>(N) * n_cand * 8, 256);
+}
+}  // namespace
+
+cham_status chameleon_group_candidates(uint32_t palette_mask, uint32_t group_mask, int* g_out, int* fmt_out, int cap,
+                                       int* n_out) {
+  if (n_out == nullptr || cap < 0 || (cap > 0 && (g_out == nullptr || fmt_out == nullptr)))
+    return fail(CHAM_ERR_INVALID_ARG, "null output");
+  cham::GroupCand c[cham::kMaxCands];
+  const int n = group_candidates(palette_mask & 0x1FFu, group_mask & 0x1Fu, c, cham::kMaxCands);
+  for (int i = 0; i < n && i < cap; ++i) {
+    g_out[i] = c[i].g;
+    fmt_out[i] = c[i].f;
+  }
+  *n_out = n;
+  return CHAM_OK;
+}
+
+cham_status chameleon_select_weight_groups_workspace_size(int N, int K, uint32_t palette_mask, uint32_t group_mask,
+                                                          size_t* ws_bytes) {
+  cham_status s = check_group_search(N, K, palette_mask, group_mask);
+  if (s != CHAM_OK) return s;
+  if (ws_bytes == nullptr) return fail(CHAM_ERR_INVALID_ARG, "ws_bytes is NULL");
+  cham::GroupCand c[cham::kMaxCands];
+  *ws_bytes = group_search_ws(N, K, group_candidates(palette_mask, group_mask, c, cham::kMaxCands));
+  return CHAM_OK;
+}
+
+cham_status chameleon_select_weight_groups(const void* W, int N, int K, uint32_t palette_mask, uint32_t group_mask,
+                                           const double* energy, double* scores, void* ws, size_t ws_bytes,
+                                           void* stream) {
+  cham_status s = check_group_search(N, K, palette_mask, group_mask);
+  if (s != CHAM_OK) return s;
+  if (W == nullptr || !aligned16(W) || scores == nullptr || ws == nullptr || !aligned16(ws))
+    return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
+  cham::GroupSearchArgs a{};
+  a.n_cand = group_candidates(palette_mask, group_mask, a.cand, cham::kMaxCands);
+  const size_t need = group_search_ws(N, K, a.n_cand);
+  if (ws_bytes < need) return fail(CHAM_ERR_WORKSPACE, "ws %zu < %zu bytes", ws_bytes, need);
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  a.W = static_cast<const __half*>(W);
+  a.N = N;
+  a.K = K;
+  a.energy = energy;
+  a.energy32 = reinterpret_cast<float*>(w);
+  a.parts = reinterpret_cast<double*>(w + round_up(static_cast<size_t>(K) * 4, 256));
+  a.scores = scores;
+  cham::launch_select_groups(a, nf4_table(), static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "group search launch");
+}
+
+int chameleon_candidate_argmin(const double* scores, int n) {
+  if (scores == nullptr || n <= 0) return -1;
+  int best = 0;
+  for (int i = 1; i < n; ++i)
+    if (scores[i] < scores[best]) best = i;
+  return best;
+}
+
+cham_status chameleon_act_channel_energy(const void* X, int M, int K, double* energy, void* stream) {
+  if (M <= 0 || K <= 0 || K % 8 != 0 || X == nullptr || !aligned16(X) || energy == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "M=%d K=%d (K a multiple of 8, X 16-byte aligned)", M, K);
+  cham::launch_channel_energy(static_cast<const __half*>(X), M, K, energy, static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "channel energy launch");
+}
+
 // ---------------------------------------------------------------- a6
 }  // extern "C"
 namespace {
@@ -532,12 +636,28 @@ cham_status chameleon_pack_plan_palette(int N, int K, uint32_t palette_mask, cha
   return CHAM_OK;
 }
 
+cham_status chameleon_pack_plan_grouped(int N, int K, int fmt, int group, cham_wpack_desc* d) {
+  if (N <= 0 || K <= 0 || K % 32 != 0 || d == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "N=%d K=%d (K must be a multiple of 32)", N, K);
+  if (fmt < 0 || fmt >= CHAM_W_NFORMATS || cham::w_is_mx(fmt))
+    return fail(CHAM_ERR_INVALID_ARG, "format %d has no group-wise form", fmt);
+  if (group < 32 || group % 32 != 0 || (K + group - 1) / group > cham::kMaxRowGroups)
+    return fail(CHAM_ERR_INVALID_ARG, "group %d (a multiple of 32, at most %d groups per row)", group,
+                cham::kMaxRowGroups);
+  std::memset(d, 0, sizeof(*d));
+  d->n_fmt[fmt] = N;
+  d->n_class[cham::w_class(fmt)] = N;
+  d->group = group;
+  finish_plan(d, N, K, cham::wbits(fmt));
+  return CHAM_OK;
+}
+
 }  // extern "C"
 
 namespace {
 void finish_plan(cham_wpack_desc* d, int N, int K, int bits) {
   d->magic = 0x574D4843u;
-  d->version = 1;
+  d->version = 2;
   d->N = N;
   d->K = K;
   d->Kp = static_cast<int>(round_up(K, 64));
@@ -558,6 +678,10 @@ void finish_plan(cham_wpack_desc* d, int N, int K, int bits) {
   off = round_up(off + np, 256);
   d->off_perm = off;
   off = round_up(off + np * 4, 256);
+  if (d->group > 0) {
+    d->off_gscale = off;
+    off = round_up(off + tiles * chunks * 128 * 4, 256);
+  }
   d->bytes = off;
 }
 }  // namespace
@@ -596,6 +720,8 @@ cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const 
   a.perm = reinterpret_cast<int32_t*>(b + d->off_perm);
   a.dev_status = dev_status;
   a.one_class = d->n_class[0] == 0 ? 1 : (d->n_class[1] == 0 ? 0 : -1);
+  a.group = d->group;
+  a.gscale = d->group > 0 ? reinterpret_cast<uint32_t*>(b + d->off_gscale) : nullptr;
   a.desc = *d;
   a.desc_out = reinterpret_cast<cham_wpack_desc*>(b);
   cham::launch_pack(a, nf4_table(), st);
@@ -720,6 +846,7 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   g.wscale = reinterpret_cast<const float*>(b + d->off_scale);
   g.wzero = b + d->off_zero;
   g.we8m0 = b + d->off_e8m0;
+  g.wgscale = d->group > 0 ? reinterpret_cast<const uint32_t*>(b + d->off_gscale) : nullptr;
   g.wfmt = b + d->off_fmt;
   g.perm = reinterpret_cast<const int32_t*>(b + d->off_perm);
   g.bias = bias;

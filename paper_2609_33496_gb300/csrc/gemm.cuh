@@ -11,7 +11,8 @@ struct GemmArgs {
   const uint8_t* codes;      // blob code region (tiled, include/chameleon.h)
   const float* wscale;       // [Np] per packed channel
   const uint8_t* wzero;      // [Np]
-  const uint8_t* we8m0;      // [tiles][chunks][128][2]
+  const uint8_t* we8m0;      // [tiles][chunks][128][2] (group-wise blobs: the blocks' zero points)
+  const uint32_t* wgscale;   // group-wise blobs: [tiles][chunks][128] two fp16 block scales, else null
   const uint8_t* wfmt;       // [Np]
   const int32_t* perm;       // [Np]
   const float* bias;         // [N] in original order, or null

@@ -42,8 +42,9 @@ template <int BN, int BITS>
 struct GemmCfg {
   static constexpr int kBBytes = BN * 128;                        // activation tile
   static constexpr int kWBytes = 128 * (BITS == 8 ? 64 : 32);     // raw codes of 128 channels
-  static constexpr int kEBytes = 256;                             // their E8M0 pairs
-  static constexpr int kStage = (kBBytes + kWBytes + kEBytes + 1023) / 1024 * 1024;
+  static constexpr int kEBytes = 256;                             // their E8M0 pairs (or zero points)
+  static constexpr int kGBytes = 512;                             // group-wise blobs: fp16 block scales
+  static constexpr int kStage = (kBBytes + kWBytes + kEBytes + kGBytes + 1023) / 1024 * 1024;
   // shared-memory ring: as deep as fits in ~200 KiB, to cover the TMA round trip (~1000 cycles)
   // plus decode and MMA time of the stages in flight
   static constexpr int kStages = (200 * 1024) / kStage > 8 ? 8 : (200 * 1024) / kStage;
@@ -123,6 +124,7 @@ CHAM_DEV uint32_t hmul2u(uint32_t a, uint32_t b) { return h2_as_u32(__hmul2(u32_
 struct ChanDecode {
   int f;          // weight format
   int off;        // stored code of the value 0: zero point (asym) or the offset-binary bias
+  int off0, off1; // the same for the chunk's two 32-element blocks (group-wise asym: their own)
   int e_off;      // MX: block exponent offset of the element scale (MXINT8 -6, MXINT4 -2, MXFP4 0)
   bool mx;
 };
@@ -132,6 +134,7 @@ CHAM_DEV ChanDecode chan_decode(int f, int z) {
   c.f = f;
   const bool asym = f == CHAM_W_INT8_ASYM || f == CHAM_W_INT4_ASYM;
   c.off = asym ? z : (wbits(f) == 8 ? 128 : 8);
+  c.off0 = c.off1 = c.off;
   c.e_off = f == CHAM_W_MXINT8 ? -6 : (f == CHAM_W_MXINT4 ? -2 : 0);
   c.mx = w_is_mx(f);
   return c;
@@ -161,8 +164,8 @@ CHAM_DEV void decode_w8(const uint32_t (&w)[16], const ChanDecode& c, uint32_t e
   if (__all_sync(0xffffffffu, fast)) {
     const int E0 = min(max(e0, -24), 5) + 25, E1 = min(max(e1, -24), 5) + 25;
     const uint32_t hi[2] = {static_cast<uint32_t>(E0) << 2, static_cast<uint32_t>(E1) << 2};
-    const uint32_t sub[2] = {dup16((static_cast<uint32_t>(E0) << 10) | static_cast<uint32_t>(c.off)),
-                             dup16((static_cast<uint32_t>(E1) << 10) | static_cast<uint32_t>(c.off))};
+    const uint32_t sub[2] = {dup16((static_cast<uint32_t>(E0) << 10) | static_cast<uint32_t>(c.off0)),
+                             dup16((static_cast<uint32_t>(E1) << 10) | static_cast<uint32_t>(c.off1))};
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       const int b = i >> 3;
@@ -174,12 +177,13 @@ CHAM_DEV void decode_w8(const uint32_t (&w)[16], const ChanDecode& c, uint32_t e
     uint32_t f1[2], f2[2];
     pow2_factors(e0, f1[0], f2[0]);
     pow2_factors(e1, f1[1], f2[1]);
-    const uint32_t sub = dup16((25u << 10) | static_cast<uint32_t>(c.off));
+    const uint32_t sub[2] = {dup16((25u << 10) | static_cast<uint32_t>(c.off0)),
+                             dup16((25u << 10) | static_cast<uint32_t>(c.off1))};
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
       const int b = i >> 3;
-      out[2 * i] = hmul2u(hmul2u(hsub2u(__byte_perm(w[i], 0x64u, 0x4140), sub), f1[b]), f2[b]);
-      out[2 * i + 1] = hmul2u(hmul2u(hsub2u(__byte_perm(w[i], 0x64u, 0x4342), sub), f1[b]), f2[b]);
+      out[2 * i] = hmul2u(hmul2u(hsub2u(__byte_perm(w[i], 0x64u, 0x4140), sub[b]), f1[b]), f2[b]);
+      out[2 * i + 1] = hmul2u(hmul2u(hsub2u(__byte_perm(w[i], 0x64u, 0x4342), sub[b]), f1[b]), f2[b]);
     }
   }
 }
@@ -253,9 +257,9 @@ CHAM_DEV void decode_w4(const uint32_t (&w)[8], const ChanDecode& c, uint32_t e8
     const int c0 = min(max(e0, -20), 5), c1 = min(max(e1, -20), 5);
     const uint32_t m0[2] = {dup16(static_cast<uint32_t>(c0 + 25) << 10), dup16(static_cast<uint32_t>(c1 + 25) << 10)};
     const uint32_t m1[2] = {dup16(static_cast<uint32_t>(c0 + 21) << 10), dup16(static_cast<uint32_t>(c1 + 21) << 10)};
-    const uint32_t o = static_cast<uint32_t>(c.off);
-    const uint32_t s0[2] = {m0[0] | dup16(o), m0[1] | dup16(o)};
-    const uint32_t s1[2] = {m1[0] | dup16(o << 4), m1[1] | dup16(o << 4)};
+    const uint32_t o0 = static_cast<uint32_t>(c.off0), o1 = static_cast<uint32_t>(c.off1);
+    const uint32_t s0[2] = {m0[0] | dup16(o0), m0[1] | dup16(o1)};
+    const uint32_t s1[2] = {m1[0] | dup16(o0 << 4), m1[1] | dup16(o1 << 4)};
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int b = i >> 2;
@@ -266,13 +270,14 @@ CHAM_DEV void decode_w4(const uint32_t (&w)[8], const ChanDecode& c, uint32_t e8
       out[4 * i + 3] = hsub2u((t & 0x00F000F0u) | m1[b], s1[b]);
     }
   } else {
-    const uint32_t sub = dup16((25u << 10) | static_cast<uint32_t>(c.off));
+    const uint32_t sub[2] = {dup16((25u << 10) | static_cast<uint32_t>(c.off0)),
+                             dup16((25u << 10) | static_cast<uint32_t>(c.off1))};
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j)
-        out[4 * i + j] =
-            hmul2u(hmul2u(hsub2u(((w[i] >> (4 * j)) & 0x000F000Fu) | 0x64006400u, sub), f1[i >> 2]), f2[i >> 2]);
+        out[4 * i + j] = hmul2u(
+            hmul2u(hsub2u(((w[i] >> (4 * j)) & 0x000F000Fu) | 0x64006400u, sub[i >> 2]), f1[i >> 2]), f2[i >> 2]);
   }
 }
 
@@ -287,8 +292,9 @@ CHAM_DEV void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)[16]) {
 }
 
 // EPI = 2 * output type (CHAM_Y_*) + per-sample scales: one epilogue variant per instantiation
-// (several inlined into one kernel raise its register count past what the split allows)
-template <int BN, int BITS, int EPI>
+// (several inlined into one kernel raise its register count past what the split allows); GW =
+// group-wise weights (per-block fp16 scales and zero points staged with every chunk)
+template <int BN, int BITS, int EPI, bool GW>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm_ts_f16(const __grid_constant__ CUtensorMap act_map, const GemmArgs a) {
   using C = GemmCfg<BN, BITS>;
@@ -308,6 +314,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nk = a.n_chunks;
+  constexpr bool grouped = GW;  // group-wise blob: per-block fp16 scales
   const int n_ch = a.n_ch_tiles;
   const int n_tiles = n_ch * ((a.M + BN - 1) / BN);
   // K-chunks this CTA processes (its tiles x nk); the last commit group may be partial
@@ -357,12 +364,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
           uint8_t* st = smem + s * C::kStage;
           const size_t chunk = static_cast<size_t>(ch) * nk + kc;
-          mbar_arrive_expect_tx(&full[s], C::kBBytes + C::kWBytes + C::kEBytes);
+          mbar_arrive_expect_tx(&full[s], C::kBBytes + C::kWBytes + C::kEBytes + (grouped ? C::kGBytes : 0));
           // test hook: the stage's transaction bytes never arrive, so every wait on it runs out
           if (blockIdx.x == 0 && static_cast<int>(it) == a.stall_chunk) continue;
           tma_load_2d(smem_u32(st), &act_map, &full[s], kc * kBK, tok0);
           bulk_load(smem_u32(st + C::kBBytes), a.codes + chunk * C::kWBytes, C::kWBytes, &full[s]);
           bulk_load(smem_u32(st + C::kBBytes + C::kWBytes), a.we8m0 + chunk * C::kEBytes, C::kEBytes, &full[s]);
+          if constexpr (grouped)
+            bulk_load(smem_u32(st + C::kBBytes + C::kWBytes + C::kEBytes), a.wgscale + chunk * 128, C::kGBytes,
+                      &full[s]);
         }
       }
       // every issued copy must have landed before the CTA may exit
@@ -449,6 +459,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         const uint8_t* st = smem + s * C::kStage;
         const uint32_t e8 = reinterpret_cast<const uint16_t*>(st + C::kBBytes + C::kWBytes)[r];
+        ChanDecode cdk = cd;
+        uint32_t gs = 0;
+        if constexpr (grouped) {  // group-wise blob: the E8M0 slot holds the blocks' zero points (asym)
+          gs = reinterpret_cast<const uint32_t*>(st + C::kBBytes + C::kWBytes + C::kEBytes)[r];
+          if (cd.f == CHAM_W_INT8_ASYM || cd.f == CHAM_W_INT4_ASYM) {
+            cdk.off0 = static_cast<int>(e8 & 0xFFu);
+            cdk.off1 = static_cast<int>((e8 >> 8) & 0xFFu);
+          }
+        }
         uint32_t raw[16];
 #pragma unroll
         for (int j = 0; j < BITS / 2; ++j) {  // slab j: bytes [16j, 16j+16) of every channel
@@ -460,10 +479,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         uint32_t out[32];
         if constexpr (BITS == 8) {
-          decode_w8(raw, cd, e8, out);
+          decode_w8(raw, cdk, e8, out);
         } else {
           const uint32_t (&r8)[8] = *reinterpret_cast<const uint32_t(*)[8]>(&raw[0]);
-          decode_w4(r8, cd, e8, a.nf4_lo, a.nf4_hi, out);
+          decode_w4(r8, cdk, e8, a.nf4_lo, a.nf4_hi, out);
+        }
+        if constexpr (grouped) {  // each block's group scale: one fp16 product, rounded once
+          const uint32_t g0 = dup16(gs & 0xFFFFu), g1 = dup16(gs >> 16);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) out[i] = hmul2u(out[i], i < 16 ? g0 : g1);
         }
         const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
         if (!__all_sync(0xffffffffu, free_ok)) {
@@ -571,7 +595,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   }
 }
 
-template <int BN, int BITS, int EPI>
+template <int BN, int BITS, int EPI, bool GW>
 static cudaError_t launch_bn(const CUtensorMap& map, const GemmArgs& a, int num_sms, cudaStream_t st) {
   using C = GemmCfg<BN, BITS>;
   static int configured_device = -1;  // the attribute is per device; set again when it changes
@@ -579,34 +603,40 @@ static cudaError_t launch_bn(const CUtensorMap& map, const GemmArgs& a, int num_
   cudaGetDevice(&dev);
   if (configured_device != dev) {
     const cudaError_t e =
-        cudaFuncSetAttribute(k_gemm_ts_f16<BN, BITS, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+        cudaFuncSetAttribute(k_gemm_ts_f16<BN, BITS, EPI, GW>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
   const long tiles = static_cast<long>(a.n_ch_tiles) * ((a.M + BN - 1) / BN);
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  return launch_pdl(k_gemm_ts_f16<BN, BITS, EPI>, dim3(grid), dim3(kGemmThreads), C::kSmem, st, map, a);
+  return launch_pdl(k_gemm_ts_f16<BN, BITS, EPI, GW>, dim3(grid), dim3(kGemmThreads), C::kSmem, st, map, a);
 }
 
-template <int BITS, int EPI>
+template <int BITS, int EPI, bool GW>
 static cudaError_t launch_bits(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
   switch (bn) {
-    case 16: return launch_bn<16, BITS, EPI>(map, a, num_sms, st);
-    case 32: return launch_bn<32, BITS, EPI>(map, a, num_sms, st);
-    case 64: return launch_bn<64, BITS, EPI>(map, a, num_sms, st);
-    case 128: return launch_bn<128, BITS, EPI>(map, a, num_sms, st);
-    default: return launch_bn<192, BITS, EPI>(map, a, num_sms, st);
+    case 16: return launch_bn<16, BITS, EPI, GW>(map, a, num_sms, st);
+    case 32: return launch_bn<32, BITS, EPI, GW>(map, a, num_sms, st);
+    case 64: return launch_bn<64, BITS, EPI, GW>(map, a, num_sms, st);
+    case 128: return launch_bn<128, BITS, EPI, GW>(map, a, num_sms, st);
+    default: return launch_bn<192, BITS, EPI, GW>(map, a, num_sms, st);
   }
 }
 
+template <int BITS, int EPI>
+static cudaError_t launch_gw(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
+  return a.wgscale != nullptr ? launch_bits<BITS, EPI, true>(map, a, num_sms, bn, st)
+                              : launch_bits<BITS, EPI, false>(map, a, num_sms, bn, st);
+}
+
 // The launches of one output type YT: both weight widths, every token-tile size, per-tensor or
-// per-sample activation scales.
+// per-sample activation scales, per-channel or group-wise weights.
 template <int YT>
 cudaError_t launch_gemm_yt(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
-  const bool grouped = a.act_scale != nullptr && a.rows_per_group < a.M;
+  const bool per_sample = a.act_scale != nullptr && a.rows_per_group < a.M;
   if (a.bits == 8)
-    return grouped ? launch_bits<8, 2 * YT + 1>(map, a, num_sms, bn, st) : launch_bits<8, 2 * YT>(map, a, num_sms, bn, st);
-  return grouped ? launch_bits<4, 2 * YT + 1>(map, a, num_sms, bn, st) : launch_bits<4, 2 * YT>(map, a, num_sms, bn, st);
+    return per_sample ? launch_gw<8, 2 * YT + 1>(map, a, num_sms, bn, st) : launch_gw<8, 2 * YT>(map, a, num_sms, bn, st);
+  return per_sample ? launch_gw<4, 2 * YT + 1>(map, a, num_sms, bn, st) : launch_gw<4, 2 * YT>(map, a, num_sms, bn, st);
 }
 
 }  // namespace cham

@@ -214,7 +214,87 @@ CHAM_DEV size_t code_offset(int p, int k0, int n_chunks, int bits) {
   return chunk_base + static_cast<size_t>(kk >> 5) * 2048 + r * 16 + ((kk & 31) >> 3) * 4;
 }
 
+// Stores the 8 codes of elements [8v, 8v+8) of packed slot p in the tiled layout: symmetric
+// integer codes in offset binary (q + 128, q + 8); 4-bit words with nibble j (j < 4) = element 2j
+// and nibble 4 + j = element 2j + 1 (the integer and E2M1 decodes isolate a pair with one mask),
+// NF4 with nibble j = element j (the register-table decode).
+CHAM_DEV void store_codes(const PackArgs& a, int p, int v, int f, int (&code)[8]) {
+  const int bias = (f == CHAM_W_INT8_SYM || f == CHAM_W_MXINT8) ? 0x80
+                   : ((f == CHAM_W_INT4_SYM || f == CHAM_W_MXINT4) ? 0x8 : 0);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) code[i] = (code[i] & (a.bits == 8 ? 0xFF : 0xF)) ^ bias;
+  const size_t off = code_offset(p, v * 8, a.n_chunks, a.bits);
+  if (a.bits == 8) {
+    uint32_t lo = 0, hi = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      lo |= (static_cast<uint32_t>(code[i]) & 0xFFu) << (8 * i);
+      hi |= (static_cast<uint32_t>(code[4 + i]) & 0xFFu) << (8 * i);
+    }
+    *reinterpret_cast<uint2*>(a.codes + off) = make_uint2(lo, hi);
+  } else {
+    uint32_t w = 0;
+    if (f == CHAM_W_NF4) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) w |= (static_cast<uint32_t>(code[j]) & 0xFu) << (4 * j);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        w |= (static_cast<uint32_t>(code[2 * j]) & 0xFu) << (4 * j);
+        w |= (static_cast<uint32_t>(code[2 * j + 1]) & 0xFu) << (4 * (j + 4));
+      }
+    }
+    *reinterpret_cast<uint32_t*>(a.codes + off) = w;
+  }
+}
+
+// ------------------------------------------------------------------ group-wise formats (Sec. 3.5 forks)
+struct GroupParam {  // scale, reciprocal and zero point of one group of one row
+  float s, inv;
+  int z;
+};
+
+// Statistics of elements [k0, k1) of a row, by one lane (k0, k1 multiples of 8).
+CHAM_DEV ChanStats range_stats(const __half* row, int k0, int k1) {
+  float amax = 0.f, lo = INFINITY, hi = -INFINITY;
+  for (int v = k0 / 8; v < k1 / 8; ++v) {
+    float x[8];
+    load8(row, v, x);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      amax = fmaxf(amax, fabsf(x[i]));
+      lo = fminf(lo, x[i]);
+      hi = fmaxf(hi, x[i]);
+    }
+  }
+  return ChanStats{amax, lo, hi};
+}
+
+// The scale rule of format f on every group of g elements of a row (lane j takes groups j, j + 32,
+// ...), into this warp's shared-memory table.
+CHAM_DEV void group_params(const __half* row, int K, int g, int f, int lane, GroupParam* gp) {
+  const int ng = (K + g - 1) / g;
+  for (int j = lane; j < ng; j += 32) {
+    const ChanScale cs = chan_scale(f, range_stats(row, j * g, min((j + 1) * g, K)));
+    gp[j] = GroupParam{cs.s, cs.inv, cs.z};
+  }
+  __syncwarp();
+}
+
+// The value a non-MX code stands for, before its scale: q (sym), q - z (asym), the NF4 level,
+// the E2M1 value.
+CHAM_DEV float code_value(int f, int code, int z, const NF4Table& nf4) {
+  switch (f) {
+    case CHAM_W_INT8_ASYM:
+    case CHAM_W_INT4_ASYM: return static_cast<float>(code - z);
+    case CHAM_W_NF4: return __half2float(__ushort_as_half(nf4.level[code]));
+    case CHAM_W_E2M1: return e2m1_value(static_cast<uint32_t>(code));
+    default: return static_cast<float>(code);
+  }
+}
+
 __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) {
+  __shared__ GroupParam s_gp[kWWarps][kMaxRowGroups];
   if (blockIdx.x == 0 && threadIdx.x < 64)  // the blob's header: a copy of the descriptor
     reinterpret_cast<uint32_t*>(a.desc_out)[threadIdx.x] = reinterpret_cast<const uint32_t*>(&a.desc)[threadIdx.x];
   const int lane = threadIdx.x & 31;
@@ -249,6 +329,7 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
       const size_t e = ((static_cast<size_t>(tile) * a.n_chunks + ch) * 128 + r) * 2;
       a.e8m0[e] = 127;
       a.e8m0[e + 1] = 127;
+      if (a.gscale != nullptr) a.gscale[e / 2] = 0u;
     }
     if (lane == 0) {
       a.scale[p] = 1.f;
@@ -259,6 +340,41 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
   const int f = a.fmtp[p];
   const __half* row = a.W + static_cast<size_t>(c) * a.K;
   const int nvec = a.K / 8;
+  if (a.group > 0) {
+    // group-wise: codes with their group's parameters; per 32-element block its zero point (in
+    // the E8M0 slot) and its group's scale as fp16; the per-channel scale is 1
+    if (lane == 0 && a.desc.n_fmt[f] != a.N) set_status(a.dev_status, CHAM_ERR_INVALID_ARG);  // one format per plan
+    GroupParam* gp = s_gp[threadIdx.x >> 5];
+    group_params(row, a.K, a.group, f, lane, gp);
+    const bool asym = f == CHAM_W_INT8_ASYM || f == CHAM_W_INT4_ASYM;
+    for (int v = lane; v < nvec_p; v += 32) {
+      int code[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      GroupParam q{0.f, 1.f, 0};  // beyond K: code 0, zero point 0, scale 0 -> the value 0
+      if (v < nvec) {
+        q = gp[(v * 8) / a.group];
+        float x[8];
+        load8(row, v, x);
+        const ChanScale cs{q.s, q.inv, q.z};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float err;
+          code[i] = encode_chan(f, x[i], cs, nf4, &err);
+        }
+      }
+      store_codes(a, p, v, f, code);
+      if ((v & 3) == 0) {
+        const int k0 = v * 8;
+        const size_t e = ((static_cast<size_t>(tile) * a.n_chunks + (k0 >> 6)) * 128 + r) * 2 + ((k0 & 63) >> 5);
+        a.e8m0[e] = asym ? static_cast<uint8_t>(q.z) : 0;
+        reinterpret_cast<__half*>(a.gscale)[e] = __float2half_rn(v < nvec ? q.s : 0.f);
+      }
+    }
+    if (lane == 0) {
+      a.scale[p] = 1.f;
+      a.zero[p] = 0;
+    }
+    return;
+  }
   const ChanStats st = row_stats(row, nvec, lane);
   const ChanScale cs = chan_scale(f, st);
   const bool mx = w_is_mx(f);
@@ -296,36 +412,7 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
 #pragma unroll
       for (int i = 0; i < 8; ++i) code[i] = f == CHAM_W_INT8_ASYM || f == CHAM_W_INT4_ASYM ? cs.z : 0;
     }
-    // symmetric integer codes are stored in offset binary (q + 128, q + 8)
-    const int bias = (f == CHAM_W_INT8_SYM || f == CHAM_W_MXINT8) ? 0x80
-                     : ((f == CHAM_W_INT4_SYM || f == CHAM_W_MXINT4) ? 0x8 : 0);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) code[i] = (code[i] & (a.bits == 8 ? 0xFF : 0xF)) ^ bias;
-    const size_t off = code_offset(p, v * 8, a.n_chunks, a.bits);
-    if (a.bits == 8) {
-      uint32_t lo = 0, hi = 0;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        lo |= (static_cast<uint32_t>(code[i]) & 0xFFu) << (8 * i);
-        hi |= (static_cast<uint32_t>(code[4 + i]) & 0xFFu) << (8 * i);
-      }
-      *reinterpret_cast<uint2*>(a.codes + off) = make_uint2(lo, hi);
-    } else {
-      // nibble j (j < 4) = element 2j, nibble 4 + j = element 2j + 1 (the integer and E2M1 decodes
-      // isolate a pair with one mask); NF4: nibble j = element j (the register-table decode)
-      uint32_t w = 0;
-      if (f == CHAM_W_NF4) {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) w |= (static_cast<uint32_t>(code[j]) & 0xFu) << (4 * j);
-      } else {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          w |= (static_cast<uint32_t>(code[2 * j]) & 0xFu) << (4 * j);
-          w |= (static_cast<uint32_t>(code[2 * j + 1]) & 0xFu) << (4 * (j + 4));
-        }
-      }
-      *reinterpret_cast<uint32_t*>(a.codes + off) = w;
-    }
+    store_codes(a, p, v, f, code);
     if ((lane & 3) == 0) {  // one E8M0 byte per 32-element block
       const int k0 = v * 8;
       const size_t e = ((static_cast<size_t>(tile) * a.n_chunks + (k0 >> 6)) * 128 + r) * 2 + ((k0 & 63) >> 5);
@@ -337,6 +424,130 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
     a.scale[p] = mx ? 1.f : cs.s;
     a.zero[p] = static_cast<uint8_t>(cs.z);
   }
+}
+
+// ------------------------------------------------------------------ (g, f) search (Sec. 3.5 forks)
+__global__ void __launch_bounds__(256) k_energy_f32(const double* __restrict__ energy, int K, float* __restrict__ out) {
+  for (int k = blockIdx.x * blockDim.x + threadIdx.x; k < K; k += gridDim.x * blockDim.x)
+    out[k] = energy != nullptr ? static_cast<float>(energy[k]) : 1.f;
+}
+
+// Per channel (one warp) and candidate: sum_k e_k (w - DQ(w))^2, with the element error rounded
+// once to fp32, weighted and squared in fp32, summed in fp32 over 8 elements, then in fp64.
+__global__ void __launch_bounds__(kWThreads) k_w_select_groups(GroupSearchArgs a, NF4Table nf4) {
+  __shared__ GroupParam s_gp[kWWarps][kMaxRowGroups];
+  const int lane = threadIdx.x & 31;
+  const int c = blockIdx.x * kWWarps + (threadIdx.x >> 5);
+  if (c >= a.N) return;  // whole warps: no block-wide barrier follows
+  GroupParam* gp = s_gp[threadIdx.x >> 5];
+  const __half* row = a.W + static_cast<size_t>(c) * a.K;
+  const int nvec = a.K / 8;
+  const int iters = (nvec + 31) / 32;  // same trip count in every lane (shuffles)
+  for (int ci = 0; ci < a.n_cand; ++ci) {
+    const int g = a.cand[ci].g, f = a.cand[ci].f;
+    double acc = 0.0;
+    if (w_is_mx(f)) {
+      for (int it = 0; it < iters; ++it) {
+        const int v = it * 32 + lane;
+        float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        if (v < nvec) load8(row, v, x);
+        float am = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
+        am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 1));  // 4 lanes = one 32-element block
+        am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 2));
+        const int X = mx_exponent(f, am);
+        if (v < nvec) {
+          float e2[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            float dq;
+            encode_mx(f, x[i], X, &dq);
+            const float e = __fsub_rn(x[i], dq);
+            e2[i] = __fmul_rn(__fmul_rn(e, e), a.energy32[v * 8 + i]);
+          }
+          acc += static_cast<double>(sum8(e2));
+        }
+      }
+    } else {
+      __syncwarp();  // the previous candidate's table is no longer read
+      group_params(row, a.K, g, f, lane, gp);
+      for (int v = lane; v < nvec; v += 32) {
+        const GroupParam q = gp[(v * 8) / g];
+        const ChanScale cs{q.s, q.inv, q.z};
+        const float s16 = __half2float(__float2half_rn(q.s));
+        float x[8], e2[8];
+        load8(row, v, x);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          float err;
+          const int code = encode_chan(f, x[i], cs, nf4, &err);
+          // DQ = fp16(value * fp16(s)): the product of two fp16 values is exact in fp32
+          const float dq = __half2float(__float2half_rn(__fmul_rn(code_value(f, code, q.z, nf4), s16)));
+          const float e = __fsub_rn(x[i], dq);
+          e2[i] = __fmul_rn(__fmul_rn(e, e), a.energy32[v * 8 + i]);
+        }
+        acc += static_cast<double>(sum8(e2));
+      }
+    }
+    const double tot = warp_reduce(acc, DAdd());
+    if (lane == 0) a.parts[static_cast<size_t>(c) * a.n_cand + ci] = tot;
+  }
+}
+
+// scores[i] = sum over channels, in channel order, of the per-channel errors of candidate i.
+__global__ void __launch_bounds__(64) k_w_select_groups_finish(GroupSearchArgs a) {
+  for (int ci = threadIdx.x; ci < a.n_cand; ci += blockDim.x) {
+    double t = 0.0;
+    for (int c = 0; c < a.N; ++c) t += a.parts[static_cast<size_t>(c) * a.n_cand + ci];
+    a.scores[ci] = t;
+  }
+}
+
+void launch_select_groups(const GroupSearchArgs& a, const NF4Table& nf4, cudaStream_t st) {
+  k_energy_f32<<<(a.K + 255) / 256, 256, 0, st>>>(a.energy, a.K, a.energy32);
+  k_w_select_groups<<<(a.N + kWWarps - 1) / kWWarps, kWThreads, 0, st>>>(a, nf4);
+  k_w_select_groups_finish<<<1, 64, 0, st>>>(a);
+}
+
+// energy[k] += sum_m x[m, k]^2.  A CTA of 32 x 32 threads owns 32 column vectors (lane = vector,
+// warp = one of 32 row strides); each thread sums its rows' squares in fp32 over runs of 8 rows
+// and in fp64 across runs; the 32 row strides are then added in warp order (deterministic).
+__global__ void __launch_bounds__(1024) k_channel_energy(const __half* __restrict__ X, int M, int K,
+                                                        double* __restrict__ energy) {
+  __shared__ double sh[32][33];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nv = K / 8;
+  const int v = blockIdx.x * 32 + lane;
+  double acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  if (v < nv) {
+    for (int m0 = warp * 8; m0 < M; m0 += 32 * 8) {
+      float part[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      for (int m = m0; m < min(m0 + 8, M); ++m) {
+        float x[8];
+        load8(X + static_cast<size_t>(m) * K, v, x);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) part[i] = __fadd_rn(part[i], __fmul_rn(x[i], x[i]));
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] += static_cast<double>(part[i]);
+    }
+  }
+#pragma unroll 1
+  for (int i = 0; i < 8; ++i) {
+    sh[warp][lane] = acc[i];
+    __syncthreads();
+    if (warp == 0 && v < nv) {
+      double t = 0.0;
+      for (int w = 0; w < 32; ++w) t += sh[w][lane];
+      energy[v * 8 + i] += t;
+    }
+    __syncthreads();
+  }
+}
+
+void launch_channel_energy(const __half* X, int M, int K, double* energy, cudaStream_t st) {
+  k_channel_energy<<<(K / 8 + 31) / 32, 1024, 0, st>>>(X, M, K, energy);
 }
 
 void launch_pack(const PackArgs& a, const NF4Table& nf4, cudaStream_t st) {

@@ -150,6 +150,24 @@ CHAM_DEV int encode_mx(int fmt, float w, int X, float* dq) {
   return static_cast<int>(n);
 }
 
+constexpr int kMaxRowGroups = 256;  // groups per row of a group-wise blob (K <= 8192 at g = 32)
+constexpr int kMaxCands = 48;       // (g, f) candidates of one search
+
+struct GroupCand {
+  int g, f;
+};
+
+struct GroupSearchArgs {
+  const __half* W;
+  int N, K;
+  const double* energy;   // [K] or null (e_k = 1)
+  float* energy32;        // [K] scratch: energy as fp32
+  double* parts;          // [N][n_cand] per-channel weighted errors
+  double* scores;         // [n_cand] output
+  int n_cand;
+  GroupCand cand[kMaxCands];
+};
+
 struct PackArgs {
   const __half* W;
   const uint8_t* fmt_dev;   // selected format of each original channel
@@ -166,11 +184,15 @@ struct PackArgs {
   uint8_t* e8m0;
   uint8_t* fmtp;
   int32_t* perm;
+  int group;                // group-wise blob: g input channels per scale (0: per channel)
+  uint32_t* gscale;         // group-wise blob: [tiles][chunks][128] two fp16 block scales
   int* dev_status;
 };
 
 void launch_select(const __half* W, int N, int K, uint32_t mask, uint8_t* fmt_out, double* sse_out,
                    const NF4Table& nf4, cudaStream_t st);
 void launch_pack(const PackArgs& a, const NF4Table& nf4, cudaStream_t st);
+void launch_select_groups(const GroupSearchArgs& a, const NF4Table& nf4, cudaStream_t st);
+void launch_channel_energy(const __half* X, int M, int K, double* energy, cudaStream_t st);
 
 }  // namespace cham

@@ -8,11 +8,12 @@ CLASS0 = (3, 4, 6, 7, 8)
 def desc_fields(blob_bytes):
     hdr = np.frombuffer(blob_bytes[:256], dtype=np.uint8)
     i32 = hdr[:80].view(np.int32)
-    u64 = hdr[80:136].view(np.uint64)
-    keys = ["off_codes", "off_scale", "off_zero", "off_e8m0", "off_fmt", "off_perm", "bytes"]
+    u64 = hdr[80:144].view(np.uint64)
+    keys = ["off_codes", "off_scale", "off_zero", "off_e8m0", "off_fmt", "off_perm", "bytes", "off_gscale"]
     d = {"magic": int(hdr[:4].view(np.uint32)[0]), "N": int(i32[2]), "K": int(i32[3]),
          "Kp": int(i32[4]), "bits": int(i32[5]), "n_class": [int(i32[6]), int(i32[7])],
-         "n_tiles": [int(i32[8]), int(i32[9])], "n_fmt": [int(v) for v in i32[10:19]]}
+         "n_tiles": [int(i32[8]), int(i32[9])], "n_fmt": [int(v) for v in i32[10:19]],
+         "version": int(hdr[4:8].view(np.uint32)[0]), "group": int(i32[19])}
     d.update({k: int(v) for k, v in zip(keys, u64)})
     return d
 
@@ -30,6 +31,9 @@ def unpack(blob_bytes):
     scale = b[d["off_scale"]:d["off_scale"] + 4 * Np].view(np.float32)
     zero = b[d["off_zero"]:d["off_zero"] + Np]
     e8 = b[d["off_e8m0"]:d["off_e8m0"] + tiles * nch * 256].reshape(tiles, nch, 128, 2)
+    gsc = None
+    if d["group"] > 0:   # group-wise blob: fp16 scale of each 32-element block
+        gsc = b[d["off_gscale"]:d["off_gscale"] + tiles * nch * 512].view(np.float16).reshape(tiles, nch, 128, 2)
     CB = 64 if bits == 8 else 32
     codes_raw = b[d["off_codes"]:d["off_codes"] + tiles * nch * 128 * CB].reshape(tiles, nch, CB // 16, 128, 16)
     # per slot: bytes of each chunk in order
@@ -69,4 +73,6 @@ def unpack(blob_bytes):
             vals = vals ^ 0x8
         out[c] = {"fmt": f, "codes": vals, "s": np.float32(scale[p]), "z": int(zero[p]), "e8m0": e8c,
                   "slot": p}
+        if gsc is not None:
+            out[c]["gscale16"] = gsc[t, :, r, :].reshape(-1)[:K // 32]
     return d, out

@@ -177,3 +177,33 @@ def test_act_format_argmin_host_helper(cl):
     w = ctypes.c_size_t()
     assert cl.lib().chameleon_act_format_sse_workspace_size(16, 48, ctypes.byref(w)) == cl.ERR_INVALID_ARG
     assert cl.lib().chameleon_act_format_sse_workspace_size(16, 64, ctypes.byref(w)) == cl.OK and w.value >= 256
+
+
+def test_group_candidates_match_oracle(cl):
+    for pal, groups in [([F.W_INT4_ASYM, F.W_NF4, F.W_E2M1], F.GROUP_SIZES),
+                        ([F.W_INT4_ASYM, F.W_NF4, F.W_E2M1, F.W_MXINT4, F.W_MXFP4], F.GROUP_SIZES),
+                        ([F.W_INT8_SYM, F.W_INT8_ASYM, F.W_MXINT8], (32, 128)),
+                        ([F.W_MXFP4], (64,))]:
+        mask = sum(1 << f for f in pal)
+        assert cl.group_candidates(mask, cl.group_mask(groups)) == SEL.group_candidates(pal, groups)
+    assert cl.candidate_argmin([3.0, 1.0, 1.0, 2.0]) == 1
+    assert cl.lib().chameleon_candidate_argmin(None, 3) == -1
+
+
+def test_pack_plan_grouped_layout_and_checks(cl):
+    d = cl.pack_plan_grouped(300, 320, F.W_INT4_ASYM, 192)
+    assert (d.group, d.bits, list(d.n_class), d.n_fmt[F.W_INT4_ASYM], d.version) == (192, 4, [300, 0], 300, 2)
+    assert d.off_gscale % 256 == 0 and d.off_gscale >= d.off_perm + 4 * 384
+    assert d.bytes >= d.off_gscale + 3 * 5 * 128 * 4
+    assert cl.pack_plan(300, 320, np.full(300, F.W_INT4_ASYM, np.uint8)).off_gscale == 0
+    for fmt, g, K in [(F.W_MXFP4, 32, 320), (F.W_NF4, 48, 320), (F.W_NF4, 0, 320), (F.W_E2M1, 32, 32 * 257),
+                      (9, 32, 320)]:
+        with pytest.raises(cl.ChameleonError) as e:
+            cl.pack_plan_grouped(64, K, fmt, g)
+        assert e.value.status == cl.ERR_INVALID_ARG
+    w = ctypes.c_size_t()
+    L = cl.lib()
+    assert L.chameleon_select_weight_groups_workspace_size(64, 320, 0x070, 0, ctypes.byref(w)) == cl.ERR_INVALID_ARG
+    assert L.chameleon_select_weight_groups_workspace_size(64, 320, 0x1F8 | 0x1, 1, ctypes.byref(w)) == cl.ERR_INVALID_ARG
+    assert L.chameleon_select_weight_groups_workspace_size(64, 32 * 257, 0x070, 1, ctypes.byref(w)) == cl.ERR_INVALID_ARG
+    assert L.chameleon_select_weight_groups_workspace_size(64, 320, 0x070, 0x1F, ctypes.byref(w)) == cl.OK
