@@ -247,12 +247,11 @@ def main():
         blobs[li] = torch.empty(descs[li].bytes, dtype=torch.uint8, device=device)
 
     def select_pack():
-        """a5 + a6 for every layer: GPU selection into the layer's slice of one format buffer,
-        GPU pack into the layer's blob."""
+        """a5 + a6 for every layer in one launch each: GPU selection into the layer's slice of one
+        format buffer and, from the same warp, the pack into the layer's blob."""
         for li in range(len(layers)):
             f = fmt_all[fmt_off[li]:fmt_off[li + 1]]
-            cl.select_weight_formats(W[li], cl.PALETTE_W8, fmt_out=f)
-            cl.pack_weights(W[li], f, descs[li], dev_status=st, blob=blobs[li])
+            cl.select_pack_palette(W[li], cl.PALETTE_W8, descs[li], fmt_out=f, blob=blobs[li], dev_status=st)
 
     flops_step = nb * sum(layer_flops(M, K, N) for (_, M, K, N) in layers)
     quant_bytes_step = 0.0
@@ -302,9 +301,9 @@ def main():
         else:
             run_step(key)
 
-    # kernel launches per step: select 1 + pack 1 per layer (one MMA class: no slot ranking);
+    # kernel launches per step: one fused select + pack per layer (one MMA class: slot = channel);
     # per linear 1 quantizer kernel (static scales or MX; 2 with dynamic per-tensor scales) + 1 GEMM
-    launches = 2 * len(layers) + sum(
+    launches = len(layers) + sum(
         (2 if args.dynamic_scales and lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(nb))
     for li, (_, M, K, N) in enumerate(layers):
         for bk in range(nb):
@@ -368,7 +367,7 @@ def main():
                    "layers": len(layers), "buckets": nb, "global_batch": 2 * world,
                    "tokens": [M for (_, M, _, _) in layers], "weight_palette": "W8 {INT8-sym, INT8-asym, MXINT8}",
                    "activation_formats_used": sorted(set(int(v) for v in lut.ravel())),
-                   "step": "select+pack 10 layers, then 10 buckets x 10 layers of act-quant (%s) + GEMM, one "
+                   "step": "fused select+pack of 10 layers, then 10 buckets x 10 layers of act-quant (%s) + GEMM, one "
                            "CUDA graph" % ("dynamic per-tensor scales, Alg. 3" if args.dynamic_scales else
                                            "static calibrated per-(layer, bucket) scales, Alg. 2"),
                    "l2": "inputs larger than L2 (%.0f MB of activations per step)" %
@@ -452,8 +451,8 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, qp, device, stream, world, f
         stream.wait_event(w_ready)
         for li in range(len(layers)):
             f = fmt_all[fmt_off[li]:fmt_off[li + 1]]
-            cl.select_weight_formats(Wd[li], cl.PALETTE_W8, fmt_out=f, stream=stream)
-            cl.pack_weights(Wd[li], f, descs[li], dev_status=st, blob=blobs[li], stream=stream)
+            cl.select_pack_palette(Wd[li], cl.PALETTE_W8, descs[li], fmt_out=f, blob=blobs[li], dev_status=st,
+                                   stream=stream)
         for bk in range(nb):
             for li in range(len(layers)):
                 with torch.cuda.stream(s_h2d):
@@ -567,7 +566,14 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
         blob, _ = cl.pack_weights(W[li], fmt, desc, dev_status=st)
         t_pack = timed(lambda: cl.pack_weights(W[li], fmt, desc, dev_status=st, blob=blob))
         pack_bytes = 2 * N * K + N * K * bits / 8 + 10 * N
+        t_fused = None
+        if mask == cl.PALETTE_W8:   # one MMA class: the fused select + pack of the step
+            d_pal = cl.pack_plan_palette(N, K, mask)
+            blob_pal = torch.empty(d_pal.bytes, dtype=torch.uint8, device=dev)
+            t_fused = timed(lambda: cl.select_pack_palette(W[li], mask, d_pal, fmt_out=fmt, blob=blob_pal,
+                                                           dev_status=st))
         out["weights"].append({"palette": pal_name, "select_us": round(t_sel * 1e3, 2),
+                               "select_pack_fused_us": None if t_fused is None else round(t_fused * 1e3, 2),
                                "pack_us": round(t_pack * 1e3, 2),
                                "pack_gbs": round(pack_bytes / (t_pack * 1e-3) / 1e9, 1),
                                "pack_frac_hbm": round(pack_bytes / (t_pack * 1e-3) / hbm, 4),

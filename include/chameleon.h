@@ -264,6 +264,16 @@ typedef struct {
  * bit width).  desc->bytes is the blob size. */
 cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* desc);
 
+/* Selection (a5) and pack (a6) in one launch, for a palette whose members share one MMA class
+ * (e.g. CHAM_PALETTE_W8): desc comes from chameleon_pack_plan_palette(N, K, palette_mask); the
+ * warp that selects channel c's format encodes c right away.  Writes fmt_out (device, uint8 [N],
+ * the formats chameleon_select_weight_formats would give) and the blob (device, as
+ * chameleon_pack_weights would write it for those formats).  CHAM_ERR_INVALID_ARG when desc is not
+ * a one-class plan of these N x K weights, or a palette member lies outside its class / width. */
+cham_status chameleon_select_pack_palette(const void* W, int N, int K, uint32_t palette_mask,
+                                          const cham_wpack_desc* desc, uint8_t* fmt_out, void* blob,
+                                          size_t blob_bytes, int* dev_status, void* stream);
+
 /* A group-wise plan (the DiT and few-step forks, Sec. 3.5): every channel in format fmt (a non-MX
  * format: INT8-sym, INT8-asym, INT4-sym, INT4-asym, NF4 or E2M1), one scale (and zero point) per
  * run of `group` input channels along K -- group a multiple of 32 with at most 256 groups per row

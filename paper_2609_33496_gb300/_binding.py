@@ -38,6 +38,7 @@ EXPORTS = [
     "chameleon_act_format_sse_workspace_size", "chameleon_act_format_sse", "chameleon_act_format_argmin",
     "chameleon_pack_plan_grouped", "chameleon_group_candidates", "chameleon_select_weight_groups_workspace_size",
     "chameleon_select_weight_groups", "chameleon_candidate_argmin", "chameleon_act_channel_energy",
+    "chameleon_select_pack_palette",
 ]
 
 
@@ -128,6 +129,7 @@ def lib():
         "chameleon_select_weight_groups": (i32, [vp, i32, i32, u32, u32, vp, vp, vp, sz, vp]),
         "chameleon_candidate_argmin": (i32, [ctypes.POINTER(ctypes.c_double), i32]),
         "chameleon_act_channel_energy": (i32, [vp, i32, i32, vp, vp]),
+        "chameleon_select_pack_palette": (i32, [vp, i32, i32, u32, pdesc, vp, vp, sz, vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -354,6 +356,22 @@ def pack_plan(N, K, fmt_host):
     d = WPackDesc()
     check(lib().chameleon_pack_plan(N, K, f.ctypes.data_as(ctypes.c_void_p), ctypes.byref(d)))
     return d
+
+
+def select_pack_palette(W, palette_mask, desc, fmt_out=None, blob=None, dev_status=None, stream=None):
+    """Selection and pack in one launch for a one-class palette plan (pack_plan_palette).  Returns
+    (fmt device uint8 [N], blob, dev_status)."""
+    import torch
+    N, K = W.shape
+    if fmt_out is None:
+        fmt_out = torch.empty(N, dtype=torch.uint8, device=W.device)
+    if blob is None or blob.numel() < desc.bytes:
+        blob = _bytes(desc.bytes, W.device)
+    if dev_status is None:
+        dev_status = torch.zeros(1, dtype=torch.int32, device=W.device)
+    check(lib().chameleon_select_pack_palette(_ptr(W), N, K, palette_mask, ctypes.byref(desc), _ptr(fmt_out),
+                                              _ptr(blob), blob.numel(), _ptr(dev_status), _stream(stream)))
+    return fmt_out, blob, dev_status
 
 
 def pack_weights(W, fmt_dev, desc, dev_status=None, stream=None, blob=None):

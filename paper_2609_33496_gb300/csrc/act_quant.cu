@@ -143,11 +143,12 @@ CHAM_DEV void encode8_tensor(const uint4& v, const TensorParams& p, uint2& code,
 // per-tensor range) writes its gridDim.x partials at parts[blockIdx.y * gridDim.x ...].
 __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, int64_t nvec,
                                                   RangePartial* __restrict__ parts) {
+  // X may be the previous kernel's output (a linear's fp16 Y fed to the next linear), and that
+  // kernel lets its dependents start early: wait for it before the first read
+  griddep_wait();
   griddep_launch_dependents();
   X += static_cast<int64_t>(blockIdx.y) * nvec;
   parts += static_cast<int64_t>(blockIdx.y) * gridDim.x;
-  // X is a caller input that no kernel of the chain writes: it is read before the wait, so this
-  // pass overlaps the tail of the previous kernel; the partial is written after it
   __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
   uint32_t nonfinite = 0;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
@@ -165,7 +166,6 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
   float lo = fminf(__low2float(lo2), __high2float(lo2));
   float hi = fmaxf(__low2float(hi2), __high2float(hi2));
   block_range(lo, hi, nonfinite);
-  griddep_wait();
   if (threadIdx.x == 0) parts[blockIdx.x] = RangePartial{lo, hi, static_cast<int>(nonfinite), 0};
 }
 

@@ -686,18 +686,8 @@ void finish_plan(cham_wpack_desc* d, int N, int K, int bits) {
 }
 }  // namespace
 
-
-extern "C" {
-
-cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const cham_wpack_desc* d, void* blob,
-                                   size_t blob_bytes, int* dev_status, void* stream) {
-  cham_status s = check_desc(d);
-  if (s != CHAM_OK) return s;
-  if (W == nullptr || fmt_dev == nullptr || blob == nullptr || !aligned16(W) || !aligned16(blob))
-    return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
-  if (blob_bytes < d->bytes) return fail(CHAM_ERR_WORKSPACE, "blob %zu < %llu bytes", blob_bytes,
-                                          static_cast<unsigned long long>(d->bytes));
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
+namespace {
+cham::PackArgs pack_args(const cham_wpack_desc* d, const void* W, const uint8_t* fmt_dev, void* blob, int* dev_status) {
   uint8_t* b = static_cast<uint8_t*>(blob);
   cham::PackArgs a{};
   a.W = static_cast<const __half*>(W);
@@ -724,9 +714,46 @@ cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const 
   a.gscale = d->group > 0 ? reinterpret_cast<uint32_t*>(b + d->off_gscale) : nullptr;
   a.desc = *d;
   a.desc_out = reinterpret_cast<cham_wpack_desc*>(b);
-  cham::launch_pack(a, nf4_table(), st);
+  return a;
+}
+}  // namespace
+
+extern "C" {
+
+cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const cham_wpack_desc* d, void* blob,
+                                   size_t blob_bytes, int* dev_status, void* stream) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  if (W == nullptr || fmt_dev == nullptr || blob == nullptr || !aligned16(W) || !aligned16(blob))
+    return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
+  if (blob_bytes < d->bytes) return fail(CHAM_ERR_WORKSPACE, "blob %zu < %llu bytes", blob_bytes,
+                                          static_cast<unsigned long long>(d->bytes));
+  cham::launch_pack(pack_args(d, W, fmt_dev, blob, dev_status), nf4_table(), static_cast<cudaStream_t>(stream));
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "pack launch");
+}
+
+cham_status chameleon_select_pack_palette(const void* W, int N, int K, uint32_t palette_mask,
+                                          const cham_wpack_desc* d, uint8_t* fmt_out, void* blob, size_t blob_bytes,
+                                          int* dev_status, void* stream) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  if (d->N != N || d->K != K || d->group != 0 || (d->n_class[0] != 0 && d->n_class[1] != 0))
+    return fail(CHAM_ERR_INVALID_ARG, "descriptor is not a one-class plan of %d x %d weights", N, K);
+  if (palette_mask == 0 || (palette_mask & ~0x1FFu) != 0) return fail(CHAM_ERR_INVALID_ARG, "palette mask 0x%x", palette_mask);
+  const int cls = d->n_class[0] == 0 ? 1 : 0;
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f)
+    if (((palette_mask >> f) & 1u) && (cham::w_class(f) != cls || cham::wbits(f) != d->bits))
+      return fail(CHAM_ERR_INVALID_ARG, "palette 0x%x does not match the plan's class and width", palette_mask);
+  if (W == nullptr || fmt_out == nullptr || blob == nullptr || !aligned16(W) || !aligned16(blob))
+    return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
+  if (blob_bytes < d->bytes) return fail(CHAM_ERR_WORKSPACE, "blob %zu < %llu bytes", blob_bytes,
+                                          static_cast<unsigned long long>(d->bytes));
+  cham::PackArgs a = pack_args(d, W, nullptr, blob, dev_status);
+  a.fmt_out = fmt_out;
+  cham::launch_select_pack(a, palette_mask, nf4_table(), static_cast<cudaStream_t>(stream));
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "select+pack launch");
 }
 
 // ---------------------------------------------------------------- a7/a8

@@ -80,32 +80,31 @@ CHAM_DEV float sum8(const float (&e2)[8]) {
   return __fadd_rn(__fadd_rn(a, b), __fadd_rn(c, d));
 }
 
-__global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict__ W, int N, int K, uint32_t mask,
-                                                       uint8_t* __restrict__ fmt_out, double* __restrict__ sse_out,
-                                                       NF4Table nf4) {
-  const int lane = threadIdx.x & 31;
-  const int c = blockIdx.x * kWWarps + (threadIdx.x >> 5);
-  if (c >= N) return;  // whole warps: no block-wide barrier follows
-  const __half* row = W + static_cast<size_t>(c) * K;
+// The selection of one channel (one warp): the first format of the palette with the least
+// SSE; sse_row (9 slots, +inf for non-members) may be null.  Every lane returns the result.
+CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const NF4Table& nf4, double* sse_row) {
   const int nvec = K / 8;
   const ChanStats st = row_stats(row, nvec, lane);
   const int iters = (nvec + 31) / 32;  // same trip count in every lane (shuffles)
   int best = -1;
   double best_e = 0.0;
   for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
-    if (!((mask >> f) & 1u)) continue;
+    if (!((mask >> f) & 1u)) {
+      if (lane == 0 && sse_row != nullptr) sse_row[f] = INFINITY;
+      continue;
+    }
     double acc = 0.0;
     if (w_is_mx(f)) {
       for (int it = 0; it < iters; ++it) {
         const int v = it * 32 + lane;
         float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
         if (v < nvec) load8(row, v, x);
-        float a = 0.f;
+        float am = 0.f;
 #pragma unroll
-        for (int i = 0; i < 8; ++i) a = fmaxf(a, fabsf(x[i]));
-        a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, 1));  // 4 lanes = one 32-element block
-        a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, 2));
-        const int X = mx_exponent(f, a);
+        for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
+        am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 1));  // 4 lanes = one 32-element block
+        am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 2));
+        const int X = mx_exponent(f, am);
         if (v < nvec) {
           float e2[8];
 #pragma unroll
@@ -137,14 +136,20 @@ __global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict
       best = f;
       best_e = tot;
     }
-    if (lane == 0 && sse_out != nullptr) sse_out[static_cast<size_t>(c) * CHAM_W_NFORMATS + f] = tot;
+    if (lane == 0 && sse_row != nullptr) sse_row[f] = tot;
   }
-  if (lane == 0) {
-    if (sse_out != nullptr)
-      for (int f = 0; f < CHAM_W_NFORMATS; ++f)
-        if (!((mask >> f) & 1u)) sse_out[static_cast<size_t>(c) * CHAM_W_NFORMATS + f] = INFINITY;
-    fmt_out[c] = static_cast<uint8_t>(best);
-  }
+  return best;
+}
+
+__global__ void __launch_bounds__(kWThreads) k_w_select(const __half* __restrict__ W, int N, int K, uint32_t mask,
+                                                       uint8_t* __restrict__ fmt_out, double* __restrict__ sse_out,
+                                                       NF4Table nf4) {
+  const int lane = threadIdx.x & 31;
+  const int c = blockIdx.x * kWWarps + (threadIdx.x >> 5);
+  if (c >= N) return;  // whole warps: no block-wide barrier follows
+  const int best = select_row(W + static_cast<size_t>(c) * K, K, mask, lane, nf4,
+                              sse_out != nullptr ? sse_out + static_cast<size_t>(c) * CHAM_W_NFORMATS : nullptr);
+  if (lane == 0) fmt_out[c] = static_cast<uint8_t>(best);
 }
 
 void launch_select(const __half* W, int N, int K, uint32_t mask, uint8_t* fmt_out, double* sse_out,
@@ -293,30 +298,8 @@ CHAM_DEV float code_value(int f, int code, int z, const NF4Table& nf4) {
   }
 }
 
-__global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) {
-  __shared__ GroupParam s_gp[kWWarps][kMaxRowGroups];
-  if (blockIdx.x == 0 && threadIdx.x < 64)  // the blob's header: a copy of the descriptor
-    reinterpret_cast<uint32_t*>(a.desc_out)[threadIdx.x] = reinterpret_cast<const uint32_t*>(&a.desc)[threadIdx.x];
-  const int lane = threadIdx.x & 31;
-  const int p = blockIdx.x * kWWarps + (threadIdx.x >> 5);  // one warp per packed slot
-  if (p >= a.n_packed) return;
-  int c;
-  if (a.one_class >= 0) {
-    // one MMA class: slot p holds channel p - base in original order, the rest is padding
-    const int rank = p - a.cls_base[a.one_class];
-    c = (rank >= 0 && rank < a.cls_count[a.one_class]) ? rank : -1;
-    if (lane == 0) {
-      const int f = c >= 0 ? a.fmt_dev[c] : -1;
-      const bool valid = f >= 0 && f < CHAM_W_NFORMATS && w_class(f) == a.one_class;
-      if (c >= 0 && !valid) set_status(a.dev_status, CHAM_ERR_INVALID_ARG);  // formats must match the plan
-      a.perm[p] = c;
-      a.fmtp[p] = c >= 0 ? static_cast<uint8_t>(valid ? f : 0xFF) : static_cast<uint8_t>(0xFF);
-    }
-    __syncwarp();
-    if (c >= 0 && (a.fmtp[p] == 0xFF)) return;  // invalid format: nothing to encode
-  } else {
-    c = a.perm[p];
-  }
+// Encodes packed slot p holding original channel c (-1: padding) in format f (one warp).
+CHAM_DEV void pack_slot(const PackArgs& a, int p, int c, int f, int lane, const NF4Table& nf4, GroupParam* s_gp_warp) {
   const int nvec_p = a.Kp / 8;
   const int tile = p >> 7, r = p & 127;
   if (c < 0) {  // padding slot: zero codes, unit scale
@@ -337,14 +320,13 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
     }
     return;
   }
-  const int f = a.fmtp[p];
   const __half* row = a.W + static_cast<size_t>(c) * a.K;
   const int nvec = a.K / 8;
   if (a.group > 0) {
     // group-wise: codes with their group's parameters; per 32-element block its zero point (in
     // the E8M0 slot) and its group's scale as fp16; the per-channel scale is 1
     if (lane == 0 && a.desc.n_fmt[f] != a.N) set_status(a.dev_status, CHAM_ERR_INVALID_ARG);  // one format per plan
-    GroupParam* gp = s_gp[threadIdx.x >> 5];
+    GroupParam* gp = s_gp_warp;
     group_params(row, a.K, a.group, f, lane, gp);
     const bool asym = f == CHAM_W_INT8_ASYM || f == CHAM_W_INT4_ASYM;
     for (int v = lane; v < nvec_p; v += 32) {
@@ -424,6 +406,58 @@ __global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) 
     a.scale[p] = mx ? 1.f : cs.s;
     a.zero[p] = static_cast<uint8_t>(cs.z);
   }
+}
+
+__global__ void __launch_bounds__(kWThreads) k_w_pack(PackArgs a, NF4Table nf4) {
+  __shared__ GroupParam s_gp[kWWarps][kMaxRowGroups];
+  if (blockIdx.x == 0 && threadIdx.x < 64)  // the blob's header: a copy of the descriptor
+    reinterpret_cast<uint32_t*>(a.desc_out)[threadIdx.x] = reinterpret_cast<const uint32_t*>(&a.desc)[threadIdx.x];
+  const int lane = threadIdx.x & 31;
+  const int p = blockIdx.x * kWWarps + (threadIdx.x >> 5);  // one warp per packed slot
+  if (p >= a.n_packed) return;
+  int c;
+  if (a.one_class >= 0) {
+    // one MMA class: slot p holds channel p - base in original order, the rest is padding
+    const int rank = p - a.cls_base[a.one_class];
+    c = (rank >= 0 && rank < a.cls_count[a.one_class]) ? rank : -1;
+    if (lane == 0) {
+      const int f = c >= 0 ? a.fmt_dev[c] : -1;
+      const bool valid = f >= 0 && f < CHAM_W_NFORMATS && w_class(f) == a.one_class;
+      if (c >= 0 && !valid) set_status(a.dev_status, CHAM_ERR_INVALID_ARG);  // formats must match the plan
+      a.perm[p] = c;
+      a.fmtp[p] = c >= 0 ? static_cast<uint8_t>(valid ? f : 0xFF) : static_cast<uint8_t>(0xFF);
+    }
+    __syncwarp();
+    if (c >= 0 && (a.fmtp[p] == 0xFF)) return;  // invalid format: nothing to encode
+  } else {
+    c = a.perm[p];
+  }
+  pack_slot(a, p, c, c >= 0 ? a.fmtp[p] : -1, lane, nf4, s_gp[threadIdx.x >> 5]);
+}
+
+// Selection and pack in one pass for a one-class plan (slot = channel): the warp that selects
+// channel c's format (Sec. 3.4) encodes the channel right away, so the row is read from DRAM once
+// and one launch serves both steps.
+__global__ void __launch_bounds__(kWThreads) k_w_select_pack(PackArgs a, uint32_t mask, NF4Table nf4) {
+  if (blockIdx.x == 0 && threadIdx.x < 64)  // the blob's header: a copy of the descriptor
+    reinterpret_cast<uint32_t*>(a.desc_out)[threadIdx.x] = reinterpret_cast<const uint32_t*>(&a.desc)[threadIdx.x];
+  const int lane = threadIdx.x & 31;
+  const int p = blockIdx.x * kWWarps + (threadIdx.x >> 5);
+  if (p >= a.n_packed) return;
+  const int rank = p - a.cls_base[a.one_class];
+  const int c = (rank >= 0 && rank < a.cls_count[a.one_class]) ? rank : -1;
+  int f = -1;
+  if (c >= 0) f = select_row(a.W + static_cast<size_t>(c) * a.K, a.K, mask, lane, nf4, nullptr);
+  if (lane == 0) {
+    if (c >= 0) a.fmt_out[c] = static_cast<uint8_t>(f);
+    a.perm[p] = c;
+    a.fmtp[p] = c >= 0 ? static_cast<uint8_t>(f) : static_cast<uint8_t>(0xFF);
+  }
+  pack_slot(a, p, c, f, lane, nf4, nullptr);
+}
+
+void launch_select_pack(const PackArgs& a, uint32_t mask, const NF4Table& nf4, cudaStream_t st) {
+  k_w_select_pack<<<(a.n_packed + kWWarps - 1) / kWWarps, kWThreads, 0, st>>>(a, mask, nf4);
 }
 
 // ------------------------------------------------------------------ (g, f) search (Sec. 3.5 forks)

@@ -171,6 +171,7 @@ struct GroupSearchArgs {
 struct PackArgs {
   const __half* W;
   const uint8_t* fmt_dev;   // selected format of each original channel
+  uint8_t* fmt_out;         // fused selection + pack: where the selected formats go
   int N, K, Kp, bits, n_chunks;
   int n_packed;             // Np
   int cls_base[2];          // first packed slot of each MMA class
@@ -192,6 +193,8 @@ struct PackArgs {
 void launch_select(const __half* W, int N, int K, uint32_t mask, uint8_t* fmt_out, double* sse_out,
                    const NF4Table& nf4, cudaStream_t st);
 void launch_pack(const PackArgs& a, const NF4Table& nf4, cudaStream_t st);
+// Fused selection + pack of a one-class plan (every palette member in one MMA class).
+void launch_select_pack(const PackArgs& a, uint32_t mask, const NF4Table& nf4, cudaStream_t st);
 void launch_select_groups(const GroupSearchArgs& a, const NF4Table& nf4, cudaStream_t st);
 void launch_channel_energy(const __half* X, int M, int K, double* energy, cudaStream_t st);
 

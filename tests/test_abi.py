@@ -207,3 +207,16 @@ def test_pack_plan_grouped_layout_and_checks(cl):
     assert L.chameleon_select_weight_groups_workspace_size(64, 320, 0x1F8 | 0x1, 1, ctypes.byref(w)) == cl.ERR_INVALID_ARG
     assert L.chameleon_select_weight_groups_workspace_size(64, 32 * 257, 0x070, 1, ctypes.byref(w)) == cl.ERR_INVALID_ARG
     assert L.chameleon_select_weight_groups_workspace_size(64, 320, 0x070, 0x1F, ctypes.byref(w)) == cl.OK
+
+
+def test_select_pack_palette_argument_checks(cl):
+    L = cl.lib()
+    buf = ctypes.create_string_buffer(1 << 20)
+    x = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
+    d8 = cl.pack_plan_palette(64, 320, cl.PALETTE_W8)
+    two = cl.pack_plan(64, 320, np.array([F.W_INT4_SYM, F.W_NF4] * 32, np.uint8))
+    grouped = cl.pack_plan_grouped(64, 320, F.W_INT4_ASYM, 64)
+    for d, N, K, mask in [(d8, 64, 256, cl.PALETTE_W8), (d8, 32, 320, cl.PALETTE_W8), (two, 64, 320, cl.PALETTE_W4),
+                          (grouped, 64, 320, 1 << F.W_INT4_ASYM), (d8, 64, 320, cl.PALETTE_W4), (d8, 64, 320, 0)]:
+        assert L.chameleon_select_pack_palette(x, N, K, mask, ctypes.byref(d), x, x, 1 << 19, x,
+                                               None) == cl.ERR_INVALID_ARG

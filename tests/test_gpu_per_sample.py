@@ -144,3 +144,33 @@ def test_pixart_shapes_two_samples_sampled_rows(cl, index):
         a = np.vstack([F.act_dequant(q) for q in qs])
         y_ref, bound = G.linear_rows_reference(a, w, rows, bias)
         check_rows(host(Y)[rows], y_ref, bound, "f16", "%s act %d" % ((M, K, N), act_fmt))
+
+
+@pytest.mark.parametrize("act_fmt", [F.A_E4M3, F.A_INT8_ASYM, F.A_MXFP8])
+def test_chained_linears_read_the_previous_output(cl, act_fmt):
+    """One linear's fp16 output fed straight to the next linear on the same stream: the second
+    quantizer (launched while the first GEMM may still run) must see the finished output.  The
+    output buffer starts filled with 2^14 so that an early read would change the range."""
+    import torch
+    rng = np.random.default_rng(70 + act_fmt)
+    M, K1, K2, N2 = 256, 320, 640, 257
+    X = WL.to_fp16(rng.standard_t(4, (M, K1)))
+    W1 = WL.weight_mix(rng, K2, K1)
+    W2 = WL.weight_mix(rng, N2, K2)
+    f1 = np.asarray(F.W8_PALETTE, np.uint8)[rng.integers(0, 3, K2)]
+    f2 = np.asarray(F.W8_PALETTE, np.uint8)[rng.integers(0, 3, N2)]
+    d1, d2 = cl.pack_plan(K2, K1, f1), cl.pack_plan(N2, K2, f2)
+    b1, _ = cl.pack_weights(cuda(W1), cuda(f1), d1)
+    b2, _ = cl.pack_weights(cuda(W2), cuda(f2), d2)
+    torch.cuda.synchronize()
+    Y1 = torch.full((M, K2), 16384.0, dtype=torch.float16, device="cuda")
+    for _ in range(3):
+        Y1.fill_(16384.0)
+        cl.linear_ex(cuda(X), d1, b1, F.A_E4M3, 1, Y=Y1)
+        Y2, st = cl.linear_ex(Y1, d2, b2, act_fmt, 2)
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0
+        y1 = host(Y1)
+        a = F.act_dequant_per_sample(F.act_quant_per_sample(y1, act_fmt, 2))
+        y_ref, bound = G.linear_rows_reference(a, SEL.dequant_selected(W2, f2), np.arange(M), None)
+        assert_within_bound(host(Y2), y_ref, bound, "chained act %d" % act_fmt)

@@ -125,3 +125,26 @@ def test_palette_plan_packs_the_same_blob(cl, mask, K):
     assert np.array_equal(a[:40], b[:40]) and np.array_equal(a[76:256], b[76:256])
     n_fmt = slice(40, 40 + 4 * 9)                      # int32 n_fmt[9] in the descriptor copy
     assert np.all(b[n_fmt].view(np.int32)[[f for f in range(9) if (mask >> f) & 1]] == -1)
+
+
+@pytest.mark.parametrize("mask,K", [(0x007, 320), (0x007, 1280), ((1 << 4) | (1 << 6) | (1 << 7) | (1 << 8), 96),
+                                    (1 << 5, 64)])
+def test_fused_select_pack_equals_the_two_launches(cl, mask, K):
+    """chameleon_select_pack_palette gives the formats of chameleon_select_weight_formats and the
+    blob chameleon_pack_weights writes for them from the same palette plan, byte for byte."""
+    import torch
+    W = WL.weight_mix(np.random.default_rng(K + mask), 300, K)
+    Wd = cuda(W)
+    d = cl.pack_plan_palette(W.shape[0], K, mask)
+    fmt_ref, _ = cl.select_weight_formats(Wd, mask)
+    b_ref, st1 = cl.pack_weights(Wd, fmt_ref, d)
+    fmt, b, st2 = cl.select_pack_palette(Wd, mask, d)
+    torch.cuda.synchronize()
+    assert int(st1.item()) == 0 and int(st2.item()) == 0
+    np.testing.assert_array_equal(host(fmt), host(fmt_ref))
+    a, c = host(b_ref), host(b)
+    tiles = d.n_tiles[0] + d.n_tiles[1]
+    np_, chunks, cb = 128 * tiles, d.Kp // 64, 64 if d.bits == 8 else 32
+    for off, n in [(0, 256), (d.off_codes, tiles * chunks * 128 * cb), (d.off_scale, 4 * np_), (d.off_zero, np_),
+                   (d.off_e8m0, tiles * chunks * 256), (d.off_fmt, np_), (d.off_perm, 4 * np_)]:
+        assert np.array_equal(a[off:off + n], c[off:off + n]), off
