@@ -216,8 +216,9 @@ cham_status chameleon_act_channel_energy(const void* X, int M, int K, double* en
 
 /* ------------------------------------------------------------------ a6: weight pack */
 
-/* Packed-weight descriptor.  Channels are permuted (Sec. 5: "same-format sub-GEMMs after a
- * channel permutation") into two MMA classes, each padded to 128-channel tiles:
+/* Packed-weight descriptor.  Channels are reordered (Sec. 5 proposes a permutation that groups
+ * the channels of one format so that each group runs as its own GEMM) into two MMA classes, each
+ * padded to 128-channel tiles:
  *   class 0 = 4-bit formats with an 8-bit tensor-core path (INT4-sym, INT4-asym, E2M1, MXINT4,
  *             MXFP4), class 1 = the rest (NF4, INT8-sym, INT8-asym, MXINT8);
  * inside a class in original channel order (a tile's output columns stay contiguous; the GEMM

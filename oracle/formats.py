@@ -1,9 +1,9 @@
 """Number formats of the Chameleon palette, written from their definitions.
 
 Test infrastructure (see ``oracle/__init__``).  Passages followed:
-  * activation palette and codes 0..4 -- Sec. 3.2 (F_a, "indexed by integer codes 0,1,2,3,4");
+  * activation palette and codes 0..4 -- Sec. 3.2 (F_a, numbered 0 to 4 in the runtime LUT);
   * weight palettes F_w^(8), F_w^(4) -- Sec. 3.2;
-  * INT8-asym, E4M3, E5M2, MX, 4-bit codes -- App. A.11 ("Number-Format Details");
+  * INT8-asym, E4M3, E5M2, MX, 4-bit codes -- App. A.11 (the number-format appendix);
   * ScaleZP -- App. A.7 (shared helper of Alg. 1 and Alg. 3);
   * clamp before the FP8 cast -- App. A.7, implementation note (ii);
   * MX shared exponent floor(log2 max|x|) with an E8M0 byte -- Sec. 3.6, App. A.11, App. A.12.
@@ -38,13 +38,13 @@ W_BITS = {W_INT8_SYM: 8, W_INT8_ASYM: 8, W_MXINT8: 8, W_INT4_SYM: 4, W_INT4_ASYM
           W_NF4: 4, W_E2M1: 4, W_MXINT4: 4, W_MXFP4: 4}
 W_IS_MX = {f: f in (W_MXINT8, W_MXINT4, W_MXFP4) for f in W_BITS}
 
-MX_BLOCK = 32  # "block size 32 and a shared 8-bit exponent" (Sec. 3.2)
+MX_BLOCK = 32  # MX formats: 32-element blocks sharing one 8-bit exponent (Sec. 3.2)
 
 # ---------------------------------------------------------------- binary minifloats (App. A.11)
 # name: (exponent bits, mantissa bits, bias, largest finite magnitude)
 FP_SPECS = {
-    "e4m3": (4, 3, 7, 448.0),      # "range +-448, smallest normal 2^-6", no infinities
-    "e5m2": (5, 2, 15, 57344.0),   # "range +-57344, smallest normal 2^-14"
+    "e4m3": (4, 3, 7, 448.0),      # max 448, smallest normal 2^-6, no infinities (App. A.11)
+    "e5m2": (5, 2, 15, 57344.0),   # max 57344, smallest normal 2^-14 (App. A.11)
     "e2m1": (2, 1, 1, 6.0),        # {0, +-0.5, +-1, +-1.5, +-2, +-3, +-4, +-6}
 }
 

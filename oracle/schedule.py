@@ -12,7 +12,7 @@ Test infrastructure (see ``oracle/__init__``).  Passages followed:
 
 Readings of passages the paper leaves open: timesteps are integers 0..T-1 with alpha_bar_t including beta_t (R17);
 the scaled-linear betas interpolate linearly in sqrt(beta) (Stable-Diffusion schedule named by
-App. A.11 "scaled-linear"), the linear betas linearly in beta; kappa := 0 when the variance is 0.
+App. A.11 names it scaled-linear), the linear betas linearly in beta; kappa := 0 when the variance is 0.
 """
 import numpy as np
 

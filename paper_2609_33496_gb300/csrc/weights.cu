@@ -2,13 +2,13 @@
 //
 // Selection (Sec. 3.4, Eq. weight-argmax): every output channel is round-tripped through every
 // palette format; the squared reconstruction error SSE_f(c) is accumulated from per-element
-// errors that are exact up to one fp32 rounding (fp32 sums of eight squares, added in fp64;
-// relative error below 2.4e-7); the smallest error wins, the earlier palette member on ties
+// errors that are exact up to one fp32 rounding (fp32 sums of eight squares, added exactly as
+// fp32 pairs; relative error below 2.4e-7); the smallest error wins, the earlier palette member on ties
 // (strict '<').  One warp per channel: the row (at most 10 KB for K = 5120) stays in L1 across
 // the format passes, and every reduction is a warp shuffle tree.
 //
-// Pack: channels are permuted (Sec. 5: "same-format sub-GEMMs after a channel permutation") into
-// the two MMA classes, each kept in original channel order and padded to 128-channel tiles, and
+// Pack: channels are reordered (Sec. 5 proposes grouping the channels of one format by a
+// permutation so that each group runs as its own GEMM) into the two MMA classes, each kept in original channel order and padded to 128-channel tiles, and
 // encoded in the tiled layout the GEMM reads with bulk copies (include/chameleon.h).
 #include "weights.cuh"
 
@@ -71,13 +71,46 @@ CHAM_DEV ChanStats row_stats(const __half* row, int nvec, int lane) {
 // ------------------------------------------------------------------ a5: selection
 // Pairwise fp32 sum of eight non-negative squared errors.  Each square and each of the three
 // levels of additions rounds once, so the group sum is within 4 * 2^-24 relative of the exact
-// sum; the groups are then added in fp64.  Every term being non-negative, the channel's SSE
-// keeps that relative bound (about 2.4e-7), while the fp64 pipe -- a small fraction of the
-// fp32 rate on this GPU -- sees one add per eight elements.
+// sum; the groups are then added exactly (Sum2 below).  Every term being non-negative, the
+// channel's SSE keeps that relative bound (about 2.4e-7).
 CHAM_DEV float sum8(const float (&e2)[8]) {
   const float a = __fadd_rn(e2[0], e2[1]), b = __fadd_rn(e2[2], e2[3]);
   const float c = __fadd_rn(e2[4], e2[5]), d = __fadd_rn(e2[6], e2[7]);
   return __fadd_rn(__fadd_rn(a, b), __fadd_rn(c, d));
+}
+
+// A sum kept as an unevaluated pair hi + lo of fp32 values: each addition splits the rounding
+// error of hi + x off exactly (Knuth's TwoSum; this file is compiled without FMA contraction) and
+// carries it in lo.  The pair tracks the exact sum of its fp32 inputs to about 2^-24 relative of
+// lo, far below the 4 * 2^-24 of each eight-element group sum, without the fp64 pipe (a small
+// fraction of the fp32 rate on this GPU) inside the loops.
+struct Sum2 {
+  float hi, lo;
+};
+
+CHAM_DEV Sum2 two_sum(float a, float b) {
+  const float s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  const float err = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  return Sum2{s, err};
+}
+
+CHAM_DEV void sum2_add(Sum2& acc, float x) {
+  const Sum2 t = two_sum(acc.hi, x);
+  acc.hi = t.hi;
+  acc.lo = __fadd_rn(acc.lo, t.lo);
+}
+
+// Warp-wide total of the lanes' pairs (fixed xor-tree order), as fp64, in every lane.
+CHAM_DEV double warp_sum2(Sum2 v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float h = __shfl_xor_sync(0xffffffffu, v.hi, o), l = __shfl_xor_sync(0xffffffffu, v.lo, o);
+    const Sum2 t = two_sum(v.hi, h);
+    v.hi = t.hi;
+    v.lo = __fadd_rn(__fadd_rn(v.lo, l), t.lo);
+  }
+  return static_cast<double>(v.hi) + static_cast<double>(v.lo);
 }
 
 // The selection of one channel (one warp): the first format of the palette with the least
@@ -93,7 +126,7 @@ CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const
       if (lane == 0 && sse_row != nullptr) sse_row[f] = INFINITY;
       continue;
     }
-    double acc = 0.0;
+    Sum2 acc{0.f, 0.f};
     if (w_is_mx(f)) {
       for (int it = 0; it < iters; ++it) {
         const int v = it * 32 + lane;
@@ -114,7 +147,7 @@ CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const
             const float e = __fsub_rn(x[i], dq);
             e2[i] = __fmul_rn(e, e);
           }
-          acc += static_cast<double>(sum8(e2));
+          sum2_add(acc, sum8(e2));
         }
       }
     } else {
@@ -128,10 +161,10 @@ CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const
           encode_chan(f, x[i], cs, nf4, &err);
           e2[i] = __fmul_rn(err, err);
         }
-        acc += static_cast<double>(sum8(e2));
+        sum2_add(acc, sum8(e2));
       }
     }
-    const double tot = warp_reduce(acc, DAdd());
+    const double tot = warp_sum2(acc);
     if (best < 0 || tot < best_e) {  // palette order: the earlier member wins a tie
       best = f;
       best_e = tot;
@@ -479,7 +512,7 @@ __global__ void __launch_bounds__(kWThreads) k_w_select_groups(GroupSearchArgs a
   const int iters = (nvec + 31) / 32;  // same trip count in every lane (shuffles)
   for (int ci = 0; ci < a.n_cand; ++ci) {
     const int g = a.cand[ci].g, f = a.cand[ci].f;
-    double acc = 0.0;
+    Sum2 acc{0.f, 0.f};
     if (w_is_mx(f)) {
       for (int it = 0; it < iters; ++it) {
         const int v = it * 32 + lane;
@@ -500,7 +533,7 @@ __global__ void __launch_bounds__(kWThreads) k_w_select_groups(GroupSearchArgs a
             const float e = __fsub_rn(x[i], dq);
             e2[i] = __fmul_rn(__fmul_rn(e, e), a.energy32[v * 8 + i]);
           }
-          acc += static_cast<double>(sum8(e2));
+          sum2_add(acc, sum8(e2));
         }
       }
     } else {
@@ -521,10 +554,10 @@ __global__ void __launch_bounds__(kWThreads) k_w_select_groups(GroupSearchArgs a
           const float e = __fsub_rn(x[i], dq);
           e2[i] = __fmul_rn(__fmul_rn(e, e), a.energy32[v * 8 + i]);
         }
-        acc += static_cast<double>(sum8(e2));
+        sum2_add(acc, sum8(e2));
       }
     }
-    const double tot = warp_reduce(acc, DAdd());
+    const double tot = warp_sum2(acc);
     if (lane == 0) a.parts[static_cast<size_t>(c) * a.n_cand + ci] = tot;
   }
 }

@@ -66,10 +66,10 @@ def test_e4m3_grid():
     nan = np.isnan(v)
     assert list(codes[nan]) == [0x7F, 0xFF]                 # no infinities, one NaN per sign
     fin = v[~nan]
-    assert fin.max() == 448.0 and fin.min() == -448.0       # "range +-448"
+    assert fin.max() == 448.0 and fin.min() == -448.0       # App. A.11: E4M3 spans +-448
     pos = np.unique(fin[fin > 0])
     assert pos.min() == 2.0 ** -9                           # smallest subnormal m * 2^-9
-    assert F.fp_decode(0x08, "e4m3") == 2.0 ** -6           # "smallest normal 2^-6"
+    assert F.fp_decode(0x08, "e4m3") == 2.0 ** -6           # App. A.11: smallest normal 2^-6
     assert np.all(np.diff(pos[(pos >= 1) & (pos < 2)]) == 2.0 ** -3)   # 3 mantissa bits
     np.testing.assert_array_equal(pos, GRIDS["e4m3"][0][1:])
 
@@ -77,8 +77,8 @@ def test_e4m3_grid():
 def test_e5m2_grid():
     v = F.fp_decode(np.arange(256), "e5m2")
     fin = v[np.isfinite(v)]
-    assert fin.max() == 57344.0                             # "range +-57344"
-    assert F.fp_decode(0x04, "e5m2") == 2.0 ** -14          # "smallest normal 2^-14"
+    assert fin.max() == 57344.0                             # App. A.11: E5M2 spans +-57344
+    assert F.fp_decode(0x04, "e5m2") == 2.0 ** -14          # App. A.11: smallest normal 2^-14
     assert np.sum(~np.isfinite(v)) == 8                     # exponent 31: inf and NaN
     pos = np.unique(fin[fin > 0])
     assert np.all(np.diff(pos[(pos >= 1) & (pos < 2)]) == 2.0 ** -2)   # 2 mantissa bits
