@@ -78,6 +78,13 @@ typedef int cham_status;
 
 const char* chameleon_status_string(cham_status s);
 const char* chameleon_last_error_detail(void);
+
+/* Waits for the work queued on `stream` (a cudaStream_t; NULL = the legacy default stream) and
+ * returns the device status word dev_status (device int, written by the kernels of the calls
+ * that were given it: 0 = CHAM_OK, else the first device-detected error, e.g.
+ * CHAM_ERR_NONFINITE or CHAM_ERR_TIMEOUT).  The word is left as it is.  CHAM_ERR_CUDA when the
+ * synchronisation or the copy fails; CHAM_ERR_INVALID_ARG when dev_status is NULL. */
+cham_status chameleon_check(const int* dev_status, void* stream);
 int chameleon_version(void);
 
 /* ------------------------------------------------------------------ host helpers (a1, L2) */

@@ -38,7 +38,7 @@ EXPORTS = [
     "chameleon_act_format_sse_workspace_size", "chameleon_act_format_sse", "chameleon_act_format_argmin",
     "chameleon_pack_plan_grouped", "chameleon_group_candidates", "chameleon_select_weight_groups_workspace_size",
     "chameleon_select_weight_groups", "chameleon_candidate_argmin", "chameleon_act_channel_energy",
-    "chameleon_select_pack_palette",
+    "chameleon_select_pack_palette", "chameleon_check",
 ]
 
 
@@ -130,6 +130,7 @@ def lib():
         "chameleon_candidate_argmin": (i32, [ctypes.POINTER(ctypes.c_double), i32]),
         "chameleon_act_channel_energy": (i32, [vp, i32, i32, vp, vp]),
         "chameleon_select_pack_palette": (i32, [vp, i32, i32, u32, pdesc, vp, vp, sz, vp, vp]),
+        "chameleon_check": (i32, [vp, vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -142,6 +143,11 @@ def lib():
 def check(status):
     if status != OK:
         raise ChameleonError(status, lib().chameleon_last_error_detail().decode())
+
+
+def device_status(dev_status, stream=None):
+    """Synchronise the stream and return the device status word (0 = ok) without raising."""
+    return lib().chameleon_check(_ptr(dev_status), _stream(stream))
 
 
 def _ptr(t):

@@ -256,6 +256,16 @@ const char* chameleon_last_error_detail(void) { return g_detail; }
 
 int chameleon_version(void) { return 2; }
 
+cham_status chameleon_check(const int* dev_status, void* stream) {
+  if (dev_status == nullptr) return fail(CHAM_ERR_INVALID_ARG, "dev_status is NULL");
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+  int v = 0;
+  e = cudaMemcpy(&v, dev_status, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "status copy");
+  return v;
+}
+
 // ---------------------------------------------------------------- a1 and the LUT builder
 int chameleon_bucket(int t, int T, int B) {
   if (T <= 0 || B <= 0 || t < 0) return -1;

@@ -220,3 +220,7 @@ def test_select_pack_palette_argument_checks(cl):
                           (grouped, 64, 320, 1 << F.W_INT4_ASYM), (d8, 64, 320, cl.PALETTE_W4), (d8, 64, 320, 0)]:
         assert L.chameleon_select_pack_palette(x, N, K, mask, ctypes.byref(d), x, x, 1 << 19, x,
                                                None) == cl.ERR_INVALID_ARG
+
+
+def test_check_rejects_a_null_status_word(cl):
+    assert cl.lib().chameleon_check(None, None) == cl.ERR_INVALID_ARG

@@ -130,3 +130,15 @@ def test_full_size_sdxl_static_sampled_rows(cl, layer):
         a = F.act_dequant(F.act_quant(X[rows], act_fmt, lo, hi))
         y_ref, bound = G.linear_rows_reference(a, w, np.arange(len(rows)), bias)
         assert_within_bound(host(Y)[rows], y_ref, bound, "%s bucket %d" % (name, bucket))
+
+
+def test_check_returns_the_device_status(cl):
+    """chameleon_check synchronises and hands back the first device-detected error."""
+    import torch
+    X = WL.to_fp16(np.random.default_rng(2).standard_normal((64, 256)))
+    _, st = cl.act_quant_static(cuda(X), F.A_E4M3, cl.scale_zp(F.A_E4M3, -4.0, 4.0))
+    assert cl.device_status(st) == 0
+    X[3, 3] = np.float16(np.nan)
+    _, st = cl.act_quant_static(cuda(X), F.A_E4M3, cl.scale_zp(F.A_E4M3, -4.0, 4.0))
+    assert cl.device_status(st) == cl.ERR_NONFINITE
+    assert cl.lib().chameleon_check(None, None) == cl.ERR_INVALID_ARG
