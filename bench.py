@@ -357,6 +357,8 @@ def main():
     clocks = clk.summary()
     probe = tensor_probe(torch, device)
     variants = None if args.no_variants else variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe)
+    if variants is not None:
+        variants["workloads"] = workload_variants(torch, cl, st, pk, probe)
 
     result = {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
@@ -650,6 +652,65 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
         out["layers"].append({"layer": lname, "M": Ml, "K": Kl, "N": Nl, "act_fmt": af, "us": round(t * 1e6, 2),
                               "tflops": round(fl / t / 1e12, 1), "bound": "tensor" if t_f >= t_b else "hbm",
                               "frac_f16_roofline": round(max(t_f, t_b) / t, 4)})
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0, "device status %d" % int(st.item())
+    return out
+
+
+def workload_variants(torch, cl, st, pk, probe, reps=20):
+    """The other workloads' layer shapes, each selected (4-bit palette of its fork), packed,
+    quantized and multiplied on the GPU; per shape the GEMM and the quantizer alone (reps
+    graph-captured launches between two events) with their roofline fractions.  SDXL-UNet W4A8
+    at a mid bucket (E4M3, dynamic scales); PixArt-alpha W4A8 with E5M2 and the DiT path's two
+    per-sample scales; SDXL-Turbo weight-only W4A16 rows (fp16 activations, no quantizer)."""
+    from paper_2609_33496_gb300 import workloads as WL
+    dev = torch.device("cuda", torch.cuda.current_device())
+    hbm = pk["hbm_gbs"] * 1e9
+    p16 = (probe or {}).get("f16", pk.get("bf16_tflops", 1900.0)) * 1e12
+    palette = (1 << cl.W_INT4_SYM) | (1 << cl.W_INT4_ASYM) | (1 << cl.W_NF4) | (1 << cl.W_E2M1) | \
+        (1 << cl.W_MXINT4) | (1 << cl.W_MXFP4)
+
+    def timed(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for _ in range(reps):
+                fn()
+        g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps * 1e-3  # seconds per launch
+
+    out = []
+    for cfg, name, shapes, af, groups in ((3, "sdxl-unet W4A8", WL.UNET_W4A8_SHAPES, cl.A_E4M3, 1),
+                                          (4, "pixart-alpha W4A8", WL.PIXART_W4A8_SHAPES, cl.A_E5M2, 2),
+                                          (5, "sdxl-turbo W4A16", WL.TURBO_W4A16_SHAPES, cl.A_FP16, 1)):
+        for i, (M, K, N) in enumerate(shapes):
+            X, W, bias = WL.config_layer(cfg, i, M, K, N)
+            Xd, Wd, bd = (torch.from_numpy(v).to(dev) for v in (X, W, bias))
+            fmt, _ = cl.select_weight_formats(Wd, palette)
+            desc = cl.pack_plan(N, K, fmt.cpu().numpy())
+            blob, _ = cl.pack_weights(Wd, fmt, desc, dev_status=st)
+            ws = torch.empty(cl.linear_workspace_size(M, desc, af), dtype=torch.uint8, device=dev)
+            Y = torch.empty((M, N), dtype=torch.float32, device=dev)
+            g = groups if M % groups == 0 else 1
+            cl.linear_prepare_groups(Xd, af, g, ws, st)
+            t = timed(lambda: cl.linear_gemm_ex(Xd, desc, blob, af, g, bd, Y, ws, st))
+            fl = 2.0 * M * K * N
+            a_bytes = M * K * 2                       # the fp16 operand (or X itself)
+            byts = a_bytes + N * K / 2 + 9 * N + 4 * M * N
+            row = {"workload": name, "M": M, "K": K, "N": N, "act_fmt": af, "gemm_us": round(t * 1e6, 2),
+                   "tflops": round(fl / t / 1e12, 1), "bound": "tensor" if fl / p16 >= byts / hbm else "hbm",
+                   "frac_f16_roofline": round(max(fl / p16, byts / hbm) / t, 4)}
+            if af != cl.A_FP16:
+                tq = timed(lambda: cl.linear_prepare_groups(Xd, af, g, ws, st))
+                row.update({"quant_us": round(tq * 1e6, 2), "quant_gbs": round(4 * M * K / tq / 1e9, 1),
+                            "quant_frac_hbm": round(4 * M * K / tq / hbm, 4)})
+            out.append(row)
+            del Xd, Wd, bd, blob, ws, Y
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
     return out

@@ -234,6 +234,23 @@ size_t linear_ws_need(int M, int K, int act_fmt) {
   return linear_ws(M, K).operand + round_up(static_cast<size_t>(M) * K * 2, 256);
 }
 
+// The GEMM's split-K factor and its partial-sum region, which follows the operand region.
+struct GemmPlan {
+  int bn, k_split;
+  size_t partial, need;
+};
+GemmPlan gemm_plan(int M, const cham_wpack_desc* d, int act_fmt) {
+  GemmPlan g;
+  const int num_sms = num_sms_current();
+  const int ch_tiles = d->n_tiles[0] + d->n_tiles[1];
+  g.bn = cham::gemm_pick_bn(M, ch_tiles, num_sms);
+  const int tiles = ch_tiles * ((M + g.bn - 1) / g.bn);
+  g.k_split = cham::gemm_pick_split(tiles, d->Kp / 64, num_sms);
+  g.partial = linear_ws_need(M, d->K, act_fmt);
+  g.need = g.partial + (g.k_split > 1 ? round_up(static_cast<size_t>(g.k_split) * M * 128 * ch_tiles * 4, 256) : 0);
+  return g;
+}
+
 }  // namespace
 
 extern "C" {
@@ -768,13 +785,14 @@ cham_status chameleon_select_pack_palette(const void* W, int N, int K, uint32_t 
 
 // ---------------------------------------------------------------- a7/a8
 // Workspace: [0, 256) the per-tensor scale s_a; [256, 256 + R) range partials; then the M x K
-// fp16 activation operand (exact values of the codes, R13).
+// fp16 activation operand (exact values of the codes, R13); then, when the GEMM splits K, its
+// fp32 partial sums.
 cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* d, int act_fmt, size_t* ws_bytes) {
   cham_status s = check_desc(d);
   if (s != CHAM_OK) return s;
   if (M <= 0 || act_fmt < 0 || act_fmt > CHAM_A_FP16 || ws_bytes == nullptr)
     return fail(CHAM_ERR_INVALID_ARG, "M=%d act_fmt=%d", M, act_fmt);
-  *ws_bytes = linear_ws_need(M, d->K, act_fmt);
+  *ws_bytes = gemm_plan(M, d, act_fmt).need;
   return CHAM_OK;
 }
 
@@ -867,7 +885,8 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   s = check_groups(M, n_groups);
   if (s != CHAM_OK) return s;
   const int K = d->K;
-  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
+  const GemmPlan plan = gemm_plan(M, d, act_fmt);
+  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, plan.need);
   if (s != CHAM_OK) return s;
   if (act_fmt == CHAM_A_FP16 && (X == nullptr || !aligned16(X)))
     return fail(CHAM_ERR_INVALID_ARG, "X must be a 16-byte aligned device pointer");
@@ -908,12 +927,15 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   }
   const int num_sms = num_sms_current();
   const int tiles = d->n_tiles[0] + d->n_tiles[1];
-  const int bn = cham::gemm_pick_bn(M, tiles, num_sms);
+  const int bn = plan.bn;
   CUtensorMap map;
   s = make_act_map(&map, operand, M, K, bn);
   if (s != CHAM_OK) return s;
   g.tile0 = 0;
   g.n_ch_tiles = tiles;
+  g.Np = 128 * tiles;
+  g.k_split = plan.k_split;
+  g.partial = plan.k_split > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
   const cudaError_t e = cham::launch_gemm_f16(map, g, num_sms, bn, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "gemm launch");
 }

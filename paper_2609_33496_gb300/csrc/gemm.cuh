@@ -20,6 +20,9 @@ struct GemmArgs {
   void* Y;                   // [M][N] of y_type
   int y_type;                // CHAM_Y_F32, CHAM_Y_F16 or CHAM_Y_BF16
   int rows_per_group;        // rows sharing one act_scale entry (per-sample scales); >= M: one
+  int k_split;               // split-K: each tile's K-chunks in k_split contiguous ranges (1: off)
+  float* partial;            // split-K: raw fp32 sums [k_split][M][Np], reduced by a second kernel
+  int Np;                    // packed channels (128 per channel tile)
   int M, N, n_chunks;        // n_chunks = Kp / 64
   int tile0;                 // first 128-channel tile of this launch
   int n_ch_tiles;            // 128-channel tiles of this launch
@@ -32,6 +35,9 @@ struct GemmArgs {
 
 // Token-tile (MMA N) size for M tokens: 16, 32, 64, 128 or 192.
 int gemm_pick_bn(int M, int n_tiles, int num_sms);
+// Split-K factor: 1 when the tiles fill the GPU, else enough K ranges (of at least two chunks)
+// to give every SM work.
+int gemm_pick_split(int tiles, int n_chunks, int num_sms);
 // Persistent launch: min(tiles, num_sms) CTAs walk the (channel tile, token tile) grid.
 cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
 // The launches of one output type (instantiated in gemm.cu, gemm_f16.cu, gemm_bf16.cu).

@@ -36,6 +36,7 @@ namespace cham {
 constexpr int kBK = 64;  // K elements per stage: 128 bytes of fp16 per activation row
 constexpr int kDecodeGroups = 2;  // decode warpgroups, taking alternate K-chunks
 constexpr int kEpiGroups = 2;     // epilogue warpgroups, taking alternate 16-column slices
+constexpr int kPartialOut = 3;    // epilogue "output type" of split-K units: raw fp32 partial sums
 constexpr int kGemmThreads = 128 * (1 + kDecodeGroups + kEpiGroups);
 
 template <int BN, int BITS>
@@ -317,11 +318,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   constexpr bool grouped = GW;  // group-wise blob: per-block fp16 scales
   const int n_ch = a.n_ch_tiles;
   const int n_tiles = n_ch * ((a.M + BN - 1) / BN);
-  // K-chunks this CTA processes (its tiles x nk); the last commit group may be partial
-  const uint32_t total =
-      static_cast<int>(blockIdx.x) < n_tiles
-          ? static_cast<uint32_t>((n_tiles - static_cast<int>(blockIdx.x) + gridDim.x - 1) / gridDim.x) * nk
-          : 0u;
+  // Work units: tile t = u / ks over its K-chunk range j = u % ks (ks = 1: whole tiles).  Units
+  // u = blockIdx.x, blockIdx.x + gridDim.x, ... belong to this CTA.
+  const int ks = a.k_split;
+  const int n_units = n_tiles * ks;
+  auto kc_begin = [&](int u) { return ks == 1 ? 0 : (u % ks) * nk / ks; };
+  auto kc_end = [&](int u) { return ks == 1 ? nk : (u % ks + 1) * nk / ks; };
+  // K-chunks this CTA processes; the last commit group may be partial
+  uint32_t total = 0;
+  for (int u = blockIdx.x; u < n_units; u += gridDim.x) total += static_cast<uint32_t>(kc_end(u) - kc_begin(u));
   // wait until the MMAs of chunk j have completed (the commit of its group)
   auto wait_done = [&](uint32_t j) {
     const uint32_t g = j / kGroup;
@@ -354,9 +359,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        const int t = u / ks;
         const int ch = a.tile0 + t % n_ch, tok0 = (t / n_ch) * BN;
-        for (int kc = 0; kc < nk; ++kc, ++it) {
+        const int kc1 = kc_end(u);
+        for (int kc = kc_begin(u); kc < kc1; ++kc, ++it) {
           const int s = it % S;
           if (it >= static_cast<uint32_t>(S) && !wait_done(it - S)) {  // the stage's previous chunk is consumed
             ok = false;
@@ -389,15 +396,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       constexpr uint32_t kStageDesc = C::kStage >> 4;
       uint32_t it = 0, acc_it = 0, s = 0, sa = 0, gi = 0;  // s = it % S, sa = it % kAStages, gi = it % kGroup
       bool ok = true;
-      for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++acc_it) {
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++acc_it) {
         const int b = acc_it & 1;
+        const int kc0 = kc_begin(u), kc1 = kc_end(u);
         if (!mbar_wait(&accempty[b], ((acc_it >> 1) & 1) ^ 1, abort_flag, a.dev_status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem + b * C::kAccCols;
         // One wait per group of kGroup consecutive K-chunks, on the decoded-operand barrier only:
         // the decoders arrive on it after they have themselves observed the stage's TMA barrier,
         // so the activation tile has landed too.  A group may straddle two tiles.
-        for (int kc = 0; kc < nk; ++kc, ++it) {
+        for (int kc = kc0; kc < kc1; ++kc, ++it) {
           if (gi == 0) {
             if (!mbar_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
               ok = false;
@@ -407,7 +415,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
           const uint64_t bd = desc0 + s * kStageDesc;
           const uint32_t ad = tmem + C::kACol + sa * 32;
-          mma_f16_ts(d_tmem, ad, bd, idesc, kc != 0);
+          mma_f16_ts(d_tmem, ad, bd, idesc, kc != kc0);
           mma_f16_ts(d_tmem, ad + 8, bd + 2, idesc, 1u);
           mma_f16_ts(d_tmem, ad + 16, bd + 4, idesc, 1u);
           mma_f16_ts(d_tmem, ad + 24, bd + 6, idesc, 1u);
@@ -434,19 +442,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // the last chunk of this CTA also arrives for the missing chunks of its group
     // the channel's format and zero point for the next tile are loaded one tile ahead
     int nf = 0, nz = 0;
-    if (static_cast<int>(blockIdx.x) < n_tiles) {
-      const int p0 = (a.tile0 + static_cast<int>(blockIdx.x) % n_ch) * 128 + r;
+    if (static_cast<int>(blockIdx.x) < n_units) {
+      const int p0 = (a.tile0 + (static_cast<int>(blockIdx.x) / ks) % n_ch) * 128 + r;
       nf = a.wfmt[p0];
       nz = a.wzero[p0];
     }
-    for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+    for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       const ChanDecode cd = chan_decode(nf, nz);
-      if (t + static_cast<int>(gridDim.x) < n_tiles) {
-        const int pn = (a.tile0 + (t + static_cast<int>(gridDim.x)) % n_ch) * 128 + r;
+      if (u + static_cast<int>(gridDim.x) < n_units) {
+        const int pn = (a.tile0 + ((u + static_cast<int>(gridDim.x)) / ks) % n_ch) * 128 + r;
         nf = a.wfmt[pn];
         nz = a.wzero[pn];
       }
-      for (int kc = 0; kc < nk; ++kc, ++it) {
+      const int kc1 = kc_end(u);
+      for (int kc = kc_begin(u); kc < kc1; ++kc, ++it) {
         if (static_cast<int>(it % kDecodeGroups) != grp) continue;
         const int s = it % S, sa = it % kAStages;
         const uint32_t ph = (it / S) & 1;
@@ -515,8 +524,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const float sa = a.act_scale != nullptr ? *a.act_scale : 1.f;
     uint32_t acc_it = 0;
-    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++acc_it) {
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++acc_it) {
       const int b = acc_it & 1;
+      const int t = u / ks;
       // per-channel constants first: their (dependent) loads overlap the wait for the accumulator
       const int p = (a.tile0 + t % n_ch) * 128 + r;
       const int tok0 = (t / n_ch) * BN;
@@ -530,17 +540,29 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       // y = acc * (s_a * s_w) + bias, rounded once to fp32, then (f16 / bf16 outputs) to the output
       // type; one instantiation per output type and scale granularity keeps each variant as lean
       // as the fp32 per-tensor one
+      // YT = kPartialOut (EPI = 6, split-K): the raw fp32 sums go to a.partial[u % ks][tok][p]
+      // and the reduction kernel applies scales, bias and the output type
       auto drain = [&](auto yt, auto grouped_tag) {
         constexpr int YT = decltype(yt)::value;
         constexpr bool GROUPED = decltype(grouped_tag)::value;
-        using OutT = std::conditional_t<YT == CHAM_Y_F32, float,
+        using OutT = std::conditional_t<YT == CHAM_Y_F32 || YT == kPartialOut, float,
                                         std::conditional_t<YT == CHAM_Y_F16, __half, __nv_bfloat16>>;
         OutT* yc = static_cast<OutT*>(a.Y) + (orig >= 0 ? orig : 0);
+        float* pc = a.partial + static_cast<size_t>(u % ks) * a.M * a.Np + p;
         // 16 token columns per tcgen05.ld; the load of the warp's next slice is in flight while
         // the current one is scaled and stored (a wait per load would serialise its latency)
         auto store16 = [&](const uint32_t (&v)[16], int j) {
           if (orig < 0) return;
           const int t0 = tok0 + j * 16;
+          if constexpr (YT == kPartialOut) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const int tok = t0 + i;
+              if (tok >= a.M) break;
+              pc[static_cast<size_t>(tok) * a.Np] = __uint_as_float(v[i]);
+            }
+            return;
+          }
           float sc = scale;
           int grp = 0, next = 0;
           if constexpr (GROUPED) {  // per-sample scales: the group advances at most a few times
@@ -607,8 +629,8 @@ static cudaError_t launch_bn(const CUtensorMap& map, const GemmArgs& a, int num_
     if (e != cudaSuccess) return e;
     configured_device = dev;
   }
-  const long tiles = static_cast<long>(a.n_ch_tiles) * ((a.M + BN - 1) / BN);
-  const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
+  const long units = static_cast<long>(a.n_ch_tiles) * ((a.M + BN - 1) / BN) * a.k_split;
+  const int grid = static_cast<int>(units < num_sms ? units : num_sms);
   return launch_pdl(k_gemm_ts_f16<BN, BITS, EPI, GW>, dim3(grid), dim3(kGemmThreads), C::kSmem, st, map, a);
 }
 
@@ -631,6 +653,13 @@ static cudaError_t launch_gw(const CUtensorMap& map, const GemmArgs& a, int num_
 
 // The launches of one output type YT: both weight widths, every token-tile size, per-tensor or
 // per-sample activation scales, per-channel or group-wise weights.
+// Split-K units: raw partial sums (EPI 6); the reduction applies scales, bias and output type.
+inline cudaError_t launch_gemm_partial(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn,
+                                       cudaStream_t st) {
+  if (a.bits == 8) return launch_gw<8, 2 * kPartialOut>(map, a, num_sms, bn, st);
+  return launch_gw<4, 2 * kPartialOut>(map, a, num_sms, bn, st);
+}
+
 template <int YT>
 cudaError_t launch_gemm_yt(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
   const bool per_sample = a.act_scale != nullptr && a.rows_per_group < a.M;

@@ -22,7 +22,7 @@ def test_withheld_chunk_times_out_and_context_survives():
     d = cl.pack_plan(W.shape[0], W.shape[1], fmt)
     blob, st = cl.pack_weights(cuda(W), cuda(fmt), d)
     Xd, bd = cuda(X), cuda(bias)
-    cl.debug_stall_next_gemm(3)
+    cl.debug_stall_next_gemm(1)   # CTA 0 owns at least two K-chunks, with or without split-K
     t0 = time.time()
     Y, st2 = cl.linear(Xd, d, blob, F.A_E4M3, bias=bd)
     torch.cuda.synchronize()
