@@ -501,17 +501,18 @@ def e2e_leg(args, torch, cl, host, layers, nb, lut, qp, device, stream, world, f
 
 
 # ------------------------------------------------------------------ the oracle as CPU baseline
-def oracle_sample(layers_idx=(4,), buckets=(0, 9)):
+def oracle_sample(layers_idx=(4,), buckets=(0, 5, 9)):
     """The oracle on a bounded sample of the workload: for each (layer, bucket) of the sample,
     per-channel selection over the W8 palette, the activation quantizer in the format the route
-    picks, and the fp64 GEMM over all rows.  Returns (flops, seconds, description)."""
+    picks with the static scale of the tensor's range (Alg. 1 -> Alg. 2), and the fp64 GEMM over
+    all rows, each stage timed.  Returns (flops, seconds, description, seconds per stage)."""
     from oracle import formats as F
     from oracle import gemm as G
     from oracle import schedule as S
     from oracle import select as SEL
     from paper_2609_33496_gb300 import workloads as WL
     snr = S.snr(S.betas_scaled_linear())
-    flops, t = 0.0, 0.0
+    flops, stages = 0.0, {"select": 0.0, "act_quant": 0.0, "gemm": 0.0}
     for li in layers_idx:
         name, M, K, N = WL.SDXL_PROJ_LAYERS[li]
         W, bias = WL.sdxl_layer_weights(li)
@@ -519,14 +520,20 @@ def oracle_sample(layers_idx=(4,), buckets=(0, 9)):
             X = WL.sdxl_layer_activation(li, bk)
             t0 = time.perf_counter()
             fmt, _, _ = SEL.select_formats(W, 0x007)
+            t1 = time.perf_counter()
             f = S.route(S.kurtosis(X), snr[int(S.bucket_midpoint(bk))])
-            x = X.astype(np.float32)          # Alg. 1's range on this sample, then Alg. 2's static scale
-            G.linear_reference(X, f, W, fmt, bias, float(x.min()), float(x.max()))
-            t += time.perf_counter() - t0
+            x = X.astype(np.float32)
+            a = F.act_dequant(F.act_quant(X, f, float(x.min()), float(x.max())))
+            t2 = time.perf_counter()
+            G.linear_output(a, SEL.dequant_selected(W, fmt), bias)
+            t3 = time.perf_counter()
+            stages["select"] += t1 - t0
+            stages["act_quant"] += t2 - t1
+            stages["gemm"] += t3 - t2
             flops += layer_flops(M, K, N)
-    desc = "oracle select(W8)+static act-quant+fp64 GEMM of layer(s) %s at buckets %s" % (
+    desc = "oracle select(W8)+static act-quant+fp64 GEMM of layer(s) %s at buckets %s, one BLAS thread" % (
         [WL.SDXL_PROJ_LAYERS[i][0] for i in layers_idx], list(buckets))
-    return flops, t, desc
+    return flops, sum(stages.values()), desc, stages
 
 
 def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=20):
@@ -660,13 +667,17 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
 def workload_variants(torch, cl, st, pk, probe, reps=20):
     """The other workloads' layer shapes, each selected (4-bit palette of its fork), packed,
     quantized and multiplied on the GPU; per shape the GEMM and the quantizer alone (reps
-    graph-captured launches between two events) with their roofline fractions.  SDXL-UNet W4A8
-    at a mid bucket (E4M3, dynamic scales); PixArt-alpha W4A8 with E5M2 and the DiT path's two
-    per-sample scales; SDXL-Turbo weight-only W4A16 rows (fp16 activations, no quantizer)."""
+    graph-captured launches between two events) with their roofline fractions (the f16 one, and
+    for 8-bit activations the FP8 one: max(flops / peak, bytes / HBM)).  SDXL-UNet W4A8: the 22
+    distinct shapes of one step, at a mid bucket (E4M3, dynamic scales); PixArt-alpha W4A8: the
+    5 distinct shapes of a block, E5M2 with the DiT path's two per-sample scales; SDXL-Turbo
+    weight-only W4A16 rows at batch 1 to 16 (fp16 activations, no quantizer).  Each workload also
+    gets its aggregate over its shapes (sum of flops over sum of GEMM times, one launch each)."""
     from paper_2609_33496_gb300 import workloads as WL
     dev = torch.device("cuda", torch.cuda.current_device())
     hbm = pk["hbm_gbs"] * 1e9
     p16 = (probe or {}).get("f16", pk.get("bf16_tflops", 1900.0)) * 1e12
+    p8 = (probe or {}).get("f8f6f4", 2 * p16 / 1e12) * 1e12
     palette = (1 << cl.W_INT4_SYM) | (1 << cl.W_INT4_ASYM) | (1 << cl.W_NF4) | (1 << cl.W_E2M1) | \
         (1 << cl.W_MXINT4) | (1 << cl.W_MXFP4)
 
@@ -684,10 +695,12 @@ def workload_variants(torch, cl, st, pk, probe, reps=20):
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / reps * 1e-3  # seconds per launch
 
-    out = []
-    for cfg, name, shapes, af, groups in ((3, "sdxl-unet W4A8", WL.UNET_W4A8_SHAPES, cl.A_E4M3, 1),
-                                          (4, "pixart-alpha W4A8", WL.PIXART_W4A8_SHAPES, cl.A_E5M2, 2),
-                                          (5, "sdxl-turbo W4A16", WL.TURBO_W4A16_SHAPES, cl.A_FP16, 1)):
+    turbo = tuple(shp for b in (1, 2, 4, 8, 16) for shp in WL.turbo_batch_shapes(b))
+    rows, summary = [], []
+    for cfg, name, shapes, af, groups in ((3, "sdxl-unet W4A8", WL.UNET_STEP_SHAPES, cl.A_E4M3, 1),
+                                          (4, "pixart-alpha W4A8", WL.PIXART_STEP_SHAPES, cl.A_E5M2, 2),
+                                          (5, "sdxl-turbo W4A16", turbo, cl.A_FP16, 1)):
+        tot_fl, tot_t, tot_q = 0.0, 0.0, 0.0
         for i, (M, K, N) in enumerate(shapes):
             X, W, bias = WL.config_layer(cfg, i, M, K, N)
             Xd, Wd, bd = (torch.from_numpy(v).to(dev) for v in (X, W, bias))
@@ -700,20 +713,25 @@ def workload_variants(torch, cl, st, pk, probe, reps=20):
             cl.linear_prepare_groups(Xd, af, g, ws, st)
             t = timed(lambda: cl.linear_gemm_ex(Xd, desc, blob, af, g, bd, Y, ws, st))
             fl = 2.0 * M * K * N
-            a_bytes = M * K * 2                       # the fp16 operand (or X itself)
-            byts = a_bytes + N * K / 2 + 9 * N + 4 * M * N
+            byts = M * K * (2 if af == cl.A_FP16 else 1) + N * K / 2 + 9 * N + 4 * M * N
             row = {"workload": name, "M": M, "K": K, "N": N, "act_fmt": af, "gemm_us": round(t * 1e6, 2),
                    "tflops": round(fl / t / 1e12, 1), "bound": "tensor" if fl / p16 >= byts / hbm else "hbm",
                    "frac_f16_roofline": round(max(fl / p16, byts / hbm) / t, 4)}
             if af != cl.A_FP16:
+                row["frac_fp8_roofline"] = round(max(fl / p8, byts / hbm) / t, 4)
                 tq = timed(lambda: cl.linear_prepare_groups(Xd, af, g, ws, st))
+                tot_q += tq
                 row.update({"quant_us": round(tq * 1e6, 2), "quant_gbs": round(4 * M * K / tq / 1e9, 1),
                             "quant_frac_hbm": round(4 * M * K / tq / hbm, 4)})
-            out.append(row)
+            rows.append(row)
+            tot_fl += fl
+            tot_t += t
             del Xd, Wd, bd, blob, ws, Y
+        summary.append({"workload": name, "shapes": len(shapes), "gemm_tflops": round(tot_fl / tot_t / 1e12, 1),
+                        "gemm_ms": round(tot_t * 1e3, 3), "quant_ms": round(tot_q * 1e3, 3)})
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
-    return out
+    return {"shapes": rows, "summary": summary}
 
 
 def tensor_probe(torch, device):
@@ -746,9 +764,11 @@ def tensor_probe(torch, device):
 
 
 def cpu_baseline():
-    flops, t, desc = oracle_sample()
+    # one core: the BLAS and OpenMP pools of this process are limited to one thread at start-up
+    flops, t, desc, stages = oracle_sample()
     return {"value": round(flops / t / 1e12, 6), "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
-            "sample": desc, "seconds": round(t, 2)}
+            "sample": desc, "seconds": round(t, 2), "stage_seconds": {k: round(v, 3) for k, v in stages.items()},
+            "host_cores": os.cpu_count()}
 
 
 def reference_arm(args, world):
@@ -757,7 +777,7 @@ def reference_arm(args, world):
     flops, t = 0.0, 0.0
     desc = ""
     for _ in range(args.steps):
-        f, s, desc = oracle_sample(buckets=(9,))
+        f, s, desc, _ = oracle_sample(buckets=(9,))
         flops += f
         t += s
     value = flops / t / 1e12

@@ -27,11 +27,17 @@ def linear_reference(X, act_fmt, W, wfmt, bias=None, lo=None, hi=None):
     else:
         a = F.act_dequant(F.act_quant(X, act_fmt, lo, hi))
     w = dequant_selected(W, np.asarray(wfmt))
-    y = a @ w.T
-    if bias is not None:
-        y = y + np.asarray(bias, dtype=np.float64)[None, :]
+    y = linear_output(a, w, bias)
     bound = TOL_REL * (np.abs(a) @ np.abs(w).T)
     return y, bound, a, w
+
+
+def linear_output(a_dq, w_dq, bias=None):
+    """Y = A W^T (+ bias) in fp64 on the dequantized operands (Sec. 3.6)."""
+    y = np.asarray(a_dq, dtype=np.float64) @ np.asarray(w_dq, dtype=np.float64).T
+    if bias is not None:
+        y = y + np.asarray(bias, dtype=np.float64)[None, :]
+    return y
 
 
 def linear_rows_reference(a_dq, w_dq, rows, bias=None):

@@ -101,6 +101,26 @@ UNET_W4A8_SHAPES = ((2, 320, 1280), (154, 2048, 1280), (2048, 5120, 1280), (8192
                     (32768, 960, 320))
 PIXART_W4A8_SHAPES = ((240, 1152, 1152), (8192, 1152, 4608), (8192, 4608, 1152), (240, 4096, 1152))
 TURBO_W4A16_SHAPES = ((1, 320, 1280), (16, 1280, 1280), (616, 2048, 640), (8192, 640, 640))
+# The 22 distinct (M, K, N) of the linear and 1x1-conv GEMMs of one SDXL-architecture UNet step at
+# 1024^2 (latent 128^2, batch 2): time embedding and its projections (M = 2), text cross-attention
+# K/V (M = 154), and the 32^2 / 64^2 / 128^2 stages (M = 2048 / 8192 / 32768).
+UNET_STEP_SHAPES = ((2, 320, 1280), (2, 1280, 320), (2, 1280, 640), (2, 1280, 1280), (2, 2816, 1280),
+                    (154, 2048, 640), (154, 2048, 1280), (2048, 640, 1280), (2048, 1280, 1280),
+                    (2048, 1920, 1280), (2048, 2560, 1280), (2048, 5120, 1280), (2048, 1280, 10240),
+                    (8192, 320, 640), (8192, 640, 640), (8192, 960, 640), (8192, 1280, 640),
+                    (8192, 1920, 640), (8192, 2560, 640), (8192, 640, 5120), (32768, 640, 320),
+                    (32768, 960, 320))
+# The distinct GEMMs of one PixArt-alpha XL/2 block at 1024^2, batch 2 (4096 tokens, 120 caption
+# tokens per sample): self q/k/v/out and cross q/out, cross k/v, MLP fc1 and fc2, and the caption
+# projection.
+PIXART_STEP_SHAPES = ((8192, 1152, 1152), (240, 1152, 1152), (8192, 1152, 4608), (8192, 4608, 1152),
+                      (240, 4096, 1152))
+
+
+def turbo_batch_shapes(b):
+    """SDXL-Turbo weight-only rows at batch b (512^2, one step): the time-embedding projection
+    (M = b), text cross-attention K/V (M = 77 b) and a 32^2-stage projection (M = 1024 b)."""
+    return ((b, 320, 1280), (77 * b, 2048, 1280), (1024 * b, 1280, 1280))
 
 
 def config_layer(config, index, M, K, N, nu=7):
