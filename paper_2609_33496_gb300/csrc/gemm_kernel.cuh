@@ -34,8 +34,12 @@
 namespace cham {
 
 constexpr int kBK = 64;  // K elements per stage: 128 bytes of fp16 per activation row
-constexpr int kDecodeGroups = 2;  // decode warpgroups, taking alternate K-chunks
-constexpr int kEpiGroups = 2;     // epilogue warpgroups, taking alternate 16-column slices
+// decode warpgroups (taking K-chunks in turn) and epilogue warpgroups (taking alternate 16-column
+// slices): the 4-bit decode (NF4 tables) is about three times the 8-bit one per chunk
+template <int BITS> struct Roles {
+  static constexpr int kDec = BITS == 4 ? 3 : 2, kEpi = BITS == 4 ? 1 : 2;
+};
+constexpr int kDecodeGroups = 2, kEpiGroups = 2;  // the 8-bit split; the thread count is the same
 constexpr int kPartialOut = 3;    // epilogue "output type" of split-K units: raw fp32 partial sums
 constexpr int kGemmThreads = 128 * (1 + kDecodeGroups + kEpiGroups);
 
@@ -339,7 +343,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     for (int g = 0; g < kAGroups; ++g) mbar_init(&afull[g], 4 * kGroup);  // one elected lane per warp and chunk
     for (int b = 0; b < 2; ++b) {
       mbar_init(&accfull[b], 1);
-      mbar_init(&accempty[b], 4 * kEpiGroups);  // one elected lane per epilogue warp
+      mbar_init(&accempty[b], 4 * Roles<BITS>::kEpi);  // one elected lane per epilogue warp
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -431,7 +435,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       // all issued MMAs have finished before tensor memory is released
       if (acc_it > 0) drain_wait(&accfull[(acc_it - 1) & 1], ((acc_it - 1) >> 1) & 1);
     }
-  } else if (warp >= 4 && warp < 4 + 4 * kDecodeGroups) {
+  } else if (warp >= 4 && warp < 4 + 4 * Roles<BITS>::kDec) {
     // ---------------- weight decode: one channel per thread; group g takes chunks it % G == g
     const int q = warp & 3;  // tensor-memory lane quadrant of this warp (warp % 4)
     const int grp = (warp - 4) >> 2;
@@ -456,7 +460,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
       const int kc1 = kc_end(u);
       for (int kc = kc_begin(u); kc < kc1; ++kc, ++it) {
-        if (static_cast<int>(it % kDecodeGroups) != grp) continue;
+        if (static_cast<int>(it % Roles<BITS>::kDec) != grp) continue;
         const int s = it % S, sa = it % kAStages;
         const uint32_t ph = (it / S) & 1;
         // decode as soon as the codes have landed; the tensor-memory slot (its previous chunk,
@@ -515,11 +519,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
       }
     }
-  } else if (warp >= 4 + 4 * kDecodeGroups) {
+  } else if (warp >= 4 + 4 * Roles<BITS>::kDec) {
     // ---------------- epilogue: drain one accumulator buffer per tile; warpgroup h takes the
     // 16-column slices j = h, h + kEpiGroups, ...
     const int q = warp & 3;
-    const int h = (warp - (4 + 4 * kDecodeGroups)) >> 2;
+    const int h = (warp - (4 + 4 * Roles<BITS>::kDec)) >> 2;
     const int r = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const float sa = a.act_scale != nullptr ? *a.act_scale : 1.f;
@@ -587,7 +591,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             else yc[static_cast<size_t>(tok) * a.N] = __float2bfloat16_rn(y);
           }
         };
-        constexpr int kLoads = BN / 16, kE = kEpiGroups;
+        constexpr int kLoads = BN / 16, kE = Roles<BITS>::kEpi;
         uint32_t va[16], vb[16];
         if (h < kLoads) {
           tmem_ld_32x32b_x16(d_tmem + h * 16, va);
