@@ -306,6 +306,12 @@ cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const 
 
 /* ------------------------------------------------------------------ a7/a8: quantized linear */
 
+/* Workspace (device) of the linear calls for M rows of the layer *desc in act_fmt: the activation
+ * scales of up to CHAM_MAX_GROUPS row groups, the quantizer's range partials, the exact fp16
+ * operand (M x K; none for CHAM_A_FP16) and, when the GEMM splits K -- a layer whose 128-channel
+ * x token tiles are fewer than half the SMs and whose K spans at least 8 chunks of 64 -- the fp32
+ * partial sums of the K ranges, which a second kernel adds in order.  The size depends on the
+ * current device's SM count. */
 cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* desc, int act_fmt,
                                             size_t* ws_bytes);
 
