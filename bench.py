@@ -369,6 +369,7 @@ def main():
                    "layers": len(layers), "buckets": nb, "global_batch": 2 * world,
                    "tokens": [M for (_, M, _, _) in layers], "weight_palette": "W8 {INT8-sym, INT8-asym, MXINT8}",
                    "activation_formats_used": sorted(set(int(v) for v in lut.ravel())),
+                   "lut": [[int(v) for v in row] for row in lut],   # F[layer][bucket] from Alg. 1's route
                    "step": "fused select+pack of 10 layers, then 10 buckets x 10 layers of act-quant (%s) + GEMM, one "
                            "CUDA graph" % ("dynamic per-tensor scales, Alg. 3" if args.dynamic_scales else
                                            "static calibrated per-(layer, bucket) scales, Alg. 2"),
@@ -701,11 +702,15 @@ def workload_variants(torch, cl, st, pk, probe, reps=20):
                                           (4, "pixart-alpha W4A8", WL.PIXART_STEP_SHAPES, cl.A_E5M2, 2),
                                           (5, "sdxl-turbo W4A16", turbo, cl.A_FP16, 1)):
         tot_fl, tot_t, tot_q = 0.0, 0.0, 0.0
+        hist = {}
         for i, (M, K, N) in enumerate(shapes):
             X, W, bias = WL.config_layer(cfg, i, M, K, N)
             Xd, Wd, bd = (torch.from_numpy(v).to(dev) for v in (X, W, bias))
             fmt, _ = cl.select_weight_formats(Wd, palette)
-            desc = cl.pack_plan(N, K, fmt.cpu().numpy())
+            fmt_h = fmt.cpu().numpy()
+            for f, c in zip(*np.unique(fmt_h, return_counts=True)):
+                hist[int(f)] = hist.get(int(f), 0) + int(c)
+            desc = cl.pack_plan(N, K, fmt_h)
             blob, _ = cl.pack_weights(Wd, fmt, desc, dev_status=st)
             ws = torch.empty(cl.linear_workspace_size(M, desc, af), dtype=torch.uint8, device=dev)
             Y = torch.empty((M, N), dtype=torch.float32, device=dev)
@@ -728,7 +733,8 @@ def workload_variants(torch, cl, st, pk, probe, reps=20):
             tot_t += t
             del Xd, Wd, bd, blob, ws, Y
         summary.append({"workload": name, "shapes": len(shapes), "gemm_tflops": round(tot_fl / tot_t / 1e12, 1),
-                        "gemm_ms": round(tot_t * 1e3, 3), "quant_ms": round(tot_q * 1e3, 3)})
+                        "gemm_ms": round(tot_t * 1e3, 3), "quant_ms": round(tot_q * 1e3, 3),
+                        "weight_formats": dict(sorted(hist.items()))})
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
     return {"shapes": rows, "summary": summary}
