@@ -359,6 +359,7 @@ def main():
     variants = None if args.no_variants else variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe)
     if variants is not None:
         variants["workloads"] = workload_variants(torch, cl, st, pk, probe)
+        variants["dit_sampler"] = dit_sampler(torch, cl, st)
 
     result = {
         "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world, "steps": K_,
@@ -738,6 +739,71 @@ def workload_variants(torch, cl, st, pk, probe, reps=20):
     torch.cuda.synchronize()
     assert int(st.item()) == 0, "device status %d" % int(st.item())
     return {"shapes": rows, "summary": summary}
+
+
+def dit_sampler(torch, cl, st, steps=20):
+    """The DiT path end to end on the 5 GEMMs of a PixArt-alpha block: per linear, input-channel
+    energies from the calibration activations of all 10 buckets (GPU), the (g, f) search over
+    {32, ..., 288} x {INT4-asym, NF4, E2M1} scored by the input-aware SQNR, the group-wise pack;
+    per (layer, bucket) the format the route picks from kappa and SNR on the linear schedule
+    (the LUT of Alg. 1); then a 20-step sampler (t_i = 999 - 50 i) in which every step quantizes
+    each layer's input with the two samples' own scales (Alg. 3 per sample) in F[l, b(t)] and
+    multiplies (fp32 outputs).  The 20 steps are one CUDA graph, timed after a warm replay."""
+    from paper_2609_33496_gb300 import workloads as WL
+    dev = torch.device("cuda", torch.cuda.current_device())
+    snr = cl.snr(cl.SCHEDULE_LINEAR, 1000)
+    palette = (1 << cl.W_INT4_ASYM) | (1 << cl.W_NF4) | (1 << cl.W_E2M1)
+    gmask = cl.group_mask(cl.GROUP_SIZES)
+    cands = cl.group_candidates(palette, gmask)
+    layers = []
+    for li, (M, K, N) in enumerate(WL.PIXART_STEP_SHAPES):
+        W, bias = WL.pixart_layer_weights(li)
+        Wd, bd = torch.from_numpy(W).to(dev), torch.from_numpy(bias).to(dev)
+        Xs = [torch.from_numpy(WL.pixart_layer_activation(li, b)).to(dev) for b in range(10)]
+        energy = torch.zeros(K, dtype=torch.float64, device=dev)
+        lut = []
+        for b, X in enumerate(Xs):
+            cl.act_channel_energy(X, energy=energy)
+            sums = cl.act_moments(X).cpu().numpy()
+            lut.append(cl.route(cl.kurtosis(sums[:5]), snr[b * 100 + 50], False))
+        g, f = cands[cl.candidate_argmin(cl.select_weight_groups(Wd, palette, gmask, energy=energy).cpu().numpy())]
+        desc = cl.pack_plan_grouped(N, K, f, g)
+        blob, _ = cl.pack_weights(Wd, torch.full((N,), f, dtype=torch.uint8, device=dev), desc, dev_status=st)
+        ws = torch.empty(max(cl.linear_workspace_size(M, desc, a) for a in range(6)), dtype=torch.uint8, device=dev)
+        Y = torch.empty((M, N), dtype=torch.float32, device=dev)
+        layers.append({"Xs": Xs, "desc": desc, "blob": blob, "bias": bd, "ws": ws, "Y": Y, "lut": lut,
+                       "g": g, "f": f, "M": M, "K": K, "N": N})
+    ts = [999 - 50 * i for i in range(steps)]
+
+    def run():
+        for t in ts:
+            b = cl.bucket(t)
+            for L in layers:
+                af = int(L["lut"][b])
+                X = L["Xs"][b]
+                cl.linear_prepare_groups(X, af, 2, L["ws"], st)
+                cl.linear_gemm_ex(X, L["desc"], L["blob"], af, 2, L["bias"], L["Y"], L["ws"], st)
+
+    run()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        run()
+    g.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    g.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0, "device status %d" % int(st.item())
+    ms = e0.elapsed_time(e1)
+    flops = steps * sum(2.0 * L["M"] * L["K"] * L["N"] for L in layers)
+    used = sorted(set(int(L["lut"][cl.bucket(t)]) for t in ts for L in layers))
+    return {"steps": steps, "ms": round(ms, 3), "tflops": round(flops / (ms * 1e-3) / 1e12, 1),
+            "weights_g_f": [[L["g"], L["f"]] for L in layers], "lut": [[int(v) for v in L["lut"]] for L in layers],
+            "activation_formats_used": used,
+            "shapes": [[L["M"], L["K"], L["N"]] for L in layers]}
 
 
 def tensor_probe(torch, device):

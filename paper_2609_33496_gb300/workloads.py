@@ -117,6 +117,21 @@ PIXART_STEP_SHAPES = ((8192, 1152, 1152), (240, 1152, 1152), (8192, 1152, 4608),
                       (240, 4096, 1152))
 
 
+def pixart_layer_activation(index, bucket):
+    """Input of PixArt-alpha block GEMM `index` (PIXART_STEP_SHAPES) at timestep bucket `bucket`:
+    StudentT(nu_b) * c_k as for the SDXL projections, the two samples of the batch drawn together."""
+    M, K, N = PIXART_STEP_SHAPES[index]
+    c = channel_jitter(rng(4, 100 + index), K)
+    g = rng(4, 200 + 10 * index + bucket)
+    return to_fp16(student_t(g, NU_SCHEDULE[bucket], (M, K)) * c[None, :])
+
+
+def pixart_layer_weights(index):
+    M, K, N = PIXART_STEP_SHAPES[index]
+    g = rng(4, 300 + index)
+    return weight_mix(g, N, K), g.normal(0.0, 0.02, N).astype(np.float32)
+
+
 def turbo_batch_shapes(b):
     """SDXL-Turbo weight-only rows at batch b (512^2, one step): the time-embedding projection
     (M = b), text cross-attention K/V (M = 77 b) and a 32^2-stage projection (M = 1024 b)."""
