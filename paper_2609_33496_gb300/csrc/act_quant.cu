@@ -532,8 +532,13 @@ int group_grid(int64_t nvec, int n_groups, int num_sms) {
 template <int FMT, bool CODES, bool DEQ>
 static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
   if (a.use_static) {
-    launch_pdl(k_act_encode_static<FMT, CODES, DEQ>, dim3(range_grid(a.nvec, a.num_sms)), dim3(256), 0, st, a.X,
-               a.nvec, a.stat, a.codes, a.deq, a.params, a.scale_out, a.dev_status);
+    // one pass: enough CTAs that every thread's kUnroll loads cover the tensor (up to 8 resident
+    // CTAs per SM), so no thread needs a second DRAM round trip for a tail
+    const int64_t want = (a.nvec + 256 * kUnroll - 1) / (256 * kUnroll);
+    const int64_t cap = static_cast<int64_t>(a.num_sms) * 8;
+    const int g = static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
+    launch_pdl(k_act_encode_static<FMT, CODES, DEQ>, dim3(g), dim3(256), 0, st, a.X, a.nvec, a.stat, a.codes,
+               a.deq, a.params, a.scale_out, a.dev_status);
     return;
   }
   // per-sample groups: each group's range and encode grids are the per-tensor ones split evenly
