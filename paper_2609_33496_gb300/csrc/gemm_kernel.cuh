@@ -567,6 +567,29 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
             return;
           }
+          if (t0 + 16 <= a.M) {
+            // a full slice inside one row group (always, for a per-tensor scale): no bounds or
+            // group checks, one running pointer
+            float s16 = scale;
+            bool one = true;
+            if constexpr (GROUPED) {
+              const int g0 = t0 / a.rows_per_group;
+              one = (t0 + 15) / a.rows_per_group == g0;
+              if (one) s16 = __fmul_rn(a.act_scale[g0], ws);
+            }
+            if (one) {
+              OutT* yp = yc + static_cast<size_t>(t0) * a.N;
+              const size_t stride = static_cast<size_t>(a.N);
+#pragma unroll
+              for (int i = 0; i < 16; ++i, yp += stride) {
+                const float y = fmaf(__uint_as_float(v[i]), s16, bv);
+                if constexpr (YT == CHAM_Y_F32) *yp = y;
+                else if constexpr (YT == CHAM_Y_F16) *yp = __float2half_rn(y);
+                else *yp = __float2bfloat16_rn(y);
+              }
+              return;
+            }
+          }
           float sc = scale;
           int grp = 0, next = 0;
           if constexpr (GROUPED) {  // per-sample scales: the group advances at most a few times
