@@ -224,3 +224,29 @@ def test_select_pack_palette_argument_checks(cl):
 
 def test_check_rejects_a_null_status_word(cl):
     assert cl.lib().chameleon_check(None, None) == cl.ERR_INVALID_ARG
+
+
+def test_linear_workspace_includes_split_k_partials(cl):
+    """The GEMM splits K when its 128-channel x token tiles are fewer than half the SMs and K has at
+    least 8 chunks of 64; the workspace then adds k_split x M x Np fp32 partial sums.  Without a
+    device the library assumes 148 SMs."""
+    sms = 148
+
+    def bn(M):
+        return next(b for b in (16, 32, 64, 128) if M <= b) if M <= 128 else 192
+
+    def expected_extra(M, N, K):
+        tiles = -(-N // 128) * -(-M // bn(M))
+        nk = -(-K // 64)
+        if tiles * 2 > sms or nk < 8:
+            return 0
+        ks = max(1, min(sms // tiles, nk // 2))
+        return -(-(ks * M * 128 * -(-N // 128) * 4) // 256) * 256
+
+    for M, K, N in [(16, 1280, 1280), (154, 2048, 1280), (240, 4096, 1152), (2, 320, 1280), (2048, 1280, 10240),
+                    (8192, 640, 640), (1, 512, 128)]:
+        d = cl.pack_plan(N, K, np.full(N, F.W_INT8_SYM, np.uint8))
+        base = cl.linear_workspace_size(M, d, F.A_FP16)          # FP16: 256 bytes before any partials
+        assert base - 256 == expected_extra(M, N, K), (M, K, N)
+        q = cl.linear_workspace_size(M, d, F.A_E4M3)
+        assert q - (base - 256) >= 2 * M * K                      # the fp16 operand precedes the partials
