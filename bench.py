@@ -255,7 +255,6 @@ def main():
 
     flops_step = nb * sum(layer_flops(M, K, N) for (_, M, K, N) in layers)
     quant_bytes_step = 0.0
-    gemm_bytes_step = 0.0
 
     def run_step(parts="wqg"):
         """a5 + a6 for every layer ("w"), then a2-a4 + a7 for every (bucket, layer): act-quant in
@@ -305,11 +304,10 @@ def main():
     # per linear 1 quantizer kernel (static scales or MX; 2 with dynamic per-tensor scales) + 1 GEMM
     launches = len(layers) + sum(
         (2 if args.dynamic_scales and lut[li, bk] <= 2 else 1) + 1 for li in range(len(layers)) for bk in range(nb))
+    # the quantizer's algorithmic bytes: X read, the exact fp16 operand written (MX formats fold
+    # the block exponent into the operand, so no E8M0 bytes are written on this path)
     for li, (_, M, K, N) in enumerate(layers):
-        for bk in range(nb):
-            mx = lut[li, bk] >= 3
-            quant_bytes_step += M * K * 2 + M * K * 2 + (M * K / 32 if mx else 0)
-            gemm_bytes_step += M * K * 1 + N * K * 1 + N * (4 + 1) + 4 * N + M * N * 4
+        quant_bytes_step += nb * (M * K * 2 + M * K * 2)
     # ---------------------------------------------------------------- timed region (device)
     if world > 1:
         dist.barrier()
@@ -395,7 +393,7 @@ def main():
         "weights_select_pack_ms_per_step": round(weights_ms / K_, 4),
         "act_quant": {"achieved_gbs": round(quant_gbs, 1), "peak_gbs": pk["hbm_gbs"],
                       "frac": round(quant_gbs / pk["hbm_gbs"], 4), "ms_per_step": round(quant_ms / K_, 4),
-                      "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"},
+                      "bytes": "2 B read + 2 B fp16 operand write per element"},
         "variants": variants,
         "calibration": route_vs_argmin(cl, lut, cal_sse),
         "gpu_launches": launches * K_,
@@ -609,12 +607,12 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
                 xf = x.float()
                 p_af = cl.scale_zp(af, float(xf.min()), float(xf.max())) if af <= 2 else None
                 tqs = timed(lambda: cl.linear_prepare_static(x, af, p_af, ws, st))
-                qb = 4 * M * K + (M * K / 32 if af in (3, 4) else 0)
+                qb = 4 * M * K
                 out["quant"].append({"act_fmt": af, "us": round(tq * 1e3, 2), "static_us": round(tqs * 1e3, 2),
                                      "gbs": round(qb / (tq * 1e-3) / 1e9, 1),
                                      "static_gbs": round(qb / (tqs * 1e-3) / 1e9, 1),
                                      "frac_hbm": round(qb / (tq * 1e-3) / hbm, 4),
-                                     "bytes": "2 B read + 2 B fp16 operand write per element (+1/32 B MX)"})
+                                     "bytes": "2 B read + 2 B fp16 operand write per element"})
     # output type and scale granularity of the epilogue on the largest layer and on the first
     # layer with a large fp32 output (8192 x 640 x 640): f32 / f16 / bf16 Y, one tensor scale or
     # two per-sample scales (the DiT path's), E4M3 activations, W8 weights
