@@ -140,6 +140,16 @@ def lib():
     return L
 
 
+def status_string(status):
+    """The library's name for a status code."""
+    return lib().chameleon_status_string(status).decode()
+
+
+def version():
+    """The library's ABI version (2: descriptors with group-wise weights)."""
+    return lib().chameleon_version()
+
+
 def check(status):
     if status != OK:
         raise ChameleonError(status, lib().chameleon_last_error_detail().decode())

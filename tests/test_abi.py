@@ -250,3 +250,8 @@ def test_linear_workspace_includes_split_k_partials(cl):
         assert base - 256 == expected_extra(M, N, K), (M, K, N)
         q = cl.linear_workspace_size(M, d, F.A_E4M3)
         assert q - (base - 256) >= 2 * M * K                      # the fp16 operand precedes the partials
+
+
+def test_version_and_status_names(cl):
+    assert cl.version() == 2
+    assert cl.status_string(cl.OK) and cl.status_string(cl.ERR_TIMEOUT) != cl.status_string(cl.OK)
