@@ -119,27 +119,34 @@ CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const
   const int nvec = K / 8;
   const ChanStats st = row_stats(row, nvec, lane);
   const int iters = (nvec + 31) / 32;  // same trip count in every lane (shuffles)
-  int best = -1;
-  double best_e = 0.0;
-  for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
-    if (!((mask >> f) & 1u)) {
-      if (lane == 0 && sse_row != nullptr) sse_row[f] = INFINITY;
-      continue;
-    }
-    Sum2 acc{0.f, 0.f};
-    if (w_is_mx(f)) {
-      for (int it = 0; it < iters; ++it) {
-        const int v = it * 32 + lane;
-        float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        if (v < nvec) load8(row, v, x);
-        float am = 0.f;
+  const bool any_mx = (mask & ((1u << CHAM_W_MXINT8) | (1u << CHAM_W_MXINT4) | (1u << CHAM_W_MXFP4))) != 0u;
+  // one pass over the row for every palette member: each vector is loaded once and the members'
+  // round trips are independent work for the scheduler
+  ChanScale cs[CHAM_W_NFORMATS];
+  Sum2 acc[CHAM_W_NFORMATS];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
-        am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 1));  // 4 lanes = one 32-element block
-        am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 2));
-        const int X = mx_exponent(f, am);
-        if (v < nvec) {
-          float e2[8];
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
+    cs[f] = (((mask >> f) & 1u) && !w_is_mx(f)) ? chan_scale(f, st) : ChanScale{1.f, 1.f, 0};
+    acc[f] = Sum2{0.f, 0.f};
+  }
+  for (int it = 0; it < iters; ++it) {
+    const int v = it * 32 + lane;
+    float x[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    if (v < nvec) load8(row, v, x);
+    float am = 0.f;
+    if (any_mx) {  // the palette is the same in every lane: all of them take the shuffles
+#pragma unroll
+      for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(x[i]));
+      am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 1));  // 4 lanes = one 32-element block
+      am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, 2));
+    }
+    if (v < nvec) {
+#pragma unroll
+      for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
+        if (!((mask >> f) & 1u)) continue;
+        float e2[8];
+        if (w_is_mx(f)) {
+          const int X = mx_exponent(f, am);
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             float dq;
@@ -147,24 +154,27 @@ CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const
             const float e = __fsub_rn(x[i], dq);
             e2[i] = __fmul_rn(e, e);
           }
-          sum2_add(acc, sum8(e2));
-        }
-      }
-    } else {
-      const ChanScale cs = chan_scale(f, st);
-      for (int v = lane; v < nvec; v += 32) {
-        float x[8], e2[8];
-        load8(row, v, x);
+        } else {
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          float err;
-          encode_chan(f, x[i], cs, nf4, &err);
-          e2[i] = __fmul_rn(err, err);
+          for (int i = 0; i < 8; ++i) {
+            float err;
+            encode_chan(f, x[i], cs[f], nf4, &err);
+            e2[i] = __fmul_rn(err, err);
+          }
         }
-        sum2_add(acc, sum8(e2));
+        sum2_add(acc[f], sum8(e2));
       }
     }
-    const double tot = warp_sum2(acc);
+  }
+  int best = -1;
+  double best_e = 0.0;
+#pragma unroll
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f) {
+    if (!((mask >> f) & 1u)) {
+      if (lane == 0 && sse_row != nullptr) sse_row[f] = INFINITY;
+      continue;
+    }
+    const double tot = warp_sum2(acc[f]);
     if (best < 0 || tot < best_e) {  // palette order: the earlier member wins a tie
       best = f;
       best_e = tot;
