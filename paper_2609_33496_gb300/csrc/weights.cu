@@ -115,9 +115,11 @@ CHAM_DEV double warp_sum2(Sum2 v) {
 
 // The selection of one channel (one warp): the first format of the palette with the least
 // SSE; sse_row (9 slots, +inf for non-members) may be null.  Every lane returns the result.
-CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const NF4Table& nf4, double* sse_row) {
+CHAM_DEV int select_row(const __half* row, int K, uint32_t mask, int lane, const NF4Table& nf4, double* sse_row,
+                        ChanStats* st_out = nullptr) {
   const int nvec = K / 8;
   const ChanStats st = row_stats(row, nvec, lane);
+  if (st_out != nullptr) *st_out = st;
   const int iters = (nvec + 31) / 32;  // same trip count in every lane (shuffles)
   const bool any_mx = (mask & ((1u << CHAM_W_MXINT8) | (1u << CHAM_W_MXINT4) | (1u << CHAM_W_MXFP4))) != 0u;
   // one pass over the row for every palette member: each vector is loaded once and the members'
@@ -342,7 +344,8 @@ CHAM_DEV float code_value(int f, int code, int z, const NF4Table& nf4) {
 }
 
 // Encodes packed slot p holding original channel c (-1: padding) in format f (one warp).
-CHAM_DEV void pack_slot(const PackArgs& a, int p, int c, int f, int lane, const NF4Table& nf4, GroupParam* s_gp_warp) {
+CHAM_DEV void pack_slot(const PackArgs& a, int p, int c, int f, int lane, const NF4Table& nf4, GroupParam* s_gp_warp,
+                        const ChanStats* pre = nullptr) {
   const int nvec_p = a.Kp / 8;
   const int tile = p >> 7, r = p & 127;
   if (c < 0) {  // padding slot: zero codes, unit scale
@@ -400,7 +403,7 @@ CHAM_DEV void pack_slot(const PackArgs& a, int p, int c, int f, int lane, const 
     }
     return;
   }
-  const ChanStats st = row_stats(row, nvec, lane);
+  const ChanStats st = pre != nullptr ? *pre : row_stats(row, nvec, lane);  // the selection's, when fused
   const ChanScale cs = chan_scale(f, st);
   const bool mx = w_is_mx(f);
   const int iters = (nvec_p + 31) / 32;
@@ -490,13 +493,14 @@ __global__ void __launch_bounds__(kWThreads) k_w_select_pack(PackArgs a, uint32_
   const int rank = p - a.cls_base[a.one_class];
   const int c = (rank >= 0 && rank < a.cls_count[a.one_class]) ? rank : -1;
   int f = -1;
-  if (c >= 0) f = select_row(a.W + static_cast<size_t>(c) * a.K, a.K, mask, lane, nf4, nullptr);
+  ChanStats st{0.f, 0.f, 0.f};
+  if (c >= 0) f = select_row(a.W + static_cast<size_t>(c) * a.K, a.K, mask, lane, nf4, nullptr, &st);
   if (lane == 0) {
     if (c >= 0) a.fmt_out[c] = static_cast<uint8_t>(f);
     a.perm[p] = c;
     a.fmtp[p] = c >= 0 ? static_cast<uint8_t>(f) : static_cast<uint8_t>(0xFF);
   }
-  pack_slot(a, p, c, f, lane, nf4, nullptr);
+  pack_slot(a, p, c, f, lane, nf4, nullptr, &st);
 }
 
 void launch_select_pack(const PackArgs& a, uint32_t mask, const NF4Table& nf4, cudaStream_t st) {
