@@ -255,3 +255,58 @@ def test_linear_workspace_includes_split_k_partials(cl):
 def test_version_and_status_names(cl):
     assert cl.version() == 2
     assert cl.status_string(cl.OK) and cl.status_string(cl.ERR_TIMEOUT) != cl.status_string(cl.OK)
+
+
+@pytest.mark.parametrize("bad", [0, -1, -32])
+def test_empty_and_negative_sizes_are_rejected_on_the_host(cl, bad):
+    """Every entry point that takes a size rejects an empty (0) or negative M, N, K or count with
+    CHAM_ERR_INVALID_ARG before touching the device (no GPU is present here)."""
+    L = cl.lib()
+    buf = ctypes.create_string_buffer(1 << 16)
+    x = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
+    n = ctypes.c_size_t(0)
+    d = cl.WPackDesc()
+    good = cl.pack_plan(64, 64, np.zeros(64, np.uint8))
+    p = cl.scale_zp(F.A_E4M3, -1.0, 1.0)
+    calls = {
+        "act_moments": lambda: L.chameleon_act_moments(x, bad, x, x, 1 << 15, None),
+        "act_quant_size": lambda: L.chameleon_act_quant_size(bad, 64, 1, ctypes.byref(n), ctypes.byref(n)),
+        "act_quant_size K": lambda: L.chameleon_act_quant_size(16, bad, 1, ctypes.byref(n), ctypes.byref(n)),
+        "act_quant": lambda: L.chameleon_act_quant(x, bad, 64, 1, x, 1 << 15, x, 1 << 15, x, None),
+        "act_quant K": lambda: L.chameleon_act_quant(x, 16, bad, 1, x, 1 << 15, x, 1 << 15, x, None),
+        "act_quant_noalloc": lambda: L.chameleon_act_quant_noalloc(x, bad, 64, 1, x, 1 << 15, x, None),
+        "act_quant_static": lambda: L.chameleon_act_quant_static(x, bad, 64, 1, ctypes.byref(p), x, 1 << 15, x,
+                                                                 None),
+        "act_format_sse_workspace_size": lambda: L.chameleon_act_format_sse_workspace_size(bad, 64,
+                                                                                            ctypes.byref(n)),
+        "act_format_sse": lambda: L.chameleon_act_format_sse(x, 16, bad, x, x, 1 << 15, x, None),
+        "act_channel_energy": lambda: L.chameleon_act_channel_energy(x, bad, 64, x, None),
+        "select_weight_formats": lambda: L.chameleon_select_weight_formats(x, bad, 64, cl.PALETTE_W8, x, None,
+                                                                           None),
+        "select_weight_formats K": lambda: L.chameleon_select_weight_formats(x, 16, bad, cl.PALETTE_W8, x,
+                                                                             None, None),
+        "select_weight_groups_workspace_size": lambda: L.chameleon_select_weight_groups_workspace_size(
+            bad, 64, 1 << F.W_NF4, 1, ctypes.byref(n)),
+        "select_weight_groups": lambda: L.chameleon_select_weight_groups(x, 16, bad, 1 << F.W_NF4, 1, None, x,
+                                                                         x, 1 << 15, None),
+        "select_pack_palette": lambda: L.chameleon_select_pack_palette(x, bad, 64, cl.PALETTE_W8,
+                                                                       ctypes.byref(d), x, x, 1 << 15, x, None),
+        "pack_plan": lambda: L.chameleon_pack_plan(bad, 64, x, ctypes.byref(d)),
+        "pack_plan K": lambda: L.chameleon_pack_plan(16, bad, x, ctypes.byref(d)),
+        "pack_plan_palette": lambda: L.chameleon_pack_plan_palette(bad, 64, cl.PALETTE_W8, ctypes.byref(d)),
+        "pack_plan_grouped": lambda: L.chameleon_pack_plan_grouped(16, bad, F.W_NF4, 32, ctypes.byref(d)),
+        "linear_workspace_size": lambda: L.chameleon_linear_workspace_size(bad, ctypes.byref(good), 1,
+                                                                           ctypes.byref(n)),
+        "linear_prepare": lambda: L.chameleon_linear_prepare(x, bad, 64, 1, x, 1 << 15, x, None),
+        "linear_prepare_static": lambda: L.chameleon_linear_prepare_static(x, bad, 64, 1, ctypes.byref(p), x,
+                                                                           1 << 15, x, None),
+        "linear_prepare_groups": lambda: L.chameleon_linear_prepare_groups(x, bad, 64, 1, 1, x, 1 << 15, x, None),
+        "linear": lambda: L.chameleon_linear(x, bad, ctypes.byref(good), x, 1, None, x, x, 1 << 15, x, None),
+        "linear_gemm": lambda: L.chameleon_linear_gemm(x, bad, ctypes.byref(good), x, 1, None, x, x, 1 << 15, x,
+                                                       None),
+        "linear_gemm_ex": lambda: L.chameleon_linear_gemm_ex(x, bad, ctypes.byref(good), x, 1, 1, None, x,
+                                                             cl.Y_F32, x, 1 << 15, x, None),
+    }
+    calls["act_moments_workspace_size"] = lambda: L.chameleon_act_moments_workspace_size(bad, ctypes.byref(n))
+    for name, call in calls.items():
+        assert call() == cl.ERR_INVALID_ARG, name
