@@ -310,3 +310,59 @@ def test_empty_and_negative_sizes_are_rejected_on_the_host(cl, bad):
     calls["act_moments_workspace_size"] = lambda: L.chameleon_act_moments_workspace_size(bad, ctypes.byref(n))
     for name, call in calls.items():
         assert call() == cl.ERR_INVALID_ARG, name
+
+
+def test_misaligned_device_pointers_are_rejected_on_the_host(cl):
+    """Device pointers must be 16-byte aligned: inputs, outputs and workspaces two bytes off a
+    16-byte boundary give CHAM_ERR_INVALID_ARG before any device work."""
+    L = cl.lib()
+    buf = ctypes.create_string_buffer(1 << 16)
+    a = ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16
+    x, m = ctypes.c_void_p(a), ctypes.c_void_p(a + 2)
+    good = cl.pack_plan(64, 64, np.zeros(64, np.uint8))
+    p = cl.scale_zp(F.A_E4M3, -1.0, 1.0)
+    pw4 = 1 << F.W_NF4
+    calls = {
+        "act_moments X": lambda: L.chameleon_act_moments(m, 1024, x, x, 1 << 15, None),
+        "act_quant X": lambda: L.chameleon_act_quant(m, 16, 64, 1, x, 1 << 15, x, 1 << 15, x, None),
+        "act_quant qact": lambda: L.chameleon_act_quant(x, 16, 64, 1, m, 1 << 15, x, 1 << 15, x, None),
+        "act_quant ws": lambda: L.chameleon_act_quant(x, 16, 64, 1, x, 1 << 15, m, 1 << 15, x, None),
+        "act_quant_noalloc X": lambda: L.chameleon_act_quant_noalloc(m, 16, 64, 1, x, 1 << 15, x, None),
+        "act_quant_static X": lambda: L.chameleon_act_quant_static(m, 16, 64, 1, ctypes.byref(p), x, 1 << 15, x,
+                                                                   None),
+        "act_quant_static qact": lambda: L.chameleon_act_quant_static(x, 16, 64, 1, ctypes.byref(p), m, 1 << 15,
+                                                                      x, None),
+        "act_format_sse X": lambda: L.chameleon_act_format_sse(m, 16, 64, x, x, 1 << 15, x, None),
+        "act_format_sse ws": lambda: L.chameleon_act_format_sse(x, 16, 64, x, m, 1 << 15, x, None),
+        "act_channel_energy X": lambda: L.chameleon_act_channel_energy(m, 16, 64, x, None),
+        "select_weight_formats W": lambda: L.chameleon_select_weight_formats(m, 16, 64, cl.PALETTE_W8, x, None,
+                                                                             None),
+        "select_weight_groups W": lambda: L.chameleon_select_weight_groups(m, 16, 64, pw4, 1, None, x, x, 1 << 15,
+                                                                           None),
+        "select_weight_groups ws": lambda: L.chameleon_select_weight_groups(x, 16, 64, pw4, 1, None, x, m,
+                                                                            1 << 15, None),
+        "pack_weights W": lambda: L.chameleon_pack_weights(m, x, ctypes.byref(good), x, 1 << 15, x, None),
+        "pack_weights blob": lambda: L.chameleon_pack_weights(x, x, ctypes.byref(good), m, 1 << 15, x, None),
+        "select_pack_palette W": lambda: L.chameleon_select_pack_palette(m, 64, 64, cl.PALETTE_W8,
+                                                                         ctypes.byref(good), x, x, 1 << 15, x, None),
+        "select_pack_palette blob": lambda: L.chameleon_select_pack_palette(x, 64, 64, cl.PALETTE_W8,
+                                                                            ctypes.byref(good), x, m, 1 << 15, x,
+                                                                            None),
+        "linear_prepare X": lambda: L.chameleon_linear_prepare(m, 16, 64, 1, x, 1 << 15, x, None),
+        "linear_prepare ws": lambda: L.chameleon_linear_prepare(x, 16, 64, 1, m, 1 << 15, x, None),
+        "linear_prepare_static X": lambda: L.chameleon_linear_prepare_static(m, 16, 64, 1, ctypes.byref(p), x,
+                                                                             1 << 15, x, None),
+        "linear_gemm_ex blob": lambda: L.chameleon_linear_gemm_ex(x, 16, ctypes.byref(good), m, 1, 1, None, x,
+                                                                  cl.Y_F32, x, 1 << 15, x, None),
+        "linear_gemm_ex Y": lambda: L.chameleon_linear_gemm_ex(x, 16, ctypes.byref(good), x, 1, 1, None, m,
+                                                               cl.Y_F32, x, 1 << 15, x, None),
+        "linear_gemm_ex ws": lambda: L.chameleon_linear_gemm_ex(x, 16, ctypes.byref(good), x, 1, 1, None, x,
+                                                                cl.Y_F32, m, 1 << 15, x, None),
+        "linear_gemm_ex bias": lambda: L.chameleon_linear_gemm_ex(x, 16, ctypes.byref(good), x, 1, 1, m, x,
+                                                                  cl.Y_F32, x, 1 << 15, x, None),
+        "linear_gemm_ex X (fp16 operand)": lambda: L.chameleon_linear_gemm_ex(m, 16, ctypes.byref(good), x,
+                                                                              F.A_FP16, 1, None, x, cl.Y_F32, x,
+                                                                              1 << 15, x, None),
+    }
+    for name, call in calls.items():
+        assert call() == cl.ERR_INVALID_ARG, name
