@@ -14,6 +14,11 @@ from oracle import select as SEL
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "chameleon.h")
+# Tests that hand host buffers to entry points that take device pointers: every such call must be
+# rejected on the host, so no kernel ever sees them.  They run only where no GPU is present, so a
+# regression in the host checks can never launch a kernel on host memory.
+host_buffers_only = pytest.mark.skipif(os.path.exists("/dev/nvidiactl"),
+                                       reason="host-buffer argument checks run on GPU-less hosts only")
 
 
 @pytest.fixture(scope="module")
@@ -130,6 +135,7 @@ def test_scale_zp_host_matches_oracle_bit_for_bit(cl):
             assert (np.float32(p.s), np.float32(p.inv), p.z, p.fmt) == (s, inv, z, fmt), (fmt, lo, hi)
 
 
+@host_buffers_only
 def test_scale_zp_and_static_entry_points_reject_bad_arguments(cl):
     for fmt, lo, hi in [(3, -1.0, 1.0), (5, -1.0, 1.0), (-1, 0.0, 1.0), (0, 1.0, -1.0),
                         (1, float("nan"), 1.0), (2, 0.0, float("inf")), (0, -3e38, 3e38)]:
@@ -155,6 +161,7 @@ def test_scale_zp_and_static_entry_points_reject_bad_arguments(cl):
                                         None) == cl.ERR_INVALID_ARG      # K not a multiple of 32
 
 
+@host_buffers_only
 def test_groups_and_output_type_argument_checks(cl):
     """Per-sample groups must divide M and number 1..CHAM_MAX_GROUPS; y_type is one of three.
     Every rejection happens on the host, before any launch."""
@@ -209,6 +216,7 @@ def test_pack_plan_grouped_layout_and_checks(cl):
     assert L.chameleon_select_weight_groups_workspace_size(64, 320, 0x070, 0x1F, ctypes.byref(w)) == cl.OK
 
 
+@host_buffers_only
 def test_select_pack_palette_argument_checks(cl):
     L = cl.lib()
     buf = ctypes.create_string_buffer(1 << 20)
@@ -257,6 +265,7 @@ def test_version_and_status_names(cl):
     assert cl.status_string(cl.OK) and cl.status_string(cl.ERR_TIMEOUT) != cl.status_string(cl.OK)
 
 
+@host_buffers_only
 @pytest.mark.parametrize("bad", [0, -1, -32])
 def test_empty_and_negative_sizes_are_rejected_on_the_host(cl, bad):
     """Every entry point that takes a size rejects an empty (0) or negative M, N, K or count with
@@ -312,6 +321,7 @@ def test_empty_and_negative_sizes_are_rejected_on_the_host(cl, bad):
         assert call() == cl.ERR_INVALID_ARG, name
 
 
+@host_buffers_only
 def test_misaligned_device_pointers_are_rejected_on_the_host(cl):
     """Device pointers must be 16-byte aligned: inputs, outputs and workspaces two bytes off a
     16-byte boundary give CHAM_ERR_INVALID_ARG before any device work."""
@@ -366,3 +376,51 @@ def test_misaligned_device_pointers_are_rejected_on_the_host(cl):
     }
     for name, call in calls.items():
         assert call() == cl.ERR_INVALID_ARG, name
+
+
+@host_buffers_only
+def test_undersized_buffers_are_rejected_on_the_host(cl):
+    """A buffer one byte smaller than its size query returned gives CHAM_ERR_WORKSPACE before any
+    device work: quantized activations, workspaces, weight blobs."""
+    L = cl.lib()
+    buf = ctypes.create_string_buffer(1 << 20)
+    x = ctypes.c_void_p(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 256)
+    good = cl.pack_plan(64, 64, np.zeros(64, np.uint8))
+    p = cl.scale_zp(F.A_E4M3, -1.0, 1.0)
+    q, w = cl.act_quant_size(16, 64, F.A_E4M3)
+    n = ctypes.c_size_t(0)
+
+    def size(fn, *args):
+        assert fn(*args, ctypes.byref(n)) == cl.OK
+        return n.value
+
+    sse = size(L.chameleon_act_format_sse_workspace_size, 16, 64)
+    sg = size(L.chameleon_select_weight_groups_workspace_size, 16, 64, 1 << F.W_NF4, 1)
+    lw = size(L.chameleon_linear_workspace_size, 16, ctypes.byref(good), F.A_E4M3)
+    mw = size(L.chameleon_act_moments_workspace_size, 1024)
+    e4, nf4, blob = F.A_E4M3, 1 << F.W_NF4, good.bytes
+    calls = {
+        "act_quant qact": lambda: L.chameleon_act_quant(x, 16, 64, e4, x, q - 1, x, w, x, None),
+        "act_quant ws": lambda: L.chameleon_act_quant(x, 16, 64, e4, x, q, x, w - 1, x, None),
+        "act_quant_static qact": lambda: L.chameleon_act_quant_static(x, 16, 64, e4, ctypes.byref(p), x, q - 1, x,
+                                                                      None),
+        "act_quant_noalloc qact": lambda: L.chameleon_act_quant_noalloc(x, 16, 64, e4, x, q - 1, x, None),
+        "act_format_sse ws": lambda: L.chameleon_act_format_sse(x, 16, 64, x, x, sse - 1, x, None),
+        "act_moments ws": lambda: L.chameleon_act_moments(x, 1024, x, x, mw - 1, None),
+        "select_weight_groups ws": lambda: L.chameleon_select_weight_groups(x, 16, 64, nf4, 1, None, x, x, sg - 1,
+                                                                            None),
+        "pack_weights blob": lambda: L.chameleon_pack_weights(x, x, ctypes.byref(good), x, blob - 1, x, None),
+        "select_pack_palette blob": lambda: L.chameleon_select_pack_palette(x, 64, 64, cl.PALETTE_W8,
+                                                                            ctypes.byref(good), x, x, blob - 1, x,
+                                                                            None),
+        "linear_prepare ws": lambda: L.chameleon_linear_prepare(x, 16, 64, e4, x, lw - 1, x, None),
+        "linear_prepare_static ws": lambda: L.chameleon_linear_prepare_static(x, 16, 64, e4, ctypes.byref(p), x,
+                                                                              lw - 1, x, None),
+        "linear_prepare_groups ws": lambda: L.chameleon_linear_prepare_groups(x, 16, 64, e4, 2, x, lw - 1, x,
+                                                                              None),
+        "linear_gemm ws": lambda: L.chameleon_linear_gemm(x, 16, ctypes.byref(good), x, e4, None, x, x, lw - 1, x,
+                                                          None),
+        "linear ws": lambda: L.chameleon_linear(x, 16, ctypes.byref(good), x, e4, None, x, x, lw - 1, x, None),
+    }
+    for name, call in calls.items():
+        assert call() == cl.ERR_WORKSPACE, name
