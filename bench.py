@@ -841,8 +841,8 @@ def tensor_probe(torch, device):
 
 def cpu_baseline():
     # one core: the BLAS and OpenMP pools of this process are limited to one thread at start-up
-    # about ten seconds of one Grace core: two layers (q and FF-out) at three buckets
-    flops, t, desc, stages = oracle_sample(layers_idx=(4, 9))
+    # about ten seconds of one Grace core: two layers (q and FF-out) at five buckets
+    flops, t, desc, stages = oracle_sample(layers_idx=(4, 9), buckets=(0, 3, 5, 7, 9))
     return {"value": round(flops / t / 1e12, 6), "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
             "sample": desc, "seconds": round(t, 2), "stage_seconds": {k: round(v, 3) for k, v in stages.items()},
             "host_cores": os.cpu_count()}
