@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -38,16 +39,19 @@ cham_status cuda_fail(cudaError_t e, const char* where) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// SM count of the current device, cached per device (host threads may race to fill an entry;
+// they all store the same value).  152 (GB300) when the query fails: sizes then stay valid and
+// the launch itself reports the CUDA error.
 int num_sms_current() {
-  static int cache[64];
+  static std::atomic<int> cache[64];
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-  if (cache[dev] == 0) {
-    int n = 0;
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    cache[dev] = n > 0 ? n : 148;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+  int n = cache[dev].load(std::memory_order_relaxed);
+  if (n == 0) {
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
+    cache[dev].store(n, std::memory_order_relaxed);
   }
-  return cache[dev];
+  return n;
 }
 
 // ---------------------------------------------------------------- NF4 levels (library's own)
@@ -861,7 +865,7 @@ cham_status chameleon_linear_prepare_static(const void* X, int M, int K, int act
 }
 
 namespace {
-int g_stall_next_gemm = -1;  // set by chameleon_debug_stall_next_gemm, consumed by the next launch
+std::atomic<int> g_stall_next_gemm{-1};  // set by chameleon_debug_stall_next_gemm, taken by the next launch
 }  // namespace
 
 cham_status chameleon_debug_stall_next_gemm(int chunk) {
@@ -914,8 +918,7 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   g.N = d->N;
   g.n_chunks = d->Kp / 64;
   g.bits = d->bits;
-  g.stall_chunk = g_stall_next_gemm;
-  g_stall_next_gemm = -1;
+  g.stall_chunk = g_stall_next_gemm.exchange(-1);
   g.dev_status = dev_status;
   const cham::NF4Table& nf4 = nf4_table();
   for (int r = 0; r < 4; ++r) {

@@ -237,8 +237,8 @@ def test_check_rejects_a_null_status_word(cl):
 def test_linear_workspace_includes_split_k_partials(cl):
     """The GEMM splits K when its 128-channel x token tiles are fewer than half the SMs and K has at
     least 8 chunks of 64; the workspace then adds k_split x M x Np fp32 partial sums.  Without a
-    device the library assumes 148 SMs."""
-    sms = 148
+    device the library assumes the 152 SMs of a GB300."""
+    sms = 152
 
     def bn(M):
         return next(b for b in (16, 32, 64, 128) if M <= b) if M <= 128 else 192
