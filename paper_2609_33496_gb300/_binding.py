@@ -161,7 +161,27 @@ def device_status(dev_status, stream=None):
 
 
 def _ptr(t):
-    return None if t is None else ctypes.c_void_p(t.data_ptr())
+    """Device address of a tensor the library reads or writes as one dense buffer."""
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to libchameleon must be contiguous (got strides %s)" % (t.stride(),))
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _typed(t, dtype_name, what):
+    """_ptr of t after checking its element type (None passes through)."""
+    if t is not None and str(t.dtype) != "torch." + dtype_name:
+        raise TypeError("%s must be a %s tensor (got %s)" % (what, dtype_name, t.dtype))
+    return _ptr(t)
+
+
+def _half(t, what):
+    return _typed(t, "float16", what)
+
+
+def _f32(t, what):
+    return _typed(t, "float32", what)
 
 
 def _stream(stream):
@@ -206,7 +226,7 @@ def act_moments(X, out=None, stream=None):
     ws_b = ctypes.c_size_t()
     check(lib().chameleon_act_moments_workspace_size(n, ctypes.byref(ws_b)))
     ws = _bytes(ws_b.value, X.device)
-    check(lib().chameleon_act_moments(_ptr(X), n, _ptr(out), _ptr(ws), ws_b.value, _stream(stream)))
+    check(lib().chameleon_act_moments(_half(X, "X"), n, _ptr(out), _ptr(ws), ws_b.value, _stream(stream)))
     return out
 
 
@@ -227,7 +247,7 @@ def act_quant(X, fmt, dev_status=None, stream=None):
     ws = _bytes(wb, X.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
-    check(lib().chameleon_act_quant(_ptr(X), M, K, fmt, _ptr(qact), qb, _ptr(ws), wb, _ptr(dev_status),
+    check(lib().chameleon_act_quant(_half(X, "X"), M, K, fmt, _ptr(qact), qb, _ptr(ws), wb, _ptr(dev_status),
                                     _stream(stream)))
     return qact, dev_status
 
@@ -252,7 +272,7 @@ def act_quant_static(X, fmt, params, dev_status=None, stream=None):
     qact = _bytes(qb, X.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
-    check(lib().chameleon_act_quant_static(_ptr(X), M, K, fmt, _pref(params), _ptr(qact), qb, _ptr(dev_status),
+    check(lib().chameleon_act_quant_static(_half(X, "X"), M, K, fmt, _pref(params), _ptr(qact), qb, _ptr(dev_status),
                                            _stream(stream)))
     return qact, dev_status
 
@@ -283,7 +303,7 @@ def act_format_sse(X, out=None, dev_status=None, stream=None):
     w = ctypes.c_size_t()
     check(lib().chameleon_act_format_sse_workspace_size(M, K, ctypes.byref(w)))
     ws = _bytes(w.value, X.device)
-    check(lib().chameleon_act_format_sse(_ptr(X), M, K, _ptr(out), _ptr(ws), w.value, _ptr(dev_status),
+    check(lib().chameleon_act_format_sse(_half(X, "X"), M, K, _ptr(out), _ptr(ws), w.value, _ptr(dev_status),
                                          _stream(stream)))
     return out, dev_status
 
@@ -303,7 +323,7 @@ def select_weight_formats(W, palette_mask, want_sse=False, stream=None, fmt_out=
     if fmt.numel() != N or fmt.dtype != torch.uint8 or not fmt.is_contiguous():
         raise ValueError("fmt_out must be a contiguous uint8 tensor of N elements")
     sse = torch.empty((N, 9), dtype=torch.float64, device=W.device) if want_sse else None
-    check(lib().chameleon_select_weight_formats(_ptr(W), N, K, palette_mask, _ptr(fmt), _ptr(sse),
+    check(lib().chameleon_select_weight_formats(_half(W, "W"), N, K, palette_mask, _ptr(fmt), _ptr(sse),
                                                 _stream(stream)))
     return fmt, sse
 
@@ -347,7 +367,7 @@ def select_weight_groups(W, palette_mask, gmask, energy=None, stream=None):
     check(lib().chameleon_select_weight_groups_workspace_size(N, K, palette_mask, gmask, ctypes.byref(w)))
     ws = _bytes(w.value, W.device)
     scores = torch.empty(len(group_candidates(palette_mask, gmask)), dtype=torch.float64, device=W.device)
-    check(lib().chameleon_select_weight_groups(_ptr(W), N, K, palette_mask, gmask, _ptr(energy), _ptr(scores),
+    check(lib().chameleon_select_weight_groups(_half(W, "W"), N, K, palette_mask, gmask, _ptr(energy), _ptr(scores),
                                                _ptr(ws), w.value, _stream(stream)))
     return scores
 
@@ -363,7 +383,7 @@ def act_channel_energy(X, energy=None, stream=None):
     M, K = X.shape
     if energy is None:
         energy = torch.zeros(K, dtype=torch.float64, device=X.device)
-    check(lib().chameleon_act_channel_energy(_ptr(X), M, K, _ptr(energy), _stream(stream)))
+    check(lib().chameleon_act_channel_energy(_half(X, "X"), M, K, _ptr(energy), _stream(stream)))
     return energy
 
 
@@ -385,7 +405,7 @@ def select_pack_palette(W, palette_mask, desc, fmt_out=None, blob=None, dev_stat
         blob = _bytes(desc.bytes, W.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=W.device)
-    check(lib().chameleon_select_pack_palette(_ptr(W), N, K, palette_mask, ctypes.byref(desc), _ptr(fmt_out),
+    check(lib().chameleon_select_pack_palette(_half(W, "W"), N, K, palette_mask, ctypes.byref(desc), _ptr(fmt_out),
                                               _ptr(blob), blob.numel(), _ptr(dev_status), _stream(stream)))
     return fmt_out, blob, dev_status
 
@@ -396,7 +416,7 @@ def pack_weights(W, fmt_dev, desc, dev_status=None, stream=None, blob=None):
         blob = _bytes(desc.bytes, W.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=W.device)
-    check(lib().chameleon_pack_weights(_ptr(W), _ptr(fmt_dev), ctypes.byref(desc), _ptr(blob), blob.numel(),
+    check(lib().chameleon_pack_weights(_half(W, "W"), _ptr(fmt_dev), ctypes.byref(desc), _ptr(blob), blob.numel(),
                                        _ptr(dev_status), _stream(stream)))
     return blob, dev_status
 
@@ -419,8 +439,8 @@ def linear(X, desc, blob, act_fmt, bias=None, Y=None, ws=None, dev_status=None, 
         Y = torch.empty((M, desc.N), dtype=torch.float32, device=X.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
-    check(lib().chameleon_linear(_ptr(X), M, ctypes.byref(desc), _ptr(blob), act_fmt, _ptr(bias), _ptr(Y),
-                                 _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))
+    check(lib().chameleon_linear(_half(X, "X"), M, ctypes.byref(desc), _ptr(blob), act_fmt, _f32(bias, "bias"),
+                                 _f32(Y, "Y"), _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))
     return Y, dev_status
 
 
@@ -453,15 +473,15 @@ def linear_prepare_groups(X, act_fmt, n_groups, ws, dev_status, stream=None):
     """First half of linear with per-sample scales: rows in n_groups equal groups, each quantized
     with the ScaleZP of its own range."""
     M, K = X.shape
-    check(lib().chameleon_linear_prepare_groups(_ptr(X), M, K, act_fmt, n_groups, _ptr(ws), ws.numel(),
+    check(lib().chameleon_linear_prepare_groups(_half(X, "X"), M, K, act_fmt, n_groups, _ptr(ws), ws.numel(),
                                                 _ptr(dev_status), _stream(stream)))
 
 
 def linear_gemm_ex(X, desc, blob, act_fmt, n_groups, bias, Y, ws, dev_status, stream=None):
     """Second half of linear with the operand's row groups; the output type is Y's dtype."""
-    check(lib().chameleon_linear_gemm_ex(_ptr(X), X.shape[0], ctypes.byref(desc), _ptr(blob), act_fmt, n_groups,
-                                         _ptr(bias), _ptr(Y), _y_type(Y), _ptr(ws), ws.numel(), _ptr(dev_status),
-                                         _stream(stream)))
+    check(lib().chameleon_linear_gemm_ex(_half(X, "X"), X.shape[0], ctypes.byref(desc), _ptr(blob), act_fmt,
+                                         n_groups, _f32(bias, "bias"), _ptr(Y), _y_type(Y), _ptr(ws), ws.numel(),
+                                         _ptr(dev_status), _stream(stream)))
 
 
 def linear_ex(X, desc, blob, act_fmt, n_groups=1, y_dtype=None, bias=None, Y=None, ws=None, dev_status=None,
@@ -489,21 +509,22 @@ def debug_stall_next_gemm(chunk):
 def linear_prepare(X, act_fmt, ws, dev_status, stream=None):
     """First half of linear: quantize X into the workspace operand."""
     M, K = X.shape
-    check(lib().chameleon_linear_prepare(_ptr(X), M, K, act_fmt, _ptr(ws), ws.numel(), _ptr(dev_status),
+    check(lib().chameleon_linear_prepare(_half(X, "X"), M, K, act_fmt, _ptr(ws), ws.numel(), _ptr(dev_status),
                                          _stream(stream)))
 
 
 def linear_prepare_static(X, act_fmt, params, ws, dev_status, stream=None):
     """First half of linear on the static path: quantize X with fixed parameters (QParams)."""
     M, K = X.shape
-    check(lib().chameleon_linear_prepare_static(_ptr(X), M, K, act_fmt, _pref(params), _ptr(ws), ws.numel(),
+    check(lib().chameleon_linear_prepare_static(_half(X, "X"), M, K, act_fmt, _pref(params), _ptr(ws), ws.numel(),
                                                 _ptr(dev_status), _stream(stream)))
 
 
 def linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream=None):
     """Second half of linear: the tcgen05 GEMM on the prepared operand."""
-    check(lib().chameleon_linear_gemm(_ptr(X), X.shape[0], ctypes.byref(desc), _ptr(blob), act_fmt, _ptr(bias),
-                                      _ptr(Y), _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))
+    check(lib().chameleon_linear_gemm(_half(X, "X"), X.shape[0], ctypes.byref(desc), _ptr(blob), act_fmt,
+                                      _f32(bias, "bias"), _f32(Y, "Y"), _ptr(ws), ws.numel(), _ptr(dev_status),
+                                      _stream(stream)))
 
 
 def act_quant_noalloc(X, fmt, qact, dev_status, stream=None):
@@ -511,5 +532,5 @@ def act_quant_noalloc(X, fmt, qact, dev_status, stream=None):
     the caller passes the output buffer `qact` (sized by act_quant_size) and the status word; the
     range partials live in a static device array inside the library.  Returns the raw status."""
     M, K = X.shape
-    return lib().chameleon_act_quant_noalloc(_ptr(X), M, K, fmt, _ptr(qact), qact.numel(), _ptr(dev_status),
+    return lib().chameleon_act_quant_noalloc(_half(X, "X"), M, K, fmt, _ptr(qact), qact.numel(), _ptr(dev_status),
                                              _stream(stream))
