@@ -166,6 +166,8 @@ def _ptr(t):
         return None
     if not t.is_contiguous():
         raise ValueError("tensors passed to libchameleon must be contiguous (got strides %s)" % (t.stride(),))
+    if not t.is_cuda:
+        raise ValueError("tensors passed to libchameleon must be CUDA tensors (got one on %s)" % (t.device,))
     return ctypes.c_void_p(t.data_ptr())
 
 

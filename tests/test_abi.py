@@ -427,23 +427,22 @@ def test_undersized_buffers_are_rejected_on_the_host(cl):
 
 
 @host_buffers_only
-def test_binding_rejects_strided_and_mistyped_tensors(cl):
-    """The binding hands the library one dense buffer per tensor: a non-contiguous view or a
-    tensor of the wrong element type raises in Python, before the library is called."""
+def test_binding_rejects_strided_mistyped_and_host_tensors(cl):
+    """The binding hands the library one dense CUDA buffer per tensor: a host tensor, a
+    non-contiguous view or a tensor of the wrong element type raises in Python, before the library
+    is called (element type first, then layout, then device)."""
     import torch
     X = torch.zeros(64, 32, dtype=torch.float16)
-    with pytest.raises(ValueError):
-        cl.act_quant(X.t(), F.A_E4M3)                                   # 32 x 64 transposed view
-    with pytest.raises(TypeError):
+    with pytest.raises(ValueError, match="CUDA"):
+        cl.act_quant(X, F.A_E4M3)                                       # a host tensor
+    with pytest.raises(TypeError, match="float16"):
         cl.act_quant(X.float(), F.A_E4M3)
-    with pytest.raises(TypeError):
+    with pytest.raises(TypeError, match="float16"):
         cl.select_weight_formats(torch.zeros(16, 64, dtype=torch.bfloat16), cl.PALETTE_W8)
-    d = cl.pack_plan(64, 64, np.zeros(64, np.uint8))
-    blob = torch.zeros(d.bytes, dtype=torch.uint8)
-    X64 = torch.zeros(16, 64, dtype=torch.float16)
-    with pytest.raises(TypeError):
-        cl.linear(X64, d, blob, F.A_E4M3, bias=torch.zeros(64, dtype=torch.float64))
-    with pytest.raises(TypeError):
-        cl.linear(X64, d, blob, F.A_E4M3, Y=torch.zeros(16, 64, dtype=torch.float16))
-    with pytest.raises(ValueError):
-        cl.linear(X64, d, blob, F.A_E4M3, Y=torch.zeros(64, 16, dtype=torch.float32).t())
+    with pytest.raises(ValueError, match="contiguous"):
+        cl._ptr(X.t())                                                  # 32 x 64 transposed view
+    with pytest.raises(TypeError, match="float32"):
+        cl._f32(torch.zeros(64, dtype=torch.float64), "bias")
+    with pytest.raises(TypeError, match="float32"):
+        cl._f32(torch.zeros(16, 64, dtype=torch.float16), "Y")
+    assert cl._f32(None, "bias") is None
