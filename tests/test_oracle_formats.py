@@ -156,6 +156,21 @@ def test_fp8_scale(fmt, fmax, top):
     assert q["codes"][i] & 0x7F == top                                 # amax -> +-Fmax
 
 
+def test_int8_asym_one_sided_ranges_include_zero():
+    """R4: the range is widened to include 0, so a single-signed tensor keeps an exact zero:
+    all positive -> z = 0, s = hi / 255; all negative -> z = 255, s = -lo / 255."""
+    x = np.array([[1.0, 2.0, 3.0] + [1.5] * 29], np.float16)
+    q = F.act_quant(x, F.A_INT8_ASYM)
+    assert q["z"] == 0 and q["s"] == np.float32(np.float32(3.0) / np.float32(255.0))
+    assert q["codes"][0, 2] == 255 and q["codes"][0, 0] == 85                 # 1.0 / (3/255) = 85
+    q = F.act_quant(-x, F.A_INT8_ASYM)
+    assert q["z"] == 255 and q["s"] == np.float32(np.float32(3.0) / np.float32(255.0))
+    assert q["codes"][0, 2] == 0 and q["codes"][0, 0] == 170
+    w = np.array([[0.5, 1.0, 2.0, 4.0] * 8], np.float16)                       # weight channel, INT4-asym
+    qw = F.weight_quant(w, F.W_INT4_ASYM)
+    assert qw["z"][0] == 0 and qw["s"][0] == np.float32(np.float32(4.0) / np.float32(15.0))
+
+
 def test_fp8_round_trip_on_representable_values():
     """DQ(Q(x)) == x when x already lies on the E4M3 grid and amax = 448 (inv = 1)."""
     vals = F.fp_decode(np.arange(0x7F), "e4m3")

@@ -165,6 +165,23 @@ def test_nf4_quantiles_by_bisection():
     assert np.all(v.astype(np.float16).astype(np.float64) == nf4.nf4_levels_fp16())
 
 
+def test_nf4_exact_midpoints_go_to_the_lower_level():
+    """R9: the code is the number of midpoints strictly below w/s, so a weight exactly on a
+    midpoint takes the lower level.  Nine of the fifteen midpoints are fp16 values: with a 1.0 in
+    the row (s = amax = 1) those weights sit exactly on them."""
+    L = nf4.nf4_levels_fp16()
+    mids = (L[:-1] + L[1:]) / 2.0
+    idx = [i for i in range(15) if float(np.float16(mids[i])) == mids[i]]
+    assert len(idx) >= 5
+    row = np.array([1.0] + [mids[i] for i in idx], np.float16)[None, :]
+    q = F.weight_quant(row, F.W_NF4, nf4_levels=L)
+    assert q["s"][0] == 1.0 and q["codes"][0, 0] == 15
+    assert q["codes"][0, 1:].tolist() == idx
+    nudged = np.nextafter(row.astype(np.float16), np.float16(2.0))     # one fp16 ulp above: upper level
+    nudged[0, 0] = 1.0
+    assert F.weight_quant(nudged, F.W_NF4, nf4_levels=L)["codes"][0, 1:].tolist() == [i + 1 for i in idx]
+
+
 # ---------------------------------------------------------------- activation-format argmin (Eq. format-argmin)
 def fp8_grid(ebits, mbits, bias, skip):
     """(value, mantissa-is-even) of every non-negative finite value, from the bit definition."""
