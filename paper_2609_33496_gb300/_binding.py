@@ -151,6 +151,7 @@ def version():
 
 
 def check(status):
+    """Raise ChameleonError (with the library's detail line) unless status is CHAM_OK."""
     if status != OK:
         raise ChameleonError(status, lib().chameleon_last_error_detail().decode())
 
@@ -199,21 +200,25 @@ def _bytes(n, device):
 
 # ------------------------------------------------------------------ host helpers
 def bucket(t, T=1000, B=10):
+    """Timestep bucket b = min(floor(t / (T/B)), B - 1) (Alg. 2, Alg. 3); -1 for invalid input."""
     return lib().chameleon_bucket(int(t), int(T), int(B))
 
 
 def snr(schedule=SCHEDULE_SCALED_LINEAR, T=1000):
+    """SNR(t) = abar_t / (1 - abar_t) for t = 0..T-1 of a noise schedule (host, float64 [T])."""
     out = np.zeros(T, dtype=np.float64)
     check(lib().chameleon_snr(schedule, T, out.ctypes.data_as(ctypes.POINTER(ctypes.c_double))))
     return out
 
 
 def kurtosis(sums):
+    """kappa = m4 / m2^2 from the power sums {n, S1, S2, S3, S4} (the first five of act_moments)."""
     arr = (ctypes.c_double * 5)(*[float(s) for s in sums[:5]])
     return lib().chameleon_kurtosis(arr)
 
 
 def route(kappa, snr_b, is_shortcut=False):
+    """The activation format the routing rule picks for kurtosis kappa at SNR(t_b) (Sec. 3.3)."""
     return lib().chameleon_route(float(kappa), float(snr_b), int(bool(is_shortcut)))
 
 
@@ -234,6 +239,7 @@ def act_moments(X, out=None, stream=None):
 
 # ------------------------------------------------------------------ a2-a4
 def act_quant_size(M, K, fmt):
+    """(qact bytes, workspace bytes) of chameleon_act_quant for an M x K tensor in format fmt."""
     q, w = ctypes.c_size_t(), ctypes.c_size_t()
     check(lib().chameleon_act_quant_size(M, K, fmt, ctypes.byref(q), ctypes.byref(w)))
     return q.value, w.value
@@ -332,6 +338,8 @@ def select_weight_formats(W, palette_mask, want_sse=False, stream=None, fmt_out=
 
 # ------------------------------------------------------------------ a6
 def pack_plan_palette(N, K, palette_mask):
+    """Packed layout for N x K weights whose palette shares one MMA class (no host copy of the
+    selected formats needed); the formats are written by the selection on the device."""
     d = WPackDesc()
     check(lib().chameleon_pack_plan_palette(N, K, palette_mask, ctypes.byref(d)))
     return d
@@ -375,6 +383,7 @@ def select_weight_groups(W, palette_mask, gmask, energy=None, stream=None):
 
 
 def candidate_argmin(scores_host):
+    """Index of the first smallest (g, f) search score (host list or array)."""
     a = (ctypes.c_double * len(scores_host))(*[float(v) for v in scores_host])
     return lib().chameleon_candidate_argmin(a, len(scores_host))
 
@@ -390,6 +399,7 @@ def act_channel_energy(X, energy=None, stream=None):
 
 
 def pack_plan(N, K, fmt_host):
+    """Packed layout (cham_wpack_desc) for N x K weights with the selected formats fmt_host (host uint8 [N])."""
     f = np.ascontiguousarray(np.asarray(fmt_host, dtype=np.uint8))
     d = WPackDesc()
     check(lib().chameleon_pack_plan(N, K, f.ctypes.data_as(ctypes.c_void_p), ctypes.byref(d)))
@@ -413,6 +423,8 @@ def select_pack_palette(W, palette_mask, desc, fmt_out=None, blob=None, dev_stat
 
 
 def pack_weights(W, fmt_dev, desc, dev_status=None, stream=None, blob=None):
+    """Encode each channel of W (fp16 N x K, CUDA) in its format fmt_dev (uint8 [N], CUDA) into the
+    packed blob desc describes.  Returns (blob, dev_status)."""
     import torch
     if blob is None or blob.numel() < desc.bytes:
         blob = _bytes(desc.bytes, W.device)
@@ -425,6 +437,7 @@ def pack_weights(W, fmt_dev, desc, dev_status=None, stream=None, blob=None):
 
 # ------------------------------------------------------------------ a7/a8
 def linear_workspace_size(M, desc, act_fmt):
+    """Workspace bytes of chameleon_linear for M rows, the packed weights desc and act_fmt."""
     w = ctypes.c_size_t()
     check(lib().chameleon_linear_workspace_size(M, ctypes.byref(desc), act_fmt, ctypes.byref(w)))
     return w.value
