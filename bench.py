@@ -37,6 +37,13 @@ GEMM_TRAFFIC_PER_LAUNCH = {"bytes": 43.79e6, "launch": "2048x1280x10240 (GEGLU-i
                            "algorithmic_bytes": 99.8e6}
 
 
+def traffic_fields(t=GEMM_TRAFFIC_PER_LAUNCH):
+    """roofline.traffic (DRAM bytes of one captured launch, or None) and what that launch was."""
+    if not t:
+        return {"traffic": None}
+    return {"traffic": t["bytes"], "traffic_launch": t["launch"], "traffic_algorithmic_bytes": t["algorithmic_bytes"]}
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -377,7 +384,7 @@ def main():
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
         "roofline": {"bound": "tensor", "achieved": round(gemm_tflops, 2), "peak": peak_tensor,
                      "unit": "TFLOP/s", "frac": round(gemm_tflops / peak_tensor, 4),
-                     "traffic": GEMM_TRAFFIC_PER_LAUNCH,
+                     **traffic_fields(),
                      "kernel": "k_gemm_ts_f16 (tcgen05 kind::f16, weights decoded into TMEM)",
                      "peak_source": "%s bf16_tflops_sustained (fp16 MMA rate = bf16 rate)" % pk_kind,
                      "roofline_time_frac": round(t_roof * K_ / (gemm_ms * 1e-3), 4),
