@@ -76,7 +76,10 @@ typedef int cham_status;
 #define CHAM_SCHEDULE_SCALED_LINEAR 0
 #define CHAM_SCHEDULE_LINEAR 1
 
+/* Static name of a status code ("ok", "invalid argument", ...); "unknown status" for other values. */
 const char* chameleon_status_string(cham_status s);
+/* One-line description of the last failed call on the calling host thread (a thread-local
+ * buffer, empty before any failure; its contents change at that thread's next failing call). */
 const char* chameleon_last_error_detail(void);
 
 /* Waits for the work queued on `stream` (a cudaStream_t; NULL = the legacy default stream) and
@@ -85,6 +88,7 @@ const char* chameleon_last_error_detail(void);
  * CHAM_ERR_NONFINITE or CHAM_ERR_TIMEOUT).  The word is left as it is.  CHAM_ERR_CUDA when the
  * synchronisation or the copy fails; CHAM_ERR_INVALID_ARG when dev_status is NULL. */
 cham_status chameleon_check(const int* dev_status, void* stream);
+/* ABI version of this library: 2 (packed-weight descriptors with group-wise weights). */
 int chameleon_version(void);
 
 /* ------------------------------------------------------------------ host helpers (a1, L2) */
@@ -134,6 +138,9 @@ typedef struct {
   int32_t fmt;
 } cham_qparams;
 
+/* Size query for chameleon_act_quant: *qact_bytes of the layout above and *ws_bytes of scratch
+ * (0 for the MX formats; either pointer may be NULL).  Host only.  CHAM_ERR_INVALID_ARG for
+ * M, K <= 0, K not a multiple of 32 or fmt outside 0..4. */
 cham_status chameleon_act_quant_size(int M, int K, int fmt, size_t* qact_bytes, size_t* ws_bytes);
 
 /* Quantize X (device, fp16 M x K) in activation format fmt with its own dynamic range (Alg. 3:
