@@ -18,7 +18,7 @@ MUTANTS = (
     "e5m2_decode_inf_as_nan_only_for_max", "asym_zero_point_sign", "asym_raw_range",
     "fp8_amax_from_hi_only", "mxfp8_exponent_off_by_one", "mxint_exponent_off_by_one",
     "mx_zero_block_byte_127", "int8_sym_scale_over_128", "e2m1_weight_scale_over_4",
-    "nf4_ties_to_upper_level", "static_range_ignored", "per_sample_strided_rows",
+    "nf4_ties_to_upper_level", "nf4_delta_one_minus_1_32", "static_range_ignored", "per_sample_strided_rows",
     # schedule, statistics and route
     "kurtosis_dropped_term", "alpha_bar_excludes_t", "route_kappa_high_inclusive", "bucket_rounds_to_nearest",
     # selection and search
@@ -111,6 +111,9 @@ def apply(name):
                 q["codes"] = (mids32[None, None, :] <= v[..., None]).sum(axis=2).astype(np.int64)
             return q
         F.weight_quant = weight_quant
+    elif name == "nf4_delta_one_minus_1_32":
+        from oracle import nf4 as N
+        N.NF4_DELTA = 1.0 - 1.0 / 32.0      # the 16-level offset alone instead of the mean of the two
     elif name == "kurtosis_dropped_term":
         S.kurtosis_from_sums = _kurtosis_without_cross_term
     elif name == "alpha_bar_excludes_t":

@@ -88,6 +88,16 @@ def test_kurtosis_gaussian_and_laplace():
     assert S.kurtosis(2.0 + 0.1 * rng.standard_normal(1_000_000)) == pytest.approx(3.0, abs=0.03)
 
 
+@pytest.mark.slow
+def test_kurtosis_student_t_closed_form():
+    """Student-t with nu > 4 degrees of freedom has kurtosis 3 + 6 / (nu - 4): 4 at nu = 10, the
+    heavy-tailed family the synthetic activations are drawn from.  Its eighth moment exists, so
+    the sample kurtosis of 10^7 draws has a spread of about 0.01."""
+    rng = np.random.default_rng(20260004)
+    assert S.kurtosis(rng.standard_t(10, 10_000_000)) == pytest.approx(4.0, abs=0.1)
+    assert S.kurtosis(-1.5 + 0.5 * rng.standard_t(12, 10_000_000)) == pytest.approx(3.75, abs=0.1)
+
+
 def test_power_sums_merge():
     rng = np.random.default_rng(20260003)
     a, b = rng.standard_normal(1000), rng.standard_t(5, 777)

@@ -5,6 +5,7 @@ the code list) on tiny tensors must give the same SSE and the same argmin.  Cons
 channels pin the tie rule (palette order) and zero-error cases.
 """
 import math
+import os
 
 import numpy as np
 import pytest
@@ -163,6 +164,21 @@ def test_nf4_quantiles_by_bisection():
     v = np.sort(np.array(pos + [0.0] + neg)) / max(pos)
     np.testing.assert_allclose(nf4.nf4_levels_exact(), v, atol=1e-12)
     assert np.all(v.astype(np.float16).astype(np.float64) == nf4.nf4_levels_fp16())
+
+
+def test_nf4_levels_match_the_published_qlora_table():
+    """The levels against the NF4 table that QLoRA publishes (Appendix E of Dettmers et al., 2023;
+    the source App. A.11 cites for NF4), a fact from outside this construction: a wrong outermost
+    probability (e.g. 1 - 1/32 alone), a wrong count of negative quantiles or a missing
+    normalisation moves some level by 1e-3 or more.  The published values are float32 renderings,
+    hence the 1e-6 tolerance."""
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "nf4_qlora_levels.txt")
+    rows = [line.split() for line in open(path) if line.strip() and not line.startswith("#")]
+    assert [int(r[0]) for r in rows] == list(range(16))
+    published = np.array([float(r[1]) for r in rows])
+    np.testing.assert_allclose(nf4.nf4_levels_exact(), published, rtol=0, atol=1e-6)
+    # the frozen fp16 levels are those values rounded to fp16
+    assert np.all(published.astype(np.float16).astype(np.float64) == nf4.nf4_levels_fp16())
 
 
 def test_nf4_exact_midpoints_go_to_the_lower_level():
