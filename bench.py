@@ -273,9 +273,9 @@ def main():
                 f = int(lut[li, bk])
                 if "q" in parts:
                     if args.dynamic_scales:
-                        cl.linear_prepare(X[li][bk], f, ws[li], st)
+                        cl.linear_prepare(X[li][bk], descs[li], f, ws[li], st)
                     else:
-                        cl.linear_prepare_static(X[li][bk], f, qp[li][bk], ws[li], st)
+                        cl.linear_prepare_static(X[li][bk], descs[li], f, qp[li][bk], ws[li], st)
                 if "g" in parts:
                     cl.linear_gemm(X[li][bk], descs[li], blobs[li], f, bias[li], Y[li], ws[li], st)
 
@@ -604,7 +604,7 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
         ws = torch.empty(max(cl.linear_workspace_size(M, desc, f) for f in range(6)), dtype=torch.uint8, device=dev)
         for af in ([0, 1, 2, 3, 4] + ([5] if bits == 4 else [])):
             if af != 5:
-                cl.linear_prepare(x, af, ws, st)
+                cl.linear_prepare(x, desc, af, ws, st)
             t = timed(lambda: cl.linear_gemm(x, desc, blob, af, bias[li], Y, ws, st))
             a_bytes = M * K * (2 if af == 5 else 1) + (M * K / 32 if af in (3, 4) else 0)
             byts = a_bytes + N * K * bits / 8 + 9 * N + 4 * M * N
@@ -616,10 +616,10 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
                 row["frac_fp8_roofline"] = round(max(flops / p8, byts / hbm) / t_s, 4)
             out["gemm"].append(row)
             if bits == 8 and af != 5:
-                tq = timed(lambda: cl.linear_prepare(x, af, ws, st))
+                tq = timed(lambda: cl.linear_prepare(x, desc, af, ws, st))
                 xf = x.float()
                 p_af = cl.scale_zp(af, float(xf.min()), float(xf.max())) if af <= 2 else None
-                tqs = timed(lambda: cl.linear_prepare_static(x, af, p_af, ws, st))
+                tqs = timed(lambda: cl.linear_prepare_static(x, desc, af, p_af, ws, st))
                 qb = 4 * M * K
                 out["quant"].append({"act_fmt": af, "us": round(tq * 1e3, 2), "static_us": round(tqs * 1e3, 2),
                                      "gbs": round(qb / (tq * 1e-3) / 1e9, 1),
@@ -642,7 +642,7 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
         ws_l = torch.zeros(cl.linear_workspace_size(Ml, desc_l, 1), dtype=torch.uint8, device=dev)
         fl = layer_flops(Ml, Kl, Nl)
         for groups in (1, 2):
-            cl.linear_prepare_groups(X[lj][-1], 1, groups, ws_l, st)
+            cl.linear_prepare_groups(X[lj][-1], desc_l, 1, groups, ws_l, st)
             for yn in ("f32", "f16", "bf16"):
                 Y_l = torch.empty((Ml, Nl), dtype=tdt[yn], device=dev)
                 t = timed(lambda: cl.linear_gemm_ex(X[lj][-1], desc_l, blob_l, 1, groups, bias[lj], Y_l, ws_l,
@@ -664,7 +664,7 @@ def variant_matrix(torch, cl, W, bias, X, layers, lut, qp, st, pk, probe, reps=2
         cl.pack_weights(W[lj], fmt_l, desc_l, dev_status=st, blob=blob_l)
         ws_l = torch.zeros(cl.linear_workspace_size(Ml, desc_l, af), dtype=torch.uint8, device=dev)
         Y_l = torch.empty((Ml, Nl), dtype=torch.float32, device=dev)
-        cl.linear_prepare_static(X[lj][-1], af, qp[lj][-1], ws_l, st)
+        cl.linear_prepare_static(X[lj][-1], desc_l, af, qp[lj][-1], ws_l, st)
         t = timed(lambda: cl.linear_gemm(X[lj][-1], desc_l, blob_l, af, bias[lj], Y_l, ws_l, st)) * 1e-3
         fl = layer_flops(Ml, Kl, Nl)
         byts = Ml * Kl + Nl * Kl + 9 * Nl + 4 * Ml * Nl
@@ -727,7 +727,7 @@ def workload_variants(torch, cl, st, pk, probe, reps=20):
             ws = torch.empty(cl.linear_workspace_size(M, desc, af), dtype=torch.uint8, device=dev)
             Y = torch.empty((M, N), dtype=torch.float32, device=dev)
             g = groups if M % groups == 0 else 1
-            cl.linear_prepare_groups(Xd, af, g, ws, st)
+            cl.linear_prepare_groups(Xd, desc, af, g, ws, st)
             t = timed(lambda: cl.linear_gemm_ex(Xd, desc, blob, af, g, bd, Y, ws, st))
             fl = 2.0 * M * K * N
             byts = M * K * (2 if af == cl.A_FP16 else 1) + N * K / 2 + 9 * N + 4 * M * N
@@ -736,7 +736,7 @@ def workload_variants(torch, cl, st, pk, probe, reps=20):
                    "frac_f16_roofline": round(max(fl / p16, byts / hbm) / t, 4)}
             if af != cl.A_FP16:
                 row["frac_fp8_roofline"] = round(max(fl / p8, byts / hbm) / t, 4)
-                tq = timed(lambda: cl.linear_prepare_groups(Xd, af, g, ws, st))
+                tq = timed(lambda: cl.linear_prepare_groups(Xd, desc, af, g, ws, st))
                 tot_q += tq
                 row.update({"quant_us": round(tq * 1e6, 2), "quant_gbs": round(4 * M * K / tq / 1e9, 1),
                             "quant_frac_hbm": round(4 * M * K / tq / hbm, 4)})
@@ -792,7 +792,7 @@ def dit_sampler(torch, cl, st, steps=20):
             for L in layers:
                 af = int(L["lut"][b])
                 X = L["Xs"][b]
-                cl.linear_prepare_groups(X, af, 2, L["ws"], st)
+                cl.linear_prepare_groups(X, L["desc"], af, 2, L["ws"], st)
                 cl.linear_gemm_ex(X, L["desc"], L["blob"], af, 2, L["bias"], L["Y"], L["ws"], st)
 
     run()

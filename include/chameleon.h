@@ -88,7 +88,8 @@ const char* chameleon_last_error_detail(void);
  * CHAM_ERR_NONFINITE or CHAM_ERR_TIMEOUT).  The word is left as it is.  CHAM_ERR_CUDA when the
  * synchronisation or the copy fails; CHAM_ERR_INVALID_ARG when dev_status is NULL. */
 cham_status chameleon_check(const int* dev_status, void* stream);
-/* ABI version of this library: 2 (packed-weight descriptors with group-wise weights). */
+/* ABI version of this library: 3 (packed-weight descriptors with group-wise weights and the MMA
+ * path switch; the linear prepare calls take the descriptor). */
 int chameleon_version(void);
 
 /* ------------------------------------------------------------------ host helpers (a1, L2) */
@@ -264,7 +265,7 @@ cham_status chameleon_act_channel_energy(const void* X, int M, int K, double* en
  * forks); its weights decode to fp16(value(code) * scale16), the product rounded once. */
 typedef struct {
   uint32_t magic;    /* 0x574D4843 ("CHMW") */
-  uint32_t version;  /* 2 */
+  uint32_t version;  /* 3 */
   int32_t N, K, Kp, bits;
   int32_t n_class[2];
   int32_t n_tiles[2];
@@ -272,7 +273,11 @@ typedef struct {
   int32_t group;              /* 0: per-channel (or MX) formats; g > 0: group-wise, g input channels */
   uint64_t off_codes, off_scale, off_zero, off_e8m0, off_fmt, off_perm, bytes;
   uint64_t off_gscale;        /* group-wise blobs: the gscale region, else 0 */
-  uint8_t reserved[112];      /* pads the descriptor to 256 bytes */
+  int32_t f16_only;           /* 0 (the plans' default): class-0 tiles multiply on the FP8 tensor cores
+                                 when the activation format is E4M3, E5M2 or MXFP8 (see
+                                 chameleon_linear); 1: every tile on fp16 MMAs.  The linear calls of
+                                 one layer must see the same value (it fixes the workspace layout). */
+  uint8_t reserved[108];      /* pads the descriptor to 256 bytes */
 } cham_wpack_desc;
 
 /* Fill *desc for N x K weights whose selected formats are fmt_host (host, uint8 [N], all of one
@@ -314,11 +319,13 @@ cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const 
 /* ------------------------------------------------------------------ a7/a8: quantized linear */
 
 /* Workspace (device) of the linear calls for M rows of the layer *desc in act_fmt: the activation
- * scales of up to CHAM_MAX_GROUPS row groups, the quantizer's range partials, the exact fp16
- * operand (M x K; none for CHAM_A_FP16) and, when the GEMM splits K -- a layer whose 128-channel
- * x token tiles are fewer than half the SMs and whose K spans at least 8 chunks of 64 -- the fp32
- * partial sums of the K ranges, which a second kernel adds in order.  The size depends on the
- * current device's SM count. */
+ * scales of up to CHAM_MAX_GROUPS row groups, the quantizer's range partials, the GEMM operands the
+ * layer's tiles need -- the exact fp16 operand (M x K) for tiles on fp16 MMAs, the 1-byte codes
+ * (M x K, plus for MXFP8 their E8M0 exponents chunk-major: [ceil(K/128)][round_up(M, 4)][4]) for
+ * class-0 tiles on FP8 MMAs, neither for CHAM_A_FP16 -- and, when a GEMM launch splits K (a layer
+ * whose 128-channel x token tiles are fewer than half the SMs and whose K spans at least 8
+ * chunks), the fp32 partial sums of the K ranges, which a second kernel adds in order.  The size
+ * depends on the current device's SM count. */
 cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* desc, int act_fmt,
                                             size_t* ws_bytes);
 
@@ -326,23 +333,32 @@ cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* desc, 
  * (= F[layer, bucket] resolved on the host, Alg. 2/3) with its own range, multiplied on tcgen05
  * tensor cores with the packed weights (device blob made from *desc, host), fp32 accumulation;
  * Y (device, fp32 M x desc->N) in original channel order.  bias (device, fp32 [N]) may be NULL.
- * act_fmt = CHAM_A_FP16 multiplies X itself (weight-only fork).  ws (device) >= the size query. */
+ * act_fmt = CHAM_A_FP16 multiplies X itself (weight-only fork).  ws (device) >= the size query.
+ * Which tensor cores multiply (Sec. 3.6: native FP8 and MX kernels): the class-0 tiles of a 4-bit
+ * per-channel layout (INT4-sym, INT4-asym, E2M1, MXINT4, MXFP4 -- every decoded value an exact E4M3
+ * number) against E4M3, E5M2 or MXFP8 activations run kind::mxf8f6f4 MMAs on the 1-byte codes,
+ * with the MX exponents of both sides as block scale factors, unless desc->f16_only is set; every
+ * other tile runs kind::f16 MMAs on exact fp16 operands.  Both give the same products; the sums
+ * differ only in accumulation order. */
 cham_status chameleon_linear(const void* X, int M, const cham_wpack_desc* desc, const void* blob,
                              int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
                              int* dev_status, void* stream);
 
 /* The two halves of chameleon_linear, for callers that schedule or time them separately.
- * chameleon_linear_prepare quantizes X (device, fp16 M x K) in act_fmt into ws (the GEMM operand:
- * the exact fp16 value of every code, R13, plus the per-tensor scale; nothing for CHAM_A_FP16).
- * chameleon_linear_gemm multiplies that operand (or X itself for CHAM_A_FP16; X may be NULL
- * otherwise) with the packed weights.  Same arguments, workspace and errors as chameleon_linear. */
-cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, void* ws, size_t ws_bytes,
-                                     int* dev_status, void* stream);
+ * chameleon_linear_prepare quantizes X (device, fp16 M x desc->K) in act_fmt into ws: the GEMM
+ * operands that the layer *desc's tiles need (the exact fp16 value of every code, R13, and / or the
+ * 1-byte codes, see chameleon_linear_workspace_size) plus the per-tensor scale; nothing for
+ * CHAM_A_FP16.  chameleon_linear_gemm multiplies them (or X itself for CHAM_A_FP16; X may be NULL
+ * otherwise) with the packed weights.  Same arguments, workspace and errors as chameleon_linear;
+ * prepare and gemm of one layer take the same desc (its f16_only fixes which operands exist). */
+cham_status chameleon_linear_prepare(const void* X, int M, const cham_wpack_desc* desc, int act_fmt, void* ws,
+                                     size_t ws_bytes, int* dev_status, void* stream);
 /* chameleon_linear_prepare on the static path of Alg. 2: the operand is quantized with *params
  * (host; see chameleon_act_quant_static for its checks and for MX / FP16, which ignore it) in
  * one pass.  Same workspace as chameleon_linear_prepare; chameleon_linear_gemm then multiplies it. */
-cham_status chameleon_linear_prepare_static(const void* X, int M, int K, int act_fmt, const cham_qparams* params,
-                                            void* ws, size_t ws_bytes, int* dev_status, void* stream);
+cham_status chameleon_linear_prepare_static(const void* X, int M, const cham_wpack_desc* desc, int act_fmt,
+                                            const cham_qparams* params, void* ws, size_t ws_bytes, int* dev_status,
+                                            void* stream);
 cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* desc, const void* blob,
                                   int act_fmt, const float* bias, float* Y, void* ws, size_t ws_bytes,
                                   int* dev_status, void* stream);
@@ -354,8 +370,8 @@ cham_status chameleon_linear_gemm(const void* X, int M, const cham_wpack_desc* d
  * MX formats and FP16 have no per-tensor scale: for them n_groups is only checked.
  * CHAM_ERR_INVALID_ARG unless 1 <= n_groups <= CHAM_MAX_GROUPS and n_groups divides M; otherwise
  * as chameleon_linear_prepare (same workspace). */
-cham_status chameleon_linear_prepare_groups(const void* X, int M, int K, int act_fmt, int n_groups, void* ws,
-                                            size_t ws_bytes, int* dev_status, void* stream);
+cham_status chameleon_linear_prepare_groups(const void* X, int M, const cham_wpack_desc* desc, int act_fmt,
+                                            int n_groups, void* ws, size_t ws_bytes, int* dev_status, void* stream);
 
 /* chameleon_linear_gemm with the operand's row groups and a choice of output type.  n_groups must
  * be the one the operand was prepared with (1 after chameleon_linear_prepare or
@@ -368,12 +384,13 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
                                      int act_fmt, int n_groups, const float* bias, void* Y, int y_type, void* ws,
                                      size_t ws_bytes, int* dev_status, void* stream);
 
-/* Test hook, not part of the method: the next chameleon_linear_gemm (or chameleon_linear) launch
- * on this host thread's library instance has the producer of its first CTA withhold the copies of
- * that CTA's K-chunk number `chunk` (0-based over its work), so the decoders' bounded wait for it
- * runs out: the kernel records CHAM_ERR_TIMEOUT in the call's device status word, drains its own
- * copies and MMAs, releases tensor memory and returns within a few seconds, leaving the context
- * usable (the output of that call is undefined).  chunk = -1 cancels.  Host-only, no GPU work. */
+/* Test hook, not part of the method: the next chameleon_linear_gemm (or chameleon_linear) call
+ * made by this host thread has the producer of the first CTA of its first GEMM launch withhold the
+ * copies of that CTA's K-chunk number `chunk` (0-based over its work), so the decoders' bounded
+ * wait for it runs out: the kernel records CHAM_ERR_TIMEOUT in the call's device status word,
+ * drains its own copies and MMAs, releases tensor memory and returns within a few seconds, leaving
+ * the context usable (the output of that call is undefined).  chunk = -1 cancels.  Host-only, no
+ * GPU work. */
 cham_status chameleon_debug_stall_next_gemm(int chunk);
 
 /* chameleon_act_quant without a caller-supplied workspace.  The paper has no counterpart: this
@@ -385,7 +402,8 @@ cham_status chameleon_debug_stall_next_gemm(int chunk);
  * 1024 x 16 bytes (16 KiB, held on every GPU that loads the library until exit); this fits any
  * M, K on GPUs with up to 256 SMs and returns CHAM_ERR_WORKSPACE (nothing launched) otherwise.
  * It calls no allocator.  The first call on a device looks up the array's address with that
- * device current: make it before any stream capture.  All calls share the array; calls whose
+ * device current: make it before any stream capture.  That address is kept until exit, so the
+ * entry point must not be used on a device after cudaDeviceReset (the array may then move).  All calls share the array; calls whose
  * kernels overlap on the GPU (e.g. concurrent streams) race on it and give wrong results.
  * Errors are returned as status codes only (chameleon_last_error_detail is not updated). */
 cham_status chameleon_act_quant_noalloc(const void* X, int M, int K, int fmt, void* qact, size_t qact_bytes,

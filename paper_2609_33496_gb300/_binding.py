@@ -53,7 +53,7 @@ class WPackDesc(ctypes.Structure):
                 ("off_zero", ctypes.c_uint64), ("off_e8m0", ctypes.c_uint64),
                 ("off_fmt", ctypes.c_uint64), ("off_perm", ctypes.c_uint64),
                 ("bytes", ctypes.c_uint64), ("off_gscale", ctypes.c_uint64),
-                ("reserved", ctypes.c_uint8 * 112)]
+                ("f16_only", ctypes.c_int32), ("reserved", ctypes.c_uint8 * 108)]
 
 
 assert ctypes.sizeof(WPackDesc) == 256
@@ -111,14 +111,14 @@ def lib():
         "chameleon_pack_weights": (i32, [vp, vp, pdesc, vp, sz, vp, vp]),
         "chameleon_linear_workspace_size": (i32, [i32, pdesc, i32, psz]),
         "chameleon_linear": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
-        "chameleon_linear_prepare": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
+        "chameleon_linear_prepare": (i32, [vp, i32, pdesc, i32, vp, sz, vp, vp]),
         "chameleon_linear_gemm": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
         "chameleon_act_quant_noalloc": (i32, [vp, i32, i32, i32, vp, sz, vp, vp]),
         "chameleon_debug_stall_next_gemm": (i32, [i32]),
         "chameleon_scale_zp": (i32, [i32, ctypes.c_float, ctypes.c_float, ctypes.POINTER(QParams)]),
         "chameleon_act_quant_static": (i32, [vp, i32, i32, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
-        "chameleon_linear_prepare_static": (i32, [vp, i32, i32, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
-        "chameleon_linear_prepare_groups": (i32, [vp, i32, i32, i32, i32, vp, sz, vp, vp]),
+        "chameleon_linear_prepare_static": (i32, [vp, i32, pdesc, i32, ctypes.POINTER(QParams), vp, sz, vp, vp]),
+        "chameleon_linear_prepare_groups": (i32, [vp, i32, pdesc, i32, i32, vp, sz, vp, vp]),
         "chameleon_linear_gemm_ex": (i32, [vp, i32, pdesc, vp, i32, i32, vp, vp, i32, vp, sz, vp, vp]),
         "chameleon_act_format_sse_workspace_size": (i32, [i32, i32, psz]),
         "chameleon_act_format_sse": (i32, [vp, i32, i32, vp, vp, sz, vp, vp]),
@@ -471,7 +471,7 @@ def linear_static(X, desc, blob, act_fmt, params, bias=None, Y=None, ws=None, de
         Y = torch.empty((M, desc.N), dtype=torch.float32, device=X.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
-    linear_prepare_static(X, act_fmt, params, ws, dev_status, stream)
+    linear_prepare_static(X, desc, act_fmt, params, ws, dev_status, stream)
     linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream)
     return Y, dev_status
 
@@ -484,12 +484,11 @@ def _y_type(Y):
     return t
 
 
-def linear_prepare_groups(X, act_fmt, n_groups, ws, dev_status, stream=None):
+def linear_prepare_groups(X, desc, act_fmt, n_groups, ws, dev_status, stream=None):
     """First half of linear with per-sample scales: rows in n_groups equal groups, each quantized
-    with the ScaleZP of its own range."""
-    M, K = X.shape
-    check(lib().chameleon_linear_prepare_groups(_half(X, "X"), M, K, act_fmt, n_groups, _ptr(ws), ws.numel(),
-                                                _ptr(dev_status), _stream(stream)))
+    with the ScaleZP of its own range, into the operands the layer desc's tiles need."""
+    check(lib().chameleon_linear_prepare_groups(_half(X, "X"), X.shape[0], ctypes.byref(desc), act_fmt, n_groups,
+                                                _ptr(ws), ws.numel(), _ptr(dev_status), _stream(stream)))
 
 
 def linear_gemm_ex(X, desc, blob, act_fmt, n_groups, bias, Y, ws, dev_status, stream=None):
@@ -511,7 +510,7 @@ def linear_ex(X, desc, blob, act_fmt, n_groups=1, y_dtype=None, bias=None, Y=Non
         Y = torch.empty((M, desc.N), dtype=y_dtype or torch.float32, device=X.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
-    linear_prepare_groups(X, act_fmt, n_groups, ws, dev_status, stream)
+    linear_prepare_groups(X, desc, act_fmt, n_groups, ws, dev_status, stream)
     linear_gemm_ex(X, desc, blob, act_fmt, n_groups, bias, Y, ws, dev_status, stream)
     return Y, dev_status
 
@@ -521,18 +520,17 @@ def debug_stall_next_gemm(chunk):
     check(lib().chameleon_debug_stall_next_gemm(chunk))
 
 
-def linear_prepare(X, act_fmt, ws, dev_status, stream=None):
-    """First half of linear: quantize X into the workspace operand."""
-    M, K = X.shape
-    check(lib().chameleon_linear_prepare(_half(X, "X"), M, K, act_fmt, _ptr(ws), ws.numel(), _ptr(dev_status),
-                                         _stream(stream)))
+def linear_prepare(X, desc, act_fmt, ws, dev_status, stream=None):
+    """First half of linear: quantize X into the workspace operands the layer desc's tiles need."""
+    check(lib().chameleon_linear_prepare(_half(X, "X"), X.shape[0], ctypes.byref(desc), act_fmt, _ptr(ws),
+                                         ws.numel(), _ptr(dev_status), _stream(stream)))
 
 
-def linear_prepare_static(X, act_fmt, params, ws, dev_status, stream=None):
+def linear_prepare_static(X, desc, act_fmt, params, ws, dev_status, stream=None):
     """First half of linear on the static path: quantize X with fixed parameters (QParams)."""
-    M, K = X.shape
-    check(lib().chameleon_linear_prepare_static(_half(X, "X"), M, K, act_fmt, _pref(params), _ptr(ws), ws.numel(),
-                                                _ptr(dev_status), _stream(stream)))
+    check(lib().chameleon_linear_prepare_static(_half(X, "X"), X.shape[0], ctypes.byref(desc), act_fmt,
+                                                _pref(params), _ptr(ws), ws.numel(), _ptr(dev_status),
+                                                _stream(stream)))
 
 
 def linear_gemm(X, desc, blob, act_fmt, bias, Y, ws, dev_status, stream=None):

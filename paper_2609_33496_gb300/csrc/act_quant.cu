@@ -316,7 +316,8 @@ CHAM_DEV void encode8_mx(const uint4& v, int lane, uint2& code, uint4& deq, int&
 template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_mx(const uint4* __restrict__ X, int64_t nvec, uint2* __restrict__ codes, uint4* __restrict__ deq,
-                    uint8_t* __restrict__ e8m0, cham_qparams* __restrict__ params, int* dev_status) {
+                    uint8_t* __restrict__ e8m0, uint8_t* __restrict__ e8cm, int kblocks, int64_t cm_plane,
+                    cham_qparams* __restrict__ params, int* dev_status) {
   griddep_wait();  // its outputs may still be read by the previous kernel
   griddep_launch_dependents();
   if (blockIdx.x == 0 && threadIdx.x == 0 && params != nullptr) *params = cham_qparams{1.f, 0, 1.f, FMT};
@@ -343,6 +344,11 @@ __global__ void __launch_bounds__(256)
         if constexpr (CODES) codes[i] = c;
         if constexpr (DEQ) deq[i] = d;
         if (e8m0 != nullptr && (lane & 3) == 0) e8m0[i >> 2] = static_cast<uint8_t>(byte);
+        if (e8cm != nullptr && (lane & 3) == 0) {  // chunk-major copy for the FP8 GEMM
+          const int64_t blk = i >> 2, m = blk / kblocks;
+          const int kb = static_cast<int>(blk - m * kblocks);
+          e8cm[(kb >> 2) * cm_plane + m * 4 + (kb & 3)] = static_cast<uint8_t>(byte);
+        }
       }
     }
   }
@@ -559,7 +565,7 @@ static void launch_mx(const ActQuantArgs& a, cudaStream_t st) {
   if (g > cap) g = cap;
   if (g < 1) g = 1;
   launch_pdl(k_act_encode_mx<FMT, CODES, DEQ>, dim3(static_cast<int>(g)), dim3(256), 0, st, a.X, a.nvec, a.codes,
-             a.deq, a.e8m0, a.params, a.dev_status);
+             a.deq, a.e8m0, a.e8cm, a.kblocks, a.cm_plane, a.params, a.dev_status);
 }
 
 template <bool CODES, bool DEQ>

@@ -31,6 +31,10 @@ struct ActQuantArgs {
   uint2* codes;            // 8 code bytes per vector, or null
   uint4* deq;              // 8 exact fp16 operand values per vector, or null
   uint8_t* e8m0;           // MX formats: one byte per 4 vectors, or null
+  uint8_t* e8cm;           // MX formats, FP8 GEMM operand: the same bytes chunk-major, or null:
+                           // block kb of row m at e8cm[(kb / 4) * cm_plane + 4 m + kb % 4]
+  int kblocks;             // K / 32 (blocks per row), with e8cm
+  int64_t cm_plane;        // bytes per chunk of 4 blocks in e8cm
   cham_qparams* params;    // per-tensor parameters, or null
   float* scale_out;        // the per-tensor (per-group) scale s as bare floats (GEMM epilogue), or null
   int* dev_status;

@@ -131,15 +131,17 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// Row-major fp16 matrix rows x cols, box = 64 columns (128 bytes) x box_rows, 128-byte swizzle.
-cham_status make_act_map(CUtensorMap* map, const void* base, int rows, int cols, int box_rows) {
+// Row-major matrix rows x cols of fp16 (esize 2) or bytes (esize 1), box = 128 bytes of a row x
+// box_rows rows, 128-byte swizzle.
+cham_status make_act_map(CUtensorMap* map, const void* base, int rows, int cols, int box_rows, int esize) {
   EncodeTiledFn fn = encode_fn();
   if (fn == nullptr) return fail(CHAM_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
-  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * esize};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(128 / esize), static_cast<cuuint32_t>(box_rows)};
   const cuuint32_t estr[2] = {1, 1};
-  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  const CUresult r = fn(map, esize == 2 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 2,
+                        const_cast<void*>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(CHAM_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
@@ -198,25 +200,62 @@ const int kClassOrder[2][5] = {{CHAM_W_INT4_SYM, CHAM_W_INT4_ASYM, CHAM_W_E2M1, 
 
 cham_status check_desc(const cham_wpack_desc* d) {
   if (d == nullptr) return fail(CHAM_ERR_INVALID_ARG, "descriptor is NULL");
-  if (d->magic != 0x574D4843u || d->version != 2) return fail(CHAM_ERR_INVALID_ARG, "not a packed-weight descriptor");
+  if (d->magic != 0x574D4843u || d->version != 3) return fail(CHAM_ERR_INVALID_ARG, "not a packed-weight descriptor");
   if (d->N <= 0 || d->K <= 0 || d->K % 32 != 0 || (d->bits != 4 && d->bits != 8))
     return fail(CHAM_ERR_INVALID_ARG, "descriptor sizes are invalid");
   if (d->group < 0 || d->group % 32 != 0 || (d->group > 0 && (d->K + d->group - 1) / d->group > cham::kMaxRowGroups))
     return fail(CHAM_ERR_INVALID_ARG, "descriptor group size %d", d->group);
+  if (d->f16_only != 0 && d->f16_only != 1) return fail(CHAM_ERR_INVALID_ARG, "descriptor f16_only %d", d->f16_only);
   return CHAM_OK;
 }
 
 
-// Byte offsets inside the linear workspace.
-struct LinearWs {
-  size_t scale, parts, operand;
+// Which GEMM operands a layer's tiles need (Sec. 3.6): the class-0 tiles of a 4-bit per-channel
+// layout run on FP8 MMAs against E4M3 / E5M2 / MXFP8 codes (unless the descriptor asks for fp16
+// only); every other tile needs the exact fp16 operand (none for CHAM_A_FP16, which reads X).
+struct OperandPlan {
+  bool fp8;   // class-0 tiles on the FP8 kernel (1-byte codes, MXFP8: chunk-major exponents)
+  bool f16;   // tiles on the fp16 kernel
+  int f16_tile0, f16_tiles;
 };
-// scale: one float per row group (kMaxGroups); parts: the range partials of every group
-LinearWs linear_ws(int M, int K) {
+OperandPlan operand_plan(const cham_wpack_desc* d, int act_fmt) {
+  const bool fp8_act = act_fmt == CHAM_A_E4M3 || act_fmt == CHAM_A_E5M2 || act_fmt == CHAM_A_MXFP8;
+  OperandPlan o;
+  o.fp8 = fp8_act && d->bits == 4 && d->group == 0 && d->f16_only == 0 && d->n_tiles[0] > 0;
+  o.f16_tile0 = o.fp8 ? d->n_tiles[0] : 0;
+  o.f16_tiles = d->n_tiles[0] + d->n_tiles[1] - o.f16_tile0;
+  o.f16 = o.f16_tiles > 0;
+  return o;
+}
+
+// Byte offsets inside the linear workspace (each region 256-byte aligned): the activation scale
+// per row group, the range partials, the fp16 operand, the 1-byte codes, the MXFP8 exponents
+// chunk-major, then (gemm_plan) the split-K partial sums.
+struct LinearWs {
+  size_t scale, parts, operand, codes, e8, end;
+  int mp;  // rows per chunk of the exponent region
+};
+LinearWs linear_ws(int M, const cham_wpack_desc* d, int act_fmt) {
   static_assert(cham::kMaxGroups == CHAM_MAX_GROUPS && cham::kMaxGroups * sizeof(float) <= 256, "scale slots");
+  const int K = d->K;
   const int64_t nvec = static_cast<int64_t>(M) * K / 8;
   const int parts = std::max(cham::range_grid(nvec, num_sms_current()), cham::kMaxGroups);
-  return LinearWs{0, 256, 256 + round_up(static_cast<size_t>(parts) * sizeof(cham::RangePartial), 256)};
+  const OperandPlan o = operand_plan(d, act_fmt);
+  LinearWs L{};
+  L.scale = 0;
+  L.parts = 256;
+  // CHAM_A_FP16 multiplies X itself: no quantizer, only the scale slot precedes the partial sums
+  size_t off = act_fmt == CHAM_A_FP16 ? 256 : 256 + round_up(static_cast<size_t>(parts) * sizeof(cham::RangePartial), 256);
+  L.mp = (M + 3) / 4 * 4;
+  const size_t mk = static_cast<size_t>(M) * K;
+  L.operand = off;
+  if (o.f16 && act_fmt != CHAM_A_FP16) off += round_up(mk * 2, 256);
+  L.codes = off;
+  if (o.fp8) off += round_up(mk, 256);
+  L.e8 = off;
+  if (o.fp8 && act_fmt == CHAM_A_MXFP8) off += round_up(static_cast<size_t>((K + 127) / 128) * L.mp * 4, 256);
+  L.end = off;
+  return L;
 }
 
 cham_status check_groups(int M, int n_groups) {
@@ -233,25 +272,31 @@ cham_status check_linear_common(int M, int K, int act_fmt, void* ws, size_t ws_b
   return CHAM_OK;
 }
 
-size_t linear_ws_need(int M, int K, int act_fmt) {
-  if (act_fmt == CHAM_A_FP16) return 256;
-  return linear_ws(M, K).operand + round_up(static_cast<size_t>(M) * K * 2, 256);
-}
-
-// The GEMM's split-K factor and its partial-sum region, which follows the operand region.
+// The GEMM launches of a layer (FP8 kernel over the class-0 tiles, fp16 kernel over the rest):
+// token tile and split-K factor of each, and the partial-sum region after the operands (shared:
+// the two launches write disjoint packed channels of it).
 struct GemmPlan {
-  int bn, k_split;
+  int bn8, ks8, bn16, ks16;
   size_t partial, need;
 };
 GemmPlan gemm_plan(int M, const cham_wpack_desc* d, int act_fmt) {
-  GemmPlan g;
+  GemmPlan g{};
   const int num_sms = num_sms_current();
+  const OperandPlan o = operand_plan(d, act_fmt);
   const int ch_tiles = d->n_tiles[0] + d->n_tiles[1];
-  g.bn = cham::gemm_pick_bn(M, ch_tiles, num_sms);
-  const int tiles = ch_tiles * ((M + g.bn - 1) / g.bn);
-  g.k_split = cham::gemm_pick_split(tiles, d->Kp / 64, num_sms);
-  g.partial = linear_ws_need(M, d->K, act_fmt);
-  g.need = g.partial + (g.k_split > 1 ? round_up(static_cast<size_t>(g.k_split) * M * 128 * ch_tiles * 4, 256) : 0);
+  int ks_max = 1;
+  if (o.fp8) {
+    g.bn8 = cham::gemm_pick_bn_f8(M);
+    g.ks8 = cham::gemm_pick_split(d->n_tiles[0] * ((M + g.bn8 - 1) / g.bn8), (d->Kp / 64 + 1) / 2, num_sms);
+    ks_max = std::max(ks_max, g.ks8);
+  }
+  if (o.f16) {
+    g.bn16 = cham::gemm_pick_bn(M, o.f16_tiles, num_sms);
+    g.ks16 = cham::gemm_pick_split(o.f16_tiles * ((M + g.bn16 - 1) / g.bn16), d->Kp / 64, num_sms);
+    ks_max = std::max(ks_max, g.ks16);
+  }
+  g.partial = linear_ws(M, d, act_fmt).end;
+  g.need = g.partial + (ks_max > 1 ? round_up(static_cast<size_t>(ks_max) * M * 128 * ch_tiles * 4, 256) : 0);
   return g;
 }
 
@@ -275,7 +320,7 @@ const char* chameleon_status_string(cham_status s) {
 
 const char* chameleon_last_error_detail(void) { return g_detail; }
 
-int chameleon_version(void) { return 2; }
+int chameleon_version(void) { return 3; }
 
 cham_status chameleon_check(const int* dev_status, void* stream) {
   if (dev_status == nullptr) return fail(CHAM_ERR_INVALID_ARG, "dev_status is NULL");
@@ -688,7 +733,7 @@ cham_status chameleon_pack_plan_grouped(int N, int K, int fmt, int group, cham_w
 namespace {
 void finish_plan(cham_wpack_desc* d, int N, int K, int bits) {
   d->magic = 0x574D4843u;
-  d->version = 2;
+  d->version = 3;
   d->N = N;
   d->K = K;
   d->Kp = static_cast<int>(round_up(K, 64));
@@ -803,69 +848,80 @@ cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* d, int
 }  // extern "C"
 
 
-extern "C" {
-
-cham_status chameleon_linear_prepare(const void* X, int M, int K, int act_fmt, void* ws, size_t ws_bytes,
-                                     int* dev_status, void* stream) {
-  return chameleon_linear_prepare_groups(X, M, K, act_fmt, 1, ws, ws_bytes, dev_status, stream);
-}
-
-cham_status chameleon_linear_prepare_groups(const void* X, int M, int K, int act_fmt, int n_groups, void* ws,
-                                            size_t ws_bytes, int* dev_status, void* stream) {
-  cham_status s = check_act_args(X, M, K, act_fmt, true);
+namespace {
+// The prepare calls (Alg. 3 dynamic per tensor or per sample, or Alg. 2 static): quantize X into
+// the operands the layer's tiles need (operand_plan) -- one quantizer pass writes both when both
+// kernels run.
+cham_status prepare_common(const void* X, int M, const cham_wpack_desc* d, int act_fmt, int n_groups,
+                           const cham_qparams* params, bool is_static, void* ws, size_t ws_bytes, int* dev_status,
+                           void* stream) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  const int K = d->K;
+  s = check_act_args(X, M, K, act_fmt, true);
   if (s != CHAM_OK) return s;
   s = check_groups(M, n_groups);
   if (s != CHAM_OK) return s;
-  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
+  if (is_static) {
+    s = check_static_params(act_fmt, params);
+    if (s != CHAM_OK) return s;
+  }
+  const LinearWs L = linear_ws(M, d, act_fmt);
+  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, L.end);
   if (s != CHAM_OK) return s;
   if (act_fmt == CHAM_A_FP16) return CHAM_OK;
+  const OperandPlan o = operand_plan(d, act_fmt);
   uint8_t* w = static_cast<uint8_t*>(ws);
-  const LinearWs L = linear_ws(M, K);
   cham::ActQuantArgs a{};
   a.X = static_cast<const uint4*>(X);
   a.nvec = static_cast<int64_t>(M) * K / 8;
   a.num_sms = num_sms_current();
-  a.parts = reinterpret_cast<cham::RangePartial*>(w + L.parts);
-  a.n_groups = act_fmt <= CHAM_A_E5M2 ? n_groups : 1;
-  a.nparts = cham::group_grid(a.nvec, a.n_groups, a.num_sms);
-  a.codes = nullptr;
-  a.deq = reinterpret_cast<uint4*>(w + L.operand);
+  a.codes = o.fp8 ? reinterpret_cast<uint2*>(w + L.codes) : nullptr;
+  a.deq = o.f16 ? reinterpret_cast<uint4*>(w + L.operand) : nullptr;
   a.e8m0 = nullptr;
+  if (o.fp8 && act_fmt == CHAM_A_MXFP8) {
+    a.e8cm = w + L.e8;
+    a.kblocks = K / 32;
+    a.cm_plane = static_cast<int64_t>(L.mp) * 4;
+  }
   a.params = nullptr;
   a.scale_out = act_fmt <= CHAM_A_E5M2 ? reinterpret_cast<float*>(w + L.scale) : nullptr;
   a.dev_status = dev_status;
-  cham::launch_act_quant(act_fmt, a, false, true, static_cast<cudaStream_t>(stream));
+  if (is_static) {
+    a.use_static = true;
+    a.stat = tensor_params(params);
+  } else {
+    a.parts = reinterpret_cast<cham::RangePartial*>(w + L.parts);
+    a.n_groups = act_fmt <= CHAM_A_E5M2 ? n_groups : 1;
+    a.nparts = cham::group_grid(a.nvec, a.n_groups, a.num_sms);
+  }
+  cham::launch_act_quant(act_fmt, a, a.codes != nullptr, a.deq != nullptr, static_cast<cudaStream_t>(stream));
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "linear_prepare launch");
 }
+}  // namespace
 
-cham_status chameleon_linear_prepare_static(const void* X, int M, int K, int act_fmt, const cham_qparams* params,
-                                            void* ws, size_t ws_bytes, int* dev_status, void* stream) {
-  cham_status s = check_act_args(X, M, K, act_fmt, true);
-  if (s != CHAM_OK) return s;
-  s = check_static_params(act_fmt, params);
-  if (s != CHAM_OK) return s;
-  s = check_linear_common(M, K, act_fmt, ws, ws_bytes, linear_ws_need(M, K, act_fmt));
-  if (s != CHAM_OK) return s;
-  if (act_fmt == CHAM_A_FP16) return CHAM_OK;
-  uint8_t* w = static_cast<uint8_t*>(ws);
-  const LinearWs L = linear_ws(M, K);
-  cham::ActQuantArgs a{};
-  a.X = static_cast<const uint4*>(X);
-  a.nvec = static_cast<int64_t>(M) * K / 8;
-  a.num_sms = num_sms_current();
-  a.deq = reinterpret_cast<uint4*>(w + L.operand);
-  a.scale_out = act_fmt <= CHAM_A_E5M2 ? reinterpret_cast<float*>(w + L.scale) : nullptr;
-  a.dev_status = dev_status;
-  a.use_static = true;
-  a.stat = tensor_params(params);
-  cham::launch_act_quant(act_fmt, a, false, true, static_cast<cudaStream_t>(stream));
-  const cudaError_t e = cudaGetLastError();
-  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "linear_prepare_static launch");
+extern "C" {
+
+cham_status chameleon_linear_prepare(const void* X, int M, const cham_wpack_desc* d, int act_fmt, void* ws,
+                                     size_t ws_bytes, int* dev_status, void* stream) {
+  return prepare_common(X, M, d, act_fmt, 1, nullptr, false, ws, ws_bytes, dev_status, stream);
+}
+
+cham_status chameleon_linear_prepare_groups(const void* X, int M, const cham_wpack_desc* d, int act_fmt,
+                                            int n_groups, void* ws, size_t ws_bytes, int* dev_status, void* stream) {
+  return prepare_common(X, M, d, act_fmt, n_groups, nullptr, false, ws, ws_bytes, dev_status, stream);
+}
+
+cham_status chameleon_linear_prepare_static(const void* X, int M, const cham_wpack_desc* d, int act_fmt,
+                                            const cham_qparams* params, void* ws, size_t ws_bytes, int* dev_status,
+                                            void* stream) {
+  return prepare_common(X, M, d, act_fmt, 1, params, true, ws, ws_bytes, dev_status, stream);
 }
 
 namespace {
-std::atomic<int> g_stall_next_gemm{-1};  // set by chameleon_debug_stall_next_gemm, taken by the next launch
+// set by chameleon_debug_stall_next_gemm, taken by the next GEMM call of the same host thread
+thread_local int g_stall_next_gemm = -1;
 }  // namespace
 
 cham_status chameleon_debug_stall_next_gemm(int chunk) {
@@ -897,10 +953,11 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   if (blob == nullptr || Y == nullptr || !aligned16(blob) || !aligned16(Y) || (bias != nullptr && !aligned16(bias)))
     return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
   uint8_t* w = static_cast<uint8_t*>(ws);
-  const LinearWs L = linear_ws(M, K);
-  const void* operand = act_fmt == CHAM_A_FP16 ? X : static_cast<const void*>(w + L.operand);
+  const LinearWs L = linear_ws(M, d, act_fmt);
+  const OperandPlan o = operand_plan(d, act_fmt);
   const float* act_scale = act_fmt <= CHAM_A_E5M2 ? reinterpret_cast<const float*>(w + L.scale) : nullptr;
   const uint8_t* b = static_cast<const uint8_t*>(blob);
+  const int tiles = d->n_tiles[0] + d->n_tiles[1];
   cham::GemmArgs g{};
   g.codes = b + d->off_codes;
   g.wscale = reinterpret_cast<const float*>(b + d->off_scale);
@@ -916,9 +973,12 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   g.rows_per_group = act_fmt <= CHAM_A_E5M2 ? M / n_groups : M;
   g.M = M;
   g.N = d->N;
-  g.n_chunks = d->Kp / 64;
   g.bits = d->bits;
-  g.stall_chunk = g_stall_next_gemm.exchange(-1);
+  g.Np = 128 * tiles;
+  g.nk64 = d->Kp / 64;
+  g.kblocks = K / 32;
+  g.stall_chunk = g_stall_next_gemm;
+  g_stall_next_gemm = -1;
   g.dev_status = dev_status;
   const cham::NF4Table& nf4 = nf4_table();
   for (int r = 0; r < 4; ++r) {
@@ -929,25 +989,49 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
     }
   }
   const int num_sms = num_sms_current();
-  const int tiles = d->n_tiles[0] + d->n_tiles[1];
-  const int bn = plan.bn;
-  CUtensorMap map;
-  s = make_act_map(&map, operand, M, K, bn);
-  if (s != CHAM_OK) return s;
-  g.tile0 = 0;
-  g.n_ch_tiles = tiles;
-  g.Np = 128 * tiles;
-  g.k_split = plan.k_split;
-  g.partial = plan.k_split > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
-  const cudaError_t e = cham::launch_gemm_f16(map, g, num_sms, bn, static_cast<cudaStream_t>(stream));
-  return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "gemm launch");
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (o.fp8) {
+    // class-0 tiles on FP8 MMAs: the 1-byte codes (K-major rows of K bytes), chunks of 128
+    cham::GemmArgs g8 = g;
+    CUtensorMap map8;
+    s = make_act_map(&map8, w + L.codes, M, K, plan.bn8, 1);
+    if (s != CHAM_OK) return s;
+    g8.tile0 = 0;
+    g8.n_ch_tiles = d->n_tiles[0];
+    g8.n_chunks = (g.nk64 + 1) / 2;
+    g8.k_split = plan.ks8;
+    g8.partial = plan.ks8 > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
+    g8.b_fmt = act_fmt == CHAM_A_E5M2 ? 1 : 0;
+    if (act_fmt == CHAM_A_MXFP8) {
+      g8.act_e8 = w + L.e8;
+      g8.act_mp = L.mp;
+      g8.act_e8_plane = static_cast<int64_t>(L.mp) * 4;
+    }
+    const cudaError_t e = cham::launch_gemm_f8(map8, g8, num_sms, plan.bn8, st);
+    if (e != cudaSuccess) return cuda_fail(e, "fp8 gemm launch");
+    g.stall_chunk = -1;
+  }
+  if (o.f16) {
+    const void* operand = act_fmt == CHAM_A_FP16 ? X : static_cast<const void*>(w + L.operand);
+    CUtensorMap map;
+    s = make_act_map(&map, operand, M, K, plan.bn16, 2);
+    if (s != CHAM_OK) return s;
+    g.tile0 = o.f16_tile0;
+    g.n_ch_tiles = o.f16_tiles;
+    g.n_chunks = g.nk64;
+    g.k_split = plan.ks16;
+    g.partial = plan.ks16 > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
+    const cudaError_t e = cham::launch_gemm_f16(map, g, num_sms, plan.bn16, st);
+    if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
+  }
+  return CHAM_OK;
 }
 
 cham_status chameleon_linear(const void* X, int M, const cham_wpack_desc* d, const void* blob, int act_fmt,
                              const float* bias, float* Y, void* ws, size_t ws_bytes, int* dev_status, void* stream) {
   cham_status s = check_desc(d);
   if (s != CHAM_OK) return s;
-  s = chameleon_linear_prepare(X, M, d->K, act_fmt, ws, ws_bytes, dev_status, stream);
+  s = chameleon_linear_prepare(X, M, d, act_fmt, ws, ws_bytes, dev_status, stream);
   if (s != CHAM_OK) return s;
   return chameleon_linear_gemm(X, M, d, blob, act_fmt, bias, Y, ws, ws_bytes, dev_status, stream);
 }

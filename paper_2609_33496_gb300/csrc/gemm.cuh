@@ -31,20 +31,49 @@ struct GemmArgs {
   int* dev_status;
   uint32_t nf4_lo[4];        // NF4 levels as fp16: low bytes of levels 4r..4r+3 in word r
   uint32_t nf4_hi[4];        // high bytes, same layout
+  // FP8 kernel only (n_chunks then counts chunks of 128 elements)
+  const uint8_t* act_e8;     // MXFP8 activations: E8M0 [n_chunks][act_mp][4] (chunk-major), else null
+  int64_t act_e8_plane;      // bytes per chunk of act_e8 (act_mp * 4)
+  int act_mp;                // rows per chunk of act_e8: M rounded up to 4
+  int kblocks;               // K / 32
+  int nk64;                  // 64-element chunks of the blob (Kp / 64)
+  int b_fmt;                 // activation element type of the MMA: 0 E4M3, 1 E5M2
 };
+
+// Token tile of the FP8 kernel for M > 128: 160 leaves room in tensor memory for the scale factors
+// next to two accumulators and four decoded-weight slots.
+constexpr int kF8TokenTile = 160;
 
 // Token-tile (MMA N) size for M tokens: 16, 32, 64, 128 or 192.
 int gemm_pick_bn(int M, int n_tiles, int num_sms);
 // Split-K factor: 1 when the tiles fill the GPU, else enough K ranges (of at least two chunks)
 // to give every SM work.
 int gemm_pick_split(int tiles, int n_chunks, int num_sms);
+// Token tile of the FP8 kernel: 32, 64, 128 or kF8TokenTile.
+int gemm_pick_bn_f8(int M);
 // Persistent launch: min(tiles, num_sms) CTAs walk the (channel tile, token tile) grid.
 cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
+// The FP8 kernel (gemm_f8_kernel.cuh) over the launch's class-0 channel tiles; act_map holds the
+// activation codes (uint8).
+cudaError_t launch_gemm_f8(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
+template <int YT, bool MXA>
+cudaError_t launch_gemm_f8_yt(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
+// Split-K units' raw sums (EPI 6) and the reduction over the launch's tiles.
+cudaError_t launch_splitk_reduce(const GemmArgs& a, int num_sms, cudaStream_t st);
 // The launches of one output type (instantiated in gemm.cu, gemm_f16.cu, gemm_bf16.cu).
 template <int YT>
 cudaError_t launch_gemm_yt(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
 extern template cudaError_t launch_gemm_yt<CHAM_Y_F32>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
 extern template cudaError_t launch_gemm_yt<CHAM_Y_F16>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
 extern template cudaError_t launch_gemm_yt<CHAM_Y_BF16>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+constexpr int kPartialYT = 3;  // "output type" of split-K units: raw fp32 partial sums
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_f8_yt<kPartialYT, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+extern template cudaError_t launch_gemm_f8_yt<kPartialYT, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
 
 }  // namespace cham

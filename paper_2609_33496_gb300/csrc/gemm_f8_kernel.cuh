@@ -1,0 +1,414 @@
+// gemm_f8_kernel.cuh -- the mixed-format linear on 8-bit tensor cores (steps a7, Sec. 3.6): the
+// kernel template for the 4-bit weight channels whose every decoded value is an exact E4M3 number,
+// against FP8 activation codes (E4M3 or E5M2 with a per-tensor scale, or MXFP8 blocks).
+// Instantiated in gemm_f8.cu (per-tensor activations) and gemm_f8_mx.cu (MXFP8 activations).
+//
+// Y[m, perm[p]] = s_a * s_w[p] * sum_b 2^(e_w[p, b] + e_a[m, b]) sum_{k in block b} A^[m, k] W^[p, k] + bias
+//
+// Which weights qualify (MMA class 0 of the packed layout): INT4-sym and INT4-asym (q - z in
+// [-15, 15]), E2M1, and the element values of MXINT4 (code / 4) and MXFP4 -- all are E4M3 values, so
+// the FP8 operand is exact, and the per-32 block exponents of the MX formats ride in the MMA's block
+// scale factors.  The activation codes are the quantizer's own bytes: E4M3 / E5M2 bit patterns with
+// the per-tensor scale s_a applied in the epilogue, or MXFP8 E4M3 elements whose E8M0 exponents are
+// the activation-side scale factors.  The product is the same sum the fp16 path forms from the
+// dequantized operands; only the accumulation order inside the tensor core differs.
+//
+// Structure (as the fp16 kernel in gemm_kernel.cuh, whose epilogue role it shares):
+//   * MMA "A" (M = 128) = 128 packed weight channels decoded into tensor memory, one thread per
+//     channel: every 4-bit code indexes that channel's own 16-entry table of E4M3 bytes (built once
+//     per tile from the format and zero point), so channels of different formats in one tile take
+//     the same instructions.  Two byte permutes per four codes look the table up; the channel's
+//     four block exponents of the chunk go to the A scale-factor columns.
+//   * MMA "B" (N = BN tokens) = 128 activation code bytes per row, loaded by TMA with 128-byte
+//     swizzling; MXFP8 activations also bring their chunk's exponents (4 bytes per token).
+//   * K-chunks of 128 elements: 4 MMAs (kind::mxf8f6f4, K = 32 each, scale vector 1X: one E8M0
+//     per row per MMA, selected by the instruction's scale-factor ids); the last chunk issues only
+//     the MMAs of the 32-element blocks inside K.
+// Tensor-memory columns: two accumulators, four decoded-weight slots of 32 columns, the A scale
+// factors of each slot (8 columns apart, lane m reads column base + m / 32), and the B scale
+// factors (every lane quadrant holds all BN tokens: lane 32q + n % 32, column base + n / 32) --
+// one constant copy for per-tensor activations, one per slot for MXFP8.
+#pragma once
+
+#include "gemm_kernel.cuh"
+
+namespace cham {
+
+constexpr int kBK8 = 128;  // K elements per FP8 chunk: 128 bytes per activation row
+
+template <int BN, bool MXA>
+struct F8Cfg {
+  static constexpr int kBBytes = BN * 128;       // activation codes
+  static constexpr int kWBytes = 2 * 128 * 32;   // two 64-element blob chunks of 4-bit codes
+  static constexpr int kEBytes = 2 * 256;        // their E8M0 pairs
+  static constexpr int kSBytes = MXA ? 1024 : 0; // MXFP8: 4 exponent bytes per token, up to 256 tokens
+  static constexpr int kStage = (kBBytes + kWBytes + kEBytes + kSBytes + 1023) / 1024 * 1024;
+  static constexpr int kStages = (200 * 1024) / kStage > 8 ? 8 : (200 * 1024) / kStage;
+  static constexpr int kData = kStages * kStage;
+  static constexpr int kAccCols = BN < 32 ? 32 : BN;
+  static constexpr int kACol = 2 * kAccCols;
+  static constexpr int kAStages = 4, kGroup = 2, kDone = 8;
+  static constexpr int kSFA = kACol + kAStages * 32;          // slot s: columns kSFA + 8 s .. + 3
+  static constexpr int kSFB = kSFA + kAStages * 8;            // per-tensor: one copy; MXFP8: slot s at + 8 s
+  static constexpr int kSFBCols = (BN + 31) / 32;
+  static constexpr int kNeedCols = kSFB + (MXA ? kAStages * 8 : 8);
+  static constexpr int kTmemCols = kNeedCols <= 256 ? 256 : 512;
+  static constexpr int kMisc = 8 * (kStages + kDone + kAStages / kGroup + 4) + 16;
+  static constexpr int kNeed = 1024 + kData + kMisc;
+  static constexpr int kSmem = kNeed > 116 * 1024 ? kNeed : 116 * 1024;  // one CTA per SM
+  static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "token tile: a multiple of 32 (accumulator columns)");
+  static_assert(kStages >= 4, "ring depth");
+  static_assert(kSmem <= 227 * 1024, "within the opt-in shared-memory limit");
+  static_assert(kNeedCols <= 512, "tensor memory budget");
+  static_assert(kSFBCols <= 8, "B scale factors: 8 columns per copy");
+  static_assert(kDone * kGroup > kStages + kGroup, "group barrier rotation");
+};
+
+// D[tmem] (+)= A[tmem] * B[smem]^T with per-32 block scale factors, kind::mxf8f6f4.
+CHAM_DEV void mma_mxf8_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc, uint32_t sfa,
+                          uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], [%1], %2, %3, [%4], [%5], p;\n\t}\n" ::"r"(
+          d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
+// Instruction descriptor of kind::mxf8f6f4: A E4M3 (weights), B E4M3 or E5M2 (btype 0 / 1), both
+// K-major, M x N, UE8M0 scale factors (bit 23); the A / B scale-factor ids (bits 29-30 / 4-5) pick
+// the byte of the scale-factor column each MMA uses.
+__host__ __device__ constexpr uint32_t idesc_mxf8(int M, int N, int btype) {
+  return (0u << 7) | (static_cast<uint32_t>(btype) << 10) | (static_cast<uint32_t>(N >> 3) << 17) | (1u << 23) |
+         (static_cast<uint32_t>(M >> 4) << 24);
+}
+__host__ __device__ constexpr uint32_t idesc_sf_ids(uint32_t idesc, int i) {
+  return idesc | (static_cast<uint32_t>(i) << 4) | (static_cast<uint32_t>(i) << 29);
+}
+
+CHAM_DEV void tmem_st_32x32b_x1(uint32_t taddr, uint32_t v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(v) : "memory");
+}
+CHAM_DEV void tmem_st_32x32b_x8(uint32_t taddr, const uint32_t (&v)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
+               "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
+
+// Value of 4-bit code n of a class-0 channel in format f (zero point z for INT4-asym): INT4-sym and
+// MXINT4 store q + 8 (MXINT4 elements are q / 4, the block exponent apart), INT4-asym stores q with
+// value q - z, E2M1 and MXFP4 store the sign-exponent-mantissa bits.  Other formats (padding): 0.
+CHAM_DEV float f8_level(int f, int z, int n) {
+  switch (f) {
+    case CHAM_W_INT4_SYM: return static_cast<float>(n - 8);
+    case CHAM_W_MXINT4: return 0.25f * static_cast<float>(n - 8);
+    case CHAM_W_INT4_ASYM: return static_cast<float>(n - z);
+    case CHAM_W_E2M1:
+    case CHAM_W_MXFP4: {
+      const int e = (n >> 1) & 3, m = n & 1;
+      const float mag = e == 0 ? 0.5f * m : exp2i_f32(e - 1) * (1.f + 0.5f * m);
+      return (n & 8) ? -mag : mag;
+    }
+    default: return 0.f;
+  }
+}
+
+// The channel's 16-entry E4M3 table: byte n % 4 of word n / 4 holds the code of f8_level(n)
+// (every level is an E4M3 value, so the conversion is exact).
+CHAM_DEV void f8_table(int f, int z, uint32_t (&T)[4]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) T[i] = 0;
+#pragma unroll
+  for (int n = 0; n < 16; n += 2) {
+    const uint32_t e = cvt_e4m3x2(f8_level(f, z, n + 1), f8_level(f, z, n));
+    T[n >> 2] |= e << (8 * (n & 2));
+  }
+}
+
+// Four codes (the selector nibbles of sel; bit 3 of each code in the byte mask m) -> four table bytes.
+CHAM_DEV uint32_t f8_lookup4(uint32_t sel, uint32_t m, const uint32_t (&T)[4]) {
+  const uint32_t lo = prmt(T[0], T[1], sel), hi = prmt(T[2], T[3], sel);
+  return (lo & ~m) | (hi & m);
+}
+
+// 128 codes of one channel (16 words, word i = elements 8i..8i+7 with nibble j = element 2j for
+// j < 4 and element 2(j - 4) + 1 for j >= 4, the blob's 4-bit order) -> 32 columns of E4M3 bytes,
+// column c = elements 4c..4c+3 (byte order = element order, the MMA's K order in tensor memory).
+CHAM_DEV void decode_f8(const uint32_t (&w)[16], const uint32_t (&T)[4], uint32_t (&out)[32]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const uint32_t x = w[i];
+    const uint32_t s = x & 0x77777777u, x4 = x << 4;
+    // byte mask of each code's bit 3: PRMT with the sign-replicate selector bit copies bit 7 of the
+    // byte that holds that bit (x << 4 for the low nibble of a byte, x for the high one)
+    const uint32_t mlo = prmt(x4, x, 0xD9C8u), mhi = prmt(x4, x, 0xFBEAu);
+    const uint32_t even = f8_lookup4(s, mlo, T);         // elements 0, 2, 4, 6
+    const uint32_t odd = f8_lookup4(s >> 16, mhi, T);    // elements 1, 3, 5, 7
+    out[2 * i] = prmt(even, odd, 0x5140u);
+    out[2 * i + 1] = prmt(even, odd, 0x7362u);
+  }
+}
+
+// MXA: the activations are MXFP8 (their exponents come with every stage); otherwise E4M3 / E5M2
+// codes with a per-tensor (or per-sample) scale and constant unit B scale factors.
+template <int BN, int EPI, bool MXA>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    k_gemm_ts_f8(const __grid_constant__ CUtensorMap act_map, const GemmArgs a) {
+  using C = F8Cfg<BN, MXA>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint32_t* misc = reinterpret_cast<uint32_t*>(smem + C::kData);
+  constexpr int S = C::kStages;
+  constexpr int kAStages = C::kAStages, kGroup = C::kGroup, kAGroups = kAStages / kGroup;
+  constexpr int kDone = C::kDone;
+  constexpr int kDec = Roles<4>::kDec, kEpi = Roles<4>::kEpi;
+  uint64_t* full = reinterpret_cast<uint64_t*>(misc);       // [S] producer -> decoders (tx bytes)
+  uint64_t* done = full + S;                                 // [kDone] MMA group commit -> producer, decoders
+  uint64_t* afull = done + kDone;                            // [kAGroups] decode warps -> MMA
+  uint64_t* accfull = afull + kAGroups;                      // [2] MMA commit -> epilogue
+  uint64_t* accempty = accfull + 2;                          // [2] epilogue warps -> MMA
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nk = a.n_chunks;  // 128-element chunks
+  const int n_ch = a.n_ch_tiles;
+  const int n_tiles = n_ch * ((a.M + BN - 1) / BN);
+  const int ks = a.k_split;
+  const int n_units = n_tiles * ks;
+  auto kc_begin = [&](int u) { return ks == 1 ? 0 : (u % ks) * nk / ks; };
+  auto kc_end = [&](int u) { return ks == 1 ? nk : (u % ks + 1) * nk / ks; };
+  uint32_t total = 0;
+  for (int u = blockIdx.x; u < n_units; u += gridDim.x) total += static_cast<uint32_t>(kc_end(u) - kc_begin(u));
+  auto wait_done = [&](uint32_t j) {
+    const uint32_t g = j / kGroup;
+    return mbar_wait(&done[g % kDone], (g / kDone) & 1, abort_flag, a.dev_status);
+  };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) mbar_init(&full[s], 1);
+    for (int g = 0; g < kDone; ++g) mbar_init(&done[g], 1);
+    for (int g = 0; g < kAGroups; ++g) mbar_init(&afull[g], 4 * kGroup);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accfull[b], 1);
+      mbar_init(&accempty[b], 4 * kEpi);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) tma_prefetch_desc(&act_map);
+  if (warp == 2) tmem_alloc(tmem_slot, C::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  griddep_wait();
+  griddep_launch_dependents();
+
+  if (warp == 0) {
+    // ---------------- producer: activation codes (TMA), two blob chunks of weight codes and their
+    // E8M0 bytes (bulk), MXFP8: the chunk's activation exponents of the tile's tokens (bulk)
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+        const int t = u / ks;
+        const int ch = a.tile0 + t % n_ch, tok0 = (t / n_ch) * BN;
+        const int kc1 = kc_end(u);
+        const uint32_t sf_bytes = MXA ? static_cast<uint32_t>(min(BN, a.act_mp - tok0)) * 4u : 0u;
+        for (int kc = kc_begin(u); kc < kc1; ++kc, ++it) {
+          const int s = it % S;
+          if (it >= static_cast<uint32_t>(S) && !wait_done(it - S)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + s * C::kStage;
+          const int nh = 2 * kc + 1 < a.nk64 ? 2 : 1;  // the last chunk may hold one blob chunk
+          const size_t chunk64 = static_cast<size_t>(ch) * a.nk64 + 2 * kc;
+          mbar_arrive_expect_tx(&full[s], C::kBBytes + nh * (C::kWBytes / 2 + C::kEBytes / 2) + sf_bytes);
+          if (blockIdx.x == 0 && static_cast<int>(it) == a.stall_chunk) continue;  // test hook (see the fp16 kernel)
+          tma_load_2d(smem_u32(st), &act_map, &full[s], kc * kBK8, tok0);
+          bulk_load(smem_u32(st + C::kBBytes), a.codes + chunk64 * (C::kWBytes / 2), nh * (C::kWBytes / 2), &full[s]);
+          bulk_load(smem_u32(st + C::kBBytes + C::kWBytes), a.we8m0 + chunk64 * (C::kEBytes / 2),
+                    nh * (C::kEBytes / 2), &full[s]);
+          if constexpr (MXA)
+            bulk_load(smem_u32(st + C::kBBytes + C::kWBytes + C::kEBytes),
+                      a.act_e8 + static_cast<size_t>(kc) * a.act_e8_plane + static_cast<size_t>(tok0) * 4, sf_bytes,
+                      &full[s]);
+        }
+      }
+      const uint32_t first = it > S ? it - S : 0;
+      for (uint32_t j = first; j < it; ++j) drain_wait(&full[j % S], (j / S) & 1);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = idesc_mxf8(128, BN, a.b_fmt);
+      const uint64_t desc0 = smem_desc_sw128(smem_u32(smem));
+      constexpr uint32_t kStageDesc = C::kStage >> 4;
+      uint32_t it = 0, acc_it = 0, s = 0, sa = 0, gi = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++acc_it) {
+        const int b = acc_it & 1;
+        const int kc0 = kc_begin(u), kc1 = kc_end(u);
+        if (!mbar_wait(&accempty[b], ((acc_it >> 1) & 1) ^ 1, abort_flag, a.dev_status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + b * C::kAccCols;
+        for (int kc = kc0; kc < kc1; ++kc, ++it) {
+          if (gi == 0) {
+            if (!mbar_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+          }
+          const uint64_t bd = desc0 + s * kStageDesc;
+          const uint32_t ad = tmem + C::kACol + sa * 32;
+          const uint32_t sfa = tmem + C::kSFA + sa * 8;
+          const uint32_t sfb = tmem + C::kSFB + (MXA ? sa * 8 : 0);
+          const int nmma = min(4, a.kblocks - 4 * kc);  // 32-element blocks of this chunk inside K
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if (i < nmma) mma_mxf8_ts(d_tmem, ad + 8 * i, bd + 2 * i, idesc_sf_ids(idesc, i), sfa, sfb, kc != kc0 || i > 0);
+          if (++gi == kGroup || it + 1 == total) {
+            mma_commit(&done[(it / kGroup) % kDone]);
+            gi = gi == kGroup ? 0 : gi;
+          }
+          s = s + 1 == static_cast<uint32_t>(S) ? 0 : s + 1;
+          sa = sa + 1 == static_cast<uint32_t>(kAStages) ? 0 : sa + 1;
+        }
+        if (!ok) break;
+        mma_commit(&accfull[b]);
+      }
+      // every issued MMA has finished before tensor memory is released: one more commit covers them all
+      if (it > 0 || acc_it > 0) {
+        mma_commit(&accfull[acc_it & 1]);
+        drain_wait(&accfull[acc_it & 1], (acc_it >> 1) & 1);
+      }
+    }
+  } else if (warp >= 4 && warp < 4 + 4 * kDec) {
+    // ---------------- weight decode: one channel per thread; group g takes chunks it % kDec == g
+    const int q = warp & 3;
+    const int grp = (warp - 4) >> 2;
+    const int r = q * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    if constexpr (!MXA) {
+      // unit B scale factors for the whole launch, before this group's first arrival
+      if (grp == 0) {
+        uint32_t one[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) one[c] = 0x7F7F7F7Fu;
+        tmem_st_32x32b_x8(tmem + lane_off + C::kSFB, one);
+      }
+    }
+    uint32_t it = 0;
+    bool ok = true;
+    int nf = 0, nz = 0;
+    if (static_cast<int>(blockIdx.x) < n_units) {
+      const int p0 = (a.tile0 + (static_cast<int>(blockIdx.x) / ks) % n_ch) * 128 + r;
+      nf = a.wfmt[p0];
+      nz = a.wzero[p0];
+    }
+    for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      uint32_t T[4];
+      f8_table(nf, nz, T);
+      if (u + static_cast<int>(gridDim.x) < n_units) {
+        const int pn = (a.tile0 + ((u + static_cast<int>(gridDim.x)) / ks) % n_ch) * 128 + r;
+        nf = a.wfmt[pn];
+        nz = a.wzero[pn];
+      }
+      const int kc1 = kc_end(u);
+      for (int kc = kc_begin(u); kc < kc1; ++kc, ++it) {
+        if (static_cast<int>(it % kDec) != grp) continue;
+        const int s = it % S, sa = it % kAStages;
+        const uint32_t ph = (it / S) & 1;
+        if (!warp_wait(&full[s], ph, abort_flag, a.dev_status)) {
+          ok = false;
+          break;
+        }
+        const uint8_t* st = smem + s * C::kStage;
+        const int nh = 2 * kc + 1 < a.nk64 ? 2 : 1;
+        const uint16_t* e8 = reinterpret_cast<const uint16_t*>(st + C::kBBytes + C::kWBytes);
+        // block exponents of the chunk's four 32-element blocks (a missing second half is never read)
+        const uint32_t sfa = static_cast<uint32_t>(e8[r]) | (nh == 2 ? static_cast<uint32_t>(e8[128 + r]) << 16 : 0x7F7F0000u);
+        uint32_t raw[16];
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (h < nh) v = *reinterpret_cast<const uint4*>(st + C::kBBytes + h * 4096 + j * 2048 + r * 16);
+            raw[8 * h + 4 * j] = v.x;
+            raw[8 * h + 4 * j + 1] = v.y;
+            raw[8 * h + 4 * j + 2] = v.z;
+            raw[8 * h + 4 * j + 3] = v.w;
+          }
+        uint32_t out[32];
+        decode_f8(raw, T, out);
+        uint32_t sfb[8];
+        if constexpr (MXA) {
+          // this lane's tokens n = 32 c + lane of the tile, in every lane quadrant
+          const uint32_t* se = reinterpret_cast<const uint32_t*>(st + C::kBBytes + C::kWBytes + C::kEBytes);
+#pragma unroll
+          for (int c = 0; c < 8; ++c) sfb[c] = c < C::kSFBCols ? se[32 * c + lane] : 0x7F7F7F7Fu;
+        }
+        const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
+        if (!__all_sync(0xffffffffu, free_ok)) {
+          ok = false;
+          break;
+        }
+        __syncwarp();
+        tc_fence_after();
+        tmem_st_32x32b_x32(tmem + C::kACol + lane_off + sa * 32, out);
+        tmem_st_32x32b_x1(tmem + C::kSFA + lane_off + sa * 8 + q, sfa);
+        if constexpr (MXA) tmem_st_32x32b_x8(tmem + C::kSFB + lane_off + sa * 8, sfb);
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          const int missing = it + 1 == total ? kGroup - 1 - static_cast<int>(it % kGroup) : 0;
+          for (int m = 0; m <= missing; ++m) mbar_arrive(&afull[(it / kGroup) % kAGroups]);
+        }
+      }
+    }
+  } else if (warp >= 4 + 4 * kDec) {
+    epilogue_role<BN, EPI, kEpi, C::kAccCols>(a, tmem, accfull, accempty, abort_flag, warp, 4 + 4 * kDec, n_units,
+                                              ks, n_ch);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
+template <int BN, int EPI, bool MXA>
+static cudaError_t launch_f8_bn(const CUtensorMap& map, const GemmArgs& a, int num_sms, cudaStream_t st) {
+  using C = F8Cfg<BN, MXA>;
+  static int configured_device = -1;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (configured_device != dev) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(k_gemm_ts_f8<BN, EPI, MXA>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem);
+    if (e != cudaSuccess) return e;
+    configured_device = dev;
+  }
+  const long units = static_cast<long>(a.n_ch_tiles) * ((a.M + BN - 1) / BN) * a.k_split;
+  const int grid = static_cast<int>(units < num_sms ? units : num_sms);
+  return launch_pdl(k_gemm_ts_f8<BN, EPI, MXA>, dim3(grid), dim3(kGemmThreads), C::kSmem, st, map, a);
+}
+
+template <int EPI, bool MXA>
+static cudaError_t launch_f8_epi(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
+  switch (bn) {
+    case 32: return launch_f8_bn<32, EPI, MXA>(map, a, num_sms, st);
+    case 64: return launch_f8_bn<64, EPI, MXA>(map, a, num_sms, st);
+    case 128: return launch_f8_bn<128, EPI, MXA>(map, a, num_sms, st);
+    default: return launch_f8_bn<kF8TokenTile, EPI, MXA>(map, a, num_sms, st);
+  }
+}
+
+}  // namespace cham

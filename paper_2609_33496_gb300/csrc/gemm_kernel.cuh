@@ -40,7 +40,7 @@ template <int BITS> struct Roles {
   static constexpr int kDec = BITS == 4 ? 3 : 2, kEpi = BITS == 4 ? 1 : 2;
 };
 constexpr int kDecodeGroups = 2, kEpiGroups = 2;  // the 8-bit split; the thread count is the same
-constexpr int kPartialOut = 3;    // epilogue "output type" of split-K units: raw fp32 partial sums
+constexpr int kPartialOut = kPartialYT;  // epilogue "output type" of split-K units: raw fp32 partial sums
 constexpr int kGemmThreads = 128 * (1 + kDecodeGroups + kEpiGroups);
 
 template <int BN, int BITS>
@@ -296,6 +296,128 @@ CHAM_DEV void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&v)[16]) {
       : "memory");
 }
 
+// Epilogue role, shared by the fp16 and FP8 kernels: the warps first_warp .. first_warp + 4 * kEpiGrp - 1
+// drain one accumulator buffer per tile (buffer b at column b * kAccCols); warpgroup h takes the
+// 16-column slices j = h, h + kEpiGrp, ...
+template <int BN, int EPI, int kEpiGrp, int kAccCols>
+CHAM_DEV void epilogue_role(const GemmArgs& a, uint32_t tmem, uint64_t* accfull, uint64_t* accempty,
+                            volatile int* abort_flag, int warp, int first_warp, int n_units, int ks, int n_ch) {
+  const int lane = threadIdx.x & 31;
+  const int q = warp & 3;
+  const int h = (warp - first_warp) >> 2;
+  const int r = q * 32 + lane;
+  const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+  const float sa = a.act_scale != nullptr ? *a.act_scale : 1.f;
+  uint32_t acc_it = 0;
+  for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++acc_it) {
+    const int b = acc_it & 1;
+    const int t = u / ks;
+    // per-channel constants first: their (dependent) loads overlap the wait for the accumulator
+    const int p = (a.tile0 + t % n_ch) * 128 + r;
+    const int tok0 = (t / n_ch) * BN;
+    const int orig = a.perm[p];
+    const float ws = a.wscale[p];
+    const float scale = __fmul_rn(sa, ws);
+    const float bv = (a.bias != nullptr && orig >= 0) ? a.bias[orig] : 0.f;
+    if (!warp_wait(&accfull[b], (acc_it >> 1) & 1, abort_flag, a.dev_status)) break;
+    tc_fence_after();
+    const uint32_t d_tmem = tmem + b * kAccCols + lane_off;
+    // y = acc * (s_a * s_w) + bias, rounded once to fp32, then (f16 / bf16 outputs) to the output
+    // type; one instantiation per output type and scale granularity keeps each variant as lean
+    // as the fp32 per-tensor one
+    // YT = kPartialOut (EPI = 6, split-K): the raw fp32 sums go to a.partial[u % ks][tok][p]
+    // and the reduction kernel applies scales, bias and the output type
+    auto drain = [&](auto yt, auto grouped_tag) {
+      constexpr int YT = decltype(yt)::value;
+      constexpr bool GROUPED = decltype(grouped_tag)::value;
+      using OutT = std::conditional_t<YT == CHAM_Y_F32 || YT == kPartialOut, float,
+                                      std::conditional_t<YT == CHAM_Y_F16, __half, __nv_bfloat16>>;
+      OutT* yc = static_cast<OutT*>(a.Y) + (orig >= 0 ? orig : 0);
+      float* pc = a.partial + static_cast<size_t>(u % ks) * a.M * a.Np + p;
+      // 16 token columns per tcgen05.ld; the load of the warp's next slice is in flight while
+      // the current one is scaled and stored (a wait per load would serialise its latency)
+      auto store16 = [&](const uint32_t (&v)[16], int j) {
+        if (orig < 0) return;
+        const int t0 = tok0 + j * 16;
+        if constexpr (YT == kPartialOut) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int tok = t0 + i;
+            if (tok >= a.M) break;
+            pc[static_cast<size_t>(tok) * a.Np] = __uint_as_float(v[i]);
+          }
+          return;
+        }
+        if (t0 + 16 <= a.M) {
+          // a full slice inside one row group (always, for a per-tensor scale): no bounds or
+          // group checks, one running pointer
+          float s16 = scale;
+          bool one = true;
+          if constexpr (GROUPED) {
+            const int g0 = t0 / a.rows_per_group;
+            one = (t0 + 15) / a.rows_per_group == g0;
+            if (one) s16 = __fmul_rn(a.act_scale[g0], ws);
+          }
+          if (one) {
+            OutT* yp = yc + static_cast<size_t>(t0) * a.N;
+            const size_t stride = static_cast<size_t>(a.N);
+#pragma unroll
+            for (int i = 0; i < 16; ++i, yp += stride) {
+              const float y = fmaf(__uint_as_float(v[i]), s16, bv);
+              if constexpr (YT == CHAM_Y_F32) *yp = y;
+              else if constexpr (YT == CHAM_Y_F16) *yp = __float2half_rn(y);
+              else *yp = __float2bfloat16_rn(y);
+            }
+            return;
+          }
+        }
+        float sc = scale;
+        int grp = 0, next = 0;
+        if constexpr (GROUPED) {  // per-sample scales: the group advances at most a few times
+          grp = t0 / a.rows_per_group;
+          next = (grp + 1) * a.rows_per_group;
+          sc = __fmul_rn(a.act_scale[grp], ws);
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int tok = t0 + i;
+          if (tok >= a.M) break;
+          if constexpr (GROUPED) {
+            if (tok >= next) {
+              ++grp;
+              next += a.rows_per_group;
+              sc = __fmul_rn(a.act_scale[grp], ws);
+            }
+          }
+          const float y = fmaf(__uint_as_float(v[i]), sc, bv);
+          if constexpr (YT == CHAM_Y_F32) yc[static_cast<size_t>(tok) * a.N] = y;
+          else if constexpr (YT == CHAM_Y_F16) yc[static_cast<size_t>(tok) * a.N] = __float2half_rn(y);
+          else yc[static_cast<size_t>(tok) * a.N] = __float2bfloat16_rn(y);
+        }
+      };
+      constexpr int kLoads = BN / 16, kE = kEpiGrp;
+      uint32_t va[16], vb[16];
+      if (h < kLoads) {
+        tmem_ld_32x32b_x16(d_tmem + h * 16, va);
+        tmem_wait_ld();
+      }
+#pragma unroll 1
+      for (int j = h; j < kLoads; j += 2 * kE) {
+        if (j + kE < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + kE) * 16, vb);
+        store16(va, j);
+        tmem_wait_ld();
+        if (j + 2 * kE < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + 2 * kE) * 16, va);
+        if (j + kE < kLoads) store16(vb, j + kE);
+        tmem_wait_ld();
+      }
+    };
+    drain(std::integral_constant<int, EPI / 2>{}, std::bool_constant<(EPI % 2) == 1>{});
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&accempty[b]);
+  }
+}
+
 // EPI = 2 * output type (CHAM_Y_*) + per-sample scales: one epilogue variant per instantiation
 // (several inlined into one kernel raise its register count past what the split allows); GW =
 // group-wise weights (per-block fp16 scales and zero points staged with every chunk)
@@ -430,7 +552,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           s = s + 1 == static_cast<uint32_t>(S) ? 0 : s + 1;
           sa = sa + 1 == static_cast<uint32_t>(kAStages) ? 0 : sa + 1;
         }
-        mma_commit(&accfull[b]);
+        mma_commit(&accfull[b]);  // after an abort inside the tile this still covers every MMA issued
       }
       // all issued MMAs have finished before tensor memory is released
       if (acc_it > 0) drain_wait(&accfull[(acc_it - 1) & 1], ((acc_it - 1) >> 1) & 1);
@@ -520,121 +642,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
     }
   } else if (warp >= 4 + 4 * Roles<BITS>::kDec) {
-    // ---------------- epilogue: drain one accumulator buffer per tile; warpgroup h takes the
-    // 16-column slices j = h, h + kEpiGroups, ...
-    const int q = warp & 3;
-    const int h = (warp - (4 + 4 * Roles<BITS>::kDec)) >> 2;
-    const int r = q * 32 + lane;
-    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    const float sa = a.act_scale != nullptr ? *a.act_scale : 1.f;
-    uint32_t acc_it = 0;
-    for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++acc_it) {
-      const int b = acc_it & 1;
-      const int t = u / ks;
-      // per-channel constants first: their (dependent) loads overlap the wait for the accumulator
-      const int p = (a.tile0 + t % n_ch) * 128 + r;
-      const int tok0 = (t / n_ch) * BN;
-      const int orig = a.perm[p];
-      const float ws = a.wscale[p];
-      const float scale = __fmul_rn(sa, ws);
-      const float bv = (a.bias != nullptr && orig >= 0) ? a.bias[orig] : 0.f;
-      if (!warp_wait(&accfull[b], (acc_it >> 1) & 1, abort_flag, a.dev_status)) break;
-      tc_fence_after();
-      const uint32_t d_tmem = tmem + b * C::kAccCols + lane_off;
-      // y = acc * (s_a * s_w) + bias, rounded once to fp32, then (f16 / bf16 outputs) to the output
-      // type; one instantiation per output type and scale granularity keeps each variant as lean
-      // as the fp32 per-tensor one
-      // YT = kPartialOut (EPI = 6, split-K): the raw fp32 sums go to a.partial[u % ks][tok][p]
-      // and the reduction kernel applies scales, bias and the output type
-      auto drain = [&](auto yt, auto grouped_tag) {
-        constexpr int YT = decltype(yt)::value;
-        constexpr bool GROUPED = decltype(grouped_tag)::value;
-        using OutT = std::conditional_t<YT == CHAM_Y_F32 || YT == kPartialOut, float,
-                                        std::conditional_t<YT == CHAM_Y_F16, __half, __nv_bfloat16>>;
-        OutT* yc = static_cast<OutT*>(a.Y) + (orig >= 0 ? orig : 0);
-        float* pc = a.partial + static_cast<size_t>(u % ks) * a.M * a.Np + p;
-        // 16 token columns per tcgen05.ld; the load of the warp's next slice is in flight while
-        // the current one is scaled and stored (a wait per load would serialise its latency)
-        auto store16 = [&](const uint32_t (&v)[16], int j) {
-          if (orig < 0) return;
-          const int t0 = tok0 + j * 16;
-          if constexpr (YT == kPartialOut) {
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const int tok = t0 + i;
-              if (tok >= a.M) break;
-              pc[static_cast<size_t>(tok) * a.Np] = __uint_as_float(v[i]);
-            }
-            return;
-          }
-          if (t0 + 16 <= a.M) {
-            // a full slice inside one row group (always, for a per-tensor scale): no bounds or
-            // group checks, one running pointer
-            float s16 = scale;
-            bool one = true;
-            if constexpr (GROUPED) {
-              const int g0 = t0 / a.rows_per_group;
-              one = (t0 + 15) / a.rows_per_group == g0;
-              if (one) s16 = __fmul_rn(a.act_scale[g0], ws);
-            }
-            if (one) {
-              OutT* yp = yc + static_cast<size_t>(t0) * a.N;
-              const size_t stride = static_cast<size_t>(a.N);
-#pragma unroll
-              for (int i = 0; i < 16; ++i, yp += stride) {
-                const float y = fmaf(__uint_as_float(v[i]), s16, bv);
-                if constexpr (YT == CHAM_Y_F32) *yp = y;
-                else if constexpr (YT == CHAM_Y_F16) *yp = __float2half_rn(y);
-                else *yp = __float2bfloat16_rn(y);
-              }
-              return;
-            }
-          }
-          float sc = scale;
-          int grp = 0, next = 0;
-          if constexpr (GROUPED) {  // per-sample scales: the group advances at most a few times
-            grp = t0 / a.rows_per_group;
-            next = (grp + 1) * a.rows_per_group;
-            sc = __fmul_rn(a.act_scale[grp], ws);
-          }
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int tok = t0 + i;
-            if (tok >= a.M) break;
-            if constexpr (GROUPED) {
-              if (tok >= next) {
-                ++grp;
-                next += a.rows_per_group;
-                sc = __fmul_rn(a.act_scale[grp], ws);
-              }
-            }
-            const float y = fmaf(__uint_as_float(v[i]), sc, bv);
-            if constexpr (YT == CHAM_Y_F32) yc[static_cast<size_t>(tok) * a.N] = y;
-            else if constexpr (YT == CHAM_Y_F16) yc[static_cast<size_t>(tok) * a.N] = __float2half_rn(y);
-            else yc[static_cast<size_t>(tok) * a.N] = __float2bfloat16_rn(y);
-          }
-        };
-        constexpr int kLoads = BN / 16, kE = Roles<BITS>::kEpi;
-        uint32_t va[16], vb[16];
-        if (h < kLoads) {
-          tmem_ld_32x32b_x16(d_tmem + h * 16, va);
-          tmem_wait_ld();
-        }
-#pragma unroll 1
-        for (int j = h; j < kLoads; j += 2 * kE) {
-          if (j + kE < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + kE) * 16, vb);
-          store16(va, j);
-          tmem_wait_ld();
-          if (j + 2 * kE < kLoads) tmem_ld_32x32b_x16(d_tmem + (j + 2 * kE) * 16, va);
-          if (j + kE < kLoads) store16(vb, j + kE);
-          tmem_wait_ld();
-        }
-      };
-      drain(std::integral_constant<int, EPI / 2>{}, std::bool_constant<(EPI % 2) == 1>{});
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&accempty[b]);
-    }
+    epilogue_role<BN, EPI, Roles<BITS>::kEpi, C::kAccCols>(a, tmem, accfull, accempty, abort_flag, warp,
+                                                          4 + 4 * Roles<BITS>::kDec, n_units, ks, n_ch);
   }
   tc_fence_before();
   __syncthreads();
@@ -680,12 +689,6 @@ static cudaError_t launch_gw(const CUtensorMap& map, const GemmArgs& a, int num_
 
 // The launches of one output type YT: both weight widths, every token-tile size, per-tensor or
 // per-sample activation scales, per-channel or group-wise weights.
-// Split-K units: raw partial sums (EPI 6); the reduction applies scales, bias and output type.
-inline cudaError_t launch_gemm_partial(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn,
-                                       cudaStream_t st) {
-  if (a.bits == 8) return launch_gw<8, 2 * kPartialOut>(map, a, num_sms, bn, st);
-  return launch_gw<4, 2 * kPartialOut>(map, a, num_sms, bn, st);
-}
 
 template <int YT>
 cudaError_t launch_gemm_yt(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {

@@ -15,7 +15,9 @@
 //     overwrites every partial the second launch reads.  Calls whose kernels overlap on the GPU
 //     (for example on two streams at once) race on the array and produce wrong scales.
 //   * the first call on a device looks up the array's device address for that device (with that
-//     device current); make that first call before any stream capture.
+//     device current); make that first call before any stream capture.  The address is kept for
+//     the life of the process: after cudaDeviceReset the module is loaded again and the array may
+//     move, so the entry point must not be called on a device that has been reset.
 #include <cuda_runtime.h>
 
 #include <mutex>

@@ -20,7 +20,7 @@ int main(void) {
   /* layouts shared with the Python binding */
   CHECK(sizeof(cham_wpack_desc) == 256);
   CHECK(sizeof(cham_qparams) == 16);
-  CHECK(chameleon_version() == 2);
+  CHECK(chameleon_version() == 3);
   CHECK(chameleon_status_string(CHAM_ERR_WORKSPACE) != NULL);
 
   /* Alg. 2 / Alg. 3 bucket: b = min(floor(t / (T/B)), B-1) */
@@ -57,7 +57,7 @@ int main(void) {
     cham_wpack_desc d;
     memset(fmt, CHAM_W_INT8_SYM, sizeof fmt);
     CHECK(chameleon_pack_plan(256, 320, fmt, &d) == CHAM_OK);
-    CHECK(d.magic == 0x574D4843u && d.version == 2 && d.N == 256 && d.K == 320 && d.Kp == 320);
+    CHECK(d.magic == 0x574D4843u && d.version == 3 && d.N == 256 && d.K == 320 && d.Kp == 320);
     CHECK(d.bits == 8 && d.n_tiles[0] + d.n_tiles[1] == 2 && d.n_fmt[CHAM_W_INT8_SYM] == 256);
     CHECK(d.bytes > (uint64_t)256 * 320 && d.off_codes % 256 == 0);
   }

@@ -143,6 +143,7 @@ def test_scale_zp_and_static_entry_points_reject_bad_arguments(cl):
             cl.scale_zp(fmt, lo, hi)
         assert e.value.status == cl.ERR_INVALID_ARG
     L = cl.lib()
+    dp = ctypes.byref(cl.pack_plan(64, 64, np.zeros(64, np.uint8)))  # a 64-input layer for the prepare calls
     buf = ctypes.create_string_buffer(1 << 16)
     x = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
     good = cl.scale_zp(F.A_INT8_ASYM, -1.0, 3.0)
@@ -151,7 +152,7 @@ def test_scale_zp_and_static_entry_points_reject_bad_arguments(cl):
     for p in bad:
         ref = None if p is None else ctypes.byref(p)
         assert L.chameleon_act_quant_static(x, 16, 64, F.A_INT8_ASYM, ref, x, 1 << 15, x, None) == cl.ERR_INVALID_ARG
-        assert L.chameleon_linear_prepare_static(x, 16, 64, F.A_INT8_ASYM, ref, x, 1 << 15, x,
+        assert L.chameleon_linear_prepare_static(x, 16, dp, F.A_INT8_ASYM, ref, x, 1 << 15, x,
                                                  None) == cl.ERR_INVALID_ARG
     fp8 = cl.scale_zp(F.A_E4M3, -1.0, 3.0)
     fp8.z = 1
@@ -166,10 +167,11 @@ def test_groups_and_output_type_argument_checks(cl):
     """Per-sample groups must divide M and number 1..CHAM_MAX_GROUPS; y_type is one of three.
     Every rejection happens on the host, before any launch."""
     L = cl.lib()
+    dp = ctypes.byref(cl.pack_plan(64, 64, np.zeros(64, np.uint8)))  # a 64-input layer for the prepare calls
     buf = ctypes.create_string_buffer(1 << 20)
     x = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
     for M, n in [(64, 0), (64, 65), (64, 3), (60, -1), (128, 128)]:
-        assert L.chameleon_linear_prepare_groups(x, M, 64, F.A_E4M3, n, x, 1 << 19, x, None) == cl.ERR_INVALID_ARG
+        assert L.chameleon_linear_prepare_groups(x, M, dp, F.A_E4M3, n, x, 1 << 19, x, None) == cl.ERR_INVALID_ARG
     d = cl.pack_plan(64, 64, np.zeros(64, np.uint8))
     for n, yt in [(3, cl.Y_F32), (0, cl.Y_F16), (1, 3), (1, -1), (65, cl.Y_BF16)]:
         assert L.chameleon_linear_gemm_ex(x, 64, ctypes.byref(d), x, F.A_E4M3, n, None, x, yt, x, 1 << 19, x,
@@ -199,7 +201,7 @@ def test_group_candidates_match_oracle(cl):
 
 def test_pack_plan_grouped_layout_and_checks(cl):
     d = cl.pack_plan_grouped(300, 320, F.W_INT4_ASYM, 192)
-    assert (d.group, d.bits, list(d.n_class), d.n_fmt[F.W_INT4_ASYM], d.version) == (192, 4, [300, 0], 300, 2)
+    assert (d.group, d.bits, list(d.n_class), d.n_fmt[F.W_INT4_ASYM], d.version) == (192, 4, [300, 0], 300, 3)
     assert d.off_gscale % 256 == 0 and d.off_gscale >= d.off_perm + 4 * 384
     assert d.bytes >= d.off_gscale + 3 * 5 * 128 * 4
     assert cl.pack_plan(300, 320, np.full(300, F.W_INT4_ASYM, np.uint8)).off_gscale == 0
@@ -261,7 +263,7 @@ def test_linear_workspace_includes_split_k_partials(cl):
 
 
 def test_version_and_status_names(cl):
-    assert cl.version() == 2
+    assert cl.version() == 3
     assert cl.status_string(cl.OK) and cl.status_string(cl.ERR_TIMEOUT) != cl.status_string(cl.OK)
 
 
@@ -271,6 +273,7 @@ def test_empty_and_negative_sizes_are_rejected_on_the_host(cl, bad):
     """Every entry point that takes a size rejects an empty (0) or negative M, N, K or count with
     CHAM_ERR_INVALID_ARG before touching the device (no GPU is present here)."""
     L = cl.lib()
+    dp = ctypes.byref(cl.pack_plan(64, 64, np.zeros(64, np.uint8)))  # a 64-input layer for the prepare calls
     buf = ctypes.create_string_buffer(1 << 16)
     x = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
     n = ctypes.c_size_t(0)
@@ -306,10 +309,10 @@ def test_empty_and_negative_sizes_are_rejected_on_the_host(cl, bad):
         "pack_plan_grouped": lambda: L.chameleon_pack_plan_grouped(16, bad, F.W_NF4, 32, ctypes.byref(d)),
         "linear_workspace_size": lambda: L.chameleon_linear_workspace_size(bad, ctypes.byref(good), 1,
                                                                            ctypes.byref(n)),
-        "linear_prepare": lambda: L.chameleon_linear_prepare(x, bad, 64, 1, x, 1 << 15, x, None),
-        "linear_prepare_static": lambda: L.chameleon_linear_prepare_static(x, bad, 64, 1, ctypes.byref(p), x,
+        "linear_prepare": lambda: L.chameleon_linear_prepare(x, bad, dp, 1, x, 1 << 15, x, None),
+        "linear_prepare_static": lambda: L.chameleon_linear_prepare_static(x, bad, dp, 1, ctypes.byref(p), x,
                                                                            1 << 15, x, None),
-        "linear_prepare_groups": lambda: L.chameleon_linear_prepare_groups(x, bad, 64, 1, 1, x, 1 << 15, x, None),
+        "linear_prepare_groups": lambda: L.chameleon_linear_prepare_groups(x, bad, dp, 1, 1, x, 1 << 15, x, None),
         "linear": lambda: L.chameleon_linear(x, bad, ctypes.byref(good), x, 1, None, x, x, 1 << 15, x, None),
         "linear_gemm": lambda: L.chameleon_linear_gemm(x, bad, ctypes.byref(good), x, 1, None, x, x, 1 << 15, x,
                                                        None),
@@ -326,6 +329,7 @@ def test_misaligned_device_pointers_are_rejected_on_the_host(cl):
     """Device pointers must be 16-byte aligned: inputs, outputs and workspaces two bytes off a
     16-byte boundary give CHAM_ERR_INVALID_ARG before any device work."""
     L = cl.lib()
+    dp = ctypes.byref(cl.pack_plan(64, 64, np.zeros(64, np.uint8)))  # a 64-input layer for the prepare calls
     buf = ctypes.create_string_buffer(1 << 16)
     a = ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16
     x, m = ctypes.c_void_p(a), ctypes.c_void_p(a + 2)
@@ -358,9 +362,9 @@ def test_misaligned_device_pointers_are_rejected_on_the_host(cl):
         "select_pack_palette blob": lambda: L.chameleon_select_pack_palette(x, 64, 64, cl.PALETTE_W8,
                                                                             ctypes.byref(good), x, m, 1 << 15, x,
                                                                             None),
-        "linear_prepare X": lambda: L.chameleon_linear_prepare(m, 16, 64, 1, x, 1 << 15, x, None),
-        "linear_prepare ws": lambda: L.chameleon_linear_prepare(x, 16, 64, 1, m, 1 << 15, x, None),
-        "linear_prepare_static X": lambda: L.chameleon_linear_prepare_static(m, 16, 64, 1, ctypes.byref(p), x,
+        "linear_prepare X": lambda: L.chameleon_linear_prepare(m, 16, dp, 1, x, 1 << 15, x, None),
+        "linear_prepare ws": lambda: L.chameleon_linear_prepare(x, 16, dp, 1, m, 1 << 15, x, None),
+        "linear_prepare_static X": lambda: L.chameleon_linear_prepare_static(m, 16, dp, 1, ctypes.byref(p), x,
                                                                              1 << 15, x, None),
         "linear_gemm_ex blob": lambda: L.chameleon_linear_gemm_ex(x, 16, ctypes.byref(good), m, 1, 1, None, x,
                                                                   cl.Y_F32, x, 1 << 15, x, None),
@@ -383,6 +387,7 @@ def test_undersized_buffers_are_rejected_on_the_host(cl):
     """A buffer one byte smaller than its size query returned gives CHAM_ERR_WORKSPACE before any
     device work: quantized activations, workspaces, weight blobs."""
     L = cl.lib()
+    dp = ctypes.byref(cl.pack_plan(64, 64, np.zeros(64, np.uint8)))  # a 64-input layer for the prepare calls
     buf = ctypes.create_string_buffer(1 << 20)
     x = ctypes.c_void_p(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 256)
     good = cl.pack_plan(64, 64, np.zeros(64, np.uint8))
@@ -413,10 +418,10 @@ def test_undersized_buffers_are_rejected_on_the_host(cl):
         "select_pack_palette blob": lambda: L.chameleon_select_pack_palette(x, 64, 64, cl.PALETTE_W8,
                                                                             ctypes.byref(good), x, x, blob - 1, x,
                                                                             None),
-        "linear_prepare ws": lambda: L.chameleon_linear_prepare(x, 16, 64, e4, x, lw - 1, x, None),
-        "linear_prepare_static ws": lambda: L.chameleon_linear_prepare_static(x, 16, 64, e4, ctypes.byref(p), x,
+        "linear_prepare ws": lambda: L.chameleon_linear_prepare(x, 16, dp, e4, x, lw - 1, x, None),
+        "linear_prepare_static ws": lambda: L.chameleon_linear_prepare_static(x, 16, dp, e4, ctypes.byref(p), x,
                                                                               lw - 1, x, None),
-        "linear_prepare_groups ws": lambda: L.chameleon_linear_prepare_groups(x, 16, 64, e4, 2, x, lw - 1, x,
+        "linear_prepare_groups ws": lambda: L.chameleon_linear_prepare_groups(x, 16, dp, e4, 2, x, lw - 1, x,
                                                                               None),
         "linear_gemm ws": lambda: L.chameleon_linear_gemm(x, 16, ctypes.byref(good), x, e4, None, x, x, lw - 1, x,
                                                           None),
@@ -446,3 +451,42 @@ def test_binding_rejects_strided_mistyped_and_host_tensors(cl):
     with pytest.raises(TypeError, match="float32"):
         cl._f32(torch.zeros(16, 64, dtype=torch.float16), "Y")
     assert cl._f32(None, "bias") is None
+
+
+def test_linear_workspace_holds_the_operands_the_tiles_need(cl):
+    """The workspace layout of include/chameleon.h: class-0 tiles of a 4-bit per-channel layout
+    against E4M3 / E5M2 / MXFP8 activations take the 1-byte codes (M x K; MXFP8 adds its exponents
+    chunk-major, ceil(K/128) x round_up(M, 4) x 4 bytes); every other tile takes the exact fp16
+    operand (2 M x K); f16_only = 1 sends every tile to the fp16 path.  Differences against the
+    CHAM_A_FP16 size (which holds no operand and no range partials) isolate the operand regions;
+    no launch of this shape splits K (no partial sums)."""
+    M, K, N = 8192, 640, 1280
+
+    def r256(n):
+        return -(-n // 256) * 256
+
+    parts = r256(max(min(-(-(M * K // 8) // 256), 152 * 4), 64) * 16)   # range partials, 152 SMs
+    codes, fp16 = r256(M * K), r256(2 * M * K)
+    e8 = r256(-(-K // 128) * -(-M // 4) * 4 * 4)
+    c0 = cl.pack_plan(N, K, np.full(N, F.W_INT4_ASYM, np.uint8))
+    mixed = cl.pack_plan(N, K, np.array([F.W_MXFP4, F.W_NF4] * (N // 2), np.uint8))
+    w8 = cl.pack_plan(N, K, np.full(N, F.W_INT8_SYM, np.uint8))
+
+    def extra(d, af, f16_only=0):
+        d.f16_only = f16_only
+        return cl.linear_workspace_size(M, d, af) - cl.linear_workspace_size(M, d, F.A_FP16)
+
+    for af in (F.A_E4M3, F.A_E5M2):
+        assert extra(c0, af) == parts + codes
+        assert extra(c0, af, 1) == parts + fp16
+        assert extra(mixed, af) == parts + codes + fp16
+        assert extra(w8, af) == parts + fp16
+    assert extra(c0, F.A_MXFP8) == parts + codes + e8
+    assert extra(mixed, F.A_MXFP8) == parts + codes + e8 + fp16
+    for af in (F.A_INT8_ASYM, F.A_MXINT8):
+        assert extra(c0, af) == parts + fp16 and extra(mixed, af) == parts + fp16
+    g = cl.pack_plan_grouped(N, K, F.W_INT4_ASYM, 64)                  # group-wise blobs: fp16 path
+    assert extra(g, F.A_E4M3) == parts + fp16
+    c0.f16_only = 2
+    with pytest.raises(cl.ChameleonError):
+        cl.linear_workspace_size(M, c0, F.A_E4M3)

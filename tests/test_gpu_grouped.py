@@ -43,7 +43,7 @@ def test_packed_blob_matches_oracle(cl, fmt, g):
     W = WL.weight_mix(rng, N, K)
     d, blob = pack_grouped(cl, W, fmt, g)
     desc, chans = B.unpack(host(blob).tobytes())
-    assert desc["group"] == g and desc["version"] == 2
+    assert desc["group"] == g and desc["version"] == 3
     L = nf4_levels_fp16()
     q = F.weight_quant_grouped(W, fmt, g, nf4_levels=L)
     asym = fmt in (F.W_INT8_ASYM, F.W_INT4_ASYM)

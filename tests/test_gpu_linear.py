@@ -18,9 +18,10 @@ def cl():
     return lib_module()
 
 
-def gpu_linear(cl, X, W, fmt, act_fmt, bias):
+def gpu_linear(cl, X, W, fmt, act_fmt, bias, f16_only=0):
     import torch
     d = cl.pack_plan(W.shape[0], W.shape[1], fmt)
+    d.f16_only = f16_only
     blob, st = cl.pack_weights(cuda(W), cuda(fmt), d)
     Y, st2 = cl.linear(cuda(X), d, blob, act_fmt, bias=None if bias is None else cuda(bias))
     torch.cuda.synchronize()
@@ -28,18 +29,21 @@ def gpu_linear(cl, X, W, fmt, act_fmt, bias):
     return host(Y)
 
 
-def check(cl, X, W, fmt, act_fmt, bias, what):
-    Y = gpu_linear(cl, X, W, fmt, act_fmt, bias)
+def check(cl, X, W, fmt, act_fmt, bias, what, f16_only=0):
+    Y = gpu_linear(cl, X, W, fmt, act_fmt, bias, f16_only)
     Y_ref, bound, _, _ = G.linear_reference(X, act_fmt, W, fmt, bias)
     assert_within_bound(Y, Y_ref, bound, what)
 
 
+@pytest.mark.parametrize("f16_only", [0, 1])
 @pytest.mark.parametrize("act_fmt", ACT)
 @pytest.mark.parametrize("mask", [0x007, 0x1F8])
-def test_single_layer_w8a8_w4a8(cl, act_fmt, mask):
+def test_single_layer_w8a8_w4a8(cl, act_fmt, mask, f16_only):
+    """Config 1; with f16_only = 0 the 4-bit class-0 tiles run on FP8 MMAs for E4M3 / E5M2 / MXFP8
+    activations, with 1 every tile runs on fp16 MMAs."""
     X, W, bias = WL.single_layer()
     fmt, _, _ = SEL.select_formats(W, mask)
-    check(cl, X, W, fmt, act_fmt, bias, "act %d mask %#x" % (act_fmt, mask))
+    check(cl, X, W, fmt, act_fmt, bias, "act %d mask %#x f16_only %d" % (act_fmt, mask, f16_only), f16_only)
 
 
 def test_weight_only_fp16_activations(cl):
@@ -50,8 +54,8 @@ def test_weight_only_fp16_activations(cl):
 
 @pytest.mark.parametrize("M,K,N", [(1, 32, 1), (2, 96, 130), (17, 160, 129), (200, 64, 300),
                                    (300, 320, 257), (130, 352, 64)])
-@pytest.mark.parametrize("bits", [8, 4])
-def test_ragged_shapes_every_format(cl, M, K, N, bits):
+@pytest.mark.parametrize("bits,f16_only", [(8, 0), (4, 0), (4, 1)])
+def test_ragged_shapes_every_format(cl, M, K, N, bits, f16_only):
     g = np.random.default_rng(M * 1000 + K + N)
     X = WL.to_fp16(g.standard_t(4, (M, K)))
     W = WL.weight_mix(g, N, K)
@@ -60,7 +64,26 @@ def test_ragged_shapes_every_format(cl, M, K, N, bits):
     bias = g.normal(0, 0.02, N).astype(np.float32)
     for act_fmt in ACT + [F.A_FP16]:
         check(cl, X, W, fmt, act_fmt, bias if act_fmt % 2 else None,
-              "M%d K%d N%d bits %d act %d" % (M, K, N, bits, act_fmt))
+              "M%d K%d N%d bits %d act %d f16_only %d" % (M, K, N, bits, act_fmt, f16_only), f16_only)
+
+
+CLASS0 = [F.W_INT4_SYM, F.W_INT4_ASYM, F.W_E2M1, F.W_MXINT4, F.W_MXFP4]
+
+
+@pytest.mark.parametrize("wfmt", CLASS0)
+@pytest.mark.parametrize("act_fmt", [F.A_E4M3, F.A_E5M2, F.A_MXFP8])
+@pytest.mark.parametrize("M,K,N", [(300, 352, 300), (161, 4608, 129)])
+def test_fp8_path_every_activation_weight_pair(cl, act_fmt, wfmt, M, K, N):
+    """Each FP8 activation format x each class-0 weight format on the 8-bit tensor cores
+    (kind::mxf8f6f4): several channel and token tiles, a ragged last K-chunk (352 = 2 x 128 + 3
+    blocks of 32, the last 64-element blob chunk alone) and a long K; every channel in one format,
+    MX weights with block exponents that vary along K (outlier channels, mixed distributions)."""
+    g = np.random.default_rng(7 * M + K + N + 13 * wfmt + act_fmt)
+    X = WL.to_fp16(g.standard_t(5, (M, K)) * np.exp(0.1 * g.standard_normal(K))[None, :])
+    W = WL.weight_mix(g, N, K)
+    fmt = np.full(N, wfmt, np.uint8)
+    bias = g.normal(0, 0.02, N).astype(np.float32)
+    check(cl, X, W, fmt, act_fmt, bias, "act %d w %d M%d K%d N%d" % (act_fmt, wfmt, M, K, N))
 
 
 def test_exact_special_operands(cl):
