@@ -138,6 +138,14 @@ CHAM_DEV void encode8_tensor(const uint4& v, const TensorParams& p, uint2& code,
   deq = make_uint4(d[0], d[1], d[2], d[3]);
 }
 
+// Eight code bytes (element 0 in the low byte) -> the group order 0, 2, 4, 6, 1, 3, 5, 7.
+CHAM_DEV uint2 kperm8(const uint2& c) {
+  uint32_t lo, hi;
+  asm("prmt.b32 %0, %1, %2, 0x6420;" : "=r"(lo) : "r"(c.x), "r"(c.y));
+  asm("prmt.b32 %0, %1, %2, 0x7531;" : "=r"(hi) : "r"(c.x), "r"(c.y));
+  return make_uint2(lo, hi);
+}
+
 // ------------------------------------------------------------------ a2: range partials
 // Group blockIdx.y (rows split into gridDim.y equal groups, nvec vectors each; one group for a
 // per-tensor range) writes its gridDim.x partials at parts[blockIdx.y * gridDim.x ...].
@@ -183,7 +191,7 @@ CHAM_DEV uint32_t nonfinite8(const uint4& v) {
 // lane was non-finite (the static path has no range pass to find out).
 template <int FMT, bool CODES, bool DEQ, bool CHECK>
 CHAM_DEV uint32_t encode_tensor_body(const uint4* __restrict__ X, int64_t nvec, const TensorParams& p,
-                                     uint2* __restrict__ codes, uint4* __restrict__ deq) {
+                                     uint2* __restrict__ codes, uint4* __restrict__ deq, bool kperm) {
   uint32_t nf = 0;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec; i0 += stride * kUnroll) {
@@ -201,7 +209,7 @@ CHAM_DEV uint32_t encode_tensor_body(const uint4* __restrict__ X, int64_t nvec, 
         uint2 c;
         uint4 d;
         encode8_tensor<FMT, DEQ>(v[u], p, c, d);
-        if constexpr (CODES) codes[i] = c;
+        if constexpr (CODES) codes[i] = kperm ? kperm8(c) : c;
         if constexpr (DEQ) deq[i] = d;
       }
     }
@@ -216,7 +224,7 @@ template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_tensor(const uint4* __restrict__ X, int64_t nvec, const RangePartial* __restrict__ parts,
                         int nparts, uint2* __restrict__ codes, uint4* __restrict__ deq,
-                        cham_qparams* __restrict__ params, float* __restrict__ scale_out, int* dev_status) {
+                        cham_qparams* __restrict__ params, float* __restrict__ scale_out, int* dev_status, bool kperm) {
   griddep_wait();  // the range partials
   griddep_launch_dependents();
   const int64_t g = blockIdx.y;
@@ -230,7 +238,7 @@ __global__ void __launch_bounds__(256)
     if (nf) set_status(dev_status, CHAM_ERR_NONFINITE);
   }
   encode_tensor_body<FMT, CODES, DEQ, false>(X + g * nvec, nvec, p, codes == nullptr ? nullptr : codes + g * nvec,
-                                             deq == nullptr ? nullptr : deq + g * nvec);
+                                             deq == nullptr ? nullptr : deq + g * nvec, kperm);
 }
 
 // Static path (Alg. 2): (s, z) fixed beforehand -- ScaleZP of the calibration range that Alg. 1
@@ -240,14 +248,14 @@ template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_static(const uint4* __restrict__ X, int64_t nvec, TensorParams p, uint2* __restrict__ codes,
                         uint4* __restrict__ deq, cham_qparams* __restrict__ params, float* __restrict__ scale_out,
-                        int* dev_status) {
+                        int* dev_status, bool kperm) {
   griddep_wait();  // X may be the previous kernel's output; the outputs may still be read by it
   griddep_launch_dependents();
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     if (params != nullptr) *params = cham_qparams{p.s, p.z, p.inv, FMT};
     if (scale_out != nullptr) *scale_out = p.s;
   }
-  const uint32_t nf = encode_tensor_body<FMT, CODES, DEQ, true>(X, nvec, p, codes, deq);
+  const uint32_t nf = encode_tensor_body<FMT, CODES, DEQ, true>(X, nvec, p, codes, deq, kperm);
   if (__any_sync(0xffffffffu, nf != 0) && (threadIdx.x & 31) == 0) set_status(dev_status, CHAM_ERR_NONFINITE);
 }
 
@@ -317,7 +325,7 @@ template <int FMT, bool CODES, bool DEQ>
 __global__ void __launch_bounds__(256)
     k_act_encode_mx(const uint4* __restrict__ X, int64_t nvec, uint2* __restrict__ codes, uint4* __restrict__ deq,
                     uint8_t* __restrict__ e8m0, uint8_t* __restrict__ e8cm, int kblocks, int64_t cm_plane,
-                    cham_qparams* __restrict__ params, int* dev_status) {
+                    cham_qparams* __restrict__ params, int* dev_status, bool kperm) {
   griddep_wait();  // its outputs may still be read by the previous kernel
   griddep_launch_dependents();
   if (blockIdx.x == 0 && threadIdx.x == 0 && params != nullptr) *params = cham_qparams{1.f, 0, 1.f, FMT};
@@ -341,7 +349,7 @@ __global__ void __launch_bounds__(256)
       int byte;
       encode8_mx<FMT, DEQ>(v[u], lane, c, d, byte, nonfinite);
       if (i < nvec) {
-        if constexpr (CODES) codes[i] = c;
+        if constexpr (CODES) codes[i] = kperm ? kperm8(c) : c;
         if constexpr (DEQ) deq[i] = d;
         if (e8m0 != nullptr && (lane & 3) == 0) e8m0[i >> 2] = static_cast<uint8_t>(byte);
         if (e8cm != nullptr && (lane & 3) == 0) {  // chunk-major copy for the FP8 GEMM
@@ -544,7 +552,7 @@ static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
     const int64_t cap = static_cast<int64_t>(a.num_sms) * 8;
     const int g = static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
     launch_pdl(k_act_encode_static<FMT, CODES, DEQ>, dim3(g), dim3(256), 0, st, a.X, a.nvec, a.stat, a.codes,
-               a.deq, a.params, a.scale_out, a.dev_status);
+               a.deq, a.params, a.scale_out, a.dev_status, a.kperm);
     return;
   }
   // per-sample groups: each group's range and encode grids are the per-tensor ones split evenly
@@ -554,7 +562,7 @@ static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
   const int eg = group_grid(a.nvec, G, a.num_sms);
   launch_pdl(k_act_encode_tensor<FMT, CODES, DEQ>, dim3(eg, G), dim3(256), 0, st, a.X, nvg,
              static_cast<const RangePartial*>(a.parts), a.nparts, a.codes, a.deq, a.params, a.scale_out,
-             a.dev_status);
+             a.dev_status, a.kperm);
 }
 
 template <int FMT, bool CODES, bool DEQ>
@@ -565,7 +573,7 @@ static void launch_mx(const ActQuantArgs& a, cudaStream_t st) {
   if (g > cap) g = cap;
   if (g < 1) g = 1;
   launch_pdl(k_act_encode_mx<FMT, CODES, DEQ>, dim3(static_cast<int>(g)), dim3(256), 0, st, a.X, a.nvec, a.codes,
-             a.deq, a.e8m0, a.e8cm, a.kblocks, a.cm_plane, a.params, a.dev_status);
+             a.deq, a.e8m0, a.e8cm, a.kblocks, a.cm_plane, a.params, a.dev_status, a.kperm);
 }
 
 template <bool CODES, bool DEQ>

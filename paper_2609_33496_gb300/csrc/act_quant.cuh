@@ -35,6 +35,9 @@ struct ActQuantArgs {
                            // block kb of row m at e8cm[(kb / 4) * cm_plane + 4 m + kb % 4]
   int kblocks;             // K / 32 (blocks per row), with e8cm
   int64_t cm_plane;        // bytes per chunk of 4 blocks in e8cm
+  bool kperm;              // codes of each 8-element group stored in the order 0, 2, 4, 6, 1, 3, 5, 7
+                           // (the FP8 GEMM operand: the order in which the 4-bit weight codes
+                           // decode; both operands permuted alike leave the dot product unchanged)
   cham_qparams* params;    // per-tensor parameters, or null
   float* scale_out;        // the per-tensor (per-group) scale s as bare floats (GEMM epilogue), or null
   int* dev_status;

@@ -212,19 +212,18 @@ cham_status check_desc(const cham_wpack_desc* d) {
 
 // Which GEMM operands a layer's tiles need (Sec. 3.6): the class-0 tiles of a 4-bit per-channel
 // layout run on FP8 MMAs against E4M3 / E5M2 / MXFP8 codes (unless the descriptor asks for fp16
-// only); every other tile needs the exact fp16 operand (none for CHAM_A_FP16, which reads X).
+// only) -- one launch of the FP8 kernel, whose NF4 tiles take its fp16 mainloop; every other layer
+// runs on the fp16 kernel.  fp16 tiles need the exact fp16 operand (none for CHAM_A_FP16, which
+// reads X).
 struct OperandPlan {
-  bool fp8;   // class-0 tiles on the FP8 kernel (1-byte codes, MXFP8: chunk-major exponents)
-  bool f16;   // tiles on the fp16 kernel
-  int f16_tile0, f16_tiles;
+  bool fp8;   // the FP8 kernel (1-byte codes, MXFP8: chunk-major exponents) over all tiles
+  bool f16;   // some tiles multiply the fp16 operand (or X)
 };
 OperandPlan operand_plan(const cham_wpack_desc* d, int act_fmt) {
   const bool fp8_act = act_fmt == CHAM_A_E4M3 || act_fmt == CHAM_A_E5M2 || act_fmt == CHAM_A_MXFP8;
   OperandPlan o;
   o.fp8 = fp8_act && d->bits == 4 && d->group == 0 && d->f16_only == 0 && d->n_tiles[0] > 0;
-  o.f16_tile0 = o.fp8 ? d->n_tiles[0] : 0;
-  o.f16_tiles = d->n_tiles[0] + d->n_tiles[1] - o.f16_tile0;
-  o.f16 = o.f16_tiles > 0;
+  o.f16 = !o.fp8 || d->n_tiles[1] > 0;
   return o;
 }
 
@@ -272,31 +271,25 @@ cham_status check_linear_common(int M, int K, int act_fmt, void* ws, size_t ws_b
   return CHAM_OK;
 }
 
-// The GEMM launches of a layer (FP8 kernel over the class-0 tiles, fp16 kernel over the rest):
-// token tile and split-K factor of each, and the partial-sum region after the operands (shared:
-// the two launches write disjoint packed channels of it).
+// The GEMM launch of a layer (the FP8 kernel over all tiles, or the fp16 kernel): token tile,
+// split-K factor, and the partial-sum region after the operands.
 struct GemmPlan {
-  int bn8, ks8, bn16, ks16;
+  int bn, k_split;
   size_t partial, need;
 };
 GemmPlan gemm_plan(int M, const cham_wpack_desc* d, int act_fmt) {
   GemmPlan g{};
   const int num_sms = num_sms_current();
-  const OperandPlan o = operand_plan(d, act_fmt);
   const int ch_tiles = d->n_tiles[0] + d->n_tiles[1];
-  int ks_max = 1;
-  if (o.fp8) {
-    g.bn8 = cham::gemm_pick_bn_f8(M);
-    g.ks8 = cham::gemm_pick_split(d->n_tiles[0] * ((M + g.bn8 - 1) / g.bn8), (d->Kp / 64 + 1) / 2, num_sms);
-    ks_max = std::max(ks_max, g.ks8);
-  }
-  if (o.f16) {
-    g.bn16 = cham::gemm_pick_bn(M, o.f16_tiles, num_sms);
-    g.ks16 = cham::gemm_pick_split(o.f16_tiles * ((M + g.bn16 - 1) / g.bn16), d->Kp / 64, num_sms);
-    ks_max = std::max(ks_max, g.ks16);
+  if (operand_plan(d, act_fmt).fp8) {
+    g.bn = cham::gemm_pick_bn_f8(M);
+    g.k_split = cham::gemm_pick_split(ch_tiles * ((M + g.bn - 1) / g.bn), (d->Kp / 64 + 1) / 2, num_sms);
+  } else {
+    g.bn = cham::gemm_pick_bn(M, ch_tiles, num_sms);
+    g.k_split = cham::gemm_pick_split(ch_tiles * ((M + g.bn - 1) / g.bn), d->Kp / 64, num_sms);
   }
   g.partial = linear_ws(M, d, act_fmt).end;
-  g.need = g.partial + (ks_max > 1 ? round_up(static_cast<size_t>(ks_max) * M * 128 * ch_tiles * 4, 256) : 0);
+  g.need = g.partial + (g.k_split > 1 ? round_up(static_cast<size_t>(g.k_split) * M * 128 * ch_tiles * 4, 256) : 0);
   return g;
 }
 
@@ -877,6 +870,7 @@ cham_status prepare_common(const void* X, int M, const cham_wpack_desc* d, int a
   a.nvec = static_cast<int64_t>(M) * K / 8;
   a.num_sms = num_sms_current();
   a.codes = o.fp8 ? reinterpret_cast<uint2*>(w + L.codes) : nullptr;
+  a.kperm = o.fp8;  // the FP8 GEMM operand in the weight codes' group order
   a.deq = o.f16 ? reinterpret_cast<uint4*>(w + L.operand) : nullptr;
   a.e8m0 = nullptr;
   if (o.fp8 && act_fmt == CHAM_A_MXFP8) {
@@ -990,40 +984,35 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   }
   const int num_sms = num_sms_current();
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (o.fp8) {
-    // class-0 tiles on FP8 MMAs: the 1-byte codes (K-major rows of K bytes), chunks of 128
-    cham::GemmArgs g8 = g;
-    CUtensorMap map8;
-    s = make_act_map(&map8, w + L.codes, M, K, plan.bn8, 1);
-    if (s != CHAM_OK) return s;
-    g8.tile0 = 0;
-    g8.n_ch_tiles = d->n_tiles[0];
-    g8.n_chunks = (g.nk64 + 1) / 2;
-    g8.k_split = plan.ks8;
-    g8.partial = plan.ks8 > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
-    g8.b_fmt = act_fmt == CHAM_A_E5M2 ? 1 : 0;
-    if (act_fmt == CHAM_A_MXFP8) {
-      g8.act_e8 = w + L.e8;
-      g8.act_mp = L.mp;
-      g8.act_e8_plane = static_cast<int64_t>(L.mp) * 4;
-    }
-    const cudaError_t e = cham::launch_gemm_f8(map8, g8, num_sms, plan.bn8, st);
-    if (e != cudaSuccess) return cuda_fail(e, "fp8 gemm launch");
-    g.stall_chunk = -1;
-  }
+  g.tile0 = 0;
+  g.n_ch_tiles = tiles;
+  g.k_split = plan.k_split;
+  g.partial = plan.k_split > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
+  CUtensorMap map16;
   if (o.f16) {
     const void* operand = act_fmt == CHAM_A_FP16 ? X : static_cast<const void*>(w + L.operand);
-    CUtensorMap map;
-    s = make_act_map(&map, operand, M, K, plan.bn16, 2);
+    s = make_act_map(&map16, operand, M, K, plan.bn, 2);
     if (s != CHAM_OK) return s;
-    g.tile0 = o.f16_tile0;
-    g.n_ch_tiles = o.f16_tiles;
-    g.n_chunks = g.nk64;
-    g.k_split = plan.ks16;
-    g.partial = plan.ks16 > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
-    const cudaError_t e = cham::launch_gemm_f16(map, g, num_sms, plan.bn16, st);
-    if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
   }
+  if (o.fp8) {
+    // class-0 tiles on FP8 MMAs (the 1-byte codes, K-major rows of K bytes), NF4 tiles on fp16
+    CUtensorMap map8;
+    s = make_act_map(&map8, w + L.codes, M, K, plan.bn, 1);
+    if (s != CHAM_OK) return s;
+    g.f8_tiles = d->n_tiles[0];
+    g.n_chunks = (g.nk64 + 1) / 2;
+    g.b_fmt = act_fmt == CHAM_A_E5M2 ? 1 : 0;
+    if (act_fmt == CHAM_A_MXFP8) {
+      g.act_e8 = w + L.e8;
+      g.act_mp = L.mp;
+      g.act_e8_plane = static_cast<int64_t>(L.mp) * 4;
+    }
+    const cudaError_t e = cham::launch_gemm_f8(map8, o.f16 ? map16 : map8, g, num_sms, plan.bn, st);
+    return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "fp8 gemm launch");
+  }
+  g.n_chunks = g.nk64;
+  const cudaError_t e = cham::launch_gemm_f16(map16, g, num_sms, plan.bn, st);
+  if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
   return CHAM_OK;
 }
 

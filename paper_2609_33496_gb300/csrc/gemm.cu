@@ -65,24 +65,25 @@ int gemm_pick_bn_f8(int M) {
   return kF8TokenTile;
 }
 
-cudaError_t launch_gemm_f8(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
+cudaError_t launch_gemm_f8(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms, int bn,
+                           cudaStream_t st) {
   const bool mxa = a.act_e8 != nullptr;
   if (a.k_split > 1) {
-    const cudaError_t e = mxa ? launch_gemm_f8_yt<kPartialYT, true>(map, a, num_sms, bn, st)
-                              : launch_gemm_f8_yt<kPartialYT, false>(map, a, num_sms, bn, st);
+    const cudaError_t e = mxa ? launch_gemm_f8_yt<kPartialYT, true>(map8, map16, a, num_sms, bn, st)
+                              : launch_gemm_f8_yt<kPartialYT, false>(map8, map16, a, num_sms, bn, st);
     if (e != cudaSuccess) return e;
     return launch_splitk_reduce(a, num_sms, st);
   }
   switch (a.y_type) {
     case CHAM_Y_F16:
-      return mxa ? launch_gemm_f8_yt<CHAM_Y_F16, true>(map, a, num_sms, bn, st)
-                 : launch_gemm_f8_yt<CHAM_Y_F16, false>(map, a, num_sms, bn, st);
+      return mxa ? launch_gemm_f8_yt<CHAM_Y_F16, true>(map8, map16, a, num_sms, bn, st)
+                 : launch_gemm_f8_yt<CHAM_Y_F16, false>(map8, map16, a, num_sms, bn, st);
     case CHAM_Y_BF16:
-      return mxa ? launch_gemm_f8_yt<CHAM_Y_BF16, true>(map, a, num_sms, bn, st)
-                 : launch_gemm_f8_yt<CHAM_Y_BF16, false>(map, a, num_sms, bn, st);
+      return mxa ? launch_gemm_f8_yt<CHAM_Y_BF16, true>(map8, map16, a, num_sms, bn, st)
+                 : launch_gemm_f8_yt<CHAM_Y_BF16, false>(map8, map16, a, num_sms, bn, st);
     default:
-      return mxa ? launch_gemm_f8_yt<CHAM_Y_F32, true>(map, a, num_sms, bn, st)
-                 : launch_gemm_f8_yt<CHAM_Y_F32, false>(map, a, num_sms, bn, st);
+      return mxa ? launch_gemm_f8_yt<CHAM_Y_F32, true>(map8, map16, a, num_sms, bn, st)
+                 : launch_gemm_f8_yt<CHAM_Y_F32, false>(map8, map16, a, num_sms, bn, st);
   }
 }
 

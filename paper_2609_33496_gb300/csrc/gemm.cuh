@@ -38,6 +38,8 @@ struct GemmArgs {
   int kblocks;               // K / 32
   int nk64;                  // 64-element chunks of the blob (Kp / 64)
   int b_fmt;                 // activation element type of the MMA: 0 E4M3, 1 E5M2
+  int f8_tiles;              // the first f8_tiles channel tiles of the launch run on FP8 MMAs, the rest
+                             // (NF4) on fp16 MMAs
 };
 
 // Token tile of the FP8 kernel for M > 128: 160 leaves room in tensor memory for the scale factors
@@ -53,11 +55,14 @@ int gemm_pick_split(int tiles, int n_chunks, int num_sms);
 int gemm_pick_bn_f8(int M);
 // Persistent launch: min(tiles, num_sms) CTAs walk the (channel tile, token tile) grid.
 cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
-// The FP8 kernel (gemm_f8_kernel.cuh) over the launch's class-0 channel tiles; act_map holds the
-// activation codes (uint8).
-cudaError_t launch_gemm_f8(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
+// The FP8 kernel (gemm_f8_kernel.cuh) over a 4-bit layout: its first f8_tiles channel tiles on
+// FP8 MMAs with the activation codes (map8, uint8), the rest (NF4) on fp16 MMAs with the fp16
+// operand (map16).
+cudaError_t launch_gemm_f8(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms, int bn,
+                           cudaStream_t st);
 template <int YT, bool MXA>
-cudaError_t launch_gemm_f8_yt(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
+cudaError_t launch_gemm_f8_yt(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms,
+                              int bn, cudaStream_t st);
 // Split-K units' raw sums (EPI 6) and the reduction over the launch's tiles.
 cudaError_t launch_splitk_reduce(const GemmArgs& a, int num_sms, cudaStream_t st);
 // The launches of one output type (instantiated in gemm.cu, gemm_f16.cu, gemm_bf16.cu).
@@ -67,13 +72,15 @@ extern template cudaError_t launch_gemm_yt<CHAM_Y_F32>(const CUtensorMap&, const
 extern template cudaError_t launch_gemm_yt<CHAM_Y_F16>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
 extern template cudaError_t launch_gemm_yt<CHAM_Y_BF16>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
 constexpr int kPartialYT = 3;  // "output type" of split-K units: raw fp32 partial sums
-extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-extern template cudaError_t launch_gemm_f8_yt<kPartialYT, false>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-extern template cudaError_t launch_gemm_f8_yt<kPartialYT, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+// the FP8 launcher's signature, instantiated per output type and activation kind
+#define CHAM_F8_LAUNCH_ARGS const CUtensorMap&, const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, false>(CHAM_F8_LAUNCH_ARGS);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, false>(CHAM_F8_LAUNCH_ARGS);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, false>(CHAM_F8_LAUNCH_ARGS);
+extern template cudaError_t launch_gemm_f8_yt<kPartialYT, false>(CHAM_F8_LAUNCH_ARGS);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, true>(CHAM_F8_LAUNCH_ARGS);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, true>(CHAM_F8_LAUNCH_ARGS);
+extern template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, true>(CHAM_F8_LAUNCH_ARGS);
+extern template cudaError_t launch_gemm_f8_yt<kPartialYT, true>(CHAM_F8_LAUNCH_ARGS);
 
 }  // namespace cham

@@ -1,7 +1,7 @@
-// gemm_f8_kernel.cuh -- the mixed-format linear on 8-bit tensor cores (steps a7, Sec. 3.6): the
-// kernel template for the 4-bit weight channels whose every decoded value is an exact E4M3 number,
-// against FP8 activation codes (E4M3 or E5M2 with a per-tensor scale, or MXFP8 blocks).
-// Instantiated in gemm_f8.cu (per-tensor activations) and gemm_f8_mx.cu (MXFP8 activations).
+// gemm_f8_kernel.cuh -- the 4-bit mixed-format linear on 8-bit tensor cores (steps a7, Sec. 3.6):
+// the kernel template for the 4-bit per-channel layouts whose class-0 channels (every decoded value
+// an exact E4M3 number) meet FP8 activation codes (E4M3 or E5M2 with a per-tensor scale, or MXFP8
+// blocks).  Instantiated in gemm_f8.cu (per-tensor activations) and gemm_f8_mx.cu (MXFP8).
 //
 // Y[m, perm[p]] = s_a * s_w[p] * sum_b 2^(e_w[p, b] + e_a[m, b]) sum_{k in block b} A^[m, k] W^[p, k] + bias
 //
@@ -13,17 +13,25 @@
 // the activation-side scale factors.  The product is the same sum the fp16 path forms from the
 // dequantized operands; only the accumulation order inside the tensor core differs.
 //
+// One launch covers every tile of the layer: the class-1 tiles of a 4-bit layout (NF4, whose levels
+// are not 8-bit floats) take a second mainloop in the same kernel -- kind::f16 MMAs on the exact
+// fp16 activation operand, NF4 levels decoded to fp16 -- so that the two classes' output columns,
+// which interleave in Y, are written at the same time (two launches would each leave fp32 output
+// sectors half written, and the second one's writes would miss in L2), and neither class waits for
+// the other's last wave.
+//
 // Structure (as the fp16 kernel in gemm_kernel.cuh, whose epilogue role it shares):
 //   * MMA "A" (M = 128) = 128 packed weight channels decoded into tensor memory, one thread per
-//     channel: every 4-bit code indexes that channel's own 16-entry table of E4M3 bytes (built once
-//     per tile from the format and zero point), so channels of different formats in one tile take
-//     the same instructions.  Two byte permutes per four codes look the table up; the channel's
-//     four block exponents of the chunk go to the A scale-factor columns.
-//   * MMA "B" (N = BN tokens) = 128 activation code bytes per row, loaded by TMA with 128-byte
-//     swizzling; MXFP8 activations also bring their chunk's exponents (4 bytes per token).
-//   * K-chunks of 128 elements: 4 MMAs (kind::mxf8f6f4, K = 32 each, scale vector 1X: one E8M0
-//     per row per MMA, selected by the instruction's scale-factor ids); the last chunk issues only
-//     the MMAs of the 32-element blocks inside K.
+//     channel.  FP8 tiles: every 4-bit code indexes that channel's own 16-entry table of E4M3 bytes
+//     (built once per tile from the format and zero point), so channels of different formats in
+//     one tile take the same instructions; the channel's four block exponents of the chunk go to
+//     the A scale-factor columns.  NF4 tiles: the levels as fp16 pairs from byte tables.
+//   * MMA "B" (N = BN tokens) = 128 bytes per activation row, loaded by TMA with 128-byte
+//     swizzling: 128 FP8 codes (MXFP8 also brings its chunk's exponents, 4 bytes per token) or 64
+//     fp16 operand values.
+//   * K-chunks of 128 (FP8: 4 MMAs kind::mxf8f6f4, K = 32 each, scale vector 1X -- one E8M0 per row
+//     per MMA, selected by the instruction's scale-factor ids -- the last chunk issuing only the
+//     MMAs of the 32-element blocks inside K) or of 64 (NF4: 4 MMAs kind::f16, K = 16).
 // Tensor-memory columns: two accumulators, four decoded-weight slots of 32 columns, the A scale
 // factors of each slot (8 columns apart, lane m reads column base + m / 32), and the B scale
 // factors (every lane quadrant holds all BN tokens: lane 32q + n % 32, column base + n / 32) --
@@ -126,6 +134,9 @@ CHAM_DEV void f8_table(int f, int z, uint32_t (&T)[4]) {
   }
 }
 
+// Sign-magnitude formats (E2M1, MXFP4: bit 3 of the code is the sign, bits 0-2 the magnitude).
+CHAM_DEV bool f8_sign_magnitude(int f) { return f == CHAM_W_E2M1 || f == CHAM_W_MXFP4; }
+
 // Four codes (the selector nibbles of sel; bit 3 of each code in the byte mask m) -> four table bytes.
 CHAM_DEV uint32_t f8_lookup4(uint32_t sel, uint32_t m, const uint32_t (&T)[4]) {
   const uint32_t lo = prmt(T[0], T[1], sel), hi = prmt(T[2], T[3], sel);
@@ -133,8 +144,12 @@ CHAM_DEV uint32_t f8_lookup4(uint32_t sel, uint32_t m, const uint32_t (&T)[4]) {
 }
 
 // 128 codes of one channel (16 words, word i = elements 8i..8i+7 with nibble j = element 2j for
-// j < 4 and element 2(j - 4) + 1 for j >= 4, the blob's 4-bit order) -> 32 columns of E4M3 bytes,
-// column c = elements 4c..4c+3 (byte order = element order, the MMA's K order in tensor memory).
+// j < 4 and element 2(j - 4) + 1 for j >= 4, the blob's 4-bit order) -> 32 columns of E4M3 bytes in
+// the same group order: column 2i holds elements 8i, 8i+2, 8i+4, 8i+6 and column 2i+1 holds 8i+1,
+// 8i+3, 8i+5, 8i+7 (the activation codes of the FP8 operand are stored in that order too, so the
+// MMA still pairs element k with element k).  SM: every lane's table is sign-magnitude (entries
+// 8..15 are 0..7 with the sign bit), so one permute of the magnitudes and the sign bit suffice.
+template <bool SM>
 CHAM_DEV void decode_f8(const uint32_t (&w)[16], const uint32_t (&T)[4], uint32_t (&out)[32]) {
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
@@ -143,18 +158,24 @@ CHAM_DEV void decode_f8(const uint32_t (&w)[16], const uint32_t (&T)[4], uint32_
     // byte mask of each code's bit 3: PRMT with the sign-replicate selector bit copies bit 7 of the
     // byte that holds that bit (x << 4 for the low nibble of a byte, x for the high one)
     const uint32_t mlo = prmt(x4, x, 0xD9C8u), mhi = prmt(x4, x, 0xFBEAu);
-    const uint32_t even = f8_lookup4(s, mlo, T);         // elements 0, 2, 4, 6
-    const uint32_t odd = f8_lookup4(s >> 16, mhi, T);    // elements 1, 3, 5, 7
-    out[2 * i] = prmt(even, odd, 0x5140u);
-    out[2 * i + 1] = prmt(even, odd, 0x7362u);
+    if constexpr (SM) {
+      out[2 * i] = prmt(T[0], T[1], s) | (mlo & 0x80808080u);
+      out[2 * i + 1] = prmt(T[0], T[1], s >> 16) | (mhi & 0x80808080u);
+    } else {
+      out[2 * i] = f8_lookup4(s, mlo, T);
+      out[2 * i + 1] = f8_lookup4(s >> 16, mhi, T);
+    }
   }
 }
 
-// MXA: the activations are MXFP8 (their exponents come with every stage); otherwise E4M3 / E5M2
-// codes with a per-tensor (or per-sample) scale and constant unit B scale factors.
+// MXA: the activations are MXFP8 (their exponents come with every FP8 stage); otherwise E4M3 /
+// E5M2 codes with a per-tensor (or per-sample) scale and constant unit B scale factors.  Channel
+// tiles tile0 .. tile0 + f8_tiles - 1 take the FP8 mainloop (map8: the codes), the rest of the
+// launch's tiles the NF4 / fp16 one (map16: the fp16 operand).
 template <int BN, int EPI, bool MXA>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-    k_gemm_ts_f8(const __grid_constant__ CUtensorMap act_map, const GemmArgs a) {
+    k_gemm_ts_f8(const __grid_constant__ CUtensorMap map8, const __grid_constant__ CUtensorMap map16,
+                 const GemmArgs a) {
   using C = F8Cfg<BN, MXA>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -172,13 +193,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nk = a.n_chunks;  // 128-element chunks
+  const int nk8 = (a.nk64 + 1) / 2;  // chunks of 128 (FP8 tiles); NF4 tiles walk the nk64 chunks of 64
   const int n_ch = a.n_ch_tiles;
   const int n_tiles = n_ch * ((a.M + BN - 1) / BN);
   const int ks = a.k_split;
   const int n_units = n_tiles * ks;
-  auto kc_begin = [&](int u) { return ks == 1 ? 0 : (u % ks) * nk / ks; };
-  auto kc_end = [&](int u) { return ks == 1 ? nk : (u % ks + 1) * nk / ks; };
+  auto is_f8 = [&](int u) { return (u / ks) % n_ch < a.f8_tiles; };
+  auto kc_begin = [&](int u) { return ks == 1 ? 0 : (u % ks) * (is_f8(u) ? nk8 : a.nk64) / ks; };
+  auto kc_end = [&](int u) { const int nk = is_f8(u) ? nk8 : a.nk64; return ks == 1 ? nk : (u % ks + 1) * nk / ks; };
   uint32_t total = 0;
   for (int u = blockIdx.x; u < n_units; u += gridDim.x) total += static_cast<uint32_t>(kc_end(u) - kc_begin(u));
   auto wait_done = [&](uint32_t j) {
@@ -197,7 +219,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) tma_prefetch_desc(&act_map);
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&map8);
+    if (a.f8_tiles < n_ch) tma_prefetch_desc(&map16);
+  }
   if (warp == 2) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
   __syncthreads();
@@ -207,14 +232,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   griddep_launch_dependents();
 
   if (warp == 0) {
-    // ---------------- producer: activation codes (TMA), two blob chunks of weight codes and their
-    // E8M0 bytes (bulk), MXFP8: the chunk's activation exponents of the tile's tokens (bulk)
+    // ---------------- producer.  FP8 chunk: activation codes (TMA), two blob chunks of weight codes
+    // and their E8M0 bytes (bulk), MXFP8: the chunk's activation exponents of the tile's tokens
+    // (bulk).  NF4 chunk: fp16 operand (TMA) and one blob chunk of codes.
     if (lane == 0) {
       uint32_t it = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
         const int t = u / ks;
         const int ch = a.tile0 + t % n_ch, tok0 = (t / n_ch) * BN;
+        const bool f8 = is_f8(u);
         const int kc1 = kc_end(u);
         const uint32_t sf_bytes = MXA ? static_cast<uint32_t>(min(BN, a.act_mp - tok0)) * 4u : 0u;
         for (int kc = kc_begin(u); kc < kc1; ++kc, ++it) {
@@ -224,18 +251,22 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             break;
           }
           uint8_t* st = smem + s * C::kStage;
-          const int nh = 2 * kc + 1 < a.nk64 ? 2 : 1;  // the last chunk may hold one blob chunk
-          const size_t chunk64 = static_cast<size_t>(ch) * a.nk64 + 2 * kc;
-          mbar_arrive_expect_tx(&full[s], C::kBBytes + nh * (C::kWBytes / 2 + C::kEBytes / 2) + sf_bytes);
+          // FP8: the last chunk may hold one blob chunk; NF4: always one
+          const int nh = f8 ? (2 * kc + 1 < a.nk64 ? 2 : 1) : 1;
+          const size_t chunk64 = static_cast<size_t>(ch) * a.nk64 + (f8 ? 2 * kc : kc);
+          const uint32_t e_bytes = f8 ? nh * (C::kEBytes / 2) : 0u;
+          mbar_arrive_expect_tx(&full[s], C::kBBytes + nh * (C::kWBytes / 2) + e_bytes + (f8 ? sf_bytes : 0u));
           if (blockIdx.x == 0 && static_cast<int>(it) == a.stall_chunk) continue;  // test hook (see the fp16 kernel)
-          tma_load_2d(smem_u32(st), &act_map, &full[s], kc * kBK8, tok0);
+          if (f8) tma_load_2d(smem_u32(st), &map8, &full[s], kc * kBK8, tok0);
+          else tma_load_2d(smem_u32(st), &map16, &full[s], kc * kBK, tok0);
           bulk_load(smem_u32(st + C::kBBytes), a.codes + chunk64 * (C::kWBytes / 2), nh * (C::kWBytes / 2), &full[s]);
-          bulk_load(smem_u32(st + C::kBBytes + C::kWBytes), a.we8m0 + chunk64 * (C::kEBytes / 2),
-                    nh * (C::kEBytes / 2), &full[s]);
-          if constexpr (MXA)
-            bulk_load(smem_u32(st + C::kBBytes + C::kWBytes + C::kEBytes),
-                      a.act_e8 + static_cast<size_t>(kc) * a.act_e8_plane + static_cast<size_t>(tok0) * 4, sf_bytes,
-                      &full[s]);
+          if (f8) {
+            bulk_load(smem_u32(st + C::kBBytes + C::kWBytes), a.we8m0 + chunk64 * (C::kEBytes / 2), e_bytes, &full[s]);
+            if constexpr (MXA)
+              bulk_load(smem_u32(st + C::kBBytes + C::kWBytes + C::kEBytes),
+                        a.act_e8 + static_cast<size_t>(kc) * a.act_e8_plane + static_cast<size_t>(tok0) * 4,
+                        sf_bytes, &full[s]);
+          }
         }
       }
       const uint32_t first = it > S ? it - S : 0;
@@ -244,7 +275,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   } else if (warp == 1) {
     // ---------------- MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = idesc_mxf8(128, BN, a.b_fmt);
+      const uint32_t idesc8 = idesc_mxf8(128, BN, a.b_fmt);
+      constexpr uint32_t idesc16 = idesc_f16(128, BN);
       const uint64_t desc0 = smem_desc_sw128(smem_u32(smem));
       constexpr uint32_t kStageDesc = C::kStage >> 4;
       uint32_t it = 0, acc_it = 0, s = 0, sa = 0, gi = 0;
@@ -252,6 +284,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++acc_it) {
         const int b = acc_it & 1;
         const int kc0 = kc_begin(u), kc1 = kc_end(u);
+        const bool f8 = is_f8(u);
         if (!mbar_wait(&accempty[b], ((acc_it >> 1) & 1) ^ 1, abort_flag, a.dev_status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem + b * C::kAccCols;
@@ -265,12 +298,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           }
           const uint64_t bd = desc0 + s * kStageDesc;
           const uint32_t ad = tmem + C::kACol + sa * 32;
-          const uint32_t sfa = tmem + C::kSFA + sa * 8;
-          const uint32_t sfb = tmem + C::kSFB + (MXA ? sa * 8 : 0);
-          const int nmma = min(4, a.kblocks - 4 * kc);  // 32-element blocks of this chunk inside K
+          if (f8) {
+            const uint32_t sfa = tmem + C::kSFA + sa * 8;
+            const uint32_t sfb = tmem + C::kSFB + (MXA ? sa * 8 : 0);
+            const int nmma = min(4, a.kblocks - 4 * kc);  // 32-element blocks of this chunk inside K
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            if (i < nmma) mma_mxf8_ts(d_tmem, ad + 8 * i, bd + 2 * i, idesc_sf_ids(idesc, i), sfa, sfb, kc != kc0 || i > 0);
+            for (int i = 0; i < 4; ++i)
+              if (i < nmma)
+                mma_mxf8_ts(d_tmem, ad + 8 * i, bd + 2 * i, idesc_sf_ids(idesc8, i), sfa, sfb, kc != kc0 || i > 0);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) mma_f16_ts(d_tmem, ad + 8 * i, bd + 2 * i, idesc16, kc != kc0 || i > 0);
+          }
           if (++gi == kGroup || it + 1 == total) {
             mma_commit(&done[(it / kGroup) % kDone]);
             gi = gi == kGroup ? 0 : gi;
@@ -278,14 +317,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           s = s + 1 == static_cast<uint32_t>(S) ? 0 : s + 1;
           sa = sa + 1 == static_cast<uint32_t>(kAStages) ? 0 : sa + 1;
         }
-        if (!ok) break;
-        mma_commit(&accfull[b]);
+        mma_commit(&accfull[b]);  // after an abort inside the tile this still covers every MMA issued
       }
-      // every issued MMA has finished before tensor memory is released: one more commit covers them all
-      if (it > 0 || acc_it > 0) {
-        mma_commit(&accfull[acc_it & 1]);
-        drain_wait(&accfull[acc_it & 1], (acc_it >> 1) & 1);
-      }
+      // all issued MMAs have finished before tensor memory is released
+      if (acc_it > 0) drain_wait(&accfull[(acc_it - 1) & 1], ((acc_it - 1) >> 1) & 1);
     }
   } else if (warp >= 4 && warp < 4 + 4 * kDec) {
     // ---------------- weight decode: one channel per thread; group g takes chunks it % kDec == g
@@ -311,8 +346,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       nz = a.wzero[p0];
     }
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+      const bool f8 = is_f8(u);
       uint32_t T[4];
       f8_table(nf, nz, T);
+      const bool sm = __all_sync(0xffffffffu, f8_sign_magnitude(nf));  // the warp's channels
       if (u + static_cast<int>(gridDim.x) < n_units) {
         const int pn = (a.tile0 + ((u + static_cast<int>(gridDim.x)) / ks) % n_ch) * 128 + r;
         nf = a.wfmt[pn];
@@ -328,30 +365,50 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           break;
         }
         const uint8_t* st = smem + s * C::kStage;
-        const int nh = 2 * kc + 1 < a.nk64 ? 2 : 1;
-        const uint16_t* e8 = reinterpret_cast<const uint16_t*>(st + C::kBBytes + C::kWBytes);
-        // block exponents of the chunk's four 32-element blocks (a missing second half is never read)
-        const uint32_t sfa = static_cast<uint32_t>(e8[r]) | (nh == 2 ? static_cast<uint32_t>(e8[128 + r]) << 16 : 0x7F7F0000u);
-        uint32_t raw[16];
+        uint32_t out[32];
+        uint32_t sfa = 0;
+        uint32_t sfb[8];
+        if (f8) {
+          const int nh = 2 * kc + 1 < a.nk64 ? 2 : 1;
+          const uint16_t* e8 = reinterpret_cast<const uint16_t*>(st + C::kBBytes + C::kWBytes);
+          // block exponents of the chunk's four 32-element blocks (a missing second half is never read)
+          sfa = static_cast<uint32_t>(e8[r]) | (nh == 2 ? static_cast<uint32_t>(e8[128 + r]) << 16 : 0x7F7F0000u);
+          uint32_t raw[16];
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+              uint4 v = make_uint4(0, 0, 0, 0);
+              if (h < nh) v = *reinterpret_cast<const uint4*>(st + C::kBBytes + h * 4096 + j * 2048 + r * 16);
+              raw[8 * h + 4 * j] = v.x;
+              raw[8 * h + 4 * j + 1] = v.y;
+              raw[8 * h + 4 * j + 2] = v.z;
+              raw[8 * h + 4 * j + 3] = v.w;
+            }
+          if (sm) decode_f8<true>(raw, T, out);
+          else decode_f8<false>(raw, T, out);
+          if constexpr (MXA) {
+            // this lane's tokens n = 32 c + lane of the tile, in every lane quadrant
+            const uint32_t* se = reinterpret_cast<const uint32_t*>(st + C::kBBytes + C::kWBytes + C::kEBytes);
+#pragma unroll
+            for (int c = 0; c < 8; ++c) sfb[c] = c < C::kSFBCols ? se[32 * c + lane] : 0x7F7F7F7Fu;
+          }
+        } else {
+          // NF4 (element order in the codes): levels as fp16 pairs; the scale stays in the epilogue
+          uint32_t raw[8];
 #pragma unroll
           for (int j = 0; j < 2; ++j) {
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (h < nh) v = *reinterpret_cast<const uint4*>(st + C::kBBytes + h * 4096 + j * 2048 + r * 16);
-            raw[8 * h + 4 * j] = v.x;
-            raw[8 * h + 4 * j + 1] = v.y;
-            raw[8 * h + 4 * j + 2] = v.z;
-            raw[8 * h + 4 * j + 3] = v.w;
+            const uint4 v = *reinterpret_cast<const uint4*>(st + C::kBBytes + j * 2048 + r * 16);
+            raw[4 * j] = v.x;
+            raw[4 * j + 1] = v.y;
+            raw[4 * j + 2] = v.z;
+            raw[4 * j + 3] = v.w;
           }
-        uint32_t out[32];
-        decode_f8(raw, T, out);
-        uint32_t sfb[8];
-        if constexpr (MXA) {
-          // this lane's tokens n = 32 c + lane of the tile, in every lane quadrant
-          const uint32_t* se = reinterpret_cast<const uint32_t*>(st + C::kBBytes + C::kWBytes + C::kEBytes);
 #pragma unroll
-          for (int c = 0; c < 8; ++c) sfb[c] = c < C::kSFBCols ? se[32 * c + lane] : 0x7F7F7F7Fu;
+          for (int i = 0; i < 8; ++i) {
+            nf4_lookup4(raw[i] & 0xFFFFu, a.nf4_lo, a.nf4_hi, out[4 * i], out[4 * i + 1]);
+            nf4_lookup4(raw[i] >> 16, a.nf4_lo, a.nf4_hi, out[4 * i + 2], out[4 * i + 3]);
+          }
         }
         const bool free_ok = it < static_cast<uint32_t>(kAStages) || wait_done(it - kAStages);
         if (!__all_sync(0xffffffffu, free_ok)) {
@@ -361,8 +418,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         __syncwarp();
         tc_fence_after();
         tmem_st_32x32b_x32(tmem + C::kACol + lane_off + sa * 32, out);
-        tmem_st_32x32b_x1(tmem + C::kSFA + lane_off + sa * 8 + q, sfa);
-        if constexpr (MXA) tmem_st_32x32b_x8(tmem + C::kSFB + lane_off + sa * 8, sfb);
+        if (f8) {
+          tmem_st_32x32b_x1(tmem + C::kSFA + lane_off + sa * 8 + q, sfa);
+          if constexpr (MXA) tmem_st_32x32b_x8(tmem + C::kSFB + lane_off + sa * 8, sfb);
+        }
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
@@ -385,7 +444,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 }
 
 template <int BN, int EPI, bool MXA>
-static cudaError_t launch_f8_bn(const CUtensorMap& map, const GemmArgs& a, int num_sms, cudaStream_t st) {
+static cudaError_t launch_f8_bn(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms,
+                                cudaStream_t st) {
   using C = F8Cfg<BN, MXA>;
   static int configured_device = -1;
   int dev = 0;
@@ -398,16 +458,17 @@ static cudaError_t launch_f8_bn(const CUtensorMap& map, const GemmArgs& a, int n
   }
   const long units = static_cast<long>(a.n_ch_tiles) * ((a.M + BN - 1) / BN) * a.k_split;
   const int grid = static_cast<int>(units < num_sms ? units : num_sms);
-  return launch_pdl(k_gemm_ts_f8<BN, EPI, MXA>, dim3(grid), dim3(kGemmThreads), C::kSmem, st, map, a);
+  return launch_pdl(k_gemm_ts_f8<BN, EPI, MXA>, dim3(grid), dim3(kGemmThreads), C::kSmem, st, map8, map16, a);
 }
 
 template <int EPI, bool MXA>
-static cudaError_t launch_f8_epi(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
+static cudaError_t launch_f8_epi(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms,
+                                 int bn, cudaStream_t st) {
   switch (bn) {
-    case 32: return launch_f8_bn<32, EPI, MXA>(map, a, num_sms, st);
-    case 64: return launch_f8_bn<64, EPI, MXA>(map, a, num_sms, st);
-    case 128: return launch_f8_bn<128, EPI, MXA>(map, a, num_sms, st);
-    default: return launch_f8_bn<kF8TokenTile, EPI, MXA>(map, a, num_sms, st);
+    case 32: return launch_f8_bn<32, EPI, MXA>(map8, map16, a, num_sms, st);
+    case 64: return launch_f8_bn<64, EPI, MXA>(map8, map16, a, num_sms, st);
+    case 128: return launch_f8_bn<128, EPI, MXA>(map8, map16, a, num_sms, st);
+    default: return launch_f8_bn<kF8TokenTile, EPI, MXA>(map8, map16, a, num_sms, st);
   }
 }
 

@@ -6,13 +6,14 @@
 namespace cham {
 
 template <int YT, bool MXA>
-cudaError_t launch_gemm_f8_yt(const CUtensorMap& map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st) {
-  return launch_f8_epi<2 * YT, MXA>(map, a, num_sms, bn, st);
+cudaError_t launch_gemm_f8_yt(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms, int bn,
+                              cudaStream_t st) {
+  return launch_f8_epi<2 * YT, MXA>(map8, map16, a, num_sms, bn, st);
 }
 
-template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
-template cudaError_t launch_gemm_f8_yt<kPartialYT, true>(const CUtensorMap&, const GemmArgs&, int, int, cudaStream_t);
+template cudaError_t launch_gemm_f8_yt<CHAM_Y_F32, true>(CHAM_F8_LAUNCH_ARGS);
+template cudaError_t launch_gemm_f8_yt<CHAM_Y_F16, true>(CHAM_F8_LAUNCH_ARGS);
+template cudaError_t launch_gemm_f8_yt<CHAM_Y_BF16, true>(CHAM_F8_LAUNCH_ARGS);
+template cudaError_t launch_gemm_f8_yt<kPartialYT, true>(CHAM_F8_LAUNCH_ARGS);
 
 }  // namespace cham

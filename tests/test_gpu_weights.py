@@ -148,3 +148,34 @@ def test_fused_select_pack_equals_the_two_launches(cl, mask, K):
     for off, n in [(0, 256), (d.off_codes, tiles * chunks * 128 * cb), (d.off_scale, 4 * np_), (d.off_zero, np_),
                    (d.off_e8m0, tiles * chunks * 256), (d.off_fmt, np_), (d.off_perm, 4 * np_)]:
         assert np.array_equal(a[off:off + n], c[off:off + n]), off
+
+
+@pytest.mark.parametrize("layer", range(len(WL.SDXL_PROJ_LAYERS)))
+def test_fused_select_pack_against_oracle_on_benchmark_weights(cl, layer):
+    """The fused selection + pack the benchmark's step runs (chameleon_select_pack_palette, W8
+    palette), checked directly against the oracle on the ten SDXL projection weights the benchmark
+    packs: formats equal except at oracle near-ties, and the blob's codes, scales, zero points and
+    E8M0 bytes of each channel equal the oracle's encoding of the format the kernel chose.  Layers
+    with more than 1280 channels are checked on 1024 seeded channels."""
+    import torch
+    name, M, K, N = WL.SDXL_PROJ_LAYERS[layer]
+    W, _ = WL.sdxl_layer_weights(layer)
+    d = cl.pack_plan_palette(N, K, cl.PALETTE_W8)
+    fmt_d, blob, st = cl.select_pack_palette(cuda(W), cl.PALETTE_W8, d)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    fmt_g = host(fmt_d)
+    rows = np.arange(N) if N <= 1280 else np.sort(np.random.default_rng(layer).choice(N, 1024, replace=False))
+    fmt_o, sse_o, _ = SEL.select_formats(W[rows], cl.PALETTE_W8)
+    for i in np.nonzero(fmt_g[rows] != fmt_o)[0]:
+        assert SEL.near_tie(sse_o[i]), (name, rows[i], fmt_g[rows[i]], fmt_o[i])
+    _, got = unpack(host(blob).tobytes())
+    ref = SEL.quantize_selected(W[rows], fmt_g[rows])
+    for c, r in zip(rows, ref):
+        g = got[int(c)]
+        assert g["fmt"] == r["fmt"] == fmt_g[c]
+        np.testing.assert_array_equal(g["codes"], r["codes"], err_msg="%s channel %d" % (name, c))
+        if F.W_IS_MX[r["fmt"]]:
+            np.testing.assert_array_equal(g["e8m0"], r["e8m0"])
+        else:
+            assert np.float32(g["s"]).tobytes() == np.float32(r["s"]).tobytes() and g["z"] == r["z"]

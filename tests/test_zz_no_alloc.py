@@ -46,3 +46,30 @@ def test_noalloc_rejects_bad_arguments():
     assert cl.act_quant_noalloc(X, 1, out, st) == cl.ERR_INVALID_ARG        # K not a multiple of 32
     X = torch.zeros((64, 64), dtype=torch.float16, device="cuda")
     assert cl.act_quant_noalloc(X, 1, out[:16], st) == cl.ERR_WORKSPACE     # output buffer too small
+
+
+def test_noalloc_reports_nonfinite_input_and_takes_exactly_sized_outputs():
+    """An Inf in X reaches the caller's status word as CHAM_ERR_NONFINITE for every format, and an
+    output buffer of exactly the size act_quant_size gives is accepted for shapes whose M * K is not
+    a multiple of 256 (the parameter and exponent regions then start at rounded offsets)."""
+    import torch
+    cl = lib_module()
+    g = np.random.default_rng(20260101)
+    for M, K in [(3, 32), (7, 96), (333, 640)]:
+        X = (g.standard_normal((M, K)) * 0.5).astype(np.float16)
+        for fmt in range(5):
+            qb, _ = cl.act_quant_size(M, K, fmt)
+            Xd = cuda(X)
+            out = torch.empty((qb,), dtype=torch.uint8, device=Xd.device)
+            st = torch.zeros(1, dtype=torch.int32, device=Xd.device)
+            assert cl.act_quant_noalloc(Xd, fmt, out, st) == cl.OK
+            ref, st_ref = cl.act_quant(Xd, fmt)
+            torch.cuda.synchronize()
+            assert int(st.item()) == 0 and int(st_ref.item()) == 0
+            np.testing.assert_array_equal(host(cl.split_qact(out, M, K)[0]), host(cl.split_qact(ref, M, K)[0]))
+            bad = X.copy()
+            bad[M // 2, K - 1] = np.float16(np.inf)
+            st.zero_()
+            assert cl.act_quant_noalloc(cuda(bad), fmt, out, st) == cl.OK
+            torch.cuda.synchronize()
+            assert int(st.item()) == cl.ERR_NONFINITE, (M, K, fmt)
