@@ -329,6 +329,15 @@ cham_status chameleon_pack_weights(const void* W, const uint8_t* fmt_dev, const 
 cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* desc, int act_fmt,
                                             size_t* ws_bytes);
 
+/* The kernels the linear calls launch for M rows of the layer *desc in act_fmt (host only, no GPU
+ * work): *prepare_launches for chameleon_linear_prepare (is_static = 0, n_groups row groups) or
+ * chameleon_linear_prepare_static (is_static = 1) -- 0 for CHAM_A_FP16, 1 for the static path and
+ * the MX formats, 2 (range, encode) for a per-tensor format's dynamic scales -- and
+ * *gemm_launches for chameleon_linear_gemm(_ex): 1, or 2 when the GEMM splits K (the partial sums'
+ * reduction).  CHAM_ERR_INVALID_ARG as the size query, or for a NULL output pointer. */
+cham_status chameleon_linear_launches(int M, const cham_wpack_desc* desc, int act_fmt, int n_groups, int is_static,
+                                      int* prepare_launches, int* gemm_launches);
+
 /* Y = DQ(Q_act_fmt(X)) . DQ(W)^T + bias: X (device, fp16 M x desc->K) is quantized in act_fmt
  * (= F[layer, bucket] resolved on the host, Alg. 2/3) with its own range, multiplied on tcgen05
  * tensor cores with the packed weights (device blob made from *desc, host), fp32 accumulation;

@@ -31,7 +31,7 @@ EXPORTS = [
     "chameleon_act_moments_workspace_size", "chameleon_act_moments",
     "chameleon_act_quant_size", "chameleon_act_quant",
     "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_plan_palette", "chameleon_pack_weights",
-    "chameleon_linear_workspace_size", "chameleon_linear", "chameleon_linear_prepare",
+    "chameleon_linear_workspace_size", "chameleon_linear_launches", "chameleon_linear", "chameleon_linear_prepare",
     "chameleon_linear_gemm", "chameleon_act_quant_noalloc", "chameleon_debug_stall_next_gemm",
     "chameleon_scale_zp", "chameleon_act_quant_static", "chameleon_linear_prepare_static",
     "chameleon_linear_prepare_groups", "chameleon_linear_gemm_ex",
@@ -110,6 +110,8 @@ def lib():
         "chameleon_pack_plan_palette": (i32, [i32, i32, ctypes.c_uint32, pdesc]),
         "chameleon_pack_weights": (i32, [vp, vp, pdesc, vp, sz, vp, vp]),
         "chameleon_linear_workspace_size": (i32, [i32, pdesc, i32, psz]),
+        "chameleon_linear_launches": (i32, [i32, pdesc, i32, i32, i32, ctypes.POINTER(ctypes.c_int),
+                                            ctypes.POINTER(ctypes.c_int)]),
         "chameleon_linear": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
         "chameleon_linear_prepare": (i32, [vp, i32, pdesc, i32, vp, sz, vp, vp]),
         "chameleon_linear_gemm": (i32, [vp, i32, pdesc, vp, i32, vp, vp, vp, sz, vp, vp]),
@@ -245,18 +247,21 @@ def act_quant_size(M, K, fmt):
     return q.value, w.value
 
 
-def act_quant(X, fmt, dev_status=None, stream=None):
+def act_quant(X, fmt, dev_status=None, stream=None, qact=None, ws=None):
     """Quantize fp16 X (M x K, CUDA) in activation format fmt.  Returns the raw qact byte buffer
-    (layout of include/chameleon.h) and the device status word."""
+    (layout of include/chameleon.h) and the device status word.  qact and ws may be passed in for
+    reuse (uint8 CUDA tensors of at least the size query's bytes)."""
     import torch
     M, K = X.shape
     qb, wb = act_quant_size(M, K, fmt)
-    qact = _bytes(qb, X.device)
-    ws = _bytes(wb, X.device)
+    if qact is None or qact.numel() < qb:
+        qact = _bytes(qb, X.device)
+    if ws is None or ws.numel() < wb:
+        ws = _bytes(wb, X.device)
     if dev_status is None:
         dev_status = torch.zeros(1, dtype=torch.int32, device=X.device)
-    check(lib().chameleon_act_quant(_half(X, "X"), M, K, fmt, _ptr(qact), qb, _ptr(ws), wb, _ptr(dev_status),
-                                    _stream(stream)))
+    check(lib().chameleon_act_quant(_half(X, "X"), M, K, fmt, _ptr(qact), qact.numel(), _ptr(ws), ws.numel(),
+                                    _ptr(dev_status), _stream(stream)))
     return qact, dev_status
 
 
@@ -441,6 +446,15 @@ def linear_workspace_size(M, desc, act_fmt):
     w = ctypes.c_size_t()
     check(lib().chameleon_linear_workspace_size(M, ctypes.byref(desc), act_fmt, ctypes.byref(w)))
     return w.value
+
+
+def linear_launches(M, desc, act_fmt, n_groups=1, is_static=False):
+    """(prepare launches, gemm launches): the kernels chameleon_linear_prepare* and
+    chameleon_linear_gemm* launch for M rows of the layer desc in act_fmt (host only)."""
+    p, g = ctypes.c_int(), ctypes.c_int()
+    check(lib().chameleon_linear_launches(M, ctypes.byref(desc), act_fmt, n_groups, int(bool(is_static)),
+                                          ctypes.byref(p), ctypes.byref(g)))
+    return p.value, g.value
 
 
 def linear(X, desc, blob, act_fmt, bias=None, Y=None, ws=None, dev_status=None, stream=None):

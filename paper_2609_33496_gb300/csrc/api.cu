@@ -838,6 +838,19 @@ cham_status chameleon_linear_workspace_size(int M, const cham_wpack_desc* d, int
   return CHAM_OK;
 }
 
+cham_status chameleon_linear_launches(int M, const cham_wpack_desc* d, int act_fmt, int n_groups, int is_static,
+                                      int* prepare_launches, int* gemm_launches) {
+  cham_status s = check_desc(d);
+  if (s != CHAM_OK) return s;
+  if (M <= 0 || act_fmt < 0 || act_fmt > CHAM_A_FP16 || prepare_launches == nullptr || gemm_launches == nullptr)
+    return fail(CHAM_ERR_INVALID_ARG, "M=%d act_fmt=%d", M, act_fmt);
+  s = check_groups(M, n_groups);
+  if (s != CHAM_OK) return s;
+  *prepare_launches = act_fmt == CHAM_A_FP16 ? 0 : (is_static || act_fmt >= CHAM_A_MXFP8 ? 1 : 2);
+  *gemm_launches = gemm_plan(M, d, act_fmt).k_split > 1 ? 2 : 1;
+  return CHAM_OK;
+}
+
 }  // extern "C"
 
 

@@ -147,3 +147,63 @@ def config_layer(config, index, M, K, N, nu=7):
     W = weight_mix(g, N, K)
     bias = g.normal(0.0, 0.02, N).astype(np.float32)
     return X, W, bias
+
+
+# ------------------------------------------------------------------ PixArt-alpha DiT, whole model
+# PixArt-alpha XL/2 at 1024^2, batch 2 (4096 image tokens and 120 caption tokens per sample): the
+# caption projection (two linears on the 240 caption tokens), then 28 blocks of ten linears each --
+# self-attention q, k, v, out; cross-attention q, k, v (k and v on the caption tokens), out; MLP fc1
+# and fc2 -- 282 GEMMs per sampler step.  Each entry: (name, M, K, N, input); linears that read the
+# same tensor in the network (q, k, v of one attention; cross k and v) share an input key.
+PIXART_BLOCKS = 28
+PIXART_CAPTION_LINEARS = (("caption.fc1", 240, 4096, 1152, "caption"),
+                          ("caption.fc2", 240, 1152, 1152, "caption_hidden"))
+PIXART_BLOCK_LINEARS = (("self.q", 8192, 1152, 1152, "hidden"), ("self.k", 8192, 1152, 1152, "hidden"),
+                        ("self.v", 8192, 1152, 1152, "hidden"), ("self.out", 8192, 1152, 1152, "attn"),
+                        ("cross.q", 8192, 1152, 1152, "hidden"), ("cross.k", 240, 1152, 1152, "text"),
+                        ("cross.v", 240, 1152, 1152, "text"), ("cross.out", 8192, 1152, 1152, "cross_attn"),
+                        ("mlp.fc1", 8192, 1152, 4608, "hidden"), ("mlp.fc2", 8192, 4608, 1152, "mlp"))
+PIXART_INPUTS = {"caption": (240, 4096), "caption_hidden": (240, 1152), "hidden": (8192, 1152),
+                 "attn": (8192, 1152), "text": (240, 1152), "cross_attn": (8192, 1152), "mlp": (8192, 4608)}
+PIXART_SAMPLER_T = tuple(999 - 50 * i for i in range(20))   # 20 steps, two per timestep bucket
+
+
+def pixart_model_linears():
+    """The 282 linears of one PixArt-alpha sampler step, in execution order: (name, M, K, N, input)."""
+    out = [tuple(L) for L in PIXART_CAPTION_LINEARS]
+    for b in range(PIXART_BLOCKS):
+        out += [("block%d.%s" % (b, n), M, K, N, x) for (n, M, K, N, x) in PIXART_BLOCK_LINEARS]
+    return out
+
+
+def weight_mix_rows(g, N, K, scale=0.02):
+    """The weight_mix distributions (channel n: kind n % 5 of Gaussian, Laplace, uniform, Student-t
+    nu = 4, Gaussian with K/64 outliers x12), drawn kind by kind for all rows at once."""
+    W = np.empty((N, K))
+    rows = [np.arange(k, N, 5) for k in range(5)]
+    W[rows[0]] = g.normal(0, scale, (len(rows[0]), K))
+    W[rows[1]] = g.laplace(0, scale / np.sqrt(2), (len(rows[1]), K))
+    W[rows[2]] = g.uniform(-scale * np.sqrt(3), scale * np.sqrt(3), (len(rows[2]), K))
+    W[rows[3]] = g.standard_t(4, (len(rows[3]), K)) * scale / np.sqrt(2)
+    W[rows[4]] = g.normal(0, scale, (len(rows[4]), K))
+    n_out = max(1, K // 64)
+    for r in rows[4]:
+        W[r, g.choice(K, n_out, replace=False)] *= 12.0
+    return to_fp16(W)
+
+
+def pixart_model_weights(layer_index):
+    """Weights (per-channel distribution diversity, config 3's recipe) and bias of linear
+    `layer_index` of pixart_model_linears()."""
+    _, M, K, N, _ = pixart_model_linears()[layer_index]
+    g = rng(4, 1000 + layer_index)
+    return weight_mix_rows(g, N, K), g.normal(0.0, 0.02, N).astype(np.float32)
+
+
+def pixart_model_input(key, bucket):
+    """Input tensor `key` (PIXART_INPUTS) at timestep bucket `bucket`: StudentT(nu_b) * c_k with the
+    per-bucket nu of the SDXL projections (heavier tails at high noise) and per-channel jitter."""
+    M, K = PIXART_INPUTS[key]
+    i = sorted(PIXART_INPUTS).index(key)
+    c = channel_jitter(rng(4, 2000 + i), K)
+    return to_fp16(student_t(rng(4, 2100 + 10 * i + bucket), NU_SCHEDULE[bucket], (M, K)) * c[None, :])
