@@ -2,12 +2,14 @@
 """Benchmark of the Chameleon format-adaptive quantized linear path on GB300.
 
 Headline workload: every linear of a PixArt-alpha-architecture DiT (28 blocks, hidden 1152, MLP
-4608, 4096 image + 120 caption tokens per sample, batch 2: 282 GEMMs per sampler step) over a
+4608, 4096 image + 120 caption tokens per sample, batch 2: 282 linears per sampler step) over a
 20-step sampler, W4A8.  One benchmark step is one pass of the whole hot path: per-channel
 weight-format selection over the 4-bit palette {INT4-asym, NF4, E2M1, MXINT4, MXFP4} and the pack
 of all 282 layers, then 20 sampler steps (t = 999 - 50 i) in which every linear quantizes its input
 with each sample's own range (Alg. 3) in the format its (layer, timestep-bucket) table entry names
-and multiplies (fp32 outputs).  Random-init weights, seeded synthetic activations.
+and multiplies (fp32 outputs).  Linears that read the same tensor (q, k, v; cross k, v) run as one
+GEMM with their weights stacked along N: 198 GEMMs per sampler step, the same per-channel formats,
+activation codes and outputs.  Random-init weights, seeded synthetic activations.
 
 Sub-objects: the SDXL-UNet W8A8 projection step (static calibrated scales, Alg. 2), the GEMM for
 every activation x weight format, the public quantizer per format and shape, selection and pack,
@@ -189,10 +191,11 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
     the sub-objects reuse."""
     import torch.distributed as dist
     Wn, bn, Xn = host
-    linears = WL.pixart_model_linears()
+    n_linears = len(WL.pixart_model_linears())
+    linears = WL.pixart_model_gemms()   # (names, M, K, N, input, indices): q/k/v and cross k/v stacked
     n = len(linears)
-    W = [torch.from_numpy(w).to(device) for w in Wn]
-    bias = [torch.from_numpy(b).to(device) for b in bn]
+    W = [torch.from_numpy(np.concatenate([Wn[i] for i in ix])).to(device) for (_, M, K, N, _, ix) in linears]
+    bias = [torch.from_numpy(np.concatenate([bn[i] for i in ix])).to(device) for (_, M, K, N, _, ix) in linears]
     X = {kb: torch.from_numpy(x).to(device) for kb, x in Xn.items()}
     lut = pixart_calibrate(cl, X)
     ts = WL.PIXART_SAMPLER_T[:args.sampler_steps]
@@ -201,7 +204,7 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
 
     # a5: selection into one format buffer; the packed layout needs the formats on the host (the
     # palette spans both MMA classes), so the step copies them back once for all layers
-    offs = np.cumsum([0] + [N for (_, M, K, N, _) in linears])
+    offs = np.cumsum([0] + [N for (_, M, K, N, _, _) in linears])
     fmt_all = torch.empty(int(offs[-1]), dtype=torch.uint8, device=device)
     fmt_host = torch.empty(int(offs[-1]), dtype=torch.uint8).pin_memory()
 
@@ -213,7 +216,7 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
     select_all()
     torch.cuda.synchronize()
     f_ref = fmt_host.numpy().copy()
-    descs = [cl.pack_plan(N, K, f_ref[offs[i]:offs[i + 1]]) for i, (_, M, K, N, _) in enumerate(linears)]
+    descs = [cl.pack_plan(N, K, f_ref[offs[i]:offs[i + 1]]) for i, (_, M, K, N, _, _) in enumerate(linears)]
     blobs = [torch.empty(d.bytes, dtype=torch.uint8, device=device) for d in descs]
 
     def plan_and_pack():
@@ -227,21 +230,21 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
             cl.pack_weights(W[i], fmt_all[offs[i]:offs[i + 1]], descs[i], dev_status=st, blob=blobs[i])
 
     acts = sorted(set(lut.values()))
-    ws = torch.empty(max(cl.linear_workspace_size(M, descs[i], a) for i, (_, M, K, N, _) in enumerate(linears)
+    ws = torch.empty(max(cl.linear_workspace_size(M, descs[i], a) for i, (_, M, K, N, _, _) in enumerate(linears)
                          for a in acts), dtype=torch.uint8, device=device)
-    kinds = sorted(set(name.split(".", 1)[1] if name.startswith("block") else name for (name, *_r) in linears))
+    # one output buffer per kind of GEMM (the blocks run in order; the benchmark keeps no model state)
+    kind = [names[0].split(".", 1)[1] if names[0].startswith("block") else names[0] for (names, *_r) in linears]
     Ybuf = {}
-    for (name, M, K, N, _) in linears:
-        k = name.split(".", 1)[1] if name.startswith("block") else name
+    for k, (names, M, K, N, _, _) in zip(kind, linears):
         if k not in Ybuf:
             Ybuf[k] = torch.empty((M, N), dtype=torch.float32, device=device)
-    Y = [Ybuf[name.split(".", 1)[1] if name.startswith("block") else name] for (name, *_r) in linears]
+    Y = [Ybuf[k] for k in kind]
 
     def sampler(parts="qg"):
         """20 sampler steps: per linear the quantizer with the two samples' own scales (Alg. 3) in
         F[l, b(t)] ("q") and the GEMM ("g")."""
         for b in buckets:
-            for i, (name, M, K, N, key) in enumerate(linears):
+            for i, (names, M, K, N, key, _) in enumerate(linears):
                 af = lut[(key, b)]
                 x = X[(key, b)]
                 if "q" in parts:
@@ -272,13 +275,13 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
     # encode for the per-tensor formats, one launch for MX) and the GEMM (+ the split-K reduction)
     per_linear = {}
     for b in buckets:
-        for i, (_, M, K, N, key) in enumerate(linears):
+        for i, (_, M, K, N, key, _) in enumerate(linears):
             k = (i, lut[(key, b)])
             if k not in per_linear:
                 per_linear[k] = sum(cl.linear_launches(M, descs[i], lut[(key, b)], 2))
     launches = 2 * n + sum(per_linear[(i, lut[(key, b)])] for b in buckets
-                           for i, (_, M, K, N, key) in enumerate(linears))
-    flops_step = len(buckets) * sum(layer_flops(M, K, N) for (_, M, K, N, _) in linears)
+                           for i, (_, M, K, N, key, _) in enumerate(linears))
+    flops_step = len(buckets) * sum(layer_flops(M, K, N) for (_, M, K, N, _, _) in linears)
 
     if world > 1:
         dist.barrier()
@@ -321,7 +324,7 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
     fl8 = fl16 = 0.0
     qbytes = 0.0
     for b in buckets:
-        for i, (_, M, K, N, key) in enumerate(linears):
+        for i, (_, M, K, N, key, _) in enumerate(linears):
             d, af = descs[i], lut[(key, b)]
             fl = layer_flops(M, K, N)
             share8 = d.n_class[0] / N if (af in (1, 2, 3)) else 0.0
@@ -334,7 +337,7 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
         "flops_step": flops_step, "fl8": fl8, "fl16": fl16, "qbytes": qbytes, "classes_ms": cls,
         "launches": launches, "clocks": clk.summary(), "linears": linears, "lut": lut, "buckets": buckets,
         "descs": descs, "weight_formats": {int(f): int(c) for f, c in enumerate(hist) if c},
-        "acts": acts, "kinds": kinds,
+        "acts": acts, "n_linears": n_linears,
     }
 
 
@@ -735,13 +738,13 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     linears run."""
     import torch.distributed as dist
     Wn, bn, Xn = host
-    linears = WL.pixart_model_linears()
+    linears = WL.pixart_model_gemms()
     n = len(linears)
     keys = sorted(WL.PIXART_INPUTS)
     ts = WL.PIXART_SAMPLER_T[:args.sampler_steps]
     buckets = [cl.bucket(t) for t in ts]
-    Wh = [torch.from_numpy(w).pin_memory() for w in Wn]
-    bh = [torch.from_numpy(b).pin_memory() for b in bn]
+    Wh = [torch.from_numpy(np.concatenate([Wn[i] for i in ix])).pin_memory() for (_, M, K, N, _, ix) in linears]
+    bh = [torch.from_numpy(np.concatenate([bn[i] for i in ix])).pin_memory() for (_, M, K, N, _, ix) in linears]
     Xh = {kb: torch.from_numpy(x).pin_memory() for kb, x in Xn.items() if kb[1] in set(buckets)}
     Wd = [torch.empty_like(w, device=device) for w in Wh]
     bd = [torch.empty_like(b, device=device) for b in bh]
@@ -750,7 +753,7 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     Yd_last = torch.empty((last[1], last[3]), dtype=torch.float32, device=device)
     Yh = torch.empty((last[1], last[3]), dtype=torch.float32).pin_memory()
     st = torch.zeros(1, dtype=torch.int32, device=device)
-    offs = np.cumsum([0] + [N for (_, M, K, N, _) in linears])
+    offs = np.cumsum([0] + [N for (_, M, K, N, _, _) in linears])
     fmt_all = torch.empty(int(offs[-1]), dtype=torch.uint8, device=device)
     fmt_host = torch.empty(int(offs[-1]), dtype=torch.uint8).pin_memory()
     compute = torch.cuda.current_stream()
@@ -760,17 +763,17 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     for i in range(n):
         cl.select_weight_formats(Wd[i], W4_PALETTE, fmt_out=fmt_all[offs[i]:offs[i + 1]])
     f_ref = fmt_all.cpu().numpy()
-    descs = [cl.pack_plan(N, K, f_ref[offs[i]:offs[i + 1]]) for i, (_, M, K, N, _) in enumerate(linears)]
+    descs = [cl.pack_plan(N, K, f_ref[offs[i]:offs[i + 1]]) for i, (_, M, K, N, _, _) in enumerate(linears)]
     blobs = [torch.empty(d.bytes, dtype=torch.uint8, device=device) for d in descs]
     acts = sorted(set(lut.values()))
-    ws = torch.empty(max(cl.linear_workspace_size(M, descs[i], a) for i, (_, M, K, N, _) in enumerate(linears)
+    ws = torch.empty(max(cl.linear_workspace_size(M, descs[i], a) for i, (_, M, K, N, _, _) in enumerate(linears)
                          for a in acts), dtype=torch.uint8, device=device)
+    kind = [names[0].split(".", 1)[1] if names[0].startswith("block") else names[0] for (names, *_r) in linears]
     Ys = {}
-    for (name, M, K, N, _) in linears[:-1]:
-        k = name.split(".", 1)[1] if name.startswith("block") else name
+    for k, (names, M, K, N, _, _) in zip(kind[:-1], linears[:-1]):
         if k not in Ys:
             Ys[k] = torch.empty((M, N), dtype=torch.float32, device=device)
-    Y = [Ys[name.split(".", 1)[1] if name.startswith("block") else name] for (name, *_r) in linears[:-1]] + [Yd_last]
+    Y = [Ys[k] for k in kind[:-1]] + [Yd_last]
     x_ready = [torch.cuda.Event() for _ in range(2)]
     x_free = [torch.cuda.Event() for _ in range(2)]
     w_ready, y_done = torch.cuda.Event(), torch.cuda.Event()
@@ -802,7 +805,7 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
                     Xd[buf][k].copy_(Xh[(k, b)], non_blocking=True)
                 x_ready[buf].record(copy)
             compute.wait_event(x_ready[buf])
-            for i, (name, M, K, N, key) in enumerate(linears):
+            for i, (names, M, K, N, key, _) in enumerate(linears):
                 cl.linear_ex(Xd[buf][key], descs[i], blobs[i], lut[(key, b)], 2, bias=bd[i], Y=Y[i], ws=ws,
                              dev_status=st, stream=compute)
             x_free[buf].record(compute)
@@ -984,15 +987,17 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "fp8 (e4m3 x e4m3/e5m2 MMA, fp32 accumulate; fp16 on NF4 tiles)",
         "data": "synthetic (seeded random-init weights, Student-t activations)",
         "config": {"workload": WORKLOAD if args.sampler_steps == 20 else WORKLOAD + " (%d sampler steps)" % args.sampler_steps,
-                   "model": "PixArt-alpha-architecture DiT", "linears": len(h["linears"]),
+                   "model": "PixArt-alpha-architecture DiT", "linears": h["n_linears"], "gemms": len(h["linears"]),
+                   "stacked": "q/k/v and cross k/v of each block read the same input: one quantizer pass and one "
+                              "GEMM with their weights stacked along N (per-channel formats and outputs unchanged)",
                    "sampler_steps": len(h["buckets"]), "global_batch": 2 * world, "tokens": [8192, 240],
                    "weight_palette": "W4 {INT4-asym, NF4, E2M1, MXINT4, MXFP4}, per-channel argmin",
                    "weight_formats": h["weight_formats"],
                    "lut": {str(b): v for b, v in lut_by_bucket.items()},
                    "activation_formats_used": h["acts"],
-                   "step": "selection + pack of the 282 layers, then 20 sampler steps x 282 linears (per-sample "
+                   "step": "selection + pack of the 282 layers, then 20 sampler steps x 198 GEMMs (per-sample "
                            "dynamic quantizer + GEMM, one CUDA graph)",
-                   "l2": "inputs larger than L2 (1.35 GB of activations, 0.3 GB of packed weights)",
+                   "l2": "inputs larger than L2 (1.7 GB of activations, 0.3 GB of packed weights)",
                    "parallelism": "replicas" if world > 1 else "single-gpu"},
         "roofline": {"bound": "tensor", "achieved": round(achieved, 2), "peak": round(peak_eff_s, 1), "unit": "TFLOP/s",
                      "frac": round(achieved / peak_eff_s, 4), **traffic_fields(),

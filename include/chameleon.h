@@ -277,12 +277,27 @@ typedef struct {
                                  when the activation format is E4M3, E5M2 or MXFP8 (see
                                  chameleon_linear); 1: every tile on fp16 MMAs.  The linear calls of
                                  one layer must see the same value (it fixes the workspace layout). */
-  uint8_t reserved[108];      /* pads the descriptor to 256 bytes */
+  int32_t layout;             /* channel order inside each MMA class: 0 = original order (the class
+                                 layout); 1 = format groups (chameleon_pack_plan_layout) */
+  int32_t fold;               /* layout 1: a format with fewer channels than this shares its class's
+                                 mixed tail group */
+  uint8_t reserved[100];      /* pads the descriptor to 256 bytes */
 } cham_wpack_desc;
 
 /* Fill *desc for N x K weights whose selected formats are fmt_host (host, uint8 [N], all of one
  * bit width).  desc->bytes is the blob size. */
 cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* desc);
+
+/* chameleon_pack_plan with a choice of channel order inside the MMA classes (Sec. 5: channels of
+ * one format grouped behind a permutation).  layout 0 is chameleon_pack_plan: each class in
+ * original channel order.  layout 1: format groups -- inside each class, the formats in palette
+ * order (class 0: INT4-sym, INT4-asym, E2M1, MXINT4, MXFP4; class 1: NF4, INT8-sym, INT8-asym,
+ * MXINT8), each format's channels in original order padded to whole 128-channel tiles, so that
+ * every tile holds one format; formats with fewer than `fold` channels (fold >= 0) go together, in
+ * original order, into one mixed tail group at the end of their class.  The GEMM calls take either
+ * layout.  CHAM_ERR_INVALID_ARG as chameleon_pack_plan, or for layout outside 0..1 or fold < 0. */
+cham_status chameleon_pack_plan_layout(int N, int K, const uint8_t* fmt_host, int layout, int fold,
+                                       cham_wpack_desc* desc);
 
 /* Selection (a5) and pack (a6) in one launch, for a palette whose members share one MMA class
  * (e.g. CHAM_PALETTE_W8): desc comes from chameleon_pack_plan_palette(N, K, palette_mask); the
@@ -408,7 +423,7 @@ cham_status chameleon_debug_stall_next_gemm(int chunk);
  * its plugins only their inputs and outputs, or that forbids allocation once serving starts.
  * Same arguments, output layout and results as chameleon_act_quant, minus ws / ws_bytes.  The
  * per-tensor formats keep their range partials in a library-owned static device array of
- * 1024 x 16 bytes (16 KiB, held on every GPU that loads the library until exit); this fits any
+ * 2048 x 16 bytes (32 KiB, held on every GPU that loads the library until exit); this fits any
  * M, K on GPUs with up to 256 SMs and returns CHAM_ERR_WORKSPACE (nothing launched) otherwise.
  * It calls no allocator.  The first call on a device looks up the array's address with that
  * device current: make it before any stream capture.  That address is kept until exit, so the

@@ -30,7 +30,8 @@ EXPORTS = [
     "chameleon_bucket", "chameleon_snr", "chameleon_kurtosis", "chameleon_route",
     "chameleon_act_moments_workspace_size", "chameleon_act_moments",
     "chameleon_act_quant_size", "chameleon_act_quant",
-    "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_plan_palette", "chameleon_pack_weights",
+    "chameleon_select_weight_formats", "chameleon_pack_plan", "chameleon_pack_plan_layout",
+    "chameleon_pack_plan_palette", "chameleon_pack_weights",
     "chameleon_linear_workspace_size", "chameleon_linear_launches", "chameleon_linear", "chameleon_linear_prepare",
     "chameleon_linear_gemm", "chameleon_act_quant_noalloc", "chameleon_debug_stall_next_gemm",
     "chameleon_scale_zp", "chameleon_act_quant_static", "chameleon_linear_prepare_static",
@@ -53,7 +54,8 @@ class WPackDesc(ctypes.Structure):
                 ("off_zero", ctypes.c_uint64), ("off_e8m0", ctypes.c_uint64),
                 ("off_fmt", ctypes.c_uint64), ("off_perm", ctypes.c_uint64),
                 ("bytes", ctypes.c_uint64), ("off_gscale", ctypes.c_uint64),
-                ("f16_only", ctypes.c_int32), ("reserved", ctypes.c_uint8 * 108)]
+                ("f16_only", ctypes.c_int32), ("layout", ctypes.c_int32), ("fold", ctypes.c_int32),
+                ("reserved", ctypes.c_uint8 * 100)]
 
 
 assert ctypes.sizeof(WPackDesc) == 256
@@ -107,6 +109,7 @@ def lib():
         "chameleon_act_quant": (i32, [vp, i32, i32, i32, vp, sz, vp, sz, vp, vp]),
         "chameleon_select_weight_formats": (i32, [vp, i32, i32, u32, vp, vp, vp]),
         "chameleon_pack_plan": (i32, [i32, i32, vp, pdesc]),
+        "chameleon_pack_plan_layout": (i32, [i32, i32, vp, i32, i32, pdesc]),
         "chameleon_pack_plan_palette": (i32, [i32, i32, ctypes.c_uint32, pdesc]),
         "chameleon_pack_weights": (i32, [vp, vp, pdesc, vp, sz, vp, vp]),
         "chameleon_linear_workspace_size": (i32, [i32, pdesc, i32, psz]),
@@ -403,11 +406,13 @@ def act_channel_energy(X, energy=None, stream=None):
     return energy
 
 
-def pack_plan(N, K, fmt_host):
-    """Packed layout (cham_wpack_desc) for N x K weights with the selected formats fmt_host (host uint8 [N])."""
+def pack_plan(N, K, fmt_host, layout=0, fold=0):
+    """Packed layout (cham_wpack_desc) for N x K weights with the selected formats fmt_host (host
+    uint8 [N]); layout 1 groups the channels of each format (formats with fewer than `fold`
+    channels share their class's tail group)."""
     f = np.ascontiguousarray(np.asarray(fmt_host, dtype=np.uint8))
     d = WPackDesc()
-    check(lib().chameleon_pack_plan(N, K, f.ctypes.data_as(ctypes.c_void_p), ctypes.byref(d)))
+    check(lib().chameleon_pack_plan_layout(N, K, f.ctypes.data_as(ctypes.c_void_p), layout, fold, ctypes.byref(d)))
     return d
 
 

@@ -17,7 +17,8 @@
 
 namespace cham {
 
-constexpr int kUnroll = 4;  // independent 16-byte loads in flight per thread
+constexpr int kUnroll = 4;       // independent 16-byte loads in flight per thread (encoders)
+constexpr int kRangeUnroll = 8;  // the range pass: a grid of range_grid CTAs reads the tensor in one round
 
 // min / max / non-finite flag of eight fp16 values packed in a uint4.
 CHAM_DEV void range8(const uint4& v, __half2& lo2, __half2& hi2, uint32_t& nonfinite) {
@@ -160,15 +161,16 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
   __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
   uint32_t nonfinite = 0;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec; i0 += stride * kUnroll) {
-    uint4 v[kUnroll];
+  for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec;
+       i0 += stride * kRangeUnroll) {
+    uint4 v[kRangeUnroll];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
+    for (int u = 0; u < kRangeUnroll; ++u) {
       const int64_t i = i0 + u * stride;
       v[u] = i < nvec ? __ldg(X + i) : make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);
     }
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u)
+    for (int u = 0; u < kRangeUnroll; ++u)
       if (i0 + u * stride < nvec) range8(v[u], lo2, hi2, nonfinite);
   }
   float lo = fminf(__low2float(lo2), __high2float(lo2));
@@ -532,9 +534,11 @@ __global__ void __launch_bounds__(256) k_act_moments_finish(const MomentPartial*
 }
 
 // ------------------------------------------------------------------ host-side launchers
+// Enough CTAs that each thread's kRangeUnroll loads cover the tensor in one round (the DRAM latency
+// is paid once), up to 8 resident CTAs of 256 threads per SM.
 int range_grid(int64_t nvec, int num_sms) {
-  const int64_t want = (nvec + 255) / 256;
-  const int64_t cap = static_cast<int64_t>(num_sms) * 4;
+  const int64_t want = (nvec + 256 * kRangeUnroll - 1) / (256 * kRangeUnroll);
+  const int64_t cap = static_cast<int64_t>(num_sms) * 8;
   return static_cast<int>(want < 1 ? 1 : (want < cap ? want : cap));
 }
 
@@ -559,7 +563,10 @@ static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
   const int G = a.n_groups > 1 ? a.n_groups : 1;
   const int64_t nvg = a.nvec / G;
   launch_pdl(k_act_range, dim3(a.nparts, G), dim3(256), 0, st, a.X, nvg, a.parts);
-  const int eg = group_grid(a.nvec, G, a.num_sms);
+  // the encode grid covers each group in one pass of kUnroll loads per thread (8 CTAs per SM at most)
+  const int64_t want = (nvg + 256 * kUnroll - 1) / (256 * kUnroll);
+  const int64_t cap = static_cast<int64_t>(a.num_sms) * 8 / G;
+  const int eg = static_cast<int>(want < 1 ? 1 : (want < cap ? want : (cap < 1 ? 1 : cap)));
   launch_pdl(k_act_encode_tensor<FMT, CODES, DEQ>, dim3(eg, G), dim3(256), 0, st, a.X, nvg,
              static_cast<const RangePartial*>(a.parts), a.nparts, a.codes, a.deq, a.params, a.scale_out,
              a.dev_status, a.kperm);

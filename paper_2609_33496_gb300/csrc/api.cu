@@ -206,6 +206,8 @@ cham_status check_desc(const cham_wpack_desc* d) {
   if (d->group < 0 || d->group % 32 != 0 || (d->group > 0 && (d->K + d->group - 1) / d->group > cham::kMaxRowGroups))
     return fail(CHAM_ERR_INVALID_ARG, "descriptor group size %d", d->group);
   if (d->f16_only != 0 && d->f16_only != 1) return fail(CHAM_ERR_INVALID_ARG, "descriptor f16_only %d", d->f16_only);
+  if (d->layout < 0 || d->layout > 1 || d->fold < 0 || (d->layout == 1 && d->group > 0))
+    return fail(CHAM_ERR_INVALID_ARG, "descriptor layout %d fold %d", d->layout, d->fold);
   return CHAM_OK;
 }
 
@@ -659,12 +661,62 @@ cham_status chameleon_act_channel_energy(const void* X, int M, int K, double* en
 }  // extern "C"
 namespace {
 void finish_plan(cham_wpack_desc* d, int N, int K, int bits);
+
+// The packed groups of a plan, in slot order.  Layout 0: one group per MMA class.  Layout 1: per
+// class, each format with at least `fold` channels in palette order, then the class's tail of the
+// formats with fewer.  group_of[f] is -1 for a format without channels.
+struct PackGroups {
+  int n;
+  int cls[cham::kMaxPackGroups], count[cham::kMaxPackGroups];
+  int8_t group_of[CHAM_W_NFORMATS];
+};
+PackGroups pack_groups(const cham_wpack_desc* d) {
+  PackGroups g{};
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f) g.group_of[f] = -1;
+  for (int cls = 0; cls < 2; ++cls) {
+    if (d->layout != 1) {
+      g.cls[g.n] = cls;
+      g.count[g.n] = d->n_class[cls];
+      for (int j = 0; j < 5; ++j)
+        if (kClassOrder[cls][j] >= 0) g.group_of[kClassOrder[cls][j]] = static_cast<int8_t>(g.n);
+      ++g.n;
+      continue;
+    }
+    int tail = 0;
+    for (int j = 0; j < 5; ++j) {
+      const int f = kClassOrder[cls][j];
+      if (f < 0 || d->n_fmt[f] <= 0) continue;
+      if (d->n_fmt[f] >= d->fold) {
+        g.cls[g.n] = cls;
+        g.count[g.n] = d->n_fmt[f];
+        g.group_of[f] = static_cast<int8_t>(g.n++);
+      } else {
+        tail += d->n_fmt[f];
+      }
+    }
+    if (tail > 0) {
+      for (int j = 0; j < 5; ++j) {
+        const int f = kClassOrder[cls][j];
+        if (f >= 0 && d->n_fmt[f] > 0 && d->n_fmt[f] < d->fold) g.group_of[f] = static_cast<int8_t>(g.n);
+      }
+      g.cls[g.n] = cls;
+      g.count[g.n++] = tail;
+    }
+  }
+  return g;
+}
 }  // namespace
 extern "C" {
 
 cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpack_desc* d) {
+  return chameleon_pack_plan_layout(N, K, fmt_host, 0, 0, d);
+}
+
+cham_status chameleon_pack_plan_layout(int N, int K, const uint8_t* fmt_host, int layout, int fold,
+                                       cham_wpack_desc* d) {
   if (N <= 0 || K <= 0 || K % 32 != 0 || fmt_host == nullptr || d == nullptr)
     return fail(CHAM_ERR_INVALID_ARG, "N=%d K=%d (K must be a multiple of 32)", N, K);
+  if (layout < 0 || layout > 1 || fold < 0) return fail(CHAM_ERR_INVALID_ARG, "layout %d fold %d", layout, fold);
   std::memset(d, 0, sizeof(*d));
   int bits = 0;
   for (int c = 0; c < N; ++c) {
@@ -678,6 +730,8 @@ cham_status chameleon_pack_plan(int N, int K, const uint8_t* fmt_host, cham_wpac
   for (int cls = 0; cls < 2; ++cls)
     for (int j = 0; j < 5; ++j)
       if (kClassOrder[cls][j] >= 0) d->n_class[cls] += d->n_fmt[kClassOrder[cls][j]];
+  d->layout = layout;
+  d->fold = fold;
   finish_plan(d, N, K, bits);
   return CHAM_OK;
 }
@@ -731,7 +785,16 @@ void finish_plan(cham_wpack_desc* d, int N, int K, int bits) {
   d->K = K;
   d->Kp = static_cast<int>(round_up(K, 64));
   d->bits = bits;
-  for (int cls = 0; cls < 2; ++cls) d->n_tiles[cls] = (d->n_class[cls] + 127) / 128;
+  for (int cls = 0; cls < 2; ++cls) {
+    if (d->layout == 1) {
+      const PackGroups g = pack_groups(d);
+      d->n_tiles[cls] = 0;
+      for (int i = 0; i < g.n; ++i)
+        if (g.cls[i] == cls) d->n_tiles[cls] += (g.count[i] + 127) / 128;
+    } else {
+      d->n_tiles[cls] = (d->n_class[cls] + 127) / 128;
+    }
+  }
   const size_t tiles = static_cast<size_t>(d->n_tiles[0] + d->n_tiles[1]);
   const size_t np = tiles * 128, chunks = d->Kp / 64;
   size_t off = 256;
@@ -771,6 +834,15 @@ cham::PackArgs pack_args(const cham_wpack_desc* d, const void* W, const uint8_t*
   a.cls_base[1] = 128 * d->n_tiles[0];
   a.cls_count[0] = d->n_class[0];
   a.cls_count[1] = d->n_class[1];
+  const PackGroups g = pack_groups(d);
+  a.n_groups = g.n;
+  int base = 0;
+  for (int i = 0; i < g.n; ++i) {
+    a.group_base[i] = base;
+    a.group_count[i] = g.count[i];
+    base += 128 * ((g.count[i] + 127) / 128);
+  }
+  for (int f = 0; f < CHAM_W_NFORMATS; ++f) a.group_of_fmt[f] = g.group_of[f];
   a.codes = b + d->off_codes;
   a.scale = reinterpret_cast<float*>(b + d->off_scale);
   a.zero = b + d->off_zero;
@@ -778,7 +850,8 @@ cham::PackArgs pack_args(const cham_wpack_desc* d, const void* W, const uint8_t*
   a.fmtp = b + d->off_fmt;
   a.perm = reinterpret_cast<int32_t*>(b + d->off_perm);
   a.dev_status = dev_status;
-  a.one_class = d->n_class[0] == 0 ? 1 : (d->n_class[1] == 0 ? 0 : -1);
+  // one MMA class in original order: slot = channel, no ranking pass (not for format groups)
+  a.one_class = d->layout != 0 ? -1 : (d->n_class[0] == 0 ? 1 : (d->n_class[1] == 0 ? 0 : -1));
   a.group = d->group;
   a.gscale = d->group > 0 ? reinterpret_cast<uint32_t*>(b + d->off_gscale) : nullptr;
   a.desc = *d;
@@ -807,7 +880,7 @@ cham_status chameleon_select_pack_palette(const void* W, int N, int K, uint32_t 
                                           int* dev_status, void* stream) {
   cham_status s = check_desc(d);
   if (s != CHAM_OK) return s;
-  if (d->N != N || d->K != K || d->group != 0 || (d->n_class[0] != 0 && d->n_class[1] != 0))
+  if (d->N != N || d->K != K || d->group != 0 || d->layout != 0 || (d->n_class[0] != 0 && d->n_class[1] != 0))
     return fail(CHAM_ERR_INVALID_ARG, "descriptor is not a one-class plan of %d x %d weights", N, K);
   if (palette_mask == 0 || (palette_mask & ~0x1FFu) != 0) return fail(CHAM_ERR_INVALID_ARG, "palette mask 0x%x", palette_mask);
   const int cls = d->n_class[0] == 0 ? 1 : 0;

@@ -7,7 +7,7 @@
 // the caller passes only X, the output buffer and the status word.
 //
 // Limits and sharing rules:
-//   * capacity: kScratchParts partials (16 KiB).  The quantizer launches at most 4 CTAs per SM, so
+//   * capacity: kScratchParts partials (32 KiB).  The range pass launches at most 8 CTAs per SM, so
 //     any M and K fit on GPUs with up to 256 SMs; a request that would need more partials is
 //     rejected with CHAM_ERR_WORKSPACE before anything is launched.
 //   * every GPU that loads the library holds the array until the process exits.
@@ -26,7 +26,7 @@
 
 namespace {
 
-constexpr int kScratchParts = 1024;
+constexpr int kScratchParts = 2048;
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) cham::RangePartial g_range_scratch[kScratchParts];

@@ -203,29 +203,29 @@ void launch_select(const __half* W, int N, int K, uint32_t mask, uint8_t* fmt_ou
 }
 
 // ------------------------------------------------------------------ a6: slot assignment
-// Packed slot of every channel: the first slot of its MMA class plus the number of earlier
-// channels of the same class (so each class keeps the original channel order, and a tile's Y
-// columns are contiguous).  One CTA walks the channels in chunks of 1024 with warp ballots.
+// Packed slot of every channel: the first slot of its group (its MMA class, or in the format-group
+// layout its format's group or its class's tail) plus the number of earlier channels of the same
+// group, so each group keeps the original channel order.  One CTA walks the channels in chunks of
+// 1024 with warp ballots.
 __global__ void __launch_bounds__(1024) k_w_slots(PackArgs a) {
-  __shared__ int warp_cnt[32][2];
-  __shared__ int running[2];
+  __shared__ int warp_cnt[32][kMaxPackGroups];
+  __shared__ int running[kMaxPackGroups];
   for (int p = threadIdx.x; p < a.n_packed; p += blockDim.x) {
     a.perm[p] = -1;
     a.fmtp[p] = 0xFF;
   }
-  if (threadIdx.x < 2) running[threadIdx.x] = 0;
+  if (threadIdx.x < kMaxPackGroups) running[threadIdx.x] = 0;
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int c0 = 0; c0 < a.N; c0 += blockDim.x) {
     const int c = c0 + threadIdx.x;
     const int f = c < a.N ? a.fmt_dev[c] : -1;
-    const bool valid = f >= 0 && f < CHAM_W_NFORMATS;
-    const int cls = valid ? w_class(f) : -1;
+    const bool valid = f >= 0 && f < CHAM_W_NFORMATS && a.group_of_fmt[f] >= 0;
+    const int grp = valid ? a.group_of_fmt[f] : -1;
     int my_rank_in_warp = 0;
-#pragma unroll
-    for (int g = 0; g < 2; ++g) {
-      const uint32_t m = __ballot_sync(0xffffffffu, cls == g);
-      if (cls == g) my_rank_in_warp = __popc(m & ((1u << lane) - 1u));
+    for (int g = 0; g < a.n_groups; ++g) {
+      const uint32_t m = __ballot_sync(0xffffffffu, grp == g);
+      if (grp == g) my_rank_in_warp = __popc(m & ((1u << lane) - 1u));
       if (lane == 0) warp_cnt[warp][g] = __popc(m);
     }
     __syncthreads();
@@ -233,10 +233,10 @@ __global__ void __launch_bounds__(1024) k_w_slots(PackArgs a) {
       if (!valid) {
         set_status(a.dev_status, CHAM_ERR_INVALID_ARG);
       } else {
-        int rank = running[cls] + my_rank_in_warp;
-        for (int w = 0; w < warp; ++w) rank += warp_cnt[w][cls];
-        if (rank < a.cls_count[cls]) {  // device formats must match the host plan
-          const int slot = a.cls_base[cls] + rank;
+        int rank = running[grp] + my_rank_in_warp;
+        for (int w = 0; w < warp; ++w) rank += warp_cnt[w][grp];
+        if (rank < a.group_count[grp]) {  // device formats must match the host plan
+          const int slot = a.group_base[grp] + rank;
           a.perm[slot] = c;
           a.fmtp[slot] = static_cast<uint8_t>(f);
         } else {
@@ -245,7 +245,7 @@ __global__ void __launch_bounds__(1024) k_w_slots(PackArgs a) {
       }
     }
     __syncthreads();
-    if (threadIdx.x < 2) {
+    if (threadIdx.x < a.n_groups) {
       int t = 0;
       for (int w = 0; w < 32; ++w) t += warp_cnt[w][threadIdx.x];
       running[threadIdx.x] += t;

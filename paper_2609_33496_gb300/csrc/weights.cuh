@@ -168,6 +168,8 @@ struct GroupSearchArgs {
   GroupCand cand[kMaxCands];
 };
 
+constexpr int kMaxPackGroups = 12;  // 9 formats + 2 class tails (layout 1), or the 2 classes
+
 struct PackArgs {
   const __half* W;
   const uint8_t* fmt_dev;   // selected format of each original channel
@@ -176,6 +178,12 @@ struct PackArgs {
   int n_packed;             // Np
   int cls_base[2];          // first packed slot of each MMA class
   int cls_count[2];         // channels of each class (from the host plan)
+  // the packed groups (layout 0: one per class; layout 1: per format and class tails), in slot
+  // order: group of each format, first slot and channel count of each group
+  int n_groups;
+  int8_t group_of_fmt[CHAM_W_NFORMATS];
+  int group_base[kMaxPackGroups];
+  int group_count[kMaxPackGroups];
   int one_class;            // the class of every channel when the plan has one (slot = channel), else -1
   cham_wpack_desc desc;     // copied to desc_out (the blob header) by the pack kernel
   cham_wpack_desc* desc_out;

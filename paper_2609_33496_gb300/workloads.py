@@ -154,17 +154,20 @@ def config_layer(config, index, M, K, N, nu=7):
 # caption projection (two linears on the 240 caption tokens), then 28 blocks of ten linears each --
 # self-attention q, k, v, out; cross-attention q, k, v (k and v on the caption tokens), out; MLP fc1
 # and fc2 -- 282 GEMMs per sampler step.  Each entry: (name, M, K, N, input); linears that read the
-# same tensor in the network (q, k, v of one attention; cross k and v) share an input key.
+# same tensor in the network share an input key: q, k and v read the normalised hidden state of
+# the self-attention, cross k and v the caption tokens; cross q and fc1 read their own normalised
+# states.
 PIXART_BLOCKS = 28
 PIXART_CAPTION_LINEARS = (("caption.fc1", 240, 4096, 1152, "caption"),
                           ("caption.fc2", 240, 1152, 1152, "caption_hidden"))
-PIXART_BLOCK_LINEARS = (("self.q", 8192, 1152, 1152, "hidden"), ("self.k", 8192, 1152, 1152, "hidden"),
-                        ("self.v", 8192, 1152, 1152, "hidden"), ("self.out", 8192, 1152, 1152, "attn"),
-                        ("cross.q", 8192, 1152, 1152, "hidden"), ("cross.k", 240, 1152, 1152, "text"),
+PIXART_BLOCK_LINEARS = (("self.q", 8192, 1152, 1152, "hidden_sa"), ("self.k", 8192, 1152, 1152, "hidden_sa"),
+                        ("self.v", 8192, 1152, 1152, "hidden_sa"), ("self.out", 8192, 1152, 1152, "attn"),
+                        ("cross.q", 8192, 1152, 1152, "hidden_ca"), ("cross.k", 240, 1152, 1152, "text"),
                         ("cross.v", 240, 1152, 1152, "text"), ("cross.out", 8192, 1152, 1152, "cross_attn"),
-                        ("mlp.fc1", 8192, 1152, 4608, "hidden"), ("mlp.fc2", 8192, 4608, 1152, "mlp"))
-PIXART_INPUTS = {"caption": (240, 4096), "caption_hidden": (240, 1152), "hidden": (8192, 1152),
-                 "attn": (8192, 1152), "text": (240, 1152), "cross_attn": (8192, 1152), "mlp": (8192, 4608)}
+                        ("mlp.fc1", 8192, 1152, 4608, "hidden_mlp"), ("mlp.fc2", 8192, 4608, 1152, "mlp"))
+PIXART_INPUTS = {"caption": (240, 4096), "caption_hidden": (240, 1152), "hidden_sa": (8192, 1152),
+                 "attn": (8192, 1152), "hidden_ca": (8192, 1152), "text": (240, 1152),
+                 "cross_attn": (8192, 1152), "hidden_mlp": (8192, 1152), "mlp": (8192, 4608)}
 PIXART_SAMPLER_T = tuple(999 - 50 * i for i in range(20))   # 20 steps, two per timestep bucket
 
 
@@ -173,6 +176,22 @@ def pixart_model_linears():
     out = [tuple(L) for L in PIXART_CAPTION_LINEARS]
     for b in range(PIXART_BLOCKS):
         out += [("block%d.%s" % (b, n), M, K, N, x) for (n, M, K, N, x) in PIXART_BLOCK_LINEARS]
+    return out
+
+
+def pixart_model_gemms():
+    """The GEMM launches of one sampler step: consecutive linears that read the same input (q, k, v;
+    cross k, v) stacked along N into one GEMM -- each output channel keeps its own weights, format
+    and bias, and the shared input is quantized once, so the outputs are those of the separate
+    linears.  Entries: (names, M, K, N, input, [indices into pixart_model_linears()]); 198 GEMMs."""
+    out = []
+    for i, (name, M, K, N, x) in enumerate(pixart_model_linears()):
+        short = name.split(".", 1)[1] if name.startswith("block") else name
+        if out and out[-1][4] == x and out[-1][1] == M and out[-1][2] == K and short in ("self.k", "self.v", "cross.v"):
+            names, _, _, n0, _, idx = out[-1]
+            out[-1] = (names + (name,), M, K, n0 + N, x, idx + [i])
+        else:
+            out.append(((name,), M, K, N, x, [i]))
     return out
 
 

@@ -465,7 +465,7 @@ def test_linear_workspace_holds_the_operands_the_tiles_need(cl):
     def r256(n):
         return -(-n // 256) * 256
 
-    parts = r256(max(min(-(-(M * K // 8) // 256), 152 * 4), 64) * 16)   # range partials, 152 SMs
+    parts = r256(max(min(-(-(M * K // 8) // 2048), 152 * 8), 64) * 16)  # range partials, 152 SMs
     codes, fp16 = r256(M * K), r256(2 * M * K)
     e8 = r256(-(-K // 128) * -(-M // 4) * 4 * 4)
     c0 = cl.pack_plan(N, K, np.full(N, F.W_INT4_ASYM, np.uint8))
@@ -490,3 +490,22 @@ def test_linear_workspace_holds_the_operands_the_tiles_need(cl):
     c0.f16_only = 2
     with pytest.raises(cl.ChameleonError):
         cl.linear_workspace_size(M, c0, F.A_E4M3)
+
+
+def test_format_group_layout_tile_counts(cl):
+    """chameleon_pack_plan_layout: layout 0 pads each MMA class to whole tiles; layout 1 pads each
+    format of a class (palette order) and, with fold, the class's tail of small formats."""
+    counts = {F.W_INT4_ASYM: 922, F.W_NF4: 996, F.W_E2M1: 1, F.W_MXINT4: 8, F.W_MXFP4: 2681}
+    fmt = np.concatenate([np.full(n, f, np.uint8) for f, n in counts.items()])
+    N, K = len(fmt), 1152
+    tiles = lambda n: -(-n // 128)
+    d0 = cl.pack_plan(N, K, fmt)
+    assert list(d0.n_tiles) == [tiles(922 + 1 + 8 + 2681), tiles(996)] and d0.layout == 0
+    d1 = cl.pack_plan(N, K, fmt, 1, 0)
+    assert list(d1.n_tiles) == [tiles(922) + tiles(1) + tiles(8) + tiles(2681), tiles(996)]
+    d2 = cl.pack_plan(N, K, fmt, 1, 64)
+    assert list(d2.n_tiles) == [tiles(922) + tiles(2681) + tiles(1 + 8), tiles(996)]
+    assert (d2.layout, d2.fold) == (1, 64) and d2.bytes > d0.bytes
+    for bad in ((2, 0), (-1, 0), (1, -1)):
+        with pytest.raises(cl.ChameleonError):
+            cl.pack_plan(N, K, fmt, *bad)

@@ -18,9 +18,9 @@ def cl():
     return lib_module()
 
 
-def gpu_linear(cl, X, W, fmt, act_fmt, bias, f16_only=0):
+def gpu_linear(cl, X, W, fmt, act_fmt, bias, f16_only=0, layout=0, fold=0):
     import torch
-    d = cl.pack_plan(W.shape[0], W.shape[1], fmt)
+    d = cl.pack_plan(W.shape[0], W.shape[1], fmt, layout, fold)
     d.f16_only = f16_only
     blob, st = cl.pack_weights(cuda(W), cuda(fmt), d)
     Y, st2 = cl.linear(cuda(X), d, blob, act_fmt, bias=None if bias is None else cuda(bias))
@@ -65,6 +65,22 @@ def test_ragged_shapes_every_format(cl, M, K, N, bits, f16_only):
     for act_fmt in ACT + [F.A_FP16]:
         check(cl, X, W, fmt, act_fmt, bias if act_fmt % 2 else None,
               "M%d K%d N%d bits %d act %d f16_only %d" % (M, K, N, bits, act_fmt, f16_only), f16_only)
+
+
+@pytest.mark.parametrize("fold", [0, 48])
+@pytest.mark.parametrize("M,K,N", [(17, 160, 300), (300, 352, 500)])
+def test_format_group_layout_every_activation(cl, M, K, N, fold):
+    """The format-group layout (one format per tile, small formats folded into a class tail) gives
+    the same bound on every activation format, on the FP8 and the fp16 paths."""
+    g = np.random.default_rng(M + K + N + fold)
+    X = WL.to_fp16(g.standard_t(4, (M, K)))
+    W = WL.weight_mix(g, N, K)
+    fmt = np.asarray(F.W4_PALETTE, np.uint8)[g.choice(len(F.W4_PALETTE), N, p=[0.1, 0.3, 0.2, 0.05, 0.05, 0.3])]
+    bias = g.normal(0, 0.02, N).astype(np.float32)
+    for act_fmt in ACT + [F.A_FP16]:
+        Y = gpu_linear(cl, X, W, fmt, act_fmt, bias, layout=1, fold=fold)
+        Y_ref, bound, _, _ = G.linear_reference(X, act_fmt, W, fmt, bias)
+        assert_within_bound(Y, Y_ref, bound, "layout 1 fold %d act %d" % (fold, act_fmt))
 
 
 CLASS0 = [F.W_INT4_SYM, F.W_INT4_ASYM, F.W_E2M1, F.W_MXINT4, F.W_MXFP4]

@@ -58,23 +58,24 @@ def test_select_constructed_channels(cl):
     assert fmt_g[0] == F.W_INT4_SYM and fmt_g[1] == F.W_INT4_SYM
 
 
-def unpack_blob(cl, W, fmt):
+def unpack_blob(cl, W, fmt, layout=0, fold=0):
     import torch
-    d = cl.pack_plan(W.shape[0], W.shape[1], fmt)
+    d = cl.pack_plan(W.shape[0], W.shape[1], fmt, layout, fold)
     blob, st = cl.pack_weights(cuda(W), cuda(fmt), d)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     return unpack(host(blob).tobytes())
 
 
+@pytest.mark.parametrize("layout,fold", [(0, 0), (1, 0), (1, 40)])
 @pytest.mark.parametrize("mask,K", [(0x007, 320), (0x1F8, 320), (0x1F8, 96), (0x007, 160)])
-def test_pack_matches_oracle_codes(cl, mask, K):
+def test_pack_matches_oracle_codes(cl, mask, K, layout, fold):
     W = WL.weight_mix(np.random.default_rng(K), 261, K)
     fmt_o, _, pal = SEL.select_formats(W, mask)
     fmt = fmt_o.copy()
     fmt[::7] = pal[-1]          # make sure every palette member appears
     fmt[1::7] = pal[0]
-    desc, got = unpack_blob(cl, W, fmt)
+    desc, got = unpack_blob(cl, W, fmt, layout, fold)
     ref = SEL.quantize_selected(W, fmt)
     assert sorted(got) == list(range(W.shape[0]))
     for c, r in enumerate(ref):
@@ -86,6 +87,31 @@ def test_pack_matches_oracle_codes(cl, mask, K):
         else:
             assert np.float32(g["s"]).tobytes() == np.float32(r["s"]).tobytes()
             assert g["z"] == r["z"]
+
+
+@pytest.mark.parametrize("fold", [0, 30])
+def test_pack_format_groups_order(cl, fold):
+    """Layout 1: inside each class the formats in palette order, each in original channel order and
+    padded to whole tiles (every tile one format); formats with fewer than `fold` channels share the
+    class's tail group, in original order, after the class's own groups."""
+    W = WL.weight_mix(np.random.default_rng(19), 400, 96)
+    g = np.random.default_rng(2)
+    fmt = np.concatenate([np.full(n, f) for f, n in ((3, 140), (4, 20), (5, 150), (6, 10), (7, 60), (8, 20))])
+    fmt = fmt[g.permutation(len(fmt))].astype(np.uint8)
+    desc, got = unpack_blob(cl, W, fmt, 1, fold)
+    order0, order1 = [3, 4, 6, 7, 8], [5]
+    counts = {f: int((fmt == f).sum()) for f in range(9)}
+    expect, base = {}, 0
+    for cls_order in (order0, order1):
+        own = [f for f in cls_order if counts[f] >= max(fold, 1)]
+        tail = [f for f in cls_order if 0 < counts[f] < fold]
+        for grp in [[f] for f in own] + ([tail] if tail else []):
+            chans = [c for c in range(len(fmt)) if fmt[c] in grp]
+            for r, c in enumerate(chans):
+                expect[c] = base + r
+            base += 128 * (-(-len(chans) // 128))
+    assert {c: g_["slot"] for c, g_ in got.items()} == expect
+    assert desc["n_tiles"][0] + desc["n_tiles"][1] == base // 128
 
 
 def test_pack_permutation_groups_classes(cl):
