@@ -289,8 +289,10 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
     with ClockSampler(device.index) as clk:
         t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         t0.record(stream)
+        torch.cuda.nvtx.range_push("pixart_step")   # a profiler can take exactly the timed steps
         for _ in range(args.steps):
             step(graphs)
+        torch.cuda.nvtx.range_pop()
         t1.record(stream)
         torch.cuda.synchronize()
         # kernel classes over the same period: the sampler's GEMMs alone and its quantizers alone
@@ -479,9 +481,22 @@ def gemm_matrix(torch, cl, WL, st, p16, p8, hbm, shape=(8192, 1152, 4608)):
                          "mma": "kind::mxf8f6f4" if fp8 else "kind::f16",
                          "peak_tflops": round(peak / 1e12, 1), "frac_roofline": round(t_roof / t, 4)})
             del ws
+    # the same weights with per-channel selection over the 4-bit palette (both MMA classes in one
+    # launch), E4M3 activations
+    fmt, _ = cl.select_weight_formats(W, W4_PALETTE)
+    d = cl.pack_plan(N, K, fmt.cpu().numpy())
+    blob, _ = cl.pack_weights(W, fmt, d, dev_status=st)
+    ws = torch.empty(cl.linear_workspace_size(M, d, 1), dtype=torch.uint8, device=dev)
+    cl.linear_prepare(X, d, 1, ws, st)
+    t = timed(lambda: cl.linear_gemm(X, d, blob, 1, None, Y, ws, st)) * 1e-3
+    f8 = d.n_class[0] / N
+    t_roof = fl * f8 / p8 + fl * (1 - f8) / p16
+    selected = {"act_fmt": 1, "w_fmt": "selected", "channels_fp8": int(d.n_class[0]), "channels_nf4": int(d.n_class[1]),
+                "us": round(t * 1e6, 2), "tflops": round(fl / t / 1e12, 1), "frac_roofline": round(t_roof / t, 4)}
+    del ws
     torch.cuda.synchronize()
     assert int(st.item()) == 0
-    return {"shape": [M, K, N], "reps": 20, "rows": rows,
+    return {"shape": [M, K, N], "reps": 20, "rows": rows, "selected": selected,
             "note": "act_fmt 0 INT8-asym, 1 E4M3, 2 E5M2, 3 MXFP8, 4 MXINT8, 5 fp16; w_fmt 0 INT8-sym, 1 INT8-asym, "
                     "2 MXINT8, 3 INT4-sym, 4 INT4-asym, 5 NF4, 6 E2M1, 7 MXINT4, 8 MXFP4"}
 
@@ -702,7 +717,9 @@ def dit_grouped(torch, cl, st, steps=20):
 def tensor_probe(torch, device):
     """Dense tcgen05 throughput this GPU sustains for the GEMM's instruction forms (the probe
     library of the build): kind::f16 (fp16 operands, the W8A8 path) and kind::f8f6f4 (E4M3),
-    M = 128, N = 192, on seeded finite operands.  Returns TFLOP/s per kind."""
+    M = 128, N = 192, on seeded finite operands; and, at the FP8 GEMM's N = 160, the forms that
+    GEMM issues: A from tensor memory (TS), with and without UE8M0 block scaling, and the
+    block-scaled form with A from shared memory.  Returns TFLOP/s per form."""
     import ctypes
     from paper_2609_33496_gb300 import build as B
     L = ctypes.CDLL(B.PROBE_LIB)
@@ -712,18 +729,19 @@ def tensor_probe(torch, device):
     st = torch.zeros(1, dtype=torch.int32, device=device)
     s = torch.cuda.current_stream()
     out = {}
-    for kind, name, K in ((0, "f16", 16), (2, "f8f6f4", 32)):
+    for kind, name, K, N in ((0, "f16", 16, 192), (2, "f8f6f4", 32, 192), (3, "f8f6f4_ts_n160", 32, 160),
+                             (4, "mxf8f6f4_ts_n160", 32, 160), (5, "mxf8f6f4_ss_n160", 32, 160)):
         iters, best = 4000, 0.0
         for _ in range(3):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(s)
-            rc = L.chameleon_probe_mma(kind, 192, sms, iters, ctypes.c_void_p(cyc.data_ptr()),
+            rc = L.chameleon_probe_mma(kind, N, sms, iters, ctypes.c_void_p(cyc.data_ptr()),
                                        ctypes.c_void_p(st.data_ptr()), ctypes.c_void_p(s.cuda_stream))
             e1.record(s)
             torch.cuda.synchronize()
             if rc != 0 or int(st.item()) != 0:
                 return None
-            best = max(best, sms * iters * 4 * 2.0 * 128 * 192 * K / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+            best = max(best, sms * iters * 4 * 2.0 * 128 * N * K / (e0.elapsed_time(e1) * 1e-3) / 1e12)
         out[name] = round(best, 1)
     return out
 
@@ -921,6 +939,55 @@ def reference_arm(args, world):
             "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+# ------------------------------------------------------------------ single kernel cases for profilers
+PROFILE_CASES = {
+    "gemm-pixart-qkv": "the stacked q/k/v GEMM of a PixArt-alpha block (8192 x 1152 x 3456), the 4-bit palette's "
+                       "per-channel selection, E4M3 activations with two per-sample scales: 3 GEMM launches",
+    "gemm-pixart-fc1": "PixArt-alpha fc1 (8192 x 1152 x 4608), as above: 3 GEMM launches",
+    "gemm-sdxl-geglu": "SDXL GEGLU-in (2048 x 1280 x 10240), W8 palette, E4M3: 3 GEMM launches (fp16 kernel)",
+    "quant-pixart-fc2": "the dynamic per-sample quantizer (range + encode) of PixArt-alpha fc2's input (8192 x 4608, "
+                        "E4M3, codes + fp16 operand for a layer with NF4 tiles): 3 calls",
+    "pack-w4": "selection and pack of PixArt-alpha fc1's weights (4608 x 1152) over the 4-bit palette: 3 pack launches",
+}
+
+
+def profile_case(name):
+    """Run one named case a few times (after one warm call) for a profiler; prints 'ok'."""
+    import torch
+    import paper_2609_33496_gb300 as P
+    from paper_2609_33496_gb300 import build as B
+    from paper_2609_33496_gb300 import workloads as WL
+    B.build()
+    cl = P.chameleon
+    dev = torch.device("cuda", 0)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    g = np.random.default_rng(20267000)
+    shapes = {"gemm-pixart-qkv": (8192, 1152, 3456, W4_PALETTE), "gemm-pixart-fc1": (8192, 1152, 4608, W4_PALETTE),
+              "gemm-sdxl-geglu": (2048, 1280, 10240, cl.PALETTE_W8), "quant-pixart-fc2": (8192, 4608, 1152, W4_PALETTE),
+              "pack-w4": (8192, 1152, 4608, W4_PALETTE)}
+    M, K, N, pal = shapes[name]
+    X = torch.from_numpy(WL.to_fp16(g.standard_t(7, (M, K)))).to(dev)
+    W = torch.from_numpy(WL.weight_mix_rows(g, N, K)).to(dev)
+    fmt, _ = cl.select_weight_formats(W, pal)
+    d = cl.pack_plan(N, K, fmt.cpu().numpy())
+    blob, _ = cl.pack_weights(W, fmt, d, dev_status=st)
+    ws = torch.empty(cl.linear_workspace_size(M, d, cl.A_E4M3), dtype=torch.uint8, device=dev)
+    Y = torch.empty((M, N), dtype=torch.float32, device=dev)
+    groups = 1 if name == "gemm-sdxl-geglu" else 2
+    cl.linear_prepare_groups(X, d, cl.A_E4M3, groups, ws, st)
+    for _ in range(4):
+        if name.startswith("gemm"):
+            cl.linear_gemm_ex(X, d, blob, cl.A_E4M3, groups, None, Y, ws, st)
+        elif name.startswith("quant"):
+            cl.linear_prepare_groups(X, d, cl.A_E4M3, groups, ws, st)
+        else:
+            cl.pack_weights(W, fmt, d, dev_status=st, blob=blob)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0, "device status %d" % int(st.item())
+    print("ok", name)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -932,9 +999,12 @@ def main():
     ap.add_argument("--no-variants", action="store_true", help="skip the sub-objects (config 2, per-variant tables)")
     ap.add_argument("--sampler-steps", type=int, default=20, help="sampler steps per benchmark step (smaller cases)")
     ap.add_argument("--oracle-sample", action="store_true", help=argparse.SUPPRESS)
+    ap.add_argument("--case", choices=sorted(PROFILE_CASES), help="run one kernel case for a profiler and exit")
     args = ap.parse_args()
     if args.oracle_sample:
         return oracle_sample_main()
+    if args.case:
+        return profile_case(args.case)
     args.warmup = max(args.warmup, 3)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

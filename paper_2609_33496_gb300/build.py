@@ -15,7 +15,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libchameleon.so")
 PROBE_LIB = os.path.join(HERE, "libchameleon_probe.so")   # tensor-core throughput probe (bench only)
 SOURCES = ["act_quant.cu", "weights.cu", "gemm.cu", "gemm_f16.cu", "gemm_bf16.cu", "gemm_f8.cu", "gemm_f8_mx.cu",
-           "api.cu", "noalloc.cu"]
+           "gemm_small.cu", "api.cu", "noalloc.cu"]
 # translation units whose quantizer arithmetic must not be contracted into FMAs
 NO_FMAD = {"act_quant.cu", "weights.cu"}
 HEADERS = ["common.cuh", "act_quant.cuh", "weights.cuh", "gemm.cuh", "gemm_kernel.cuh", "gemm_f8_kernel.cuh"]

@@ -20,17 +20,23 @@ namespace cham {
 constexpr int kUnroll = 4;       // independent 16-byte loads in flight per thread (encoders)
 constexpr int kRangeUnroll = 8;  // the range pass: a grid of range_grid CTAs reads the tensor in one round
 
-// min / max / non-finite flag of eight fp16 values packed in a uint4.
-CHAM_DEV void range8(const uint4& v, __half2& lo2, __half2& hi2, uint32_t& nonfinite) {
+// Running min / max of eight fp16 values packed in a uint4.  The NaN-propagating forms keep a NaN
+// lane in both results, and an infinity lands in one of them, so the non-finite test runs once
+// on the results (nonfinite_h2) instead of once per element.
+CHAM_DEV void range8(const uint4& v, __half2& lo2, __half2& hi2) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
-    // exponent field all ones in either half: Inf or NaN
-    nonfinite |= (((w[j] & 0x7C00u) == 0x7C00u) | ((w[j] & 0x7C000000u) == 0x7C000000u));
     const __half2 h = u32_as_h2(w[j]);
-    lo2 = __hmin2(lo2, h);
-    hi2 = __hmax2(hi2, h);
+    lo2 = __hmin2_nan(lo2, h);
+    hi2 = __hmax2_nan(hi2, h);
   }
+}
+
+// 1 when either half is Inf or NaN (exponent field all ones).
+CHAM_DEV uint32_t nonfinite_h2(__half2 h) {
+  const uint32_t w = h2_as_u32(h);
+  return ((w & 0x7C00u) == 0x7C00u) | ((w & 0x7C000000u) == 0x7C000000u);
 }
 
 // CTA-wide reduction of (lo, hi, nonfinite); the result is valid in every thread.
@@ -159,7 +165,6 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
   X += static_cast<int64_t>(blockIdx.y) * nvec;
   parts += static_cast<int64_t>(blockIdx.y) * gridDim.x;
   __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
-  uint32_t nonfinite = 0;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec;
        i0 += stride * kRangeUnroll) {
@@ -171,8 +176,9 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
     }
 #pragma unroll
     for (int u = 0; u < kRangeUnroll; ++u)
-      if (i0 + u * stride < nvec) range8(v[u], lo2, hi2, nonfinite);
+      if (i0 + u * stride < nvec) range8(v[u], lo2, hi2);
   }
+  uint32_t nonfinite = nonfinite_h2(lo2) | nonfinite_h2(hi2);
   float lo = fminf(__low2float(lo2), __high2float(lo2));
   float hi = fmaxf(__low2float(hi2), __high2float(hi2));
   block_range(lo, hi, nonfinite);

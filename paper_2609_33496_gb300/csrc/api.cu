@@ -221,10 +221,10 @@ struct OperandPlan {
   bool fp8;   // the FP8 kernel (1-byte codes, MXFP8: chunk-major exponents) over all tiles
   bool f16;   // some tiles multiply the fp16 operand (or X)
 };
-OperandPlan operand_plan(const cham_wpack_desc* d, int act_fmt) {
+OperandPlan operand_plan(int M, const cham_wpack_desc* d, int act_fmt) {
   const bool fp8_act = act_fmt == CHAM_A_E4M3 || act_fmt == CHAM_A_E5M2 || act_fmt == CHAM_A_MXFP8;
   OperandPlan o;
-  o.fp8 = fp8_act && d->bits == 4 && d->group == 0 && d->f16_only == 0 && d->n_tiles[0] > 0;
+  o.fp8 = fp8_act && d->bits == 4 && d->group == 0 && d->f16_only == 0 && d->n_tiles[0] > 0 && M > cham::kSmallM;
   o.f16 = !o.fp8 || d->n_tiles[1] > 0;
   return o;
 }
@@ -241,7 +241,7 @@ LinearWs linear_ws(int M, const cham_wpack_desc* d, int act_fmt) {
   const int K = d->K;
   const int64_t nvec = static_cast<int64_t>(M) * K / 8;
   const int parts = std::max(cham::range_grid(nvec, num_sms_current()), cham::kMaxGroups);
-  const OperandPlan o = operand_plan(d, act_fmt);
+  const OperandPlan o = operand_plan(M, d, act_fmt);
   LinearWs L{};
   L.scale = 0;
   L.parts = 256;
@@ -283,7 +283,10 @@ GemmPlan gemm_plan(int M, const cham_wpack_desc* d, int act_fmt) {
   GemmPlan g{};
   const int num_sms = num_sms_current();
   const int ch_tiles = d->n_tiles[0] + d->n_tiles[1];
-  if (operand_plan(d, act_fmt).fp8) {
+  if (M <= cham::kSmallM) {
+    g.bn = 0;          // the weight-streaming kernel: no token tiles, no split-K partial sums
+    g.k_split = 1;
+  } else if (operand_plan(M, d, act_fmt).fp8) {
     g.bn = cham::gemm_pick_bn_f8(M);
     g.k_split = cham::gemm_pick_split(ch_tiles * ((M + g.bn - 1) / g.bn), (d->Kp / 64 + 1) / 2, num_sms);
   } else {
@@ -949,7 +952,7 @@ cham_status prepare_common(const void* X, int M, const cham_wpack_desc* d, int a
   s = check_linear_common(M, K, act_fmt, ws, ws_bytes, L.end);
   if (s != CHAM_OK) return s;
   if (act_fmt == CHAM_A_FP16) return CHAM_OK;
-  const OperandPlan o = operand_plan(d, act_fmt);
+  const OperandPlan o = operand_plan(M, d, act_fmt);
   uint8_t* w = static_cast<uint8_t*>(ws);
   cham::ActQuantArgs a{};
   a.X = static_cast<const uint4*>(X);
@@ -1034,7 +1037,7 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
     return fail(CHAM_ERR_INVALID_ARG, "null or misaligned pointer");
   uint8_t* w = static_cast<uint8_t*>(ws);
   const LinearWs L = linear_ws(M, d, act_fmt);
-  const OperandPlan o = operand_plan(d, act_fmt);
+  const OperandPlan o = operand_plan(M, d, act_fmt);
   const float* act_scale = act_fmt <= CHAM_A_E5M2 ? reinterpret_cast<const float*>(w + L.scale) : nullptr;
   const uint8_t* b = static_cast<const uint8_t*>(blob);
   const int tiles = d->n_tiles[0] + d->n_tiles[1];
@@ -1074,6 +1077,14 @@ cham_status chameleon_linear_gemm_ex(const void* X, int M, const cham_wpack_desc
   g.n_ch_tiles = tiles;
   g.k_split = plan.k_split;
   g.partial = plan.k_split > 1 ? reinterpret_cast<float*>(w + plan.partial) : nullptr;
+  if (M <= cham::kSmallM) {
+    // a handful of tokens: weight streaming on the CUDA cores (one cluster per 64 channels)
+    const void* operand = act_fmt == CHAM_A_FP16 ? X : static_cast<const void*>(w + L.operand);
+    g.n_chunks = g.nk64;
+    const cudaError_t e = cham::launch_gemm_small(static_cast<const __half*>(operand), g,
+                                                  cham::gemm_small_split(tiles, g.nk64, num_sms), st);
+    return e == cudaSuccess ? CHAM_OK : cuda_fail(e, "small-M gemm launch");
+  }
   CUtensorMap map16;
   if (o.f16) {
     const void* operand = act_fmt == CHAM_A_FP16 ? X : static_cast<const void*>(w + L.operand);

@@ -45,6 +45,8 @@ struct GemmArgs {
 // Token tile of the FP8 kernel for M > 128: 160 leaves room in tensor memory for the scale factors
 // next to two accumulators and four decoded-weight slots.
 constexpr int kF8TokenTile = 160;
+// Up to this many tokens the linear runs on the weight-streaming kernel (gemm_small.cu).
+constexpr int kSmallM = 16;
 
 // Token-tile (MMA N) size for M tokens: 16, 32, 64, 128 or 192.
 int gemm_pick_bn(int M, int n_tiles, int num_sms);
@@ -63,6 +65,9 @@ cudaError_t launch_gemm_f8(const CUtensorMap& map8, const CUtensorMap& map16, co
 template <int YT, bool MXA>
 cudaError_t launch_gemm_f8_yt(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms,
                               int bn, cudaStream_t st);
+// The weight-streaming kernel for M <= kSmallM: ks K ranges per 64-channel CTA group (a cluster).
+int gemm_small_split(int n_ch_tiles, int n_chunks, int num_sms);
+cudaError_t launch_gemm_small(const __half* X, const GemmArgs& a, int ks, cudaStream_t st);
 // Split-K units' raw sums (EPI 6) and the reduction over the launch's tiles.
 cudaError_t launch_splitk_reduce(const GemmArgs& a, int num_sms, cudaStream_t st);
 // The launches of one output type (instantiated in gemm.cu, gemm_f16.cu, gemm_bf16.cu).

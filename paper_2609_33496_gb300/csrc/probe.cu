@@ -15,7 +15,9 @@ namespace cham {
 constexpr int kProbeOperand = 128 * 128;  // A tile: 128 rows x 128 bytes
 
 // kind: 0 = kind::f16, A from shared memory; 1 = kind::f16, A from tensor memory;
-//       2 = kind::f8f6f4 (E4M3 x E4M3), A from shared memory.
+//       2 = kind::f8f6f4 (E4M3 x E4M3), A from shared memory; 3 = the same, A from tensor memory;
+//       4 = kind::mxf8f6f4.block_scale (E4M3 x E4M3, UE8M0 scale factors in tensor memory), A from
+//       tensor memory -- the 4-bit GEMM's FP8 form; 5 = the same, A from shared memory.
 template <int KIND, int N>
 __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long long* cycles, int* status) {
   extern __shared__ uint8_t smem_raw[];
@@ -40,11 +42,20 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *slot;
-  if (KIND == 1) {  // A operand in columns 256..287 of every lane
+  const uint32_t lane_off = static_cast<uint32_t>((threadIdx.x >> 5) * 32) << 16;
+  if (KIND == 1 || KIND == 3 || KIND == 4) {  // A operand in columns 256..287 of every lane
     uint32_t z[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) z[i] = 0x30303030u + i;
-    tmem_st_32x32b_x32(tmem + 256 + ((threadIdx.x >> 5) * 32 << 16), z);
+    tmem_st_32x32b_x32(tmem + 256 + lane_off, z);
+    tmem_wait_st();
+  }
+  if (KIND >= 4) {  // scale factors 2^0 in every byte of columns 320..335 (A: 320.., B: 328..)
+    uint32_t one[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) one[i] = 0x7F7F7F7Fu;
+    tmem_st_32x32b_x8(tmem + 320 + lane_off, one);
+    tmem_st_32x32b_x8(tmem + 328 + lane_off, one);
     tmem_wait_st();
   }
   tc_fence_before();
@@ -53,7 +64,9 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
   if (threadIdx.x == 0) {
     const uint32_t a0 = smem_u32(sA), b0 = smem_u32(sB);
     uint32_t idesc = idesc_f16(128, N);
-    if (KIND == 2) idesc &= ~((7u << 7) | (7u << 10));  // E4M3 x E4M3 (format code 0), F32 D
+    if (KIND == 2 || KIND == 3) idesc &= ~((7u << 7) | (7u << 10));  // E4M3 x E4M3 (format code 0), F32 D
+    // kind::mxf8f6f4: E4M3 x E4M3, N, UE8M0 scale factors (bit 23), M; scale-factor ids added per MMA
+    const uint32_t idesc_mx = (static_cast<uint32_t>(N >> 3) << 17) | (1u << 23) | (128u >> 4 << 24);
     const unsigned long long t0 = clock64();
     for (int it = 0; it < iters; ++it) {
 #pragma unroll
@@ -67,6 +80,25 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
                        : "memory");
         } else if (KIND == 1) {
           mma_f16_ts(tmem, tmem + 256 + kk * 8, bd, idesc, 1u);
+        } else if (KIND == 3) {
+          asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+                       "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(tmem),
+                       "r"(tmem + 256 + kk * 8), "l"(bd), "r"(idesc), "r"(1u)
+                       : "memory");
+        } else if (KIND == 4) {
+          const uint32_t id = idesc_mx | (static_cast<uint32_t>(kk) << 4) | (static_cast<uint32_t>(kk) << 29);
+          asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %6, 0;\n\t"
+                       "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], [%1], %2, %3, [%4], "
+                       "[%5], p;\n\t}\n" ::"r"(tmem),
+                       "r"(tmem + 256 + kk * 8), "l"(bd), "r"(id), "r"(tmem + 320), "r"(tmem + 328), "r"(1u)
+                       : "memory");
+        } else if (KIND == 5) {
+          const uint32_t id = idesc_mx | (static_cast<uint32_t>(kk) << 4) | (static_cast<uint32_t>(kk) << 29);
+          asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %6, 0;\n\t"
+                       "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], %1, %2, %3, [%4], "
+                       "[%5], p;\n\t}\n" ::"r"(tmem),
+                       "l"(ad), "l"(bd), "r"(id), "r"(tmem + 320), "r"(tmem + 328), "r"(1u)
+                       : "memory");
         } else {
           asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
                        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(tmem),
@@ -99,7 +131,7 @@ static int launch_probe(int ctas, int iters, unsigned long long* cycles, int* st
 
 }  // namespace cham
 
-// kind 0..2 as above, n in {128, 192, 256}; ctas CTAs of 128 threads, one per SM; *cycles gets
+// kind 0..5 as above, n in {128, 160, 192, 256}; ctas CTAs of 128 threads, one per SM; *cycles gets
 // CTA 0's clock cycles.  Returns a cudaError_t value (-1 for an unsupported kind / n).
 extern "C" int chameleon_probe_mma(int kind, int n, int ctas, int iters, unsigned long long* cycles, int* status,
                                    void* stream) {
@@ -110,6 +142,9 @@ extern "C" int chameleon_probe_mma(int kind, int n, int ctas, int iters, unsigne
   PROBE_CASE(0, 128) PROBE_CASE(0, 192) PROBE_CASE(0, 256)
   PROBE_CASE(1, 128) PROBE_CASE(1, 192) PROBE_CASE(1, 256)
   PROBE_CASE(2, 128) PROBE_CASE(2, 192) PROBE_CASE(2, 256)
+  PROBE_CASE(3, 160) PROBE_CASE(3, 192)
+  PROBE_CASE(4, 160) PROBE_CASE(4, 192)
+  PROBE_CASE(5, 160) PROBE_CASE(5, 192)
 #undef PROBE_CASE
   return -1;
 }

@@ -238,14 +238,17 @@ def test_check_rejects_a_null_status_word(cl):
 
 def test_linear_workspace_includes_split_k_partials(cl):
     """The GEMM splits K when its 128-channel x token tiles are fewer than half the SMs and K has at
-    least 8 chunks of 64; the workspace then adds k_split x M x Np fp32 partial sums.  Without a
-    device the library assumes the 152 SMs of a GB300."""
+    least 8 chunks of 64; the workspace then adds k_split x M x Np fp32 partial sums.  Up to 16
+    tokens the weight-streaming kernel runs instead and needs none.  Without a device the library
+    assumes the 152 SMs of a GB300."""
     sms = 152
 
     def bn(M):
         return next(b for b in (16, 32, 64, 128) if M <= b) if M <= 128 else 192
 
     def expected_extra(M, N, K):
+        if M <= 16:          # the weight-streaming kernel: no split, no partial sums
+            return 0
         tiles = -(-N // 128) * -(-M // bn(M))
         nk = -(-K // 64)
         if tiles * 2 > sms or nk < 8:

@@ -83,6 +83,53 @@ def test_format_group_layout_every_activation(cl, M, K, N, fold):
         assert_within_bound(Y, Y_ref, bound, "layout 1 fold %d act %d" % (fold, act_fmt))
 
 
+@pytest.mark.parametrize("M", [1, 2, 8, 16])
+@pytest.mark.parametrize("K,N", [(320, 1280), (1280, 1280), (2048, 640)])
+def test_small_m_weight_streaming(cl, M, K, N):
+    """Up to 16 tokens the weight-streaming kernel runs (one cluster of K ranges per 64 channels):
+    the few-step fork's weight-only rows (SDXL-Turbo shapes at batch 1 to 16) with the mixed 4-bit
+    formats, the 8-bit palette with INT8-asym and MXFP8 activations, every element within the bound."""
+    g = np.random.default_rng(M * 7 + K + N)
+    X = WL.to_fp16(g.standard_t(4, (M, K)) * np.exp(0.1 * g.standard_normal(K))[None, :])
+    W = WL.weight_mix(g, N, K)
+    bias = g.normal(0, 0.02, N).astype(np.float32)
+    for pal, acts in ((F.W4_PALETTE, [F.A_FP16, F.A_E4M3]), (F.W8_PALETTE, [F.A_INT8_ASYM, F.A_MXFP8])):
+        fmt = np.asarray(pal, np.uint8)[g.integers(0, len(pal), N)]
+        for act_fmt in acts:
+            check(cl, X, W, fmt, act_fmt, bias, "small M%d K%d N%d act %d" % (M, K, N, act_fmt))
+
+
+def test_small_m_output_types_groups_and_group_wise_weights(cl):
+    """The weight-streaming kernel's epilogue: fp16 / bf16 outputs (the fp32 value rounded once),
+    two per-sample scales, and a group-wise blob (fp16 group scales in the decode)."""
+    import torch
+    g = np.random.default_rng(41)
+    M, K, N = 16, 640, 384
+    X = WL.to_fp16(g.standard_t(5, (M, K)))
+    W = WL.weight_mix(g, N, K)
+    fmt = np.asarray(F.W4_PALETTE, np.uint8)[g.integers(0, 6, N)]
+    d = cl.pack_plan(N, K, fmt)
+    blob, _ = cl.pack_weights(cuda(W), cuda(fmt), d)
+    for y_dtype in (torch.float32, torch.float16, torch.bfloat16):
+        Y, st = cl.linear_ex(cuda(X), d, blob, F.A_E5M2, n_groups=2, y_dtype=y_dtype)
+        torch.cuda.synchronize()
+        assert int(st.item()) == 0
+        qs = F.act_quant_per_sample(X, F.A_E5M2, 2)
+        a = F.act_dequant_per_sample(qs)
+        y_ref, bound = G.linear_rows_reference(a, SEL.dequant_selected(W, fmt), np.arange(M))
+        y = host(Y.float())
+        half = 0 if y_dtype == torch.float32 else np.abs(y_ref) * (2.0 ** -11 if y_dtype == torch.float16 else 2.0 ** -8)
+        assert_within_bound(y, y_ref, bound + half, "small M per-sample %s" % y_dtype)
+    dg = cl.pack_plan_grouped(N, K, F.W_INT4_ASYM, 64)
+    bg, _ = cl.pack_weights(cuda(W), cuda(np.full(N, F.W_INT4_ASYM, np.uint8)), dg)
+    Y, st = cl.linear(cuda(X), dg, bg, F.A_FP16)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    wq = SEL.grouped_dequant(W, 64, F.W_INT4_ASYM)
+    y_ref, bound = G.linear_rows_reference(X.astype(np.float64), wq, np.arange(M))
+    assert_within_bound(host(Y), y_ref, bound, "small M group-wise")
+
+
 CLASS0 = [F.W_INT4_SYM, F.W_INT4_ASYM, F.W_E2M1, F.W_MXINT4, F.W_MXFP4]
 
 
