@@ -287,7 +287,7 @@ GemmPlan gemm_plan(int M, const cham_wpack_desc* d, int act_fmt) {
     g.bn = 0;          // the weight-streaming kernel: no token tiles, no split-K partial sums
     g.k_split = 1;
   } else if (operand_plan(M, d, act_fmt).fp8) {
-    g.bn = cham::gemm_pick_bn_f8(M);
+    g.bn = cham::gemm_pick_bn_f8(M, act_fmt == CHAM_A_MXFP8);
     g.k_split = cham::gemm_pick_split(ch_tiles * ((M + g.bn - 1) / g.bn), (d->Kp / 64 + 1) / 2, num_sms);
   } else {
     g.bn = cham::gemm_pick_bn(M, ch_tiles, num_sms);

@@ -58,11 +58,11 @@ int gemm_pick_split(int tiles, int n_chunks, int num_sms) {
   return ks < 1 ? 1 : ks;
 }
 
-int gemm_pick_bn_f8(int M) {
+int gemm_pick_bn_f8(int M, bool mx) {
   if (M <= 32) return 32;
   if (M <= 64) return 64;
   if (M <= 128) return 128;
-  return kF8TokenTile;
+  return mx ? kF8TokenTileMx : kF8TokenTile;
 }
 
 cudaError_t launch_gemm_f8(const CUtensorMap& map8, const CUtensorMap& map16, const GemmArgs& a, int num_sms, int bn,

@@ -44,7 +44,8 @@ struct GemmArgs {
 
 // Token tile of the FP8 kernel for M > 128: 160 leaves room in tensor memory for the scale factors
 // next to two accumulators and four decoded-weight slots.
-constexpr int kF8TokenTile = 160;
+constexpr int kF8TokenTile = 192;    // per-tensor / per-sample activation scales
+constexpr int kF8TokenTileMx = 160;  // MXFP8 activations (their scale factors need tensor memory per slot)
 // Up to this many tokens the linear runs on the weight-streaming kernel (gemm_small.cu).
 constexpr int kSmallM = 16;
 
@@ -53,8 +54,8 @@ int gemm_pick_bn(int M, int n_tiles, int num_sms);
 // Split-K factor: 1 when the tiles fill the GPU, else enough K ranges (of at least two chunks)
 // to give every SM work.
 int gemm_pick_split(int tiles, int n_chunks, int num_sms);
-// Token tile of the FP8 kernel: 32, 64, 128 or kF8TokenTile.
-int gemm_pick_bn_f8(int M);
+// Token tile of the FP8 kernel: 32, 64, 128, or kF8TokenTile (kF8TokenTileMx for MXFP8 activations).
+int gemm_pick_bn_f8(int M, bool mx);
 // Persistent launch: min(tiles, num_sms) CTAs walk the (channel tile, token tile) grid.
 cudaError_t launch_gemm_f16(const CUtensorMap& act_map, const GemmArgs& a, int num_sms, int bn, cudaStream_t st);
 // The FP8 kernel (gemm_f8_kernel.cuh) over a 4-bit layout: its first f8_tiles channel tiles on

@@ -57,7 +57,7 @@ struct F8Cfg {
   static constexpr int kACol = 2 * kAccCols;
   // decoded-weight slots (32 columns each) with their A scale factors (8 columns each; MXFP8: and
   // their B scale factors, 8 more), as many as fit next to the accumulators, at most 8.  Every
-  // chunk is its own commit group: a slot goes back to the decoders as soon as its two MMAs have
+  // chunk is its own commit group: a slot goes back to the decoders as soon as its MMAs have
   // completed (pairs of chunks per commit measured 4-5 % slower on 8192 x 1152 x 4608)
   static constexpr int kPerSlot = 32 + 8 + (MXA ? 8 : 0);
   static constexpr int kAFit = (512 - kACol - (MXA ? 0 : 8)) / kPerSlot;
@@ -76,7 +76,7 @@ struct F8Cfg {
   static_assert(kSmem <= 227 * 1024, "within the opt-in shared-memory limit");
   static_assert(kNeedCols <= 512, "tensor memory budget");
   static_assert(kSFBCols <= 8, "B scale factors: 8 columns per copy");
-  static_assert(kAStages >= 4, "decoded-weight slots in flight");
+  static_assert(kAStages >= 3, "decoded-weight slots in flight");
   static_assert(kDone * kGroup > kStages + kGroup, "group barrier rotation");
 };
 
@@ -88,6 +88,21 @@ CHAM_DEV void mma_mxf8_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uin
       "setp.ne.b32 p, %6, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], [%1], %2, %3, [%4], [%5], p;\n\t}\n" ::"r"(
           d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
+// The same MMA issued by the warp's elected lane: the whole warp executes the instruction with
+// warp-uniform operands, one lane (the lowest active one, so always the same lane of a converged
+// warp) issues it.
+CHAM_DEV void mma_mxf8_ts_elect(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc, uint32_t sfa,
+                                uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred e, p;\n\t"
+      "elect.sync _|e, 0xffffffff;\n\t"
+      "setp.ne.b32 p, %6, 0;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], [%1], %2, %3, [%4], [%5], p;\n\t}\n" ::
+          "r"(d_tmem),
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
       : "memory");
 }
@@ -273,55 +288,55 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       for (uint32_t j = first; j < it; ++j) drain_wait(&full[j % S], (j / S) & 1);
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc8 = idesc_mxf8(128, BN, a.b_fmt);
-      constexpr uint32_t idesc16 = idesc_f16(128, BN);
-      const uint64_t desc0 = smem_desc_sw128(smem_u32(smem));
-      constexpr uint32_t kStageDesc = C::kStage >> 4;
-      uint32_t it = 0, acc_it = 0, s = 0, sa = 0, gi = 0;
-      bool ok = true;
-      for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++acc_it) {
-        const int b = acc_it & 1;
-        const int kc0 = kc_begin(u), kc1 = kc_end(u);
-        const bool f8 = is_f8(u);
-        if (!mbar_wait(&accempty[b], ((acc_it >> 1) & 1) ^ 1, abort_flag, a.dev_status)) break;
-        tc_fence_after();
-        const uint32_t d_tmem = tmem + b * C::kAccCols;
-        for (int kc = kc0; kc < kc1; ++kc, ++it) {
-          if (gi == 0) {
-            if (!mbar_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
+    // ---------------- MMA issuer.  The whole warp runs the loop, so the descriptors and counters
+    // are warp-uniform values; the MMAs and commits are issued by the elected lane (the lowest,
+    // the same one every time, so each commit covers every MMA issued before it)
+    const uint32_t idesc8 = idesc_mxf8(128, BN, a.b_fmt);
+    constexpr uint32_t idesc16 = idesc_f16(128, BN);
+    const uint64_t desc0 = smem_desc_sw128(smem_u32(smem));
+    constexpr uint32_t kStageDesc = C::kStage >> 4;
+    uint32_t it = 0, acc_it = 0, s = 0, sa = 0, gi = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++acc_it) {
+      const int b = acc_it & 1;
+      const int kc0 = kc_begin(u), kc1 = kc_end(u);
+      const bool f8 = is_f8(u);
+      if (!warp_wait(&accempty[b], ((acc_it >> 1) & 1) ^ 1, abort_flag, a.dev_status)) break;
+      tc_fence_after();
+      const uint32_t d_tmem = tmem + b * C::kAccCols;
+      for (int kc = kc0; kc < kc1; ++kc, ++it) {
+        if (gi == 0) {
+          if (!warp_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
+            ok = false;
+            break;
           }
-          const uint64_t bd = desc0 + s * kStageDesc;
-          const uint32_t ad = tmem + C::kACol + sa * 32;
-          if (f8) {
-            const uint32_t sfa = tmem + C::kSFA + sa * 8;
-            const uint32_t sfb = tmem + C::kSFB + (MXA ? sa * 8 : 0);
-            const int nmma = min(4, a.kblocks - 4 * kc);  // 32-element blocks of this chunk inside K
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-              if (i < nmma)
-                mma_mxf8_ts(d_tmem, ad + 8 * i, bd + 2 * i, idesc_sf_ids(idesc8, i), sfa, sfb, kc != kc0 || i > 0);
-          } else {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) mma_f16_ts(d_tmem, ad + 8 * i, bd + 2 * i, idesc16, kc != kc0 || i > 0);
-          }
-          if (++gi == kGroup || it + 1 == total) {
-            mma_commit(&done[(it / kGroup) % kDone]);
-            gi = gi == kGroup ? 0 : gi;
-          }
-          s = s + 1 == static_cast<uint32_t>(S) ? 0 : s + 1;
-          sa = sa + 1 == static_cast<uint32_t>(kAStages) ? 0 : sa + 1;
+          tc_fence_after();
         }
-        mma_commit(&accfull[b]);  // after an abort inside the tile this still covers every MMA issued
+        const uint64_t bd = desc0 + s * kStageDesc;
+        const uint32_t ad = tmem + C::kACol + sa * 32;
+        if (f8) {
+          const uint32_t sfa = tmem + C::kSFA + sa * 8;
+          const uint32_t sfb = tmem + C::kSFB + (MXA ? sa * 8 : 0);
+          const int nmma = min(4, a.kblocks - 4 * kc);  // 32-element blocks of this chunk inside K
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if (i < nmma)
+              mma_mxf8_ts_elect(d_tmem, ad + 8 * i, bd + 2 * i, idesc_sf_ids(idesc8, i), sfa, sfb, kc != kc0 || i > 0);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) mma_f16_ts_elect(d_tmem, ad + 8 * i, bd + 2 * i, idesc16, kc != kc0 || i > 0);
+        }
+        if (++gi == kGroup || it + 1 == total) {
+          mma_commit_elect(&done[(it / kGroup) % kDone]);
+          gi = gi == kGroup ? 0 : gi;
+        }
+        s = s + 1 == static_cast<uint32_t>(S) ? 0 : s + 1;
+        sa = sa + 1 == static_cast<uint32_t>(kAStages) ? 0 : sa + 1;
       }
-      // all issued MMAs have finished before tensor memory is released
-      if (acc_it > 0) drain_wait(&accfull[(acc_it - 1) & 1], ((acc_it - 1) >> 1) & 1);
+      mma_commit_elect(&accfull[b]);  // after an abort inside the tile this still covers every MMA issued
     }
+    // all issued MMAs have finished before tensor memory is released
+    if (lane == 0 && acc_it > 0) drain_wait(&accfull[(acc_it - 1) & 1], ((acc_it - 1) >> 1) & 1);
   } else if (warp >= 4 && warp < 4 + 4 * kDec) {
     // ---------------- weight decode: one channel per thread; group g takes chunks it % kDec == g
     const int q = warp & 3;
@@ -468,7 +483,10 @@ static cudaError_t launch_f8_epi(const CUtensorMap& map8, const CUtensorMap& map
     case 32: return launch_f8_bn<32, EPI, MXA>(map8, map16, a, num_sms, st);
     case 64: return launch_f8_bn<64, EPI, MXA>(map8, map16, a, num_sms, st);
     case 128: return launch_f8_bn<128, EPI, MXA>(map8, map16, a, num_sms, st);
-    default: return launch_f8_bn<kF8TokenTile, EPI, MXA>(map8, map16, a, num_sms, st);
+    default:
+      // the widest tile: kF8TokenTileMx for MXFP8 activations, kF8TokenTile otherwise
+      if constexpr (MXA) return launch_f8_bn<kF8TokenTileMx, EPI, MXA>(map8, map16, a, num_sms, st);
+      else return launch_f8_bn<kF8TokenTile, EPI, MXA>(map8, map16, a, num_sms, st);
   }
 }
 
