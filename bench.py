@@ -7,8 +7,9 @@ Headline workload: every linear of a PixArt-alpha-architecture DiT (28 blocks, h
 weight-format selection over the 4-bit palette {INT4-asym, NF4, E2M1, MXINT4, MXFP4} and the pack
 of all 282 layers, then 20 sampler steps (t = 999 - 50 i) in which every linear quantizes its input
 with each sample's own range (Alg. 3) in the format its (layer, timestep-bucket) table entry names
-and multiplies (fp32 outputs).  Linears that read the same tensor (q, k, v; cross k, v) run as one
-GEMM with their weights stacked along N: 198 GEMMs per sampler step, the same per-channel formats,
+and multiplies (fp32 outputs).  Linears that read the same tensor run as one GEMM with their
+weights stacked along N -- each block's q, k, v, and the cross-attention k, v of all 28 blocks
+(they all read the caption tokens): 171 GEMMs per sampler step, the same per-channel formats,
 activation codes and outputs.  Random-init weights, seeded synthetic activations.
 
 Sub-objects: the SDXL-UNet W8A8 projection step (static calibrated scales, Alg. 2), the GEMM for
@@ -719,7 +720,9 @@ def tensor_probe(torch, device):
     library of the build): kind::f16 (fp16 operands, the W8A8 path) and kind::f8f6f4 (E4M3),
     M = 128, N = 192, on seeded finite operands; and, at the FP8 GEMM's N = 160, the forms that
     GEMM issues: A from tensor memory (TS), with and without UE8M0 block scaling, and the
-    block-scaled form with A from shared memory.  Returns TFLOP/s per form."""
+    block-scaled form with A from shared memory; at N = 192 the TS block-scaled form alone and
+    with the GEMM's per-chunk commit + barrier wait + fence after every four MMAs.  Returns
+    TFLOP/s per form."""
     import ctypes
     from paper_2609_33496_gb300 import build as B
     L = ctypes.CDLL(B.PROBE_LIB)
@@ -730,7 +733,8 @@ def tensor_probe(torch, device):
     s = torch.cuda.current_stream()
     out = {}
     for kind, name, K, N in ((0, "f16", 16, 192), (2, "f8f6f4", 32, 192), (3, "f8f6f4_ts_n160", 32, 160),
-                             (4, "mxf8f6f4_ts_n160", 32, 160), (5, "mxf8f6f4_ss_n160", 32, 160)):
+                             (4, "mxf8f6f4_ts_n160", 32, 160), (5, "mxf8f6f4_ss_n160", 32, 160),
+                             (4, "mxf8f6f4_ts_n192", 32, 192), (6, "mxf8f6f4_ts_n192_per_chunk_commit_wait", 32, 192)):
         iters, best = 4000, 0.0
         for _ in range(3):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -1065,7 +1069,7 @@ def main():
                    "weight_formats": h["weight_formats"],
                    "lut": {str(b): v for b, v in lut_by_bucket.items()},
                    "activation_formats_used": h["acts"],
-                   "step": "selection + pack of the 282 layers, then 20 sampler steps x 198 GEMMs (per-sample "
+                   "step": "selection + pack of the 282 layers, then 20 sampler steps x 171 GEMMs (per-sample "
                            "dynamic quantizer + GEMM, one CUDA graph)",
                    "l2": "inputs larger than L2 (1.7 GB of activations, 0.3 GB of packed weights)",
                    "parallelism": "replicas" if world > 1 else "single-gpu"},

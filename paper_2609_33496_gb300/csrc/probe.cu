@@ -17,7 +17,9 @@ constexpr int kProbeOperand = 128 * 128;  // A tile: 128 rows x 128 bytes
 // kind: 0 = kind::f16, A from shared memory; 1 = kind::f16, A from tensor memory;
 //       2 = kind::f8f6f4 (E4M3 x E4M3), A from shared memory; 3 = the same, A from tensor memory;
 //       4 = kind::mxf8f6f4.block_scale (E4M3 x E4M3, UE8M0 scale factors in tensor memory), A from
-//       tensor memory -- the 4-bit GEMM's FP8 form; 5 = the same, A from shared memory.
+//       tensor memory -- the 4-bit GEMM's FP8 form; 5 = the same, A from shared memory; 6 = kind 4
+//       with the GEMM's per-chunk bookkeeping after every four MMAs: a commit to an mbarrier, an
+//       arrive-and-wait on another (a phase that is complete when tested) and the fence after it.
 template <int KIND, int N>
 __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long long* cycles, int* status) {
   extern __shared__ uint8_t smem_raw[];
@@ -25,7 +27,9 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
   uint8_t* sA = smem;
   uint8_t* sB = smem + kProbeOperand;
   uint64_t* bar = reinterpret_cast<uint64_t*>(sB + N * 128);
-  uint32_t* slot = reinterpret_cast<uint32_t*>(bar + 1);
+  uint64_t* bar2 = bar + 1;  // kind 6: per-iteration commits
+  uint64_t* bar3 = bar + 2;  // kind 6: per-iteration arrive + wait
+  uint32_t* slot = reinterpret_cast<uint32_t*>(bar + 3);
   __shared__ int abort_flag;
   // finite operands: bytes 0x30..0x3F are small positive E4M3 values, and as fp16 pairs they are
   // small positive normals
@@ -33,6 +37,8 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
     reinterpret_cast<uint32_t*>(smem)[i] = 0x30303030u + ((i * 2654435761u) >> 28) * 0x01010101u;
   if (threadIdx.x == 0) {
     mbar_init(bar, 1);
+    mbar_init(bar2, 1);
+    mbar_init(bar3, 1);
     abort_flag = 0;
     fence_mbar_init();
   }
@@ -43,7 +49,7 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
   tc_fence_after();
   const uint32_t tmem = *slot;
   const uint32_t lane_off = static_cast<uint32_t>((threadIdx.x >> 5) * 32) << 16;
-  if (KIND == 1 || KIND == 3 || KIND == 4) {  // A operand in columns 256..287 of every lane
+  if (KIND == 1 || KIND == 3 || KIND == 4 || KIND == 6) {  // A operand in columns 256..287 of every lane
     uint32_t z[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) z[i] = 0x30303030u + i;
@@ -85,7 +91,7 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
                        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(tmem),
                        "r"(tmem + 256 + kk * 8), "l"(bd), "r"(idesc), "r"(1u)
                        : "memory");
-        } else if (KIND == 4) {
+        } else if (KIND == 4 || KIND == 6) {
           const uint32_t id = idesc_mx | (static_cast<uint32_t>(kk) << 4) | (static_cast<uint32_t>(kk) << 29);
           asm volatile("{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %6, 0;\n\t"
                        "tcgen05.mma.cta_group::1.kind::mxf8f6f4.block_scale.scale_vec::1X [%0], [%1], %2, %3, [%4], "
@@ -105,6 +111,12 @@ __global__ void __launch_bounds__(128, 1) k_mma_probe(int iters, unsigned long l
                        "l"(ad), "l"(bd), "r"(idesc), "r"(1u)
                        : "memory");
         }
+      }
+      if (KIND == 6) {
+        mma_commit(bar2);
+        mbar_arrive(bar3);
+        if (!mbar_wait(bar3, it & 1, reinterpret_cast<volatile int*>(&abort_flag), status)) break;
+        tc_fence_after();
       }
     }
     mma_commit(bar);
@@ -131,7 +143,7 @@ static int launch_probe(int ctas, int iters, unsigned long long* cycles, int* st
 
 }  // namespace cham
 
-// kind 0..5 as above, n in {128, 160, 192, 256}; ctas CTAs of 128 threads, one per SM; *cycles gets
+// kind 0..6 as above, n in {128, 160, 192, 256}; ctas CTAs of 128 threads, one per SM; *cycles gets
 // CTA 0's clock cycles.  Returns a cudaError_t value (-1 for an unsupported kind / n).
 extern "C" int chameleon_probe_mma(int kind, int n, int ctas, int iters, unsigned long long* cycles, int* status,
                                    void* stream) {
@@ -145,6 +157,7 @@ extern "C" int chameleon_probe_mma(int kind, int n, int ctas, int iters, unsigne
   PROBE_CASE(3, 160) PROBE_CASE(3, 192)
   PROBE_CASE(4, 160) PROBE_CASE(4, 192)
   PROBE_CASE(5, 160) PROBE_CASE(5, 192)
+  PROBE_CASE(6, 160) PROBE_CASE(6, 192)
 #undef PROBE_CASE
   return -1;
 }

@@ -180,17 +180,25 @@ def pixart_model_linears():
 
 
 def pixart_model_gemms():
-    """The GEMM launches of one sampler step: consecutive linears that read the same input (q, k, v;
-    cross k, v) stacked along N into one GEMM -- each output channel keeps its own weights, format
-    and bias, and the shared input is quantized once, so the outputs are those of the separate
-    linears.  Entries: (names, M, K, N, input, [indices into pixart_model_linears()]); 198 GEMMs."""
+    """The GEMM launches of one sampler step.  Linears that read the same input tensor are stacked
+    along N into one GEMM -- each output channel keeps its own weights, format and bias, and the
+    shared input is quantized once, so the outputs are those of the separate linears: q, k, v of a
+    block (consecutive), and the cross-attention k and v of all 28 blocks, which read the same
+    caption tokens (they depend on nothing the blocks compute, so the one GEMM runs where block 0's
+    would).  Entries: (names, M, K, N, input, [indices into pixart_model_linears()]); 171 GEMMs."""
     out = []
+    text_at = None
     for i, (name, M, K, N, x) in enumerate(pixart_model_linears()):
         short = name.split(".", 1)[1] if name.startswith("block") else name
-        if out and out[-1][4] == x and out[-1][1] == M and out[-1][2] == K and short in ("self.k", "self.v", "cross.v"):
+        if x == "text" and text_at is not None:
+            names, _, _, n0, _, idx = out[text_at]
+            out[text_at] = (names + (name,), M, K, n0 + N, x, idx + [i])
+        elif out and out[-1][4] == x and out[-1][1] == M and out[-1][2] == K and short in ("self.k", "self.v"):
             names, _, _, n0, _, idx = out[-1]
             out[-1] = (names + (name,), M, K, n0 + N, x, idx + [i])
         else:
+            if x == "text":
+                text_at = len(out)
             out.append(((name,), M, K, N, x, [i]))
     return out
 
