@@ -47,8 +47,10 @@ FP8_OVER_BF16 = 2.0  # nominal dense FP8 / bf16 tensor rate (4.5 / 2.25 PFLOP/s 
 W4_PALETTE = (1 << 4) | (1 << 5) | (1 << 6) | (1 << 7) | (1 << 8)
 # dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant kernel from an ncu
 # capture (profiles/), with the launch it was and that launch's algorithmic bytes.  None whenever
-# the kernel has changed since the capture.
-GEMM_TRAFFIC_PER_LAUNCH = None
+# the kernel has changed since the capture.  Captured: k_gemm_ts_f8<192, 1, 0> on
+# `--case gemm-pixart-qkv`, one launch of the headline's stacked q/k/v GEMM at full size.
+GEMM_TRAFFIC_PER_LAUNCH = {"bytes": 138.6e6, "launch": "8192 x 1152 x 3456 (PixArt-alpha q/k/v stacked, E4M3, "
+                                                     "per-sample scales, fp32 Y)", "algorithmic_bytes": 143.5e6}
 
 
 def traffic_fields(t=GEMM_TRAFFIC_PER_LAUNCH):
@@ -209,16 +211,34 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
     fmt_all = torch.empty(int(offs[-1]), dtype=torch.uint8, device=device)
     fmt_host = torch.empty(int(offs[-1]), dtype=torch.uint8).pin_memory()
 
-    def select_all():
+    def select_layers():
         for i in range(n):
             cl.select_weight_formats(W[i], W4_PALETTE, fmt_out=fmt_all[offs[i]:offs[i + 1]])
-        fmt_host.copy_(fmt_all, non_blocking=True)
 
-    select_all()
+    select_layers()
+    fmt_host.copy_(fmt_all, non_blocking=True)
     torch.cuda.synchronize()
     f_ref = fmt_host.numpy().copy()
     descs = [cl.pack_plan(N, K, f_ref[offs[i]:offs[i + 1]]) for i, (_, M, K, N, _, _) in enumerate(linears)]
     blobs = [torch.empty(d.bytes, dtype=torch.uint8, device=device) for d in descs]
+
+    def pack_layers():
+        for i in range(n):
+            cl.pack_weights(W[i], fmt_all[offs[i]:offs[i + 1]], descs[i], dev_status=st, blob=blobs[i])
+
+    # the 171 selections and the 171 packs as two CUDA graphs (their arguments are the same every
+    # step; the plans are checked against the formats each step selects)
+    pack_layers()
+    torch.cuda.synchronize()
+    g_select, g_pack = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_select):
+        select_layers()
+    with torch.cuda.graph(g_pack):
+        pack_layers()
+
+    def select_all():
+        g_select.replay()
+        fmt_host.copy_(fmt_all, non_blocking=True)
 
     def plan_and_pack():
         """a6 for every layer, from the plans of the formats just selected (the same plans every
@@ -227,8 +247,7 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
         f = fmt_host.numpy()
         if not np.array_equal(f, f_ref):
             raise RuntimeError("the selected formats changed between steps")
-        for i in range(n):
-            cl.pack_weights(W[i], fmt_all[offs[i]:offs[i + 1]], descs[i], dev_status=st, blob=blobs[i])
+        g_pack.replay()
 
     acts = sorted(set(lut.values()))
     ws = torch.empty(max(cl.linear_workspace_size(M, descs[i], a) for i, (_, M, K, N, _, _) in enumerate(linears)
@@ -272,7 +291,8 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
         step(graphs)
     torch.cuda.synchronize()
 
-    # launches per benchmark step: selection and pack per layer; per linear the quantizer (range +
+    # launches per benchmark step: per layer the selection and the two pack kernels (slot plan and
+    # pack: the palette spans both MMA classes); per linear the quantizer (range +
     # encode for the per-tensor formats, one launch for MX) and the GEMM (+ the split-K reduction)
     per_linear = {}
     for b in buckets:
@@ -280,7 +300,7 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
             k = (i, lut[(key, b)])
             if k not in per_linear:
                 per_linear[k] = sum(cl.linear_launches(M, descs[i], lut[(key, b)], 2))
-    launches = 2 * n + sum(per_linear[(i, lut[(key, b)])] for b in buckets
+    launches = 3 * n + sum(per_linear[(i, lut[(key, b)])] for b in buckets
                            for i, (_, M, K, N, key, _) in enumerate(linears))
     flops_step = len(buckets) * sum(layer_flops(M, K, N) for (_, M, K, N, _, _) in linears)
 
@@ -297,7 +317,7 @@ def pixart_headline(args, torch, cl, WL, host, device, world, st):
         t1.record(stream)
         torch.cuda.synchronize()
         # kernel classes over the same period: the sampler's GEMMs alone and its quantizers alone
-        # (graph replays, once per timed step), and the selection + pack (eager)
+        # (graph replays, once per timed step), and the selection + pack (two graph replays)
         cls = {}
         for key in ("g", "q"):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -505,8 +525,8 @@ def gemm_matrix(torch, cl, WL, st, p16, p8, hbm, shape=(8192, 1152, 4608)):
 def quant_tables(torch, cl, WL, hbm):
     """The public quantizer (chameleon_act_quant: 1-byte codes, E8M0 exponents for MX, the range
     pass for per-tensor formats) per activation format: on one 8192x4608 tensor (PixArt-alpha fc2's
-    input), on each of the 22 distinct GEMM inputs of an SDXL-UNet step, and over those 22 in
-    aggregate.  Algorithmic bytes: 2 B read + 1 B code per element (+ 1/32 B for MX).  The tensors
+    input), on 8192x1152 tensors (its hidden states), on each of the 22 distinct GEMM inputs of an
+    SDXL-UNet step, and over those 22 in aggregate.  Algorithmic bytes: 2 B read + 1 B code per element (+ 1/32 B for MX).  The tensors
     are larger than L2 or, where not, their launches are back to back on distinct tensors."""
     dev = torch.device("cuda", torch.cuda.current_device())
     timed = graph_timer(torch, reps=10)
@@ -528,6 +548,27 @@ def quant_tables(torch, cl, WL, hbm):
         out["big"].append({"fmt": fmt, "M": 8192, "K": 4608, "us": round(t * 1e6, 2),
                            "gbs": round(byts / t / 1e9, 1), "frac_hbm": round(byts / t / hbm, 4)})
     del Xb
+    # PixArt-alpha's hidden-state shape (8192 x 1152, 18.9 MB): eight distinct tensors in turn, so
+    # that inputs and codes together (226 MB) exceed L2 between calls on the same tensor
+    Xh = [torch.from_numpy(WL.to_fp16(g.standard_t(5, (8192, 1152)))).to(dev) for _ in range(8)]
+    timed16 = graph_timer(torch, reps=16)
+    for fmt in range(5):
+        qb, wb = cl.act_quant_size(8192, 1152, fmt)
+        qs = [torch.empty(qb, dtype=torch.uint8, device=dev) for _ in range(8)]
+        ws = torch.empty(max(wb, 256), dtype=torch.uint8, device=dev)
+        stq = torch.zeros(1, dtype=torch.int32, device=dev)
+        turn = [0]
+
+        def call():
+            i = turn[0] % 8
+            turn[0] += 1
+            cl.act_quant(Xh[i], fmt, qact=qs[i], ws=ws, dev_status=stq)
+
+        t = timed16(call) * 1e-3
+        byts = 8192 * 1152 * (3 + (1 / 32 if fmt >= 3 else 0))
+        out["big"].append({"fmt": fmt, "M": 8192, "K": 1152, "us": round(t * 1e6, 2), "rotating_tensors": 8,
+                           "gbs": round(byts / t / 1e9, 1), "frac_hbm": round(byts / t / hbm, 4)})
+    del Xh
     tot = {f: [0.0, 0.0] for f in range(5)}
     for (M, K, N) in WL.UNET_STEP_SHAPES:
         X = torch.from_numpy(WL.to_fp16(g.standard_t(7, (M, K)))).to(dev)
@@ -952,6 +993,8 @@ PROFILE_CASES = {
     "quant-pixart-fc2": "the dynamic per-sample quantizer (range + encode) of PixArt-alpha fc2's input (8192 x 4608, "
                         "E4M3, codes + fp16 operand for a layer with NF4 tiles): 3 calls",
     "pack-w4": "selection and pack of PixArt-alpha fc1's weights (4608 x 1152) over the 4-bit palette: 3 pack launches",
+    "gemm-small-m16": "16 tokens x 1280 x 1280 (the small-M weight-streaming kernel), 4-bit palette, E4M3 with two "
+                      "per-sample scales: 3 GEMM launches",
 }
 
 
@@ -968,7 +1011,7 @@ def profile_case(name):
     g = np.random.default_rng(20267000)
     shapes = {"gemm-pixart-qkv": (8192, 1152, 3456, W4_PALETTE), "gemm-pixart-fc1": (8192, 1152, 4608, W4_PALETTE),
               "gemm-sdxl-geglu": (2048, 1280, 10240, cl.PALETTE_W8), "quant-pixart-fc2": (8192, 4608, 1152, W4_PALETTE),
-              "pack-w4": (8192, 1152, 4608, W4_PALETTE)}
+              "pack-w4": (8192, 1152, 4608, W4_PALETTE), "gemm-small-m16": (16, 1280, 1280, W4_PALETTE)}
     M, K, N, pal = shapes[name]
     X = torch.from_numpy(WL.to_fp16(g.standard_t(7, (M, K)))).to(dev)
     W = torch.from_numpy(WL.weight_mix_rows(g, N, K)).to(dev)
@@ -1082,7 +1125,7 @@ def main():
                      "fp8_flop_share": round(h["fl8"] / h["flops_step"], 4),
                      "frac_burst": round(achieved / peak_eff_b, 4), "peak_burst": round(peak_eff_b, 1),
                      "gemm_ms_per_step": round(gemm_ms, 3), "probe_tflops": probe,
-                     "timing": "value: selection + pack (eager) and one CUDA-graph replay of the sampler per step; "
+                     "timing": "value: selection + pack (two CUDA-graph replays, the formats checked on the host) and one CUDA-graph replay of the sampler per step; "
                                "GEMM class: the sampler's GEMM launches alone, graph-replayed once per timed step"},
         "act_quant": {"achieved_gbs": round(qgbs, 1), "peak_gbs": pk["hbm_gbs"], "frac": round(qgbs * 1e9 / hbm, 4),
                       "ms_per_step": round(h["classes_ms"]["q"], 3),
