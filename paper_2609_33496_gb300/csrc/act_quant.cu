@@ -13,6 +13,8 @@
 // in the order of readings R4-R8: inv by one correctly rounded division, the product x * inv
 // rounded to fp32, then the format rounding.  The same arithmetic gives the codes (public
 // chameleon_act_quant) and the exact fp16 operand values the GEMM consumes (R13).
+#include <cooperative_groups.h>
+
 #include "act_quant.cuh"
 
 namespace cham {
@@ -247,6 +249,63 @@ __global__ void __launch_bounds__(256)
   }
   encode_tensor_body<FMT, CODES, DEQ, false>(X + g * nvec, nvec, p, codes == nullptr ? nullptr : codes + g * nvec,
                                              deq == nullptr ? nullptr : deq + g * nvec, kperm);
+}
+
+// Dynamic path (Alg. 3) in one launch, for a tensor whose vectors fit in the registers of one
+// co-resident grid (a cooperative launch): every thread loads its kCoopVec vectors once, each CTA
+// writes its range partial, the grid meets at one barrier, every CTA reduces its group's
+// partials to the same ScaleZP and encodes the vectors it still holds.  X is read from DRAM once
+// and one launch replaces the range and encode launches.  Same grid shape as the range pass
+// (gridDim.x CTAs per group, 256 x kCoopVec vectors each), same results as the two-launch path.
+constexpr int kCoopVec = kRangeUnroll;
+template <int FMT, bool CODES, bool DEQ>
+__global__ void __launch_bounds__(256, 4)
+    k_act_quant_coop(const uint4* __restrict__ X, int64_t nvec, RangePartial* __restrict__ parts,
+                     uint2* __restrict__ codes, uint4* __restrict__ deq, cham_qparams* __restrict__ params,
+                     float* __restrict__ scale_out, int* dev_status, bool kperm) {
+  griddep_wait();  // X may be the previous kernel's output
+  const int64_t g = blockIdx.y;
+  const int P = gridDim.x;
+  X += g * nvec;
+  const int64_t i0 = static_cast<int64_t>(blockIdx.x) * (256 * kCoopVec) + threadIdx.x;
+  uint4 v[kCoopVec];
+  __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
+#pragma unroll
+  for (int u = 0; u < kCoopVec; ++u) {
+    const int64_t i = i0 + u * 256;
+    v[u] = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
+  }
+#pragma unroll
+  for (int u = 0; u < kCoopVec; ++u)
+    if (i0 + u * 256 < nvec) range8(v[u], lo2, hi2);
+  uint32_t nf = nonfinite_h2(lo2) | nonfinite_h2(hi2);
+  float lo = fminf(__low2float(lo2), __high2float(lo2));
+  float hi = fmaxf(__low2float(hi2), __high2float(hi2));
+  block_range(lo, hi, nf);
+  if (threadIdx.x == 0) {
+    parts[g * P + blockIdx.x] = RangePartial{lo, hi, static_cast<int>(nf), 0};
+    __threadfence();
+  }
+  cooperative_groups::this_grid().sync();
+  griddep_launch_dependents();
+  reduce_partials(parts + g * P, P, lo, hi, nf);
+  const TensorParams p = scale_zp(FMT, lo, hi);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    if (params != nullptr && g == 0) *params = cham_qparams{p.s, p.z, p.inv, FMT};
+    if (scale_out != nullptr) scale_out[g] = p.s;
+    if (nf) set_status(dev_status, CHAM_ERR_NONFINITE);
+  }
+#pragma unroll
+  for (int u = 0; u < kCoopVec; ++u) {
+    const int64_t i = i0 + u * 256;
+    if (i < nvec) {
+      uint2 c;
+      uint4 d;
+      encode8_tensor<FMT, DEQ>(v[u], p, c, d);
+      if constexpr (CODES) codes[g * nvec + i] = kperm ? kperm8(c) : c;
+      if constexpr (DEQ) deq[g * nvec + i] = d;
+    }
+  }
 }
 
 // Static path (Alg. 2): (s, z) fixed beforehand -- ScaleZP of the calibration range that Alg. 1
@@ -553,6 +612,25 @@ int group_grid(int64_t nvec, int n_groups, int num_sms) {
   return g < 1 ? 1 : g;
 }
 
+// CTAs of k_act_quant_coop that can be resident at once on this device (0 if unknown).
+template <int FMT, bool CODES, bool DEQ>
+static int64_t coop_capacity(int num_sms) {
+  static int cached_device = -1;
+  static int per_sm = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev != cached_device) {
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_act_quant_coop<FMT, CODES, DEQ>, 256, 0) != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    per_sm = n;
+    cached_device = dev;
+  }
+  return static_cast<int64_t>(per_sm) * num_sms;
+}
+
 template <int FMT, bool CODES, bool DEQ>
 static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
   if (a.use_static) {
@@ -568,6 +646,24 @@ static void launch_tensor(const ActQuantArgs& a, cudaStream_t st) {
   // per-sample groups: each group's range and encode grids are the per-tensor ones split evenly
   const int G = a.n_groups > 1 ? a.n_groups : 1;
   const int64_t nvg = a.nvec / G;
+  // one cooperative launch when the range pass's grid fits on the GPU at once and the partials'
+  // slots hold it
+  const int64_t P = (nvg + 256 * kCoopVec - 1) / (256 * kCoopVec);
+  if (P <= a.nparts && P * G <= coop_capacity<FMT, CODES, DEQ>(a.num_sms)) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(P), G);
+    cfg.blockDim = dim3(256);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, k_act_quant_coop<FMT, CODES, DEQ>, a.X, nvg, a.parts, a.codes, a.deq, a.params,
+                           a.scale_out, a.dev_status, a.kperm) == cudaSuccess)
+      return;
+    (void)cudaGetLastError();  // not launched: the two-launch path below
+  }
   launch_pdl(k_act_range, dim3(a.nparts, G), dim3(256), 0, st, a.X, nvg, a.parts);
   // the encode grid covers each group in one pass of kUnroll loads per thread (8 CTAs per SM at most)
   const int64_t want = (nvg + 256 * kUnroll - 1) / (256 * kUnroll);
