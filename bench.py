@@ -795,10 +795,11 @@ def tensor_probe(torch, device):
 def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     """The headline step through the public calls with HOST buffers: every benchmark step copies
     all 282 layers' weights and biases host->device from pinned memory (then selection and pack),
-    and every sampler step copies that step's seven input tensors host->device and reads the last
-    linear's output (block 27 fc2, the step's result) back device->host.  Uploads run on a copy
-    stream ahead of the compute; one bucket's inputs are uploaded while the previous bucket's
-    linears run."""
+    and every sampler step copies that step's input tensors host->device and reads the last
+    linear's output (block 27 fc2, the step's result) back device->host.  Copies run on a copy
+    stream beside the compute: a layer's selection starts as soon as its weights have landed, one
+    sampler step's inputs are uploaded while the previous step's linears run, and each step's
+    result is read back while the next step computes (two result buffers)."""
     import torch.distributed as dist
     Wn, bn, Xn = host
     linears = WL.pixart_model_gemms()
@@ -813,8 +814,8 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     bd = [torch.empty_like(b, device=device) for b in bh]
     Xd = [{k: torch.empty(WL.PIXART_INPUTS[k], dtype=torch.float16, device=device) for k in keys} for _ in range(2)]
     last = linears[-1]
-    Yd_last = torch.empty((last[1], last[3]), dtype=torch.float32, device=device)
-    Yh = torch.empty((last[1], last[3]), dtype=torch.float32).pin_memory()
+    Yd_last = [torch.empty((last[1], last[3]), dtype=torch.float32, device=device) for _ in range(2)]
+    Yh = [torch.empty((last[1], last[3]), dtype=torch.float32).pin_memory() for _ in range(2)]
     st = torch.zeros(1, dtype=torch.int32, device=device)
     offs = np.cumsum([0] + [N for (_, M, K, N, _, _) in linears])
     fmt_all = torch.empty(int(offs[-1]), dtype=torch.uint8, device=device)
@@ -836,13 +837,15 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     for k, (names, M, K, N, _, _) in zip(kind[:-1], linears[:-1]):
         if k not in Ys:
             Ys[k] = torch.empty((M, N), dtype=torch.float32, device=device)
-    Y = [Ys[k] for k in kind[:-1]] + [Yd_last]
+    Y = [Ys[k] for k in kind[:-1]]              # the last linear writes Yd_last (two buffers)
     x_ready = [torch.cuda.Event() for _ in range(2)]
     x_free = [torch.cuda.Event() for _ in range(2)]
-    w_ready, y_done = torch.cuda.Event(), torch.cuda.Event()
+    y_ready = [torch.cuda.Event() for _ in range(2)]
+    y_read = [torch.cuda.Event() for _ in range(2)]
+    w_ready = [torch.cuda.Event() for _ in range(n)]
     h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + \
         sum(Xh[(k, b)].numel() * 2 for b in buckets for k in keys)
-    d2h = len(buckets) * Yh.numel() * 4
+    d2h = len(buckets) * Yh[0].numel() * 4
 
     def step():
         with torch.cuda.stream(copy):
@@ -850,9 +853,9 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
             for i in range(n):
                 Wd[i].copy_(Wh[i], non_blocking=True)
                 bd[i].copy_(bh[i], non_blocking=True)
-            w_ready.record(copy)
-        compute.wait_event(w_ready)
+                w_ready[i].record(copy)
         for i in range(n):
+            compute.wait_event(w_ready[i])
             cl.select_weight_formats(Wd[i], W4_PALETTE, fmt_out=fmt_all[offs[i]:offs[i + 1]])
         fmt_host.copy_(fmt_all, non_blocking=True)
         compute.synchronize()
@@ -868,13 +871,20 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
                     Xd[buf][k].copy_(Xh[(k, b)], non_blocking=True)
                 x_ready[buf].record(copy)
             compute.wait_event(x_ready[buf])
+            compute.wait_event(y_read[buf])       # the result buffer's previous read-back is done
             for i, (names, M, K, N, key, _) in enumerate(linears):
-                cl.linear_ex(Xd[buf][key], descs[i], blobs[i], lut[(key, b)], 2, bias=bd[i], Y=Y[i], ws=ws,
+                yi = Yd_last[buf] if i == n - 1 else Y[i]
+                cl.linear_ex(Xd[buf][key], descs[i], blobs[i], lut[(key, b)], 2, bias=bd[i], Y=yi, ws=ws,
                              dev_status=st, stream=compute)
             x_free[buf].record(compute)
-            Yh.copy_(Yd_last, non_blocking=True)   # the step's result, read back on the compute stream
+            y_ready[buf].record(compute)
+            with torch.cuda.stream(copy):         # the step's result, read back beside the next step
+                copy.wait_event(y_ready[buf])
+                Yh[buf].copy_(Yd_last[buf], non_blocking=True)
+                y_read[buf].record(copy)
+        compute.wait_stream(copy)                 # every read-back of the step has landed
 
-    for e in x_free:
+    for e in x_free + y_read:
         e.record(compute)
     for _ in range(max(1, args.warmup - 1)):
         step()
