@@ -799,7 +799,7 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     linear's output (block 27 fc2, the step's result) back device->host.  Copies run on a copy
     stream beside the compute: a layer's selection starts as soon as its weights have landed, one
     sampler step's inputs are uploaded while the previous step's linears run, and each step's
-    result is read back while the next step computes (two result buffers)."""
+    result is read back on a third stream while the next step computes (two result buffers)."""
     import torch.distributed as dist
     Wn, bn, Xn = host
     linears = WL.pixart_model_gemms()
@@ -821,7 +821,8 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     fmt_all = torch.empty(int(offs[-1]), dtype=torch.uint8, device=device)
     fmt_host = torch.empty(int(offs[-1]), dtype=torch.uint8).pin_memory()
     compute = torch.cuda.current_stream()
-    copy = torch.cuda.Stream(device)
+    copy = torch.cuda.Stream(device)       # uploads
+    readback = torch.cuda.Stream(device)   # result read-backs (not queued behind the next uploads)
     for i in range(n):
         Wd[i].copy_(Wh[i])
     for i in range(n):
@@ -878,11 +879,11 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
                              dev_status=st, stream=compute)
             x_free[buf].record(compute)
             y_ready[buf].record(compute)
-            with torch.cuda.stream(copy):         # the step's result, read back beside the next step
-                copy.wait_event(y_ready[buf])
+            with torch.cuda.stream(readback):     # the step's result, read back beside the next step
+                readback.wait_event(y_ready[buf])
                 Yh[buf].copy_(Yd_last[buf], non_blocking=True)
-                y_read[buf].record(copy)
-        compute.wait_stream(copy)                 # every read-back of the step has landed
+                y_read[buf].record(readback)
+        compute.wait_stream(readback)             # every read-back of the step has landed
 
     for e in x_free + y_read:
         e.record(compute)
