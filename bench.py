@@ -1003,6 +1003,8 @@ PROFILE_CASES = {
     "gemm-sdxl-geglu": "SDXL GEGLU-in (2048 x 1280 x 10240), W8 palette, E4M3: 3 GEMM launches (fp16 kernel)",
     "quant-pixart-fc2": "the dynamic per-sample quantizer (range + encode) of PixArt-alpha fc2's input (8192 x 4608, "
                         "E4M3, codes + fp16 operand for a layer with NF4 tiles): 3 calls",
+    "quant-pixart-hidden": "the dynamic per-sample quantizer of a PixArt-alpha hidden-state input (8192 x 1152, E4M3, "
+                           "codes + fp16 operand): one cooperative launch, 3 calls",
     "pack-w4": "selection and pack of PixArt-alpha fc1's weights (4608 x 1152) over the 4-bit palette: 3 pack launches",
     "gemm-small-m16": "16 tokens x 1280 x 1280 (the small-M weight-streaming kernel), 4-bit palette, E4M3 with two "
                       "per-sample scales: 3 GEMM launches",
@@ -1022,6 +1024,7 @@ def profile_case(name):
     g = np.random.default_rng(20267000)
     shapes = {"gemm-pixart-qkv": (8192, 1152, 3456, W4_PALETTE), "gemm-pixart-fc1": (8192, 1152, 4608, W4_PALETTE),
               "gemm-sdxl-geglu": (2048, 1280, 10240, cl.PALETTE_W8), "quant-pixart-fc2": (8192, 4608, 1152, W4_PALETTE),
+              "quant-pixart-hidden": (8192, 1152, 1152, W4_PALETTE),
               "pack-w4": (8192, 1152, 4608, W4_PALETTE), "gemm-small-m16": (16, 1280, 1280, W4_PALETTE)}
     M, K, N, pal = shapes[name]
     X = torch.from_numpy(WL.to_fp16(g.standard_t(7, (M, K)))).to(dev)
