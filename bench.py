@@ -761,9 +761,9 @@ def tensor_probe(torch, device):
     library of the build): kind::f16 (fp16 operands, the W8A8 path) and kind::f8f6f4 (E4M3),
     M = 128, N = 192, on seeded finite operands; and, at the FP8 GEMM's N = 160, the forms that
     GEMM issues: A from tensor memory (TS), with and without UE8M0 block scaling, and the
-    block-scaled form with A from shared memory; at N = 192 the TS block-scaled form alone and
-    with the GEMM's per-chunk commit + barrier wait + fence after every four MMAs.  Returns
-    TFLOP/s per form."""
+    block-scaled form with A from shared memory; at N = 192 the TS block-scaled form alone, with
+    the GEMM's per-chunk commit + barrier wait + fence after every four MMAs, and the same from
+    two issuing threads into two accumulators.  Returns TFLOP/s per form."""
     import ctypes
     from paper_2609_33496_gb300 import build as B
     L = ctypes.CDLL(B.PROBE_LIB)
@@ -775,7 +775,8 @@ def tensor_probe(torch, device):
     out = {}
     for kind, name, K, N in ((0, "f16", 16, 192), (2, "f8f6f4", 32, 192), (3, "f8f6f4_ts_n160", 32, 160),
                              (4, "mxf8f6f4_ts_n160", 32, 160), (5, "mxf8f6f4_ss_n160", 32, 160),
-                             (4, "mxf8f6f4_ts_n192", 32, 192), (6, "mxf8f6f4_ts_n192_per_chunk_commit_wait", 32, 192)):
+                             (4, "mxf8f6f4_ts_n192", 32, 192), (6, "mxf8f6f4_ts_n192_per_chunk_commit_wait", 32, 192),
+                             (7, "mxf8f6f4_ts_n192_per_chunk_commit_wait_two_issuers", 32, 192)):
         iters, best = 4000, 0.0
         for _ in range(3):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
