@@ -155,6 +155,28 @@ CHAM_DEV uint2 kperm8(const uint2& c) {
   return make_uint2(lo, hi);
 }
 
+// ------------------------------------------------------------------ L2 eviction priority
+// The dynamic path reads X twice (range, then encode).  The range pass marks the lines it loads
+// as the last to evict, so that a tensor smaller than the L2 is still there for the encode pass;
+// the encode pass, their last use, marks them as the first.
+CHAM_DEV uint64_t l2_policy_keep() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+CHAM_DEV uint64_t l2_policy_drop() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+CHAM_DEV uint4 ldg_hint(const uint4* p, uint64_t pol) {
+  uint4 v;
+  asm volatile("ld.global.nc.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p), "l"(pol));
+  return v;
+}
+
 // ------------------------------------------------------------------ a2: range partials
 // Group blockIdx.y (rows split into gridDim.y equal groups, nvec vectors each; one group for a
 // per-tensor range) writes its gridDim.x partials at parts[blockIdx.y * gridDim.x ...].
@@ -167,6 +189,7 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
   X += static_cast<int64_t>(blockIdx.y) * nvec;
   parts += static_cast<int64_t>(blockIdx.y) * gridDim.x;
   __half2 lo2 = __float2half2_rn(65504.f), hi2 = __float2half2_rn(-65504.f);
+  const uint64_t keep = l2_policy_keep();
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec;
        i0 += stride * kRangeUnroll) {
@@ -174,7 +197,7 @@ __global__ void __launch_bounds__(256) k_act_range(const uint4* __restrict__ X, 
 #pragma unroll
     for (int u = 0; u < kRangeUnroll; ++u) {
       const int64_t i = i0 + u * stride;
-      v[u] = i < nvec ? __ldg(X + i) : make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);
+      v[u] = i < nvec ? ldg_hint(X + i, keep) : make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);
     }
 #pragma unroll
     for (int u = 0; u < kRangeUnroll; ++u)
@@ -199,17 +222,20 @@ CHAM_DEV uint32_t nonfinite8(const uint4& v) {
 
 // Grid-stride encode of the whole tensor with parameters p; CHECK also returns whether any input
 // lane was non-finite (the static path has no range pass to find out).
+// CHECK is the static path (one pass); otherwise X's lines are read for the last time here.
 template <int FMT, bool CODES, bool DEQ, bool CHECK>
 CHAM_DEV uint32_t encode_tensor_body(const uint4* __restrict__ X, int64_t nvec, const TensorParams& p,
                                      uint2* __restrict__ codes, uint4* __restrict__ deq, bool kperm) {
   uint32_t nf = 0;
+  const uint64_t drop = l2_policy_drop();
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i0 = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i0 < nvec; i0 += stride * kUnroll) {
     uint4 v[kUnroll];
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {
       const int64_t i = i0 + u * stride;
-      v[u] = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
+      if constexpr (CHECK) v[u] = i < nvec ? __ldg(X + i) : make_uint4(0, 0, 0, 0);
+      else v[u] = i < nvec ? ldg_hint(X + i, drop) : make_uint4(0, 0, 0, 0);
     }
 #pragma unroll
     for (int u = 0; u < kUnroll; ++u) {

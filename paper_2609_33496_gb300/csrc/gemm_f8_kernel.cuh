@@ -375,6 +375,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         if (static_cast<int>(it % kDec) != grp) continue;
         const int s = it % S, sa = it % kAStages;
         const uint32_t ph = (it / S) & 1;
+        // when S is not a multiple of the decode groups, the stage's previous chunk (it - S) is
+        // another group's, and testing this chunk's parity while that chunk's phase is still open
+        // would pass on the opposite parity.  That chunk's commit closes its phase (its MMAs
+        // follow its decode) and costs no extra wait: the producer waits for the same commit
+        // before it loads this chunk
+        if constexpr (S % kDec != 0) {
+          if (it >= static_cast<uint32_t>(S) && !__all_sync(0xffffffffu, wait_done(it - S))) {
+            ok = false;
+            break;
+          }
+        }
         if (!warp_wait(&full[s], ph, abort_flag, a.dev_status)) {
           ok = false;
           break;
