@@ -224,7 +224,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   };
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < S; ++s) mbar_init(&full[s], 1);
+    for (int s = 0; s < S; ++s) mbar_init(&full[s], 2);  // the two producer threads
     for (int g = 0; g < kDone; ++g) mbar_init(&done[g], 1);
     for (int g = 0; g < kAGroups; ++g) mbar_init(&afull[g], 4 * kGroup);
     for (int b = 0; b < 2; ++b) {
@@ -246,11 +246,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   griddep_wait();
   griddep_launch_dependents();
 
-  if (warp == 0) {
-    // ---------------- producer.  FP8 chunk: activation codes (TMA), two blob chunks of weight codes
-    // and their E8M0 bytes (bulk), MXFP8: the chunk's activation exponents of the tile's tokens
-    // (bulk).  NF4 chunk: fp16 operand (TMA) and one blob chunk of codes.
+  if (warp == 0 || warp == 3) {
+    // ---------------- producers: one chunk sequence, two threads.  Warp 0 loads the activation
+    // operand (TMA: FP8 codes, or the fp16 operand of an NF4 chunk) and, MXFP8, the chunk's
+    // activation exponents of the tile's tokens (bulk); warp 3 the weight codes (two blob chunks
+    // of 64, one for an NF4 chunk or the last FP8 chunk of an odd K) and their E8M0 bytes (bulk).
+    // Each arrives on the stage's barrier with its own byte count (the barrier counts two): issuing
+    // the copies is most of a producer's time per chunk, and one thread alone came close to the
+    // MMA thread's chunk period
     if (lane == 0) {
+      const bool act = warp == 0;
       uint32_t it = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
@@ -266,24 +271,31 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             break;
           }
           uint8_t* st = smem + s * C::kStage;
-          // FP8: the last chunk may hold one blob chunk; NF4: always one
-          const int nh = f8 ? (2 * kc + 1 < a.nk64 ? 2 : 1) : 1;
-          const size_t chunk64 = static_cast<size_t>(ch) * a.nk64 + (f8 ? 2 * kc : kc);
-          const uint32_t e_bytes = f8 ? nh * (C::kEBytes / 2) : 0u;
-          mbar_arrive_expect_tx(&full[s], C::kBBytes + nh * (C::kWBytes / 2) + e_bytes + (f8 ? sf_bytes : 0u));
-          if (blockIdx.x == 0 && static_cast<int>(it) == a.stall_chunk) continue;  // test hook (see the fp16 kernel)
-          if (f8) tma_load_2d(smem_u32(st), &map8, &full[s], kc * kBK8, tok0);
-          else tma_load_2d(smem_u32(st), &map16, &full[s], kc * kBK, tok0);
-          bulk_load(smem_u32(st + C::kBBytes), a.codes + chunk64 * (C::kWBytes / 2), nh * (C::kWBytes / 2), &full[s]);
-          if (f8) {
-            bulk_load(smem_u32(st + C::kBBytes + C::kWBytes), a.we8m0 + chunk64 * (C::kEBytes / 2), e_bytes, &full[s]);
+          const bool stall = blockIdx.x == 0 && static_cast<int>(it) == a.stall_chunk;  // test hook (see the fp16 kernel)
+          if (act) {
+            mbar_arrive_expect_tx(&full[s], C::kBBytes + (f8 ? sf_bytes : 0u));
+            if (stall) continue;
+            if (f8) tma_load_2d(smem_u32(st), &map8, &full[s], kc * kBK8, tok0);
+            else tma_load_2d(smem_u32(st), &map16, &full[s], kc * kBK, tok0);
             if constexpr (MXA)
-              bulk_load(smem_u32(st + C::kBBytes + C::kWBytes + C::kEBytes),
-                        a.act_e8 + static_cast<size_t>(kc) * a.act_e8_plane + static_cast<size_t>(tok0) * 4,
-                        sf_bytes, &full[s]);
+              if (f8)
+                bulk_load(smem_u32(st + C::kBBytes + C::kWBytes + C::kEBytes),
+                          a.act_e8 + static_cast<size_t>(kc) * a.act_e8_plane + static_cast<size_t>(tok0) * 4,
+                          sf_bytes, &full[s]);
+          } else {
+            const int nh = f8 ? (2 * kc + 1 < a.nk64 ? 2 : 1) : 1;
+            const size_t chunk64 = static_cast<size_t>(ch) * a.nk64 + (f8 ? 2 * kc : kc);
+            const uint32_t e_bytes = f8 ? nh * (C::kEBytes / 2) : 0u;
+            mbar_arrive_expect_tx(&full[s], nh * (C::kWBytes / 2) + e_bytes);
+            if (stall) continue;
+            bulk_load(smem_u32(st + C::kBBytes), a.codes + chunk64 * (C::kWBytes / 2), nh * (C::kWBytes / 2), &full[s]);
+            if (f8)
+              bulk_load(smem_u32(st + C::kBBytes + C::kWBytes), a.we8m0 + chunk64 * (C::kEBytes / 2), e_bytes,
+                        &full[s]);
           }
         }
       }
+      // every issued copy must have landed before the CTA may exit
       const uint32_t first = it > S ? it - S : 0;
       for (uint32_t j = first; j < it; ++j) drain_wait(&full[j % S], (j / S) & 1);
     }
@@ -297,6 +309,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     constexpr uint32_t kStageDesc = C::kStage >> 4;
     uint32_t it = 0, acc_it = 0, s = 0, sa = 0, gi = 0;
     bool ok = true;
+    bool ready = false;  // the chunk's decoded operands are known to be in place (tested a chunk ahead)
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++acc_it) {
       const int b = acc_it & 1;
       const int kc0 = kc_begin(u), kc1 = kc_end(u);
@@ -306,12 +319,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const uint32_t d_tmem = tmem + b * C::kAccCols;
       for (int kc = kc0; kc < kc1; ++kc, ++it) {
         if (gi == 0) {
-          if (!warp_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
+          if (!ready && !warp_wait(&afull[(it / kGroup) % kAGroups], (it / kAStages) & 1, abort_flag, a.dev_status)) {
             ok = false;
             break;
           }
           tc_fence_after();
         }
+        // test the next chunk's barrier now (its previous phases were all waited for here, in
+        // order): the result is used after this chunk's MMAs and commit, so the test's latency,
+        // a fifth of the chunk period when it sat in front of the MMAs, hides behind them
+        const uint32_t nx = it + 1;
+        const bool nready = static_cast<int>(nx % kGroup) == 0 && nx < total &&
+                            mbar_ready(&afull[(nx / kGroup) % kAGroups], (nx / kAStages) & 1);
         const uint64_t bd = desc0 + s * kStageDesc;
         const uint32_t ad = tmem + C::kACol + sa * 32;
         if (f8) {
@@ -332,6 +351,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         s = s + 1 == static_cast<uint32_t>(S) ? 0 : s + 1;
         sa = sa + 1 == static_cast<uint32_t>(kAStages) ? 0 : sa + 1;
+        ready = __all_sync(0xffffffffu, nready);
       }
       mma_commit_elect(&accfull[b]);  // after an abort inside the tile this still covers every MMA issued
     }
