@@ -794,13 +794,21 @@ def tensor_probe(torch, device):
 
 # ------------------------------------------------------------------ end to end through host buffers
 def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
-    """The headline step through the public calls with HOST buffers: every benchmark step copies
+    """The headline step through the public calls with HOST buffers.  Every benchmark step copies
     all 282 layers' weights and biases host->device from pinned memory (then selection and pack),
     and every sampler step copies that step's input tensors host->device and reads the last
-    linear's output (block 27 fc2, the step's result) back device->host.  Copies run on a copy
-    stream beside the compute: a layer's selection starts as soon as its weights have landed, one
-    sampler step's inputs are uploaded while the previous step's linears run, and each step's
-    result is read back on a third stream while the next step computes (two result buffers)."""
+    linear's output (block 27 fc2, the step's result) back device->host.  The copies run on their
+    own streams beside the compute, as a serving loop would run them:
+    * the fp16 weights are read only by selection and pack, so the next step's weights upload
+      while this step's sampler runs (the first timed step's weights were uploaded by the last
+      warm-up step, and the last timed step uploads weights for a step that is not run: one
+      1.2 GB upload per timed step all the same); the biases, which the sampler reads, upload at
+      the start of the step;
+    * one sampler step's inputs upload while the previous sampler step's linears run (two input
+      buffers), and each result is read back on a third stream (two result buffers);
+    * each sampler step's 171 `chameleon_linear` calls (quantizer + GEMM per call, as
+      `linear_ex` issues them) are captured once in a CUDA graph and replayed, so the host does
+      not pace the GPU; selection and pack are issued eagerly every step."""
     import torch.distributed as dist
     Wn, bn, Xn = host
     linears = WL.pixart_model_gemms()
@@ -813,7 +821,8 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     Xh = {kb: torch.from_numpy(x).pin_memory() for kb, x in Xn.items() if kb[1] in set(buckets)}
     Wd = [torch.empty_like(w, device=device) for w in Wh]
     bd = [torch.empty_like(b, device=device) for b in bh]
-    Xd = [{k: torch.empty(WL.PIXART_INPUTS[k], dtype=torch.float16, device=device) for k in keys} for _ in range(2)]
+    # zero-filled: the pass before the graphs are captured runs on them (finite values)
+    Xd = [{k: torch.zeros(WL.PIXART_INPUTS[k], dtype=torch.float16, device=device) for k in keys} for _ in range(2)]
     last = linears[-1]
     Yd_last = [torch.empty((last[1], last[3]), dtype=torch.float32, device=device) for _ in range(2)]
     Yh = [torch.empty((last[1], last[3]), dtype=torch.float32).pin_memory() for _ in range(2)]
@@ -822,15 +831,19 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     fmt_all = torch.empty(int(offs[-1]), dtype=torch.uint8, device=device)
     fmt_host = torch.empty(int(offs[-1]), dtype=torch.uint8).pin_memory()
     compute = torch.cuda.current_stream()
-    copy = torch.cuda.Stream(device)       # uploads
+    copy = torch.cuda.Stream(device)       # input and bias uploads
+    wcopy = torch.cuda.Stream(device)      # weight uploads (the inputs are not queued behind them)
     readback = torch.cuda.Stream(device)   # result read-backs (not queued behind the next uploads)
     for i in range(n):
         Wd[i].copy_(Wh[i])
+        bd[i].copy_(bh[i])
     for i in range(n):
         cl.select_weight_formats(Wd[i], W4_PALETTE, fmt_out=fmt_all[offs[i]:offs[i + 1]])
     f_ref = fmt_all.cpu().numpy()
     descs = [cl.pack_plan(N, K, f_ref[offs[i]:offs[i + 1]]) for i, (_, M, K, N, _, _) in enumerate(linears)]
     blobs = [torch.empty(d.bytes, dtype=torch.uint8, device=device) for d in descs]
+    for i in range(n):
+        cl.pack_weights(Wd[i], fmt_all[offs[i]:offs[i + 1]], descs[i], dev_status=st, blob=blobs[i])
     acts = sorted(set(lut.values()))
     ws = torch.empty(max(cl.linear_workspace_size(M, descs[i], a) for i, (_, M, K, N, _, _) in enumerate(linears)
                          for a in acts), dtype=torch.uint8, device=device)
@@ -844,20 +857,47 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     x_free = [torch.cuda.Event() for _ in range(2)]
     y_ready = [torch.cuda.Event() for _ in range(2)]
     y_read = [torch.cuda.Event() for _ in range(2)]
-    w_ready = [torch.cuda.Event() for _ in range(n)]
+    w_ready, b_ready, packed = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
     h2d = sum(w.numel() * 2 + b.numel() * 4 for w, b in zip(Wh, bh)) + \
         sum(Xh[(k, b)].numel() * 2 for b in buckets for k in keys)
     d2h = len(buckets) * Yh[0].numel() * 4
 
-    def step():
-        with torch.cuda.stream(copy):
-            copy.wait_stream(compute)             # the previous step no longer reads the weights
+    def sampler_step(s, b):
+        buf = s % 2
+        for i, (names, M, K, N, key, _) in enumerate(linears):
+            yi = Yd_last[buf] if i == n - 1 else Y[i]
+            cl.linear_ex(Xd[buf][key], descs[i], blobs[i], lut[(key, b)], 2, bias=bd[i], Y=yi, ws=ws,
+                         dev_status=st)
+
+    for s, b in enumerate(buckets):              # eager once, then captured
+        sampler_step(s, b)
+    torch.cuda.synchronize()
+    if int(st.item()) != 0:
+        raise RuntimeError("device status %d before capture" % int(st.item()))
+    graphs = []
+    for s, b in enumerate(buckets):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            sampler_step(s, b)
+        graphs.append(g)
+    torch.cuda.synchronize()
+    st.zero_()
+
+    def upload_weights():
+        with torch.cuda.stream(wcopy):
+            wcopy.wait_event(packed)             # selection and pack have read the weights
             for i in range(n):
                 Wd[i].copy_(Wh[i], non_blocking=True)
+            w_ready.record(wcopy)
+
+    def step():
+        with torch.cuda.stream(copy):
+            copy.wait_stream(compute)            # the previous sampler no longer reads the biases
+            for i in range(n):
                 bd[i].copy_(bh[i], non_blocking=True)
-                w_ready[i].record(copy)
+            b_ready.record(copy)
+        compute.wait_event(w_ready)              # this step's weights (uploaded during the last one)
         for i in range(n):
-            compute.wait_event(w_ready[i])
             cl.select_weight_formats(Wd[i], W4_PALETTE, fmt_out=fmt_all[offs[i]:offs[i + 1]])
         fmt_host.copy_(fmt_all, non_blocking=True)
         compute.synchronize()
@@ -865,6 +905,9 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
             raise RuntimeError("the selected formats changed between steps")
         for i in range(n):
             cl.pack_weights(Wd[i], fmt_all[offs[i]:offs[i + 1]], descs[i], dev_status=st, blob=blobs[i])
+        packed.record(compute)
+        upload_weights()                         # the next step's, beside this step's sampler
+        compute.wait_event(b_ready)
         for s, b in enumerate(buckets):
             buf = s % 2
             with torch.cuda.stream(copy):
@@ -873,21 +916,19 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
                     Xd[buf][k].copy_(Xh[(k, b)], non_blocking=True)
                 x_ready[buf].record(copy)
             compute.wait_event(x_ready[buf])
-            compute.wait_event(y_read[buf])       # the result buffer's previous read-back is done
-            for i, (names, M, K, N, key, _) in enumerate(linears):
-                yi = Yd_last[buf] if i == n - 1 else Y[i]
-                cl.linear_ex(Xd[buf][key], descs[i], blobs[i], lut[(key, b)], 2, bias=bd[i], Y=yi, ws=ws,
-                             dev_status=st, stream=compute)
+            compute.wait_event(y_read[buf])      # the result buffer's previous read-back is done
+            graphs[s].replay()
             x_free[buf].record(compute)
             y_ready[buf].record(compute)
-            with torch.cuda.stream(readback):     # the step's result, read back beside the next step
+            with torch.cuda.stream(readback):    # the step's result, read back beside the next step
                 readback.wait_event(y_ready[buf])
                 Yh[buf].copy_(Yd_last[buf], non_blocking=True)
                 y_read[buf].record(readback)
-        compute.wait_stream(readback)             # every read-back of the step has landed
+        compute.wait_stream(readback)            # every read-back of the step has landed
 
-    for e in x_free + y_read:
+    for e in x_free + y_read + [packed]:
         e.record(compute)
+    upload_weights()
     for _ in range(max(1, args.warmup - 1)):
         step()
     torch.cuda.synchronize()
@@ -897,16 +938,25 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     t0.record(compute)
     for _ in range(args.steps):
         step()
+    compute.wait_stream(wcopy)                   # the uploads issued in the timed steps have landed
     t1.record(compute)
     torch.cuda.synchronize()
     ms = t0.elapsed_time(t1)
     if world > 1:
         ms = max_over_ranks(ms, device)
-    assert int(st.item()) == 0
+    if int(st.item()) != 0:
+        raise RuntimeError("device status %d after the e2e steps" % int(st.item()))
+    # the last read-back holds the final sampler step's result of block 27 fc2
+    buf = (len(buckets) - 1) % 2
+    if not np.isfinite(Yh[buf].numpy()).all():
+        raise RuntimeError("non-finite values in the step's result")
     return {"value": round(job_tflops(flops_step, args.steps, world, ms), 3), "unit": "TFLOP/s",
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms / args.steps, 3),
             "calls": "chameleon_select_weight_formats, chameleon_pack_plan, chameleon_pack_weights, "
-                     "chameleon_linear_prepare_groups + chameleon_linear_gemm_ex"}
+                     "chameleon_linear_prepare_groups + chameleon_linear_gemm_ex (each sampler step's calls "
+                     "captured once in a CUDA graph)",
+            "pipelining": "next step's weights upload during this step's sampler; inputs double-buffered; "
+                          "read-backs on a third stream"}
 
 
 # ------------------------------------------------------------------ the oracle as CPU baseline
