@@ -17,7 +17,9 @@ Modules
   gemm      fp64 reference of the quantized linear and its error bound
   nf4       NormalFloat-4 level construction (cited at App. A.11)
 
-Parity unpinned: the NF4 level values beyond their structural invariants and an independent
-re-computation of the same quantile construction (the paper prints no NF4 table).
+Pins: every function is checked against something outside itself (closed forms, worked values,
+library routines, brute force, planted mistakes).  The NF4 levels, for which the paper cites
+QLoRA without printing a table, are checked against the table QLoRA publishes
+(``tests/golden/``).
 """
 from . import formats, schedule, select, gemm, nf4  # noqa: F401
