@@ -800,10 +800,10 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     linear's output (block 27 fc2, the step's result) back device->host.  The copies run on their
     own streams beside the compute, as a serving loop would run them:
     * the fp16 weights are read only by selection and pack, so the next step's weights upload
-      while this step's sampler runs (the first timed step's weights were uploaded by the last
-      warm-up step, and the last timed step uploads weights for a step that is not run: one
-      1.2 GB upload per timed step all the same); the biases, which the sampler reads, upload at
-      the start of the step;
+      while this step's sampler runs, one slice behind each sampler step's inputs on the input
+      stream (the first timed step's weights were uploaded by the last warm-up step, and the last
+      timed step uploads weights for a step that is not run: one 1.2 GB upload per timed step all
+      the same); the biases, which the sampler reads, upload at the start of the step;
     * one sampler step's inputs upload while the previous sampler step's linears run (two input
       buffers), and each result is read back on a third stream (two result buffers);
     * each sampler step's 171 `chameleon_linear` calls (quantizer + GEMM per call, as
@@ -883,6 +883,8 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     torch.cuda.synchronize()
     st.zero_()
 
+    wslices = np.array_split(np.arange(n), len(buckets))
+
     def upload_weights():
         with torch.cuda.stream(wcopy):
             wcopy.wait_event(packed)             # selection and pack have read the weights
@@ -906,7 +908,6 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
         for i in range(n):
             cl.pack_weights(Wd[i], fmt_all[offs[i]:offs[i + 1]], descs[i], dev_status=st, blob=blobs[i])
         packed.record(compute)
-        upload_weights()                         # the next step's, beside this step's sampler
         compute.wait_event(b_ready)
         for s, b in enumerate(buckets):
             buf = s % 2
@@ -915,6 +916,14 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
                 for k in keys:
                     Xd[buf][k].copy_(Xh[(k, b)], non_blocking=True)
                 x_ready[buf].record(copy)
+                # the next step's weights, one slice behind each sampler step's inputs on the same
+                # stream: the inputs, which the next sampler step waits for, go first on the link
+                if s == 0:
+                    copy.wait_event(packed)      # selection and pack have read the weights
+                for i in wslices[s]:
+                    Wd[i].copy_(Wh[i], non_blocking=True)
+                if s == len(buckets) - 1:
+                    w_ready.record(copy)
             compute.wait_event(x_ready[buf])
             compute.wait_event(y_read[buf])      # the result buffer's previous read-back is done
             graphs[s].replay()
@@ -938,7 +947,7 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     t0.record(compute)
     for _ in range(args.steps):
         step()
-    compute.wait_stream(wcopy)                   # the uploads issued in the timed steps have landed
+    compute.wait_stream(copy)                    # the uploads issued in the timed steps have landed
     t1.record(compute)
     torch.cuda.synchronize()
     ms = t0.elapsed_time(t1)
@@ -950,13 +959,27 @@ def pixart_e2e(args, torch, cl, WL, host, lut, device, world, flops_step):
     buf = (len(buckets) - 1) % 2
     if not np.isfinite(Yh[buf].numpy()).all():
         raise RuntimeError("non-finite values in the step's result")
+    # host->device bandwidth alone, after the timed steps: the step's weight uploads twice over,
+    # nothing else running; h2d / that rate is the copy time a step cannot go below
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    wbytes = sum(w.numel() * 2 for w in Wh)
+    with torch.cuda.stream(wcopy):
+        e0.record(wcopy)
+        for _ in range(2):
+            for i in range(n):
+                Wd[i].copy_(Wh[i], non_blocking=True)
+        e1.record(wcopy)
+    torch.cuda.synchronize()
+    h2d_gbs = 2 * wbytes / (e0.elapsed_time(e1) * 1e-3) / 1e9
     return {"value": round(job_tflops(flops_step, args.steps, world, ms), 3), "unit": "TFLOP/s",
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms / args.steps, 3),
             "calls": "chameleon_select_weight_formats, chameleon_pack_plan, chameleon_pack_weights, "
                      "chameleon_linear_prepare_groups + chameleon_linear_gemm_ex (each sampler step's calls "
                      "captured once in a CUDA graph)",
             "pipelining": "next step's weights upload during this step's sampler; inputs double-buffered; "
-                          "read-backs on a third stream"}
+                          "read-backs on a third stream",
+            "h2d_gbs_alone": round(h2d_gbs, 2),
+            "h2d_ms_per_step_at_that_rate": round(h2d / (h2d_gbs * 1e9) * 1e3, 1)}
 
 
 # ------------------------------------------------------------------ the oracle as CPU baseline
